@@ -1,0 +1,273 @@
+"""Forward-Forward CPU oracle.  TEST INFRASTRUCTURE ONLY.
+
+A plain, slow, obviously-correct fp64 NumPy statement of what the FF train
+step and FF goodness prediction compute, written from "Going Forward-Forward
+in Distributed Deep Learning" (arXiv 2404.08573).  Only ``tests/``,
+``__graft_entry__.smoke()`` and ``bench.py`` (its CPU-baseline and reference
+legs) may import this module.  The CUDA library never calls it, and it shares
+no code, header, table or constant with the CUDA path.
+
+What each function follows:
+
+* ``overlay_label``   -- §3 "Negative Data": a 1-of-C label written into a
+  10-feature area; correct label for positive rows, wrong label for negative.
+* ``normalise``       -- x / max(||x||_2, 1e-12) per row, applied to each
+  layer's input (the normalisation of Hinton's FF, cited in §2/§3; the paper
+  itself does not restate it).
+* ``layer_forward``   -- §3 "Goodness Function": rectified linear neurons,
+  y = ReLU(x_hat W^T + b); §4 notation L_i(x).
+* ``goodness``        -- Eq. 1: sum_j y_j^2.
+* ``p_real``          -- Eq. 1: sigma(sum_j y_j^2 - theta).
+* ``ff_loss``/``dloss_dg`` -- the negative log-likelihood of Eq. 1: -log p for
+  positive rows, -log(1-p) for negative rows, i.e. softplus(theta - g_pos) +
+  softplus(g_neg - theta), averaged over the B pairs.
+* ``layer_train_step`` -- one local (layer-wise, §2/§3) update: the gradient of
+  the layer's own loss w.r.t. its own W, b only (no gradient crosses layers),
+  then Adam (§5.1).
+* ``net_train_step``  -- §4: x is the concatenation of the positive and the
+  negative data; layer i trains on L_{i-1}(x) computed with the weights that
+  layer i-1 had before this step's update.
+* ``predict``         -- §3 "Prediction", Goodness method: run the input with
+  each of the 10 labels, accumulate goodness over all but the first hidden
+  layer, pick the label with the largest total.
+
+Readings of points the paper leaves open (the paper states none of them):
+
+1. Loss = mean over the B pairs of softplus(theta-g_pos) + softplus(g_neg-theta).
+2. Normalisation x/max(||x||,1e-12) of every layer input, after the overlay.
+3. Overlay *replaces* features 0..9 with a one-hot of value 1.0.
+4. Adam with beta1=0.9, beta2=0.999, eps=1e-8, bias-corrected, eps outside
+   the square root, no weight decay; the step counter t starts at 1.
+5. ReLU derivative at 0 is 0.
+6. Prediction sums goodness of layers 2..L (layer 1 when L == 1); ties go to
+   the lowest label.
+7. The layer input fed to the next layer is the ReLU activity computed with
+   the pre-update weights of the same step.
+
+``emulate_bf16=True`` rounds (round-to-nearest-even) the operands that the
+bf16-operand mode stores in bfloat16 -- the layer's input activity, W, the
+activity used in the local gradient, and the weight-gradient operand s*dZ --
+and keeps every sum in fp64.  With the rounding replaced by the identity it
+reduces to the plain definition (a test pins that).
+"""
+
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+N_CLASSES = 10
+NORM_EPS = 1e-12
+
+
+# ----------------------------------------------------------------- rounding
+def bf16_round(a):
+    """Round to the nearest bfloat16 (8 significant bits), ties to even.
+
+    Written from the format's definition: a = m * 2**e with 0.5 <= |m| < 1;
+    keep 8 significant bits of m by rounding m * 2**8 to an integer (numpy's
+    ``rint`` rounds halves to even).  Finite, normal-range values only.
+    """
+    a = np.asarray(a, dtype=np.float64)
+    m, e = np.frexp(a)
+    return np.ldexp(np.rint(m * 256.0), e - 8)
+
+
+def _identity(a):
+    return np.asarray(a, dtype=np.float64)
+
+
+# ---------------------------------------------------------------- §3 pieces
+def overlay_label(x, labels, n_classes: int = N_CLASSES):
+    """§3 Negative Data: write one-hot(label) into features 0..n_classes-1."""
+    out = np.array(x, dtype=np.float64, copy=True)
+    labels = np.asarray(labels, dtype=np.int64)
+    out[:, :n_classes] = 0.0
+    out[np.arange(out.shape[0]), labels] = 1.0
+    return out
+
+
+def row_norm(x):
+    x = np.asarray(x, dtype=np.float64)
+    return np.sqrt(np.sum(x * x, axis=1))
+
+
+def normalise(x):
+    """x_hat = x / max(||x||_2, 1e-12), row by row (a zero row stays zero)."""
+    x = np.asarray(x, dtype=np.float64)
+    return x / np.maximum(row_norm(x), NORM_EPS)[:, None]
+
+
+def layer_forward(x_hat, W, b):
+    """§3: activities of rectified linear neurons, y = ReLU(x_hat W^T + b).
+
+    Returns (Z, H): the pre-activation and the activity."""
+    Z = np.asarray(x_hat, dtype=np.float64) @ np.asarray(W, dtype=np.float64).T + np.asarray(b, dtype=np.float64)
+    return Z, np.maximum(Z, 0.0)
+
+
+def goodness(H):
+    """Eq. 1: g = sum_j y_j^2 for each row."""
+    H = np.asarray(H, dtype=np.float64)
+    return np.sum(H * H, axis=1)
+
+
+def sigmoid(t):
+    t = np.asarray(t, dtype=np.float64)
+    e = np.exp(-np.abs(t))
+    return np.where(t >= 0, 1.0 / (1.0 + e), e / (1.0 + e))
+
+
+def softplus(t):
+    """log(1 + e^t), as max(t, 0) + log1p(e^-|t|)."""
+    t = np.asarray(t, dtype=np.float64)
+    return np.maximum(t, 0.0) + np.log1p(np.exp(-np.abs(t)))
+
+
+def p_real(g, theta):
+    """Eq. 1: p(real) = sigma(g - theta)."""
+    return sigmoid(np.asarray(g, dtype=np.float64) - theta)
+
+
+def ff_loss(g, theta, B):
+    """-log p(real) on the B positive rows plus -log(1 - p(real)) on the B
+    negative rows (Eq. 1), averaged over the B pairs."""
+    g = np.asarray(g, dtype=np.float64)
+    pos, neg = g[:B], g[B:2 * B]
+    return float((np.sum(softplus(theta - pos)) + np.sum(softplus(neg - theta))) / B)
+
+
+def dloss_dg(g, theta, B):
+    """d ff_loss / d g_i: -sigma(theta - g)/B on positive rows,
+    +sigma(g - theta)/B on negative rows."""
+    g = np.asarray(g, dtype=np.float64)
+    d = np.empty_like(g)
+    d[:B] = -sigmoid(theta - g[:B]) / B
+    d[B:2 * B] = sigmoid(g[B:2 * B] - theta) / B
+    return d
+
+
+# ------------------------------------------------------------------- §5.1 Adam
+@dataclass
+class AdamHyper:
+    lr: float = 0.03
+    beta1: float = 0.9
+    beta2: float = 0.999
+    eps: float = 1e-8
+
+
+def adam_update(w, grad, m, v, t, hp: AdamHyper):
+    """Adam (Kingma & Ba), step t >= 1, bias-corrected.  Returns (w, m, v)."""
+    grad = np.asarray(grad, dtype=np.float64)
+    m = hp.beta1 * np.asarray(m, dtype=np.float64) + (1.0 - hp.beta1) * grad
+    v = hp.beta2 * np.asarray(v, dtype=np.float64) + (1.0 - hp.beta2) * grad * grad
+    m_hat = m / (1.0 - hp.beta1 ** t)
+    v_hat = v / (1.0 - hp.beta2 ** t)
+    w = np.asarray(w, dtype=np.float64) - hp.lr * m_hat / (np.sqrt(v_hat) + hp.eps)
+    return w, m, v
+
+
+# ------------------------------------------------------------ one FF layer
+@dataclass
+class LayerState:
+    W: np.ndarray          # [out, in]
+    b: np.ndarray          # [out]
+    mW: np.ndarray = None
+    vW: np.ndarray = None
+    mb: np.ndarray = None
+    vb: np.ndarray = None
+    t: int = 0
+
+    def __post_init__(self):
+        self.W = np.array(self.W, dtype=np.float64)
+        self.b = np.array(self.b, dtype=np.float64)
+        for name, like in (("mW", self.W), ("vW", self.W), ("mb", self.b), ("vb", self.b)):
+            cur = getattr(self, name)
+            setattr(self, name, np.zeros_like(like) if cur is None else np.array(cur, dtype=np.float64))
+
+    def copy(self):
+        return LayerState(self.W.copy(), self.b.copy(), self.mW.copy(), self.vW.copy(),
+                          self.mb.copy(), self.vb.copy(), self.t)
+
+
+def layer_forward_full(state: LayerState, x_in, emulate_bf16=False):
+    """L_i(x) of §4 for one layer, on the raw (un-normalised) layer input.
+
+    Returns dict(s, A, Z, H, g): s = 1/max(||x_in||, eps) per row, A the GEMM
+    operand (x_in, rounded to bf16 when emulating), Z = s*(A W^T) + b, H, g.
+    """
+    rnd = bf16_round if emulate_bf16 else _identity
+    x_in = np.asarray(x_in, dtype=np.float64)
+    s = 1.0 / np.maximum(row_norm(x_in), NORM_EPS)
+    A = rnd(x_in)
+    x_hat = s[:, None] * A                       # the normalised input
+    Z, H = layer_forward(x_hat, rnd(state.W), state.b)
+    return dict(s=s, A=A, x_hat=x_hat, Z=Z, H=H, g=goodness(H))
+
+
+def layer_train_step(state: LayerState, x_in, B: int, theta: float, hp: AdamHyper,
+                     emulate_bf16: bool = False, rounding=None):
+    """One local FF update of one layer (§3, Eq. 1; Adam of §5.1).
+
+    x_in: [2B, in] raw layer input (rows 0..B-1 positive, B..2B-1 negative;
+    for layer 1 already label-overlaid).  Mutates ``state``; returns a dict
+    with the forward quantities (H, g, s), the loss and the gradients.
+    ``rounding`` overrides the bf16 rounding function (tests use the identity).
+    """
+    rnd = rounding if rounding is not None else (bf16_round if emulate_bf16 else _identity)
+    emul = emulate_bf16 or rounding is not None
+    x_in = np.asarray(x_in, dtype=np.float64)
+    assert x_in.shape[0] == 2 * B
+    s = 1.0 / np.maximum(row_norm(x_in), NORM_EPS)
+    A = rnd(x_in)
+    x_hat = s[:, None] * A
+    Z, H = layer_forward(x_hat, rnd(state.W), state.b)
+    g = goodness(H)
+    loss = ff_loss(g, theta, B)
+    c = dloss_dg(g, theta, B)
+    # local gradient dL/dz = dL/dg * 2h * [z > 0]   (no gradient leaves the layer)
+    Hg = rnd(H) if emul else H
+    dZ = 2.0 * c[:, None] * Hg * (Z > 0)
+    if emul:
+        G = rnd(s[:, None] * dZ)               # weight-gradient operand, as stored
+        dW = G.T @ A
+    else:
+        dW = dZ.T @ x_hat                      # dL/dW = dZ^T x_hat
+    db = np.sum(dZ, axis=0)
+    state.t += 1
+    state.W, state.mW, state.vW = adam_update(state.W, dW, state.mW, state.vW, state.t, hp)
+    state.b, state.mb, state.vb = adam_update(state.b, db, state.mb, state.vb, state.t, hp)
+    return dict(H=H, g=g, s=s, loss=loss, dW=dW, db=db, c=c)
+
+
+def net_train_step(states, x_raw, labels, B: int, theta: float, hp: AdamHyper,
+                   emulate_bf16: bool = False):
+    """§4: one batch through every layer; layer k+1 trains on layer k's
+    activity from the same step (pre-update weights).  Returns per-layer dicts."""
+    x_in = overlay_label(x_raw, labels)
+    outs = []
+    for st in states:
+        o = layer_train_step(st, x_in, B, theta, hp, emulate_bf16=emulate_bf16)
+        outs.append(o)
+        x_in = o["H"]
+    return outs
+
+
+# ------------------------------------------------------------------ predict
+def predict(states, x_raw, emulate_bf16: bool = False, n_classes: int = N_CLASSES):
+    """§3 Prediction (Goodness): for every label c, overlay c, run all layers,
+    sum the goodness of layers 2..L (layer 1 if L == 1); argmax over c, the
+    lowest label winning ties.  Returns (pred [n] int64, G [n, n_classes])."""
+    x_raw = np.asarray(x_raw, dtype=np.float64)
+    n = x_raw.shape[0]
+    L = len(states)
+    G = np.zeros((n, n_classes), dtype=np.float64)
+    for c in range(n_classes):
+        a = overlay_label(x_raw, np.full(n, c))
+        for k, st in enumerate(states):
+            f = layer_forward_full(st, a, emulate_bf16=emulate_bf16)
+            if k >= 1 or L == 1:
+                G[:, c] += f["g"]
+            a = f["H"]
+    return np.argmax(G, axis=1), G

@@ -1,0 +1,334 @@
+"""Pins of the CPU oracle against facts fixed by the paper and by mathematics.
+
+None of these compares the oracle with itself: each checks a closed form, an
+invariant, a library routine, finite differences, or brute force on tiny
+inputs, chosen so that a dropped term, a wrong sign or index, or a transposed
+operand in the oracle fails at least one of them.
+"""
+
+import json
+import math
+import os
+
+import numpy as np
+import pytest
+
+from oracle import ff_oracle as fo
+from paper_2404_08573_gb300 import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _golden(name):
+    with open(os.path.join(GOLDEN, name)) as f:
+        return json.load(f)
+
+
+# ------------------------------------------------------------ bf16 rounding
+def test_bf16_round_matches_torch_conversion():
+    """RNE to bfloat16 equals PyTorch's float32 -> bfloat16 conversion."""
+    torch = pytest.importorskip("torch")
+    rng = np.random.default_rng(1)
+    vals = np.concatenate([
+        rng.standard_normal(20000).astype(np.float32),
+        (rng.standard_normal(5000) * 1e-20).astype(np.float32),
+        (rng.standard_normal(5000) * 1e20).astype(np.float32),
+    ])
+    # exact ties: 8 significant bits plus a half ulp
+    base = (rng.integers(128, 256, 2000) * 2 + 1).astype(np.float64)   # odd 9-bit ints
+    ties = (base * 2.0 ** rng.integers(-20, 20, 2000)).astype(np.float32)
+    vals = np.concatenate([vals, ties, -ties, np.zeros(3, np.float32)])
+    ref = torch.from_numpy(vals).to(torch.bfloat16).to(torch.float64).numpy()
+    got = fo.bf16_round(vals.astype(np.float64))
+    assert np.array_equal(got, ref)
+
+
+# ------------------------------------------------------------------ overlay
+def test_overlay_is_exact_one_hot_and_leaves_rest_untouched():
+    x = synth.mnist_like(64, seed=3).astype(np.float64)
+    x[:, :10] = 0.37   # nonzero under the label area: overlay must replace
+    y = synth.labels(64, seed=3)
+    o = fo.overlay_label(x, y)
+    assert np.array_equal(o[:, :10], np.eye(10)[y])
+    assert np.array_equal(o[:, 10:], x[:, 10:])
+    assert np.array_equal(x[:, :10], np.full((64, 10), 0.37))   # input not mutated
+
+
+# -------------------------------------------------------------- normalise
+def test_normalise_unit_norm_zero_row_and_scale_invariance():
+    x = synth.mnist_like(200, seed=5).astype(np.float64)
+    x[7] = 0.0
+    xh = fo.normalise(x)
+    n = np.sqrt(np.sum(xh ** 2, axis=1))
+    nz = np.arange(200) != 7
+    assert np.max(np.abs(n[nz] - 1.0)) <= 4 * np.finfo(np.float64).eps
+    assert np.all(xh[7] == 0.0)
+    assert np.allclose(fo.normalise(3.5 * x), xh, rtol=0, atol=1e-15)
+
+
+# --------------------------------------------------------------- goodness
+def test_goodness_of_hand_built_layers():
+    K = 6
+    x = np.abs(np.random.default_rng(2).standard_normal((5, K))) * 3.0   # x >= 0, not unit norm
+    st = fo.LayerState(np.eye(K), np.zeros(K))
+    f = fo.layer_forward_full(st, x)
+    assert np.allclose(f["g"], 1.0, atol=1e-14)           # W = I: g = ||x_hat||^2 = 1
+    st = fo.LayerState(-np.eye(K), np.zeros(K))
+    assert np.all(fo.layer_forward_full(st, x)["g"] == 0.0)  # W = -I: all units off
+    # one active unit: g = z^2
+    W = np.zeros((3, 2)); W[1, 0] = 2.0
+    b = np.array([-1.0, 0.25, -3.0])
+    xx = np.array([[3.0, 4.0]])                           # x_hat = (0.6, 0.8)
+    g = fo.layer_forward_full(fo.LayerState(W, b), xx)["g"]
+    assert g[0] == pytest.approx((2.0 * 0.6 + 0.25) ** 2, abs=1e-15)
+
+
+# ------------------------------------------------------------------- loss
+def test_loss_closed_forms():
+    gold = _golden("closed_forms.json")
+    B, theta = 7, 2.0
+    g = np.full(2 * B, theta)
+    assert fo.ff_loss(g, theta, B) == pytest.approx(gold["loss_at_threshold"], abs=1e-15)
+    d = fo.dloss_dg(g, theta, B)
+    assert np.allclose(d[:B], -0.5 / B, atol=1e-17) and np.allclose(d[B:], 0.5 / B, atol=1e-17)
+    # p(real) at the threshold is 1/2 (Eq. 1)
+    assert fo.p_real(theta, theta) == 0.5
+    # large margins: positives far above, negatives far below -> loss ~ 0
+    g2 = np.concatenate([np.full(B, theta + 60.0), np.full(B, theta - 60.0)])
+    assert 0.0 < fo.ff_loss(g2, theta, B) < 2 * math.exp(-59)
+    # wrong-way margins: loss ~ 2 * 60 per pair
+    g3 = np.concatenate([np.full(B, theta - 60.0), np.full(B, theta + 60.0)])
+    assert fo.ff_loss(g3, theta, B) == pytest.approx(120.0, rel=1e-12)
+    # mirror: swapping the pos/neg halves and reflecting g about theta keeps L
+    rng = np.random.default_rng(4)
+    g4 = theta + rng.standard_normal(2 * B)
+    g5 = np.concatenate([2 * theta - g4[B:], 2 * theta - g4[:B]])
+    assert fo.ff_loss(g5, theta, B) == pytest.approx(fo.ff_loss(g4, theta, B), rel=1e-14)
+    # -log p(real) definition for one positive pair member, written out
+    p = 1.0 / (1.0 + math.exp(-(g4[0] - theta)))
+    q = 1.0 / (1.0 + math.exp(-(g4[B] - theta)))
+    one = fo.ff_loss(np.array([g4[0], g4[B]]), theta, 1)
+    assert one == pytest.approx(-math.log(p) - math.log(1.0 - q), rel=1e-13)
+
+
+def test_softplus_stable_branch_agrees_with_naive():
+    t = np.linspace(-30, 30, 601)
+    assert np.allclose(fo.softplus(t), np.log1p(np.exp(t)), rtol=1e-14, atol=1e-300)
+    assert fo.softplus(np.array([800.0]))[0] == 800.0
+
+
+# -------------------------------------------------------------- gradients
+def _layer_loss(W, b, x_in, B, theta):
+    f = fo.layer_forward_full(fo.LayerState(W, b), x_in)
+    return fo.ff_loss(f["g"], theta, B)
+
+
+def _fd_check(K, N, B, seed, theta):
+    rng = np.random.default_rng(seed)
+    for _ in range(100):
+        x = np.abs(rng.standard_normal((2 * B, K)))
+        W = rng.standard_normal((N, K)) * (1.5 / math.sqrt(K))
+        b = rng.standard_normal(N) * 0.3
+        z = fo.normalise(x) @ W.T + b
+        if np.min(np.abs(z)) > 1e-3:
+            break
+    else:
+        pytest.fail("no kink-free draw")
+    st = fo.LayerState(W, b)
+    out = fo.layer_train_step(st, x, B, theta, fo.AdamHyper(lr=0.0))
+    h = 1e-6
+    num_W = np.zeros_like(W)
+    for i in range(N):
+        for j in range(K):
+            Wp = W.copy(); Wp[i, j] += h
+            Wm = W.copy(); Wm[i, j] -= h
+            num_W[i, j] = (_layer_loss(Wp, b, x, B, theta) - _layer_loss(Wm, b, x, B, theta)) / (2 * h)
+    num_b = np.zeros_like(b)
+    for i in range(N):
+        bp = b.copy(); bp[i] += h
+        bm = b.copy(); bm[i] -= h
+        num_b[i] = (_layer_loss(W, bp, x, B, theta) - _layer_loss(W, bm, x, B, theta)) / (2 * h)
+    scale_W = np.max(np.abs(num_W))
+    scale_b = np.max(np.abs(num_b))
+    assert np.max(np.abs(out["dW"] - num_W)) <= 1e-6 * scale_W
+    assert np.max(np.abs(out["db"] - num_b)) <= 1e-6 * scale_b
+
+
+def test_gradient_matches_finite_differences_4_to_3():
+    _fd_check(K=4, N=3, B=3, seed=10, theta=0.4)
+
+
+def test_gradient_matches_finite_differences_784_to_16():
+    _fd_check(K=784, N=16, B=2, seed=11, theta=0.05)
+
+
+# ------------------------------------------------------------------- Adam
+def test_adam_first_step_closed_form_and_zero_gradient():
+    hp = fo.AdamHyper(lr=0.03)
+    rng = np.random.default_rng(6)
+    w = rng.standard_normal(1000)
+    g = rng.standard_normal(1000) * 10.0 ** rng.integers(-9, 2, 1000)
+    g[:10] = 0.0
+    w1, m1, v1 = fo.adam_update(w, g, np.zeros(1000), np.zeros(1000), 1, hp)
+    # w1 - w cancels: allow a few ulps of |w| absolute
+    assert np.allclose(w1 - w, -hp.lr * g / (np.abs(g) + hp.eps), rtol=1e-12, atol=1e-15)
+    assert np.all(w1[:10] == w[:10])
+    # a constant gradient keeps the bias-corrected step at -lr*g/(|g|+eps)
+    w_t, m_t, v_t = w1, m1, v1
+    for t in range(2, 6):
+        w_n, m_t, v_t = fo.adam_update(w_t, g, m_t, v_t, t, hp)
+        assert np.allclose(w_n - w_t, -hp.lr * g / (np.abs(g) + hp.eps), rtol=1e-9, atol=1e-14)
+        w_t = w_n
+
+
+# ---------------------------------------------------------------- predict
+def _brute_predict(Ws, bs, x, n_classes=10):
+    """Pure-Python loops, no NumPy algebra: overlay, normalise, ReLU layers,
+    goodness of layers 2..L, first maximum wins."""
+    preds, Gs = [], []
+    L = len(Ws)
+    for row in x:
+        G = [0.0] * n_classes
+        for c in range(n_classes):
+            a = [0.0] * n_classes + [float(v) for v in row[n_classes:]]
+            a[c] = 1.0
+            for k in range(L):
+                nrm = math.sqrt(sum(v * v for v in a))
+                nrm = max(nrm, 1e-12)
+                xh = [v / nrm for v in a]
+                W, b = Ws[k], bs[k]
+                h = []
+                for i in range(len(b)):
+                    z = b[i]
+                    for j in range(len(xh)):
+                        z += W[i][j] * xh[j]
+                    h.append(z if z > 0 else 0.0)
+                if k >= 1 or L == 1:
+                    G[c] += sum(v * v for v in h)
+                a = h
+        best = 0
+        for c in range(1, n_classes):
+            if G[c] > G[best]:
+                best = c
+        preds.append(best)
+        Gs.append(G)
+    return np.array(preds), np.array(Gs)
+
+
+@pytest.mark.parametrize("dims", [(12, 5, 4, 3), (12, 6)])
+def test_predict_matches_brute_force(dims):
+    rng = np.random.default_rng(7)
+    Ws = [rng.standard_normal((dims[i + 1], dims[i])) for i in range(len(dims) - 1)]
+    bs = [rng.standard_normal(dims[i + 1]) * 0.2 for i in range(len(dims) - 1)]
+    x = rng.random((50, dims[0]))
+    states = [fo.LayerState(W, b) for W, b in zip(Ws, bs)]
+    pred, G = fo.predict(states, x)
+    bp, bG = _brute_predict([W.tolist() for W in Ws], [b.tolist() for b in bs], x)
+    assert np.allclose(G, bG, rtol=1e-12, atol=1e-12)
+    assert np.array_equal(pred, bp)
+
+
+def test_predict_hand_built_label_column_dominates():
+    # layer 1 copies the label area; layer 2 squares unit c strongly
+    K = 14
+    W1 = np.zeros((10, K)); W1[np.arange(10), np.arange(10)] = 1.0
+    W2 = np.eye(10) * 1.0
+    for c in (0, 3, 9):
+        W2c = W2.copy(); W2c[c, c] = 5.0
+        x = np.random.default_rng(c).random((4, K))
+        pred, G = fo.predict([fo.LayerState(W1, np.zeros(10)), fo.LayerState(W2c, np.zeros(10))], x)
+        assert np.all(pred == c)
+
+
+def test_predict_ties_go_to_lowest_label():
+    K = 12
+    W = np.zeros((3, K)); W[:, 10:] = 1.0          # ignores the label area
+    st = [fo.LayerState(W, np.zeros(3)), fo.LayerState(np.eye(3), np.zeros(3))]
+    pred, G = fo.predict(st, np.random.default_rng(0).random((5, K)))
+    assert np.all(pred == 0) and np.allclose(G, G[:, :1])
+
+
+def test_layer1_overlay_identity_used_by_predict():
+    """X^c W^T = X0 W^T + W[:, c] and ||x^c||^2 = ||x0||^2 + 1, where x0 is x
+    with the label area zeroed: the identity the GPU predict relies on."""
+    x = synth.mnist_like(30, seed=8).astype(np.float64)
+    W = synth.he_uniform(8, 20, 784).astype(np.float64)
+    x0 = x.copy(); x0[:, :10] = 0.0
+    for c in range(10):
+        xc = fo.overlay_label(x, np.full(30, c))
+        assert np.allclose(xc @ W.T, x0 @ W.T + W[:, c], rtol=0, atol=1e-12)
+        assert np.allclose(np.sum(xc ** 2, 1), np.sum(x0 ** 2, 1) + 1.0, rtol=1e-15)
+
+
+# ------------------------------------------------------- init statistic
+def test_he_uniform_goodness_expectation():
+    """Unit-norm input, He-uniform W, b = 0: E[g] = N/K (Var w = 2/K, E relu(z)^2 = Var z / 2)."""
+    gold = _golden("closed_forms.json")
+    for (K, N) in ((784, 2000), (2000, 2000), (784, 500)):
+        W = synth.he_uniform(21, N, K)
+        lo, hi = W.min(), W.max()
+        bound = math.sqrt(6.0 / K)
+        assert -bound <= lo < -0.99 * bound and 0.99 * bound < hi <= bound
+        x = synth.mnist_like(4000 if K == 784 else 1000, seed=22, features=784)
+        if K != 784:
+            x = np.abs(np.random.default_rng(23).standard_normal((1000, K)))
+        f = fo.layer_forward_full(fo.LayerState(W, np.zeros(N)), x)
+        key = f"E_g_he_uniform_{K}_{N}"
+        expect = gold[key]
+        assert expect == pytest.approx(N / K, rel=1e-3)
+        # g is a sum over N units for one row; rows share W, so allow 3%
+        assert np.mean(f["g"]) == pytest.approx(expect, rel=0.03)
+
+
+# -------------------------------------------------------- bf16 emulation
+def test_emulation_with_identity_rounding_is_the_plain_definition():
+    rng = np.random.default_rng(9)
+    B, K, N = 6, 40, 17
+    x = rng.random((2 * B, K))
+    W = rng.standard_normal((N, K)) * 0.3
+    b = rng.standard_normal(N) * 0.1
+    a = fo.layer_train_step(fo.LayerState(W, b), x, B, 1.0, fo.AdamHyper())
+    e = fo.layer_train_step(fo.LayerState(W, b), x, B, 1.0, fo.AdamHyper(), rounding=lambda v: np.asarray(v, np.float64))
+    for k in ("g", "dW", "db"):
+        assert np.allclose(a[k], e[k], rtol=1e-12, atol=1e-15)
+
+
+def test_emulation_rounds_operands_to_bf16():
+    rng = np.random.default_rng(12)
+    B, K, N = 4, 32, 9
+    x = rng.random((2 * B, K))
+    W = rng.standard_normal((N, K)) * 0.3
+    st = fo.LayerState(W, np.zeros(N))
+    f = fo.layer_forward_full(st, x, emulate_bf16=True)
+    assert np.array_equal(f["A"], fo.bf16_round(x))
+    # the product uses the rounded W and the exact norm of the unrounded input
+    s = 1.0 / np.sqrt(np.sum(x ** 2, 1))
+    assert np.allclose(f["Z"], s[:, None] * (fo.bf16_round(x) @ fo.bf16_round(W).T), rtol=1e-14)
+
+
+# ------------------------------------------------ whole-step consistency
+def test_net_step_layer_inputs_are_previous_activities():
+    B = 8
+    x = synth.mnist_like(B, seed=1)
+    y = synth.labels(B, seed=1)
+    yn = synth.negative_labels(y, seed=1)
+    x2, l2 = synth.pair_batch(x, y, yn)
+    dims = [784, 30, 20]
+    states = [fo.LayerState(synth.he_uniform(100 + i, dims[i + 1], dims[i]), np.zeros(dims[i + 1])) for i in range(2)]
+    before = [s.copy() for s in states]
+    outs = fo.net_train_step(states, x2, l2, B, 2.0, fo.AdamHyper())
+    # layer 2's forward used layer 1's pre-update activity
+    f1 = fo.layer_forward_full(before[0], fo.overlay_label(x2, l2))
+    f2 = fo.layer_forward_full(before[1], f1["H"])
+    assert np.allclose(outs[0]["H"], f1["H"], rtol=1e-14, atol=1e-15)
+    assert np.allclose(outs[1]["g"], f2["g"], rtol=1e-14, atol=1e-15)
+    assert all(s.t == 1 for s in states)
+
+
+def test_negative_labels_are_wrong_and_cover_all_offsets():
+    y = synth.labels(20000, seed=2)
+    yn = synth.negative_labels(y, seed=2)
+    assert np.all(yn != y)
+    off = (yn - y - 1) % 10
+    assert set(np.unique(off)) == set(range(9))
+    assert np.all(np.abs(np.bincount(y, minlength=10) / 20000 - 0.1) < 0.01)
