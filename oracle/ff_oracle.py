@@ -231,14 +231,16 @@ def layer_train_step(state: LayerState, x_in, B: int, theta: float, hp: AdamHype
     dZ = 2.0 * c[:, None] * Hg * (Z > 0)
     if emul:
         G = rnd(s[:, None] * dZ)               # weight-gradient operand, as stored
-        dW = G.T @ A
+        gL, gR = G, A
     else:
-        dW = dZ.T @ x_hat                      # dL/dW = dZ^T x_hat
+        gL, gR = dZ, x_hat                     # dL/dW = dZ^T x_hat
+    dW = gL.T @ gR
     db = np.sum(dZ, axis=0)
     state.t += 1
     state.W, state.mW, state.vW = adam_update(state.W, dW, state.mW, state.vW, state.t, hp)
     state.b, state.mb, state.vb = adam_update(state.b, db, state.mb, state.vb, state.t, hp)
-    return dict(H=H, g=g, s=s, loss=loss, dW=dW, db=db, c=c)
+    # gL, gR: the two operands of the weight-gradient product dW = gL^T gR
+    return dict(H=H, g=g, s=s, loss=loss, dW=dW, db=db, c=c, dZ=dZ, gL=gL, gR=gR)
 
 
 def net_train_step(states, x_raw, labels, B: int, theta: float, hp: AdamHyper,
