@@ -1,0 +1,441 @@
+#!/usr/bin/env python
+"""Benchmark of the Forward-Forward train step on one GB300.
+
+Default workload: the 784-2000-2000-2000-2000 ReLU net, bf16 operands with
+fp32 accumulation and fp32 master weights, one epoch of 60 000 synthetic
+MNIST-shaped pairs (58 batches of 1024 pairs + one of 608) per step, the four
+layers on four CUDA streams (libff's ff_net).  Metric: pairs/s.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+
+Prints one JSON line.  With torchrun (N > 1) every rank trains its own
+replica (the path does not shard); rank 0 prints the whole-job aggregate.
+``--impl reference`` times the CPU oracle (NumPy fp64) on the host cores on a
+bounded sample of the same workload.
+"""
+
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import signal
+import statistics
+import subprocess
+import sys
+import time
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "FF train samples/s (pos+neg pairs) on 4x2000 net, 1 GB300; % of bf16 TC peak"
+NET = [784, 2000, 2000, 2000, 2000]
+PAIRS_PER_EPOCH = 60000
+BATCH = 1024
+THETA, LR = 2.0, 0.03
+WORKLOAD = "ff_train_784-2000x4_bf16_epoch60000_B1024"
+
+
+def batches():
+    out, done = [], 0
+    while done < PAIRS_PER_EPOCH:
+        b = min(BATCH, PAIRS_PER_EPOCH - done)
+        out.append((done, b))
+        done += b
+    return out
+
+
+def train_flops_per_pair():
+    return 4.0 * 2 * sum(NET[i] * NET[i + 1] for i in range(len(NET) - 1))  # 2 GEMMs x 2MNK, M = 2 rows/pair
+
+
+def peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return dict(hbm=float(d["hbm_gbs"]), bf16=float(d["bf16_tflops"]),
+                    bf16_sus=float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), src="measured")
+    except Exception:
+        return dict(hbm=6800.0, bf16=1900.0, bf16_sus=1700.0, src="fallback")
+
+
+# ------------------------------------------------------------------ inputs
+def epoch_inputs(seed=0):
+    """The epoch's concatenated pair batches: x [2*60000, 784] float32 and
+    labels [2*60000] int32, batch t occupying rows 2*start .. 2*(start+B)."""
+    import numpy as np
+
+    from paper_2404_08573_gb300 import synth
+    xs, ls = [], []
+    for start, b in batches():
+        x = synth.mnist_like(b, seed=seed, start_row=start)
+        y = synth.labels(b, seed=seed, start=start)
+        yn = synth.negative_labels(y, seed=seed, start=start)
+        x2, l2 = synth.pair_batch(x, y, yn)
+        xs.append(x2)
+        ls.append(l2)
+    return np.concatenate(xs), np.concatenate(ls)
+
+
+# ------------------------------------------------------------------ clocks
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+              "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+              "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index):
+        self.index = index
+        self.p = None
+        self.path = os.path.join("/tmp", f"ff_clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            self.f = open(self.path, "w")
+            self.p = subprocess.Popen(["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                                       "--format=csv,noheader,nounits", "-lms", "200"], stdout=self.f,
+                                      stderr=subprocess.DEVNULL)
+        except Exception:
+            self.p = None
+
+    def stop(self):
+        if self.p is None:
+            return None
+        self.p.send_signal(signal.SIGTERM)
+        try:
+            self.p.wait(timeout=5)
+        except Exception:
+            self.p.kill()
+        self.f.close()
+        sm, mx, reasons = [], 0.0, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [q.strip() for q in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = max(mx, float(parts[1]))
+            except ValueError:
+                continue
+            for n, v in zip(names, parts[4:8]):
+                if v.lower() == "active":
+                    reasons.add(n)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ------------------------------------------------------------- CPU oracle
+def oracle_sample(seconds: float, min_steps: int = 1, steps: int | None = None, seed: int = 0):
+    """Times the oracle (fp64, as it stands) on config-1 batches of 1024 pairs.
+    Returns (pairs_per_s, steps_done, elapsed_s, per-step times)."""
+    from oracle import ff_oracle as fo
+    from paper_2404_08573_gb300 import synth
+    states = [fo.LayerState(synth.he_uniform(1000 + k, NET[k + 1], NET[k]), [0.0] * NET[k + 1])
+              for k in range(len(NET) - 1)]
+    hp = fo.AdamHyper(lr=LR)
+    done, t0, times = 0, time.perf_counter(), []
+    while True:
+        start = (done * BATCH) % (PAIRS_PER_EPOCH - BATCH)
+        x = synth.mnist_like(BATCH, seed=seed, start_row=start)
+        y = synth.labels(BATCH, seed=seed, start=start)
+        x2, l2 = synth.pair_batch(x, y, synth.negative_labels(y, seed=seed, start=start))
+        ts = time.perf_counter()
+        fo.net_train_step(states, x2, l2, BATCH, THETA, hp)
+        times.append(time.perf_counter() - ts)
+        done += 1
+        if steps is not None:
+            if done >= steps:
+                break
+        elif done >= min_steps and time.perf_counter() - t0 >= seconds:
+            break
+    el = sum(times)
+    return BATCH * done / el, done, el, times
+
+
+def cpu_baseline(seconds=12.0):
+    """Runs the oracle in a fresh process with every BLAS/OpenMP thread pinned
+    to the host's core count (so `cores` is what it used)."""
+    cores = os.cpu_count() or 1
+    env = dict(os.environ)
+    for v in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS", "MKL_NUM_THREADS"):
+        env[v] = str(cores)
+    env["CUDA_VISIBLE_DEVICES"] = ""
+    cmd = [sys.executable, os.path.abspath(__file__), "--cpu-worker", str(seconds)]
+    try:
+        r = subprocess.run(cmd, env=env, capture_output=True, text=True, timeout=600)
+        d = json.loads(r.stdout.strip().splitlines()[-1])
+    except Exception as e:  # reported, never fatal
+        return {"value": None, "unit": "pairs/s", "cores": cores, "kind": "oracle", "error": str(e)[:200]}
+    return {"value": d["pairs_per_s"], "unit": "pairs/s", "cores": cores, "kind": "oracle",
+            "sample": f"{d['steps']} train steps of 1024 pairs through 784-2000x4 (fp64 NumPy oracle, "
+                      f"{d['elapsed']:.1f} s)"}
+
+
+# ------------------------------------------------------------------- ours
+def run_ours(args):
+    import numpy as np
+    import torch
+
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    from paper_2404_08573_gb300 import build, ff
+    build.build()
+    lib = ff.lib()
+
+    X_h, L_h = epoch_inputs()
+    X = torch.from_numpy(X_h).to(dev)
+    Lb = torch.from_numpy(L_h).to(dev)
+    bl = batches()
+    layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", theta=THETA, lr=LR, init_seed=1000 + k, max_rows=2 * BATCH)
+              for k in range(len(NET) - 1)]
+    net = ff.Net(layers, max_B=BATCH, depth=2)
+    loss = torch.zeros(len(bl), len(layers), device=dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def epoch(xsrc=None, lsrc=None):
+        for t, (start, b) in enumerate(bl):
+            r0 = 2 * start
+            if xsrc is None:
+                net.train_step(X[r0:r0 + 2 * b], Lb[r0:r0 + 2 * b], B=b, loss=loss[t], stream=stream)
+            else:
+                xb, lb = xsrc(t, r0, b), lsrc(t, r0, b)
+                net.train_step(xb, lb, B=b, loss=loss[t], stream=stream)
+        net.sync(stream)
+
+    def barrier():
+        torch.cuda.synchronize(dev)
+        if dist is not None:
+            dist.barrier()
+
+    def max_over_ranks(v):
+        if dist is None:
+            return v
+        t = torch.tensor([v], device=dev, dtype=torch.float64)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        return float(t.item())
+
+    with torch.cuda.stream(stream):
+        for _ in range(args.warmup):
+            epoch()
+    barrier()
+
+    def timed(fn, k):
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        barrier()
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(k):
+                fn()
+            e1.record(stream)
+        barrier()
+        return max_over_ranks(e0.elapsed_time(e1))
+
+    # eager: every step a host call into libff
+    ms_eager = timed(epoch, args.steps)
+    # one epoch captured as a CUDA graph (all 4 layer streams as branches), replayed per step
+    graph, launches_per_epoch = None, None
+    if not args.no_graph:
+        l0 = lib.ff_kernel_launches()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            epoch()
+        launches_per_epoch = lib.ff_kernel_launches() - l0
+        for _ in range(args.warmup):
+            graph.replay()
+    clk = ClockSampler(local)
+    clk.start()
+    launches0 = lib.ff_kernel_launches()
+    if graph is not None:
+        ms = timed(graph.replay, args.steps)
+        launches = launches_per_epoch * args.steps
+    else:
+        ms = timed(epoch, args.steps)
+        launches = lib.ff_kernel_launches() - launches0
+    final_loss = loss[-1].cpu().numpy().tolist()
+    value = world * PAIRS_PER_EPOCH * args.steps / (ms / 1e3)
+
+    # end to end through the public API: pinned host batches copied in per batch
+    e2e = None
+    if not args.no_e2e:
+        Xp = torch.from_numpy(X_h).pin_memory()
+        Lp = torch.from_numpy(L_h).pin_memory()
+        xbuf = [torch.empty(2 * BATCH, NET[0], device=dev) for _ in range(2)]
+        lbuf = [torch.empty(2 * BATCH, dtype=torch.int32, device=dev) for _ in range(2)]
+        loss_h = torch.empty(len(layers), pin_memory=True)
+
+        def xsrc(t, r0, b):
+            xbuf[t % 2][:2 * b].copy_(Xp[r0:r0 + 2 * b], non_blocking=True)
+            return xbuf[t % 2][:2 * b]
+
+        def lsrc(t, r0, b):
+            lbuf[t % 2][:2 * b].copy_(Lp[r0:r0 + 2 * b], non_blocking=True)
+            return lbuf[t % 2][:2 * b]
+
+        with torch.cuda.stream(stream):
+            epoch(xsrc, lsrc)
+            loss_h.copy_(loss[-1], non_blocking=True)
+        barrier()
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(args.steps):
+                epoch(xsrc, lsrc)
+                loss_h.copy_(loss[-1], non_blocking=True)
+            e1.record(stream)
+        barrier()
+        ems = max_over_ranks(e0.elapsed_time(e1))
+        e2e = {"value": world * PAIRS_PER_EPOCH * args.steps / (ems / 1e3), "unit": "pairs/s",
+               "h2d_bytes_per_step": int(X_h.nbytes + L_h.nbytes), "d2h_bytes_per_step": int(loss_h.numel() * 4),
+               "ms_per_step": ems / args.steps}
+
+    # Per-kernel device time: the same epochs with the layers run one after
+    # another on one stream (each kernel alone on the GPU), every launch
+    # bracketed by CUDA events on that stream by libff's profiler.
+    kernels, roof = [], None
+    if not args.no_profile:
+        import ctypes
+        hs = [layers[k].new_activation(2 * BATCH) for k in range(len(layers) - 1)]
+        ss = [torch.empty(2 * BATCH, device=dev) for _ in range(len(layers) - 1)]
+
+        def epoch_seq():
+            for t, (start, b) in enumerate(bl):
+                r0 = 2 * start
+                for k, layer in enumerate(layers):
+                    last = k == len(layers) - 1
+                    layer.train_step(X[r0:r0 + 2 * b] if k == 0 else hs[k - 1][:2 * b],
+                                     labels=Lb[r0:r0 + 2 * b] if k == 0 else None,
+                                     row_scale=None if k == 0 else ss[k - 1][:2 * b], B=b,
+                                     h_out=None if last else hs[k][:2 * b], next_scale=None if last else ss[k][:2 * b],
+                                     loss=loss[t, k:k + 1], stream=stream)
+        with torch.cuda.stream(stream):
+            epoch_seq()
+        barrier()
+        lib.ff_profile_enable(1)
+        with torch.cuda.stream(stream):
+            for _ in range(args.steps):
+                epoch_seq()
+        barrier()
+        lib.ff_profile_enable(0)
+        cap = 32
+        names = (ctypes.c_char_p * cap)()
+        cnt = (ctypes.c_longlong * cap)()
+        tms = (ctypes.c_double * cap)()
+        wk = (ctypes.c_double * cap)()
+        lib.ff_profile_read.restype = ctypes.c_int
+        n = lib.ff_profile_read(cap, names, cnt, tms, wk)
+        total = sum(tms[i] for i in range(max(n, 0)))
+        pk = peaks()
+        for i in range(max(n, 0)):
+            nm = names[i].decode()
+            is_gemm = "gemm" in nm
+            rate = wk[i] / (tms[i] / 1e3) if tms[i] > 0 else 0.0
+            kernels.append({"kernel": nm, "launches": int(cnt[i]), "ms": round(tms[i], 3),
+                            "share": round(tms[i] / total, 4) if total else None,
+                            "achieved": round(rate / (1e12 if is_gemm else 1e9), 2),
+                            "unit": "TFLOP/s" if is_gemm else "GB/s"})
+        if kernels:
+            top = max(kernels, key=lambda k: k["ms"])
+            is_gemm = top["unit"] == "TFLOP/s"
+            peak = pk["bf16"] if is_gemm else pk["hbm"]
+            traffic = None
+            tpath = os.path.join(ROOT, "profiles", "traffic.json")
+            if os.path.exists(tpath):
+                try:
+                    traffic = json.load(open(tpath)).get(WORKLOAD, {}).get(top["kernel"])
+                except Exception:
+                    traffic = None
+            roof = {"kernel": top["kernel"], "bound": "tensor" if is_gemm else "hbm", "achieved": top["achieved"],
+                    "peak": peak, "unit": top["unit"], "frac": round(top["achieved"] / peak, 4),
+                    "peak_source": pk["src"] + (" bf16 burst (kernel timed alone)" if is_gemm else " HBM copy"),
+                    "traffic": traffic, "share": top["share"]}
+    clocks = clk.stop()
+
+    if rank == 0:
+        pk = peaks()
+        tflops = value * train_flops_per_pair() / 1e12
+        out = {
+            "metric": METRIC, "value": round(value, 1), "unit": "pairs/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+            "config": {"workload": WORKLOAD, "net": NET, "pairs_per_step": PAIRS_PER_EPOCH, "batch_pairs": BATCH,
+                       "theta": THETA, "lr": LR, "optimizer": "Adam",
+                       "parallelism": f"{world} replica(s); per GPU 4 layers on 4 CUDA streams",
+                       "l2": "inputs larger than L2 (376 MB of pair batches per step)"},
+            "launch": "one CUDA graph per step (epoch)" if graph is not None else "eager",
+            "ms_per_step_eager": round(ms_eager / args.steps, 4),
+            "tflops": round(tflops, 2),
+            "frac_of_bf16_peak": round(tflops / pk["bf16"], 4),
+            "roofline": roof, "kernels": kernels, "e2e": e2e, "gpu_launches": int(launches),
+            "clocks": clocks, "final_loss": final_loss,
+        }
+        if not args.no_cpu_baseline:
+            out["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
+        print(json.dumps(out), flush=True)
+    del graph
+    net.close()
+    if dist is not None:
+        dist.barrier()
+        dist.destroy_process_group()
+
+
+# -------------------------------------------------------------- reference
+def run_reference(args):
+    rank = int(os.environ.get("RANK", "0"))
+    if rank != 0:
+        return
+    cores = os.cpu_count() or 1
+    if args.warmup:
+        oracle_sample(0, steps=args.warmup)
+    t0 = time.perf_counter()
+    v, done, el, _ = oracle_sample(0, steps=args.steps)
+    wall = time.perf_counter() - t0
+    out = {
+        "impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": "pairs/s",
+        "n_gpus": int(os.environ.get("WORLD_SIZE", "1")), "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": round(1e3 * el / done, 2), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+        "config": {"workload": WORKLOAD, "net": NET, "batch_pairs": BATCH, "theta": THETA, "lr": LR,
+                   "sample": "each step = one train step of 1024 pairs (a bounded sample of the epoch)"},
+        "cpu_baseline": {"value": round(v, 3), "unit": "pairs/s", "cores": cores, "kind": "oracle",
+                         "sample": f"{done} train steps of 1024 pairs, fp64 NumPy oracle, {wall:.1f} s"},
+        "e2e": {"value": round(v, 3), "unit": "pairs/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0},
+    }
+    print(json.dumps(out), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-graph", action="store_true")
+    ap.add_argument("--no-profile", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0)
+    ap.add_argument("--cpu-worker", type=float, default=None, help=argparse.SUPPRESS)
+    args = ap.parse_args()
+    if args.cpu_worker is not None:
+        v, done, el, _ = oracle_sample(args.cpu_worker)
+        print(json.dumps({"pairs_per_s": v, "steps": done, "elapsed": el}))
+        return
+    if args.warmup < 3 and args.impl == "ours":
+        print("warning: fewer than 3 warm-up steps", file=sys.stderr)
+    if args.impl == "reference":
+        run_reference(args)
+    else:
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

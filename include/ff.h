@@ -1,0 +1,221 @@
+/*
+ * libff -- Forward-Forward (FF) layer-local training and goodness prediction
+ * on one NVIDIA GB300 (sm_103a).
+ *
+ * The operations follow "Going Forward-Forward in Distributed Deep Learning"
+ * (arXiv 2404.08573):
+ *   - label overlay ..................... §3 "Negative Data"
+ *   - goodness g = sum_j y_j^2, p(real) = sigma(g - theta) ... §3, Eq. 1
+ *   - L_i(x), Train(L_i, n), x = [positive; negative] ........ §4
+ *   - trainLayer(idx, batch) inside the per-layer loop ........ §4.1, Algorithm 1
+ *   - Goodness prediction over all but the first layer ....... §3 "Prediction"
+ *   - Adam for the FF layers .................................. §5.1
+ * with these readings where the paper is silent: the loss of one pair is
+ * softplus(theta - g_pos) + softplus(g_neg - theta), averaged over the pairs;
+ * every layer input is normalised to x / max(||x||_2, 1e-12) after the
+ * overlay; the overlay replaces features 0..9 with a one-hot of value 1.0;
+ * Adam is bias-corrected with eps outside the square root.
+ *
+ * Conventions that hold for every call:
+ *   - Every pointer argument is a DEVICE pointer owned by the caller unless the
+ *     call says otherwise; the library never frees caller memory.  A layer
+ *     owns its parameters, its Adam moments and its workspace.
+ *   - Every call that takes a `stream` (a cudaStream_t, NULL = legacy default
+ *     stream) is asynchronous on it.  Argument errors are detected on the host
+ *     and returned before anything is enqueued; a failed launch returns
+ *     FF_ERR_CUDA.  Errors found by kernels (a bounded wait that timed out, a
+ *     non-finite goodness) are latched in the layer and reported by
+ *     ff_layer_check().
+ *   - A layer must not be used from two streams at the same time.
+ *   - Activation buffers (the layer input when no labels are given, h_out)
+ *     are row-major in the layer's precision (float for FF_FP32, bfloat16 for
+ *     FF_BF16) with a row stride of ff_row_stride(features) elements; the pad
+ *     columns are written as zero and never read.
+ *   - Raw inputs (the `x` of a call that also takes labels, and of
+ *     ff_predict) are dense row-major float32 [rows, in_features].
+ *   - Rows 0..B-1 of a train batch are the positive rows, rows B..2B-1 the
+ *     negative rows (§4: x is the concatenation of the positive and negative
+ *     data).
+ *   - No C++ exception crosses this interface.
+ */
+#ifndef FF_H
+#define FF_H
+
+#if defined(__GNUC__)
+#define FF_API __attribute__((visibility("default")))
+#else
+#define FF_API
+#endif
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef enum {
+  FF_OK = 0,
+  FF_ERR_INVALID_ARG = 1, /* bad pointer, size, shape or precision; nothing enqueued */
+  FF_ERR_CUDA = 2,        /* a CUDA runtime/driver call or a launch failed */
+  FF_ERR_OOM = 3,         /* device allocation failed */
+  FF_ERR_TIMEOUT = 4,     /* a kernel's bounded wait gave up (latched, see ff_layer_check) */
+  FF_ERR_NONFINITE = 5,   /* a goodness value was NaN or Inf (latched) */
+  FF_ERR_UNSUPPORTED = 6  /* valid request this build or device cannot serve */
+} ff_status;
+
+typedef enum { FF_FP32 = 0, FF_BF16 = 1 } ff_precision;
+
+typedef struct {
+  int in_features;   /* fan-in K  (>= 1; >= 10 when labels are overlaid on this layer) */
+  int out_features;  /* fan-out N (>= 1) */
+  int has_bias;      /* 1: y = ReLU(x_hat W^T + b); 0: no bias (b stays 0) */
+  float theta;       /* goodness threshold of Eq. 1 */
+  float lr, beta1, beta2, eps;  /* Adam (§5.1) */
+  ff_precision prec; /* FF_FP32: fp32 everywhere. FF_BF16: bf16 GEMM operands,
+                        fp32 accumulate, fp32 master weights and moments */
+  unsigned long long init_seed; /* W ~ U(+-sqrt(6/K)) from this seed; b = 0 */
+  int max_rows;      /* workspace capacity in rows (2B); grows on demand if exceeded */
+  int keep_grad;     /* 1: keep dW, db of the last train step for ff_layer_get_grad */
+} ff_layer_config;
+
+typedef struct ff_layer ff_layer; /* opaque */
+typedef struct ff_net ff_net;     /* opaque */
+
+/* Human-readable name of a status code (static string, never NULL). */
+FF_API const char* ff_status_string(ff_status s);
+
+/* Row stride, in elements, of an activation buffer with `features` columns:
+ * features rounded up to a multiple of 8 (16-byte rows for bf16 TMA tiles). */
+FF_API int ff_row_stride(int features);
+
+/* Creates one FF layer (§4: the L_i a node trains).  Allocates W [N,K] fp32,
+ * b [N], the Adam moments (zero), the bf16 copy of W (FF_BF16) and a
+ * workspace for cfg->max_rows rows; initialises W on `stream` from
+ * cfg->init_seed with the counter-based SplitMix64 generator (He-uniform).
+ * Requires an sm_100-family GPU for FF_BF16 (FF_ERR_UNSUPPORTED otherwise).
+ * On success *out owns everything; on error *out is NULL and nothing leaks. */
+FF_API ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** out);
+
+/* Waits for the layer's last stream, frees everything it owns.  NULL-safe. */
+FF_API ff_status ff_layer_destroy(ff_layer* layer);
+
+/* Label overlay of §3 "Negative Data": out[r, 0..9] = one-hot(labels[r])
+ * (value 1.0, replacing the features), out[r, j] = x[r, j] for j >= 10, cast
+ * to `prec`; x is dense float32 [rows, features], out an activation buffer
+ * [rows, ff_row_stride(features)].  If row_scale is not NULL it receives
+ * 1 / max(||out_r||_2, 1e-12) computed in fp32 before the cast.
+ * labels should lie in 0..9; a row whose label is outside that range gets
+ * an all-zero label area.  features >= 10. */
+FF_API ff_status ff_overlay_label(const float* x, const int* labels, int rows, int features,
+                           void* out, float* row_scale, ff_precision prec, void* stream);
+
+/* L_i(x) of §4: the layer's forward pass without an update.
+ *   x          labels != NULL: raw float32 [rows, in] to overlay (§3);
+ *              labels == NULL: activation buffer [rows, ff_row_stride(in)].
+ *   row_scale  [rows] 1/||x_r|| of the layer input, or NULL to compute it
+ *              (ignored when labels are given: computed by the overlay).
+ *   h_out      [rows, ff_row_stride(out)] activation buffer: ReLU(x_hat W^T + b).
+ *   next_scale [rows] or NULL: 1 / max(sqrt(g_r), 1e-12), the next layer's
+ *              row_scale (||h_r|| = sqrt(g_r)).
+ *   goodness   [rows] or NULL: g_r = sum_j h_rj^2 (Eq. 1), from the fp32
+ *              accumulator before any rounding of h. */
+FF_API ff_status ff_layer_forward(ff_layer* layer, const void* x, const int* labels,
+                           const float* row_scale, int rows, void* h_out,
+                           float* next_scale, float* goodness, void* stream);
+
+/* trainLayer(idx, batch) of Algorithm 1 / Train(L_i, 1 batch) of §4: one
+ * local FF update on the 2B rows of x (B positive then B negative rows).
+ * Forward as ff_layer_forward (with the weights before this update), then
+ * loss = (1/B) sum_pairs softplus(theta - g_pos) + softplus(g_neg - theta)
+ * (the negative log-likelihood of Eq. 1), dL/dz = dL/dg * 2h * [z > 0],
+ * dW = dZ^T x_hat, db = sum_rows dZ, and one Adam step on W and b.
+ * No gradient leaves the layer.  h_out/next_scale/goodness as in
+ * ff_layer_forward (the pre-update forward; the next layer's input);
+ * loss [1] or NULL.  B == 0 is a no-op returning FF_OK. */
+FF_API ff_status ff_layer_train_step(ff_layer* layer, const void* x, const int* labels,
+                              const float* row_scale, int B, void* h_out,
+                              float* next_scale, float* goodness, float* loss,
+                              void* stream);
+
+/* Goodness prediction of §3 "Prediction": for every label c in 0..9 the raw
+ * input x [n, in] (float32) is overlaid with c and run through all layers;
+ * the goodness of layers 2..n_layers (layer 1 when n_layers == 1) is summed
+ * into goodness[r, c] ([n, 10] float32, or NULL) and pred[r] (int32) is the
+ * label with the largest sum, the lowest label on ties.  All layers must share
+ * one precision and chain (out_features of layer k == in_features of k+1).
+ * Scratch space is owned by layers[0] (grown on demand). n == 0 is a no-op. */
+FF_API ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n,
+                     int* pred, float* goodness, void* stream);
+
+/* Copies the layer state to/from caller buffers, which may be host or device
+ * memory: W [N,K] and its Adam moments m_W, v_W [N,K]; b, m_b, v_b [N]; the
+ * Adam step counter.  Any pointer may be NULL to skip that tensor.  Both calls
+ * first wait for the layer's last stream and are synchronous.  set_state also
+ * refreshes the bf16 copy of W. */
+FF_API ff_status ff_layer_get_state(const ff_layer* layer, float* W, float* b, float* m_W,
+                             float* v_W, float* m_b, float* v_b, long long* step);
+FF_API ff_status ff_layer_set_state(ff_layer* layer, const float* W, const float* b,
+                             const float* m_W, const float* v_W, const float* m_b,
+                             const float* v_b, long long step);
+
+/* The gradient of the last ff_layer_train_step (dW [N,K], db [N], fp32, host
+ * or device pointers; NULL skips).  Needs cfg.keep_grad = 1, else
+ * FF_ERR_UNSUPPORTED.  Synchronous. */
+FF_API ff_status ff_layer_get_grad(const ff_layer* layer, float* dW, float* db);
+
+/* Waits for the layer's last stream and returns the first latched kernel
+ * error (FF_ERR_TIMEOUT, FF_ERR_NONFINITE) or FF_ERR_CUDA, then clears it. */
+FF_API ff_status ff_layer_check(ff_layer* layer);
+
+/* A net of layers trained concurrently, one CUDA stream per layer: the
+ * single-GPU analogue of Single-Layer PFF (§4.1, Algorithm 1), where node i
+ * trains L_i on the output of L_{i-1}.  Here the hand-off is per batch: layer
+ * k+1 trains on batch t from layer k's pre-update forward of batch t, while
+ * layer k may already train on batch t+1 (inter-stream events, ring buffers
+ * of `depth` batches of activations).  The result is bitwise identical to
+ * running the same layer steps one after another on one stream.
+ * The net borrows the layers (they must outlive it) and owns its streams,
+ * events and activation buffers for up to max_B pairs. */
+FF_API ff_status ff_net_create(ff_layer* const* layers, int n_layers, int max_B, int depth,
+                        ff_net** out);
+FF_API ff_status ff_net_destroy(ff_net* net);
+
+/* Enqueues one batch for every layer: x raw float32 [2B, in], labels [2B]
+ * (true labels then wrong labels).  `stream` is ordered before layer 1 reads
+ * x, and after it finished reading x: the caller may overwrite x once
+ * `stream` reaches this point.  loss [n_layers] (device) or NULL receives
+ * each layer's loss asynchronously; call ff_net_sync before reading it. */
+FF_API ff_status ff_net_train_step(ff_net* net, const float* x, const int* labels, int B,
+                            float* loss, void* stream);
+
+/* Makes `stream` wait for all work the net has enqueued so far.  The steps
+ * enqueued between two ff_net_sync calls on one stream depend on nothing
+ * outside them but that stream, so such a sequence can be captured into a
+ * CUDA graph (the layers' workspaces must already be large enough). */
+FF_API ff_status ff_net_sync(ff_net* net, void* stream);
+
+/* ---------------------------------------------------------------------------
+ * Instrumentation (not part of the method).
+ * Every kernel launch libff makes is counted; ff_kernel_launches returns the
+ * process-wide total so far.  ff_profile_enable(1) clears earlier records and
+ * starts bracketing each launch with two CUDA events recorded on the stream
+ * the kernel is launched on; ff_profile_enable(0) stops.  ff_profile_read
+ * waits for the recorded events and writes, for up to `capacity` kernel kinds
+ * that were launched, the kind's name (static string), launch count, summed
+ * device time in ms and summed algorithmic work (FLOPs for kinds whose name
+ * contains "gemm", bytes the algorithm must move for the others).  Returns the
+ * number of kinds written, or -1 if an event query failed.  Any output array
+ * may be NULL. */
+FF_API ff_status ff_profile_enable(int on);
+FF_API int ff_profile_read(int capacity, const char** names, long long* launches, double* ms,
+                           double* work);
+FF_API unsigned long long ff_kernel_launches(void);
+/* The recorded launches in order: kind id (ff_profile_kind_name gives its
+ * name), launching stream (as an integer), start and end in ms relative to the
+ * earliest recorded start.  Returns how many were written, or -1. */
+FF_API int ff_profile_timeline(int capacity, int* kind, long long* stream_id, double* start_ms,
+                               double* end_ms);
+FF_API const char* ff_profile_kind_name(int kind);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* FF_H */

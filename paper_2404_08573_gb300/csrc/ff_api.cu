@@ -1,0 +1,598 @@
+// The libff C ABI: FF layer lifecycle, the layer-local train step, the
+// forward pass L_i(x), goodness prediction, and state access.  Host code only
+// orchestrates; every step of the path runs in the kernels of ff_elem.cu,
+// ff_gemm_tc.cu (bf16 mode) and ff_gemm_simt.cu (fp32 mode).
+#include <cmath>
+#include <cstdio>
+#include <cstdlib>
+#include <cstring>
+#include <new>
+
+#include "ff_api_internal.h"
+#include "ff_internal.cuh"
+#include "ff_prof.h"
+
+namespace ff {
+
+static bool debug_enabled() {
+  static const bool on = std::getenv("FF_DEBUG") != nullptr;
+  return on;
+}
+
+ff_status cuda_status(cudaError_t e, const char* what) {
+  if (e == cudaSuccess) return FF_OK;
+  if (debug_enabled()) std::fprintf(stderr, "libff: %s: %s\n", what, cudaGetErrorString(e));
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return FF_ERR_OOM;
+  }
+  return FF_ERR_CUDA;
+}
+
+#define FF_TRY(call, what)                                 \
+  do {                                                     \
+    ff_status s_ = ::ff::cuda_status((call), (what));      \
+    if (s_ != FF_OK) return s_;                            \
+  } while (0)
+
+// A kernel launch: counted, and timed on its stream while profiling is on.
+#define FF_LAUNCH(kind, work, st, call, what)                          \
+  do {                                                                 \
+    ff_status s_;                                                      \
+    {                                                                  \
+      ::ff::ProfScope p_((kind), (double)(work), (st));                \
+      s_ = ::ff::cuda_status((call), (what));                          \
+    }                                                                  \
+    if (s_ != FF_OK) return s_;                                        \
+  } while (0)
+
+// Host-side fault injection: FF_FAULT_ALLOC_FAIL_AT=n makes the n-th device
+// allocation (1-based, counted over the process) fail as out-of-memory.
+cudaError_t dev_alloc(void** p, size_t bytes) {
+  static long long fail_at = [] {
+    const char* e = std::getenv("FF_FAULT_ALLOC_FAIL_AT");
+    return e ? std::atoll(e) : 0ll;
+  }();
+  static long long count = 0;
+  ++count;
+  if (fail_at > 0 && count == fail_at) {
+    *p = nullptr;
+    return cudaErrorMemoryAllocation;
+  }
+  if (bytes == 0) bytes = 256;
+  return cudaMalloc(p, bytes);
+}
+
+void dev_free(void* p) {
+  if (p) cudaFree(p);
+}
+
+static size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
+
+static int gpart_tiles_max(int N) { return cdiv(N, 128); }
+
+// Grows the per-row workspace to at least `rows` rows (one allocation).
+static ff_status ensure_capacity(ff_layer* L, int rows) {
+  if (rows <= L->cap) return FF_OK;
+  const int cap = ((rows + 127) / 128) * 128;
+  const size_t es = L->is_bf16 ? 2 : 4;
+  size_t off = 0;
+  const size_t oX = off; off += align256((size_t)cap * L->ldK * es);
+  const size_t oS = off; off += align256((size_t)cap * 4);
+  const size_t oH = off; off += align256((size_t)cap * L->ldN * es);
+  const size_t oZ = off; off += align256((size_t)cap * L->ldN * es);
+  const size_t oP = off; off += align256((size_t)gpart_tiles_max(L->N) * cap * 4);
+  const size_t oG = off; off += align256((size_t)cap * 4);
+  const size_t oC = off; off += align256((size_t)cap * 4);
+  const size_t oN = off; off += align256((size_t)cap * 4);
+  const size_t oD = off; off += align256((size_t)local_grad_row_blocks(cap) * L->N * 4);
+  const size_t oL = off; off += align256((size_t)(finalize_grid(cap) > local_grad_row_blocks(cap) ? finalize_grid(cap) : local_grad_row_blocks(cap)) * 4);
+  if (L->cap > 0) {
+    FF_TRY(cudaStreamSynchronize(L->last_stream), "sync before workspace growth");
+    dev_free(L->X);
+    L->X = nullptr;
+    L->cap = 0;
+  }
+  void* base = nullptr;
+  FF_TRY(dev_alloc(&base, off), "workspace allocation");
+  char* b = static_cast<char*>(base);
+  L->X = b + oX;
+  L->s_in = reinterpret_cast<float*>(b + oS);
+  L->H = b + oH;
+  L->dZ = b + oZ;
+  L->gpart = reinterpret_cast<float*>(b + oP);
+  L->g = reinterpret_cast<float*>(b + oG);
+  L->c = reinterpret_cast<float*>(b + oC);
+  L->s_next = reinterpret_cast<float*>(b + oN);
+  L->dbpart = reinterpret_cast<float*>(b + oD);
+  L->loss_part = reinterpret_cast<float*>(b + oL);
+  L->cap = cap;
+  return FF_OK;
+}
+
+static void free_layer(ff_layer* L) {
+  if (!L) return;
+  dev_free(L->W);
+  dev_free(L->mW);
+  dev_free(L->vW);
+  dev_free(L->dW);
+  dev_free(L->b);
+  dev_free(L->Wb);
+  dev_free(L->ds);
+  dev_free(L->X);
+  dev_free(L->pws);
+  delete L;
+}
+
+static bool aligned16(const void* p) { return (reinterpret_cast<uintptr_t>(p) & 15u) == 0; }
+
+// Forward pass of one layer on M rows: operand preparation, the GEMM with the
+// fused scale/bias/ReLU/goodness epilogue.  Leaves per-tile goodness partials
+// in L->gpart and reports the row scale, activity buffer, operand buffer and
+// number of partial tiles it used.
+struct FwdResult {
+  const float* s;
+  void* H;
+  const void* X;
+  int ntiles;
+};
+
+static ff_status forward_core(ff_layer* L, const void* x, const int* labels, const float* row_scale, int M,
+                              void* h_out, cudaStream_t st, cudaEvent_t ev_input_read, FwdResult* r) {
+  const int K = L->K, N = L->N;
+  const double es = L->is_bf16 ? 2.0 : 4.0;
+  const float* s;
+  const void* X;
+  if (labels) {
+    FF_LAUNCH(K_OVERLAY, (double)M * (K * 4.0 + L->ldK * es + 8), st,
+              launch_overlay(static_cast<const float*>(x), labels, M, K, L->X, L->ldK, L->is_bf16, L->s_in, 0, st),
+              "overlay");
+    if (ev_input_read) FF_TRY(cudaEventRecord(ev_input_read, st), "event record");
+    X = L->X;
+    s = L->s_in;
+  } else {
+    X = x;
+    if (row_scale) {
+      s = row_scale;
+    } else {
+      FF_LAUNCH(K_ROW_SCALE, (double)M * (K * es + 4), st, launch_row_scale(x, L->ldK, L->is_bf16, M, K, L->s_in, st),
+                "row scale");
+      s = L->s_in;
+    }
+  }
+  void* H = h_out ? h_out : L->H;
+  EpiArgs ep{s, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
+  int ntiles;
+  if (L->is_bf16) {
+    ntiles = tc_fwd_ntiles(N);
+    FF_LAUNCH(K_FWD_TC, 2.0 * M * N * K, st,
+              tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, M, N, K, ep, &L->ds->err, st),
+              "forward GEMM (tcgen05)");
+  } else {
+    ntiles = simt_fwd_ntiles(N);
+    FF_LAUNCH(K_FWD_SIMT, 2.0 * M * N * K, st,
+              simt_gemm_fwd(static_cast<const float*>(X), L->ldK, L->W, K, M, N, K, ep, st), "forward GEMM (fp32)");
+  }
+  r->s = s;
+  r->H = H;
+  r->X = X;
+  r->ntiles = ntiles;
+  return FF_OK;
+}
+
+static ff_status check_call(ff_layer* L, const void* x, const int* labels, int rows) {
+  if (!L || !x || rows < 0) return FF_ERR_INVALID_ARG;
+  if (labels && L->K < 10) return FF_ERR_INVALID_ARG;
+  if (!labels && !aligned16(x)) return FF_ERR_INVALID_ARG;
+  if (labels && (reinterpret_cast<uintptr_t>(x) & 3u)) return FF_ERR_INVALID_ARG;
+  return FF_OK;
+}
+
+ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B, void* h_out,
+                          float* next_scale, float* goodness, float* loss, cudaStream_t st,
+                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done) {
+  ff_status cs = check_call(L, x, labels, B);
+  if (cs != FF_OK) return cs;
+  if (h_out && !aligned16(h_out)) return FF_ERR_INVALID_ARG;
+  if (B == 0) return FF_OK;
+  const int M = 2 * B;
+  if (M < B) return FF_ERR_INVALID_ARG;
+  ff_status cap_st = ensure_capacity(L, M);
+  if (cap_st != FF_OK) return cap_st;
+  L->last_stream = st;
+  const double es = L->is_bf16 ? 2.0 : 4.0;
+  FwdResult fr;
+  ff_status fs = forward_core(L, x, labels, row_scale, M, h_out, st, ev_input_read, &fr);
+  if (fs != FF_OK) return fs;
+
+  GradPrepArgs ga{};
+  ga.gpart = L->gpart;
+  ga.ntiles = fr.ntiles;
+  ga.M = M;
+  ga.N = L->N;
+  ga.ld = L->ldN;
+  ga.B = B;
+  ga.theta = L->cfg.theta;
+  ga.s = fr.s;
+  ga.g_out = goodness;
+  ga.s_next = next_scale;
+  ga.dbpart = L->dbpart;
+  ga.loss_part = L->loss_part;
+  ga.loss_out = loss ? loss : &L->ds->loss;
+  ga.ds = L->ds;
+  ga.beta1 = L->cfg.beta1;
+  ga.beta2 = L->cfg.beta2;
+  ga.err = &L->ds->err;
+  FF_LAUNCH(K_GRAD_PREP,
+            (double)M * (fr.ntiles * 4.0 + 12) + (double)M * L->ldN * es * 2 + (double)local_grad_row_blocks(M) * L->N * 4,
+            st, launch_grad_prep(ga, L->is_bf16, fr.H, L->dZ, st), "goodness/loss/local gradient");
+  if (ev_forward_done) FF_TRY(cudaEventRecord(ev_forward_done, st), "event record");
+
+  if (L->is_bf16) {
+    FF_LAUNCH(K_WGRAD_TC, 2.0 * M * L->N * L->K, st,
+              tc_gemm_wgrad(static_cast<const bf16*>(L->dZ), L->ldN, static_cast<const bf16*>(fr.X), L->ldK, M,
+                            L->N, L->K, L->dW, L->K, &L->ds->err, st),
+              "weight-gradient GEMM (tcgen05)");
+  } else {
+    FF_LAUNCH(K_WGRAD_SIMT, 2.0 * M * L->N * L->K, st,
+              simt_gemm_wgrad(static_cast<const float*>(L->dZ), L->ldN, static_cast<const float*>(fr.X), L->ldK, M,
+                              L->N, L->K, L->dW, L->K, st),
+              "weight-gradient GEMM (fp32)");
+  }
+  AdamArgs aa{};
+  aa.W = L->W;
+  aa.mW = L->mW;
+  aa.vW = L->vW;
+  aa.dW = L->dW;
+  aa.N = L->N;
+  aa.K = L->K;
+  aa.Wb = L->is_bf16 ? L->Wb : nullptr;
+  aa.ldb = L->ldK;
+  aa.b = L->b;
+  aa.mb = L->mb;
+  aa.vb = L->vb;
+  aa.dbpart = L->dbpart;
+  aa.nrb = local_grad_row_blocks(M);
+  aa.db_out = L->db;
+  aa.has_bias = L->cfg.has_bias;
+  aa.lr = L->cfg.lr;
+  aa.beta1 = L->cfg.beta1;
+  aa.beta2 = L->cfg.beta2;
+  aa.eps = L->cfg.eps;
+  aa.ds = L->ds;
+  FF_LAUNCH(K_ADAM, (double)L->N * L->K * (28.0 + (L->is_bf16 ? 2.0 : 0.0)) + (double)L->N * (aa.nrb * 4.0 + 28), st,
+            launch_adam(aa, st),
+            "Adam");
+  return FF_OK;
+}
+
+}  // namespace ff
+
+using namespace ff;
+
+extern "C" {
+
+const char* ff_status_string(ff_status s) {
+  switch (s) {
+    case FF_OK: return "FF_OK";
+    case FF_ERR_INVALID_ARG: return "FF_ERR_INVALID_ARG";
+    case FF_ERR_CUDA: return "FF_ERR_CUDA";
+    case FF_ERR_OOM: return "FF_ERR_OOM";
+    case FF_ERR_TIMEOUT: return "FF_ERR_TIMEOUT";
+    case FF_ERR_NONFINITE: return "FF_ERR_NONFINITE";
+    case FF_ERR_UNSUPPORTED: return "FF_ERR_UNSUPPORTED";
+  }
+  return "FF_ERR_UNKNOWN";
+}
+
+int ff_row_stride(int features) { return features <= 0 ? 0 : ff::row_stride(features); }
+
+ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** out) {
+  if (!out) return FF_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || cfg->in_features < 1 || cfg->out_features < 1 || cfg->max_rows < 0) return FF_ERR_INVALID_ARG;
+  if (cfg->prec != FF_FP32 && cfg->prec != FF_BF16) return FF_ERR_INVALID_ARG;
+  if (!std::isfinite(cfg->theta) || !std::isfinite(cfg->lr) || !(cfg->beta1 >= 0.f && cfg->beta1 < 1.f) ||
+      !(cfg->beta2 >= 0.f && cfg->beta2 < 1.f) || !(cfg->eps >= 0.f))
+    return FF_ERR_INVALID_ARG;
+  if ((long long)cfg->in_features * cfg->out_features > (1ll << 40)) return FF_ERR_INVALID_ARG;
+  int dev = 0;
+  FF_TRY(cudaGetDevice(&dev), "cudaGetDevice");
+  if (cfg->prec == FF_BF16 && !tc_supported()) return FF_ERR_UNSUPPORTED;
+  ff_layer* L = new (std::nothrow) ff_layer();
+  if (!L) return FF_ERR_OOM;
+  std::memset(L, 0, sizeof(*L));
+  L->cfg = *cfg;
+  L->K = cfg->in_features;
+  L->N = cfg->out_features;
+  L->ldK = row_stride(L->K);
+  L->ldN = row_stride(L->N);
+  L->device = dev;
+  L->is_bf16 = cfg->prec == FF_BF16;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  L->last_stream = st;
+  const size_t nk = (size_t)L->N * L->K;
+  ff_status s = FF_OK;
+#define FF_ALLOC(ptr, bytes)                                                      \
+  do {                                                                            \
+    s = cuda_status(dev_alloc(reinterpret_cast<void**>(&(ptr)), (bytes)), #ptr); \
+    if (s != FF_OK) {                                                             \
+      free_layer(L);                                                              \
+      return s;                                                                   \
+    }                                                                             \
+  } while (0)
+  FF_ALLOC(L->W, nk * 4);
+  FF_ALLOC(L->mW, nk * 4);
+  FF_ALLOC(L->vW, nk * 4);
+  FF_ALLOC(L->dW, nk * 4);
+  FF_ALLOC(L->b, (size_t)L->N * 4 * 4);  // b, mb, vb, db
+  if (L->is_bf16) FF_ALLOC(L->Wb, (size_t)L->N * L->ldK * 2);
+  FF_ALLOC(L->ds, sizeof(ff_dev_state));
+#undef FF_ALLOC
+  L->mb = L->b + L->N;
+  L->vb = L->b + 2 * L->N;
+  L->db = L->b + 3 * L->N;
+  cudaError_t e = cudaSuccess;
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->mW, 0, nk * 4, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->vW, 0, nk * 4, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->dW, 0, nk * 4, st);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L->b, 0, (size_t)L->N * 4 * 4, st);
+  if (e == cudaSuccess) {
+    static const ff_dev_state fresh = {0, 1.0, 1.0, 0.f, 0.f, 0, 0u, 0.f, 0};
+    e = cudaMemcpyAsync(L->ds, &fresh, sizeof(ff_dev_state), cudaMemcpyHostToDevice, st);
+    if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // `fresh` is pageable host memory
+  }
+  if (e == cudaSuccess) {
+    ProfScope p(K_INIT, (double)nk * 4, st);
+    e = launch_init_weights(L->W, L->N, L->K, cfg->init_seed, st);
+  }
+  if (e == cudaSuccess && L->is_bf16) {
+    ProfScope p(K_TO_BF16, (double)nk * 4 + (double)L->N * L->ldK * 2, st);
+    e = launch_to_bf16(L->W, L->N, L->K, L->Wb, L->ldK, st);
+  }
+  s = cuda_status(e, "layer initialisation");
+  if (s == FF_OK) s = ensure_capacity(L, cfg->max_rows > 0 ? cfg->max_rows : 256);
+  if (s != FF_OK) {
+    cudaStreamSynchronize(st);
+    free_layer(L);
+    return s;
+  }
+  *out = L;
+  return FF_OK;
+}
+
+ff_status ff_layer_destroy(ff_layer* L) {
+  if (!L) return FF_OK;
+  cudaError_t e = cudaStreamSynchronize(L->last_stream);
+  free_layer(L);
+  return cuda_status(e, "destroy sync");
+}
+
+ff_status ff_overlay_label(const float* x, const int* labels, int rows, int features, void* out, float* row_scale,
+                           ff_precision prec, void* stream) {
+  if (rows < 0 || features < 10 || (prec != FF_FP32 && prec != FF_BF16)) return FF_ERR_INVALID_ARG;
+  if (rows == 0) return FF_OK;
+  if (!x || !labels || !out) return FF_ERR_INVALID_ARG;
+  FF_LAUNCH(K_OVERLAY, (double)rows * (features * 4.0 + row_stride(features) * (prec == FF_BF16 ? 2.0 : 4.0) + 8),
+            static_cast<cudaStream_t>(stream),
+            launch_overlay(x, labels, rows, features, out, row_stride(features), prec == FF_BF16, row_scale, 0,
+                           static_cast<cudaStream_t>(stream)),
+            "overlay");
+  return FF_OK;
+}
+
+ff_status ff_layer_forward(ff_layer* L, const void* x, const int* labels, const float* row_scale, int rows,
+                           void* h_out, float* next_scale, float* goodness, void* stream) {
+  ff_status cs = check_call(L, x, labels, rows);
+  if (cs != FF_OK) return cs;
+  if (!h_out && !next_scale && !goodness) return FF_ERR_INVALID_ARG;
+  if (h_out && !aligned16(h_out)) return FF_ERR_INVALID_ARG;
+  if (rows == 0) return FF_OK;
+  ff_status es = ensure_capacity(L, rows);
+  if (es != FF_OK) return es;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  L->last_stream = st;
+  FwdResult fr;
+  ff_status fs = forward_core(L, x, labels, row_scale, rows, h_out, st, nullptr, &fr);
+  if (fs != FF_OK) return fs;
+  FinalizeArgs fa{};
+  fa.gpart = L->gpart;
+  fa.ntiles = fr.ntiles;
+  fa.M = rows;
+  fa.g_out = goodness;
+  fa.s_next = next_scale;
+  fa.err = &L->ds->err;
+  FF_LAUNCH(K_FINALIZE, (double)rows * (fr.ntiles * 4.0 + 8), st, launch_finalize(fa, st), "goodness");
+  return FF_OK;
+}
+
+ff_status ff_layer_train_step(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B,
+                              void* h_out, float* next_scale, float* goodness, float* loss, void* stream) {
+  return train_step_impl(L, x, labels, row_scale, B, h_out, next_scale, goodness, loss,
+                         static_cast<cudaStream_t>(stream), nullptr, nullptr);
+}
+
+ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n, int* pred, float* goodness,
+                     void* stream) {
+  if (!layers || n_layers < 1 || n < 0) return FF_ERR_INVALID_ARG;
+  for (int k = 0; k < n_layers; ++k) {
+    if (!layers[k]) return FF_ERR_INVALID_ARG;
+    if (layers[k]->is_bf16 != layers[0]->is_bf16) return FF_ERR_INVALID_ARG;
+    if (k > 0 && layers[k]->K != layers[k - 1]->N) return FF_ERR_INVALID_ARG;
+  }
+  if (n == 0) return FF_OK;
+  if (!x || !pred) return FF_ERR_INVALID_ARG;
+  ff_layer* L0 = layers[0];
+  if (L0->K < 10) return FF_ERR_INVALID_ARG;
+  const bool b16 = L0->is_bf16;
+  const size_t es = b16 ? 2 : 4;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  int ldmax = 0, ntmax = 0;
+  for (int k = 0; k < n_layers; ++k) {
+    if (layers[k]->ldN > ldmax) ldmax = layers[k]->ldN;
+    const int nt = b16 ? tc_fwd_ntiles(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
+    if (nt > ntmax) ntmax = nt;
+  }
+  // Samples per chunk: about 40 MB of activations per buffer, so that one
+  // chunk's two activation buffers stay resident in L2 between layers.
+  long long per = (40ll << 20) / ((long long)10 * ldmax * es);
+  int C = (int)(per < 64 ? 64 : per > 8192 ? 8192 : per);
+  if (C > n) C = n;
+  const int R = 10 * C;
+  const int N1 = L0->N;
+  size_t off = 0;
+  const size_t oX = off; off += align256((size_t)C * L0->ldK * es);
+  const size_t oS1 = off; off += align256((size_t)C * 4);
+  const size_t oBase = off; off += align256((size_t)C * L0->ldN * 4);
+  const size_t oCols = off; off += align256((size_t)10 * N1 * 4);
+  const size_t oH0 = off; off += align256((size_t)R * ldmax * es);
+  const size_t oH1 = off; off += align256((size_t)R * ldmax * es);
+  const size_t oSa = off; off += align256((size_t)R * 4);
+  const size_t oSb = off; off += align256((size_t)R * 4);
+  const size_t oP = off; off += align256((size_t)ntmax * R * 4);
+  const size_t oG = off; off += align256(goodness ? 0 : (size_t)n * 10 * 4);
+  if (off > L0->pws_bytes) {
+    FF_TRY(cudaStreamSynchronize(L0->last_stream), "sync before predict scratch growth");
+    dev_free(L0->pws);
+    L0->pws = nullptr;
+    L0->pws_bytes = 0;
+    FF_TRY(dev_alloc(&L0->pws, off), "predict scratch");
+    L0->pws_bytes = off;
+  }
+  L0->last_stream = st;
+  char* w = static_cast<char*>(L0->pws);
+  void* X0 = w + oX;
+  float* s1 = reinterpret_cast<float*>(w + oS1);
+  float* base = reinterpret_cast<float*>(w + oBase);
+  float* cols = reinterpret_cast<float*>(w + oCols);
+  void* Hb[2] = {w + oH0, w + oH1};
+  float* Sb[2] = {reinterpret_cast<float*>(w + oSa), reinterpret_cast<float*>(w + oSb)};
+  float* gpart = reinterpret_cast<float*>(w + oP);
+  float* G = goodness ? goodness : reinterpret_cast<float*>(w + oG);
+  int* err = &L0->ds->err;
+
+  FF_TRY(cudaMemsetAsync(G, 0, (size_t)n * 10 * 4, st), "zero goodness");
+  FF_LAUNCH(K_LABEL_COLS, (double)N1 * 10 * (es + 4), st,
+            launch_label_columns(b16 ? (const void*)L0->Wb : (const void*)L0->W, b16 ? L0->ldK : L0->K, b16, N1,
+                                 cols, st),
+            "label columns");
+  for (int c0 = 0; c0 < n; c0 += C) {
+    const int cn = (n - c0) < C ? (n - c0) : C;
+    const int rows = 10 * cn;
+    FF_LAUNCH(K_OVERLAY, (double)cn * (L0->K * 4.0 + L0->ldK * es + 4), st,
+              launch_overlay(x + (size_t)c0 * L0->K, nullptr, cn, L0->K, X0, L0->ldK, b16, s1, 1, st),
+              "zero label area");
+    if (b16) {
+      FF_LAUNCH(K_STORE_TC, 2.0 * cn * N1 * L0->K, st,
+                tc_gemm_store(static_cast<const bf16*>(X0), L0->ldK, L0->Wb, L0->ldK, cn, N1, L0->K, base, L0->ldN,
+                              err, st),
+                "layer-1 base GEMM (tcgen05)");
+    } else {
+      FF_LAUNCH(K_STORE_SIMT, 2.0 * cn * N1 * L0->K, st,
+                simt_gemm_store(static_cast<const float*>(X0), L0->ldK, L0->W, L0->K, cn, N1, L0->K, base, L0->ldN,
+                                st),
+                "layer-1 base GEMM (fp32)");
+    }
+    float* Gc = G + (size_t)c0 * 10;
+    FF_LAUNCH(K_EXPAND, (double)cn * (L0->ldN * 4.0 + 10.0 * L0->ldN * es + 40), st,
+              launch_expand(base, L0->ldN, cols, s1, L0->cfg.has_bias ? L0->b : nullptr, cn, N1, Hb[0], L0->ldN, b16,
+                            Sb[0], n_layers == 1 ? Gc : nullptr, err, st),
+              "layer-1 expansion");
+    int cur = 0;
+    for (int k = 1; k < n_layers; ++k) {
+      ff_layer* Lk = layers[k];
+      EpiArgs ep{Sb[cur], Lk->cfg.has_bias ? Lk->b : nullptr, Hb[cur ^ 1], Lk->ldN, gpart};
+      int nt;
+      if (b16) {
+        nt = tc_fwd_ntiles(Lk->N);
+        FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
+                  tc_gemm_fwd(static_cast<const bf16*>(Hb[cur]), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep,
+                              err, st),
+                  "predict forward GEMM (tcgen05)");
+      } else {
+        nt = simt_fwd_ntiles(Lk->N);
+        FF_LAUNCH(K_FWD_SIMT, 2.0 * rows * Lk->N * Lk->K, st,
+                  simt_gemm_fwd(static_cast<const float*>(Hb[cur]), Lk->ldK, Lk->W, Lk->K, rows, Lk->N, Lk->K, ep, st),
+                  "predict forward GEMM (fp32)");
+      }
+      FinalizeArgs fa{};
+      fa.gpart = gpart;
+      fa.ntiles = nt;
+      fa.M = rows;
+      fa.s_next = (k + 1 < n_layers) ? Sb[cur ^ 1] : nullptr;
+      fa.G_acc = Gc;
+      fa.err = err;
+      FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 12), st, launch_finalize(fa, st), "predict goodness");
+      cur ^= 1;
+    }
+  }
+  FF_LAUNCH(K_ARGMAX, (double)n * 44, st, launch_argmax(G, n, pred, nullptr, st), "argmax");
+  return FF_OK;
+}
+
+static cudaMemcpyKind kind_default() { return cudaMemcpyDefault; }
+
+ff_status ff_layer_get_state(const ff_layer* Lc, float* W, float* b, float* m_W, float* v_W, float* m_b, float* v_b,
+                             long long* step) {
+  if (!Lc) return FF_ERR_INVALID_ARG;
+  ff_layer* L = const_cast<ff_layer*>(Lc);
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  const size_t nk = (size_t)L->N * L->K * 4, n4 = (size_t)L->N * 4;
+  if (W) FF_TRY(cudaMemcpy(W, L->W, nk, kind_default()), "copy W");
+  if (m_W) FF_TRY(cudaMemcpy(m_W, L->mW, nk, kind_default()), "copy m_W");
+  if (v_W) FF_TRY(cudaMemcpy(v_W, L->vW, nk, kind_default()), "copy v_W");
+  if (b) FF_TRY(cudaMemcpy(b, L->b, n4, kind_default()), "copy b");
+  if (m_b) FF_TRY(cudaMemcpy(m_b, L->mb, n4, kind_default()), "copy m_b");
+  if (v_b) FF_TRY(cudaMemcpy(v_b, L->vb, n4, kind_default()), "copy v_b");
+  if (step) FF_TRY(cudaMemcpy(step, &L->ds->t, sizeof(long long), cudaMemcpyDeviceToHost), "copy step");
+  return FF_OK;
+}
+
+ff_status ff_layer_set_state(ff_layer* L, const float* W, const float* b, const float* m_W, const float* v_W,
+                             const float* m_b, const float* v_b, long long step) {
+  if (!L || step < 0) return FF_ERR_INVALID_ARG;
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  const size_t nk = (size_t)L->N * L->K * 4, n4 = (size_t)L->N * 4;
+  if (W) FF_TRY(cudaMemcpy(L->W, W, nk, kind_default()), "copy W");
+  if (m_W) FF_TRY(cudaMemcpy(L->mW, m_W, nk, kind_default()), "copy m_W");
+  if (v_W) FF_TRY(cudaMemcpy(L->vW, v_W, nk, kind_default()), "copy v_W");
+  if (b) FF_TRY(cudaMemcpy(L->b, b, n4, kind_default()), "copy b");
+  if (m_b) FF_TRY(cudaMemcpy(L->mb, m_b, n4, kind_default()), "copy m_b");
+  if (v_b) FF_TRY(cudaMemcpy(L->vb, v_b, n4, kind_default()), "copy v_b");
+  FF_TRY(cudaMemcpy(&L->ds->t, &step, sizeof(long long), cudaMemcpyHostToDevice), "copy step");
+  const double pw[2] = {std::pow((double)L->cfg.beta1, (double)step), std::pow((double)L->cfg.beta2, (double)step)};
+  FF_TRY(cudaMemcpy(&L->ds->pow1, pw, sizeof(pw), cudaMemcpyHostToDevice), "copy beta powers");
+  if (L->is_bf16) {
+    FF_LAUNCH(K_TO_BF16, (double)L->N * L->K * 4 + (double)L->N * L->ldK * 2, L->last_stream,
+              launch_to_bf16(L->W, L->N, L->K, L->Wb, L->ldK, L->last_stream), "refresh bf16 W");
+    FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  }
+  return FF_OK;
+}
+
+ff_status ff_layer_get_grad(const ff_layer* Lc, float* dW, float* db) {
+  if (!Lc) return FF_ERR_INVALID_ARG;
+  if (!Lc->cfg.keep_grad) return FF_ERR_UNSUPPORTED;
+  ff_layer* L = const_cast<ff_layer*>(Lc);
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  if (dW) FF_TRY(cudaMemcpy(dW, L->dW, (size_t)L->N * L->K * 4, kind_default()), "copy dW");
+  if (db) FF_TRY(cudaMemcpy(db, L->db, (size_t)L->N * 4, kind_default()), "copy db");
+  return FF_OK;
+}
+
+ff_status ff_layer_check(ff_layer* L) {
+  if (!L) return FF_ERR_INVALID_ARG;
+  cudaError_t e = cudaStreamSynchronize(L->last_stream);
+  if (e != cudaSuccess) return cuda_status(e, "check sync");
+  int err = 0;
+  FF_TRY(cudaMemcpy(&err, &L->ds->err, sizeof(int), cudaMemcpyDeviceToHost), "read error word");
+  if (err) {
+    const int zero = 0;
+    FF_TRY(cudaMemcpy(&L->ds->err, &zero, sizeof(int), cudaMemcpyHostToDevice), "clear error word");
+  }
+  if (err & DEVERR_TIMEOUT) return FF_ERR_TIMEOUT;
+  if (err & DEVERR_NONFINITE) return FF_ERR_NONFINITE;
+  return FF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,20 @@
+// Host-side helpers shared by ff_api.cu and ff_net.cu.
+#pragma once
+
+#include "ff_internal.cuh"
+
+namespace ff {
+
+ff_status cuda_status(cudaError_t e, const char* what);
+cudaError_t dev_alloc(void** p, size_t bytes);
+void dev_free(void* p);
+
+// One layer-local train step (see ff_layer_train_step).  ev_input_read, if
+// not null, is recorded once the raw input x has been consumed (after the
+// overlay; only meaningful when labels are given); ev_forward_done, if not
+// null, once the activity, goodness and next-layer scale are written.
+ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B,
+                          void* h_out, float* next_scale, float* goodness, float* loss, cudaStream_t st,
+                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done);
+
+}  // namespace ff

@@ -1,0 +1,515 @@
+// Bandwidth-bound kernels of the FF layer step and of goodness prediction:
+//   overlay      §3 "Negative Data": one-hot label in features 0..9, cast to
+//                the operand type, row norm for x / max(||x||, 1e-12)
+//   finalize     Eq. 1: goodness from the GEMM's per-tile partials and the
+//                next layer's row scale (forward and predict)
+//   grad_prep    the same goodness, the pair loss softplus(theta - g_pos) +
+//                softplus(g_neg - theta) and its derivative dL/dg, then
+//                dZ = dL/dg * 2h (h = 0 where z <= 0), the weight-gradient
+//                operand s*dZ and per-64-row partial sums for db
+//   adam         Adam (§5.1) on W and b, refreshing the bf16 copy of W
+//   init         He-uniform W from a counter-based SplitMix64 stream
+//   predict      label columns of W1, per-label expansion of layer 1,
+//                argmax over the 10 labels (§3 "Prediction")
+// Reductions use fixed orders (no floating-point atomics), so results do not
+// depend on scheduling.
+#include "ff_internal.cuh"
+
+namespace ff {
+namespace {
+
+constexpr float kNormEps = 1e-12f;
+
+// 1 / max(sqrt(ss), 1e-12), with NaN propagated (fmaxf alone would drop it).
+__device__ __forceinline__ float inv_norm(float ss) {
+  const float r = sqrtf(ss);
+  return r != r ? r : 1.f / fmaxf(r, kNormEps);
+}
+// ReLU that keeps NaN visible to the non-finite check.
+__device__ __forceinline__ float relu_nan(float z) { return z != z ? z : fmaxf(z, 0.f); }
+
+template <typename T>
+__device__ __forceinline__ T from_f(float v);
+template <>
+__device__ __forceinline__ float from_f<float>(float v) { return v; }
+template <>
+__device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_rn(v); }
+__device__ __forceinline__ float to_f(float v) { return v; }
+__device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Fixed-order block sum for blockDim.x == 256; result valid in thread 0.
+__device__ __forceinline__ float block_sum_256(float v, float* red /*[8]*/) {
+  v = warp_sum(v);
+  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
+  __syncthreads();
+  float t = 0.f;
+  if (threadIdx.x == 0) {
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[w];
+  }
+  __syncthreads();
+  return t;
+}
+
+// ------------------------------------------------------------------ overlay
+template <typename T>
+__global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ labels, int rows, int F,
+                          T* __restrict__ out, int ldo, float* __restrict__ s_out, int mode) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 8 + warp;
+  if (row >= rows) return;
+  const float* xr = x + (size_t)row * F;
+  T* orow = out + (size_t)row * ldo;
+  const int lab = (mode == 0 && labels) ? labels[row] : -1;
+  float ss = 0.f;
+  for (int f = lane; f < ldo; f += 32) {
+    float v = 0.f;
+    if (f < F) v = (f < 10) ? (f == lab ? 1.f : 0.f) : __ldg(xr + f);
+    orow[f] = from_f<T>(v);
+    ss = fmaf(v, v, ss);
+  }
+  ss = warp_sum(ss);
+  if (lane == 0 && s_out) s_out[row] = inv_norm(ss + (mode == 1 ? 1.f : 0.f));
+}
+
+template <typename T>
+__global__ void k_row_scale(const T* __restrict__ x, int ldx, int rows, int F, float* __restrict__ s_out) {
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * 8 + warp;
+  if (row >= rows) return;
+  const T* xr = x + (size_t)row * ldx;
+  float ss = 0.f;
+  for (int f = lane; f < F; f += 32) {
+    const float v = to_f(xr[f]);
+    ss = fmaf(v, v, ss);
+  }
+  ss = warp_sum(ss);
+  if (lane == 0) s_out[row] = inv_norm(ss);
+}
+
+// ----------------------------------------------------------------- finalize
+__device__ __forceinline__ float softplus_f(float t) { return fmaxf(t, 0.f) + log1pf(expf(-fabsf(t))); }
+__device__ __forceinline__ float sigmoid_f(float t) {
+  if (t >= 0.f) return 1.f / (1.f + expf(-t));
+  const float e = expf(t);
+  return e / (1.f + e);
+}
+
+__global__ void __launch_bounds__(256) k_finalize(FinalizeArgs a) {
+  const int i = blockIdx.x * 256 + threadIdx.x;
+  if (i >= a.M) return;
+  float g = 0.f;
+  for (int t = 0; t < a.ntiles; ++t) g += a.gpart[(size_t)t * a.M + i];
+  if (!isfinite(g)) atomicOr(a.err, DEVERR_NONFINITE);
+  if (a.g_out) a.g_out[i] = g;
+  if (a.s_next) a.s_next[i] = inv_norm(g);
+  if (a.G_acc) a.G_acc[i] += g;
+}
+
+// --------------------------------------------------------------- local grad
+// Block (32, 8): 256 columns (8 per thread) x 64 rows.
+template <typename T>
+struct Vec8;
+template <>
+struct Vec8<bf16> {
+  static __device__ __forceinline__ void load(const bf16* p, float (&v)[8]) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __bfloat1622float2(h[e]);
+      v[2 * e] = f.x;
+      v[2 * e + 1] = f.y;
+    }
+  }
+  static __device__ __forceinline__ void store(bf16* p, const float (&v)[8]) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+    *reinterpret_cast<uint4*>(p) = u;
+  }
+};
+template <>
+struct Vec8<float> {
+  static __device__ __forceinline__ void load(const float* p, float (&v)[8]) {
+    const float4 a = *reinterpret_cast<const float4*>(p);
+    const float4 b = *reinterpret_cast<const float4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+  static __device__ __forceinline__ void store(float* p, const float (&v)[8]) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+  }
+};
+
+// Train-step epilogue of the forward GEMM, one block per 32 rows x 256
+// columns (block 32 x 8; thread (x, y) owns columns 8x..8x+7 of rows y,
+// y+8, y+16, y+24, whose activities it loads first so that the loads
+// overlap the per-row work):
+//   warp 0: g_i from the per-tile partials (fixed order) and dL/dg_i; in the
+//     blocks of column 0 also g, the next layer's scale 1/max(sqrt g, 1e-12)
+//     and the loss terms of the rows; the last of those blocks to finish
+//     reduces the loss in block order and sets the Adam step t and the
+//     bias-correction terms for the update that follows;
+//   all: dZ'_ij = s_i * 2 dL/dg_i * h_ij (h = 0 where z <= 0) in the operand
+//     type, and the block's column sums of dZ for db.
+constexpr int kGradRows = 32;
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __restrict__ H, T* __restrict__ dZ) {
+  __shared__ float red[8][256 + 8];
+  __shared__ float c2s[kGradRows], c2[kGradRows];
+  __shared__ int is_last;
+  const int r0 = blockIdx.y * kGradRows;
+  const bool lead = blockIdx.x == 0;
+  const int cg = blockIdx.x * 256 + threadIdx.x * 8;
+  const bool cols_ok = cg < a.ld;
+  float h[4][8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int i = r0 + threadIdx.y + 8 * k;
+    if (cols_ok && i < a.M) {
+      Vec8<T>::load(H + (size_t)i * a.ld + cg, h[k]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) h[k][e] = 0.f;
+    }
+  }
+  if (threadIdx.y == 0) {
+    const int i = r0 + threadIdx.x;
+    float cc = 0.f, sc = 0.f, lv = 0.f;
+    if (i < a.M) {
+      float g = 0.f;
+      for (int t = 0; t < a.ntiles; ++t) g += a.gpart[(size_t)t * a.M + i];
+      const bool pos = i < a.B;
+      const float tt = pos ? a.theta - g : g - a.theta;  // the pair member's margin error
+      const float sg = sigmoid_f(tt);
+      cc = 2.f * (pos ? -sg : sg) / (float)a.B;
+      sc = a.s[i] * cc;
+      if (lead) {
+        if (!isfinite(g)) atomicOr(a.err, DEVERR_NONFINITE);
+        if (a.g_out) a.g_out[i] = g;
+        if (a.s_next) a.s_next[i] = inv_norm(g);
+        lv = softplus_f(tt);
+      }
+    }
+    c2[threadIdx.x] = cc;
+    c2s[threadIdx.x] = sc;
+    if (lead) {
+      lv = warp_sum(lv);
+      if (threadIdx.x == 0) {
+        a.loss_part[blockIdx.y] = lv;
+        __threadfence();
+        const unsigned prev = atomicAdd(&a.ds->counter, 1u);
+        is_last = (prev == gridDim.y - 1);
+      }
+    }
+  }
+  __syncthreads();
+  float db[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) db[e] = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int rr = threadIdx.y + 8 * k;
+    const int i = r0 + rr;
+    const float cc = c2[rr], sc = c2s[rr];
+    float z[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      z[e] = sc * h[k][e];
+      db[e] = fmaf(cc, h[k][e], db[e]);
+    }
+    if (cols_ok && i < a.M) Vec8<T>::store(dZ + (size_t)i * a.ld + cg, z);
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) red[threadIdx.y][threadIdx.x * 8 + e] = db[e];
+  __syncthreads();
+  if (threadIdx.y == 0) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int j = cg + e;
+      float t = 0.f;
+#pragma unroll
+      for (int y = 0; y < 8; ++y) t += red[y][threadIdx.x * 8 + e];
+      if (j < a.N) a.dbpart[(size_t)blockIdx.y * a.N + j] = t;
+    }
+  }
+  if (lead && is_last && threadIdx.y == 0) {
+    // warp 0 of the last block: loss partials summed lane-strided, then a
+    // fixed-order warp tree (the same order every run)
+    __threadfence();
+    const volatile float* lp = a.loss_part;
+    float tot = 0.f;
+    for (unsigned b = threadIdx.x; b < gridDim.y; b += 32) tot += lp[b];
+    tot = warp_sum(tot);
+    if (threadIdx.x == 0) {
+      a.loss_out[0] = tot / (float)a.B;
+      a.ds->counter = 0;
+      // the Adam update that follows is step t; beta^t kept as running products
+      a.ds->t += 1;
+      a.ds->pow1 *= a.beta1;
+      a.ds->pow2 *= a.beta2;
+      a.ds->bc1 = (float)(1.0 - a.ds->pow1);
+      a.ds->bc2 = (float)(1.0 - a.ds->pow2);
+    }
+  }
+}
+
+// --------------------------------------------------------------------- Adam
+__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float lr, float b1, float b2, float eps,
+                                      float bc1, float bc2) {
+  m = b1 * m + (1.f - b1) * g;
+  v = b2 * v + (1.f - b2) * g * g;
+  const float mh = m / bc1;
+  const float vh = v / bc2;
+  w -= lr * mh / (sqrtf(vh) + eps);
+}
+
+__global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
+  const float bc1 = a.ds->bc1, bc2 = a.ds->bc2;
+  if ((int)blockIdx.x < w_blocks) {
+    const long long total = (long long)a.N * a.K;
+    const long long stride = (long long)w_blocks * 256;
+    if ((a.K & 3) == 0) {
+      for (long long q = (long long)blockIdx.x * 256 + threadIdx.x; q * 4 < total; q += stride) {
+        const long long idx = q * 4;
+        float4 w = *reinterpret_cast<float4*>(a.W + idx);
+        float4 m = *reinterpret_cast<float4*>(a.mW + idx);
+        float4 v = *reinterpret_cast<float4*>(a.vW + idx);
+        const float4 g = *reinterpret_cast<const float4*>(a.dW + idx);
+        adam1(w.x, m.x, v.x, g.x, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        adam1(w.y, m.y, v.y, g.y, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        adam1(w.z, m.z, v.z, g.z, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        adam1(w.w, m.w, v.w, g.w, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        *reinterpret_cast<float4*>(a.W + idx) = w;
+        *reinterpret_cast<float4*>(a.mW + idx) = m;
+        *reinterpret_cast<float4*>(a.vW + idx) = v;
+        if (a.Wb) {
+          const long long n = idx / a.K, k = idx % a.K;
+          __nv_bfloat162 p0 = __floats2bfloat162_rn(w.x, w.y), p1 = __floats2bfloat162_rn(w.z, w.w);
+          uint2 u = make_uint2(*reinterpret_cast<uint32_t*>(&p0), *reinterpret_cast<uint32_t*>(&p1));
+          *reinterpret_cast<uint2*>(a.Wb + n * a.ldb + k) = u;
+        }
+      }
+    } else {
+      for (long long idx = (long long)blockIdx.x * 256 + threadIdx.x; idx < total; idx += stride) {
+        float w = a.W[idx], m = a.mW[idx], v = a.vW[idx];
+        adam1(w, m, v, a.dW[idx], a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        a.W[idx] = w;
+        a.mW[idx] = m;
+        a.vW[idx] = v;
+        if (a.Wb) a.Wb[(idx / a.K) * a.ldb + idx % a.K] = __float2bfloat16_rn(w);
+      }
+    }
+  } else {
+    const int j = (blockIdx.x - w_blocks) * 256 + threadIdx.x;
+    if (j >= a.N) return;
+    float db = 0.f;
+    for (int rb = 0; rb < a.nrb; ++rb) db += a.dbpart[(size_t)rb * a.N + j];
+    if (a.db_out) a.db_out[j] = db;
+    if (a.has_bias) {
+      float b = a.b[j], m = a.mb[j], v = a.vb[j];
+      adam1(b, m, v, db, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+      a.b[j] = b;
+      a.mb[j] = m;
+      a.vb[j] = v;
+    }
+  }
+}
+
+// --------------------------------------------------------------------- init
+// SplitMix64 (Steele, Lea, Flood 2014; finaliser constants of Vigna's
+// splitmix64.c), used counter-based: output i of a stream with initial
+// state s0 is mix(s0 + (i + 1) * gamma).
+__device__ __host__ __forceinline__ unsigned long long sm64_mix(unsigned long long z) {
+  z = (z ^ (z >> 30)) * 0xBF58476D1CE4E5B9ull;
+  z = (z ^ (z >> 27)) * 0x94D049BB133111EBull;
+  return z ^ (z >> 31);
+}
+constexpr unsigned long long kGamma = 0x9E3779B97F4A7C15ull;
+constexpr unsigned long long kStreamWeights = 4;
+
+__global__ void k_init_weights(float* __restrict__ W, long long total, unsigned long long s0, double bound) {
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const unsigned long long r = sm64_mix(s0 + (unsigned long long)(i + 1) * kGamma);
+    const double u = (double)(r >> 11) * 0x1.0p-53;
+    W[i] = (float)((2.0 * u - 1.0) * bound);
+  }
+}
+
+__global__ void k_to_bf16(const float* __restrict__ W, int N, int K, bf16* __restrict__ Wb, int ldb) {
+  const long long total = (long long)N * ldb;
+  for (long long i = (long long)blockIdx.x * blockDim.x + threadIdx.x; i < total;
+       i += (long long)gridDim.x * blockDim.x) {
+    const long long n = i / ldb, k = i % ldb;
+    Wb[i] = __float2bfloat16_rn(k < K ? W[n * K + k] : 0.f);
+  }
+}
+
+// ------------------------------------------------------------------ predict
+template <typename T>
+__global__ void k_label_columns(const T* __restrict__ W, int ldw, int N, float* __restrict__ cols) {
+  const int j = blockIdx.x * blockDim.x + threadIdx.x;
+  if (j >= N) return;
+#pragma unroll
+  for (int c = 0; c < 10; ++c) cols[c * N + j] = to_f(W[(size_t)j * ldw + c]);
+}
+
+// One block per sample: for each label c the layer-1 activity of the
+// overlaid input, h = ReLU(s * (base + W[:, c]) + b), using
+//   overlay(x, c) W^T = x0 W^T + W[:, c]   (x0: x with features 0..9 zeroed)
+// and the goodness/next scale of that row (row r = 10 * sample + c).
+template <typename T>
+__global__ void __launch_bounds__(256) k_expand(const float* __restrict__ base, int ldbase,
+                                                const float* __restrict__ cols, const float* __restrict__ s1,
+                                                const float* __restrict__ bias, int N, T* __restrict__ H, int ldh,
+                                                float* __restrict__ s_next, float* __restrict__ G_acc, int* err) {
+  __shared__ float red[8];
+  const int n = blockIdx.x;
+  const float s = s1[n];
+  const float* brow = base + (size_t)n * ldbase;
+  for (int c = 0; c < 10; ++c) {
+    const size_t r = (size_t)n * 10 + c;
+    T* hrow = H + r * ldh;
+    float g = 0.f;
+    for (int j = threadIdx.x; j < ldh; j += 256) {
+      float h = 0.f;
+      if (j < N) {
+        float z = s * (brow[j] + cols[c * N + j]);
+        if (bias) z += bias[j];
+        h = relu_nan(z);
+      }
+      g = fmaf(h, h, g);
+      hrow[j] = from_f<T>(h);
+    }
+    g = block_sum_256(g, red);
+    if (threadIdx.x == 0) {
+      if (!isfinite(g)) atomicOr(err, DEVERR_NONFINITE);
+      s_next[r] = inv_norm(g);
+      if (G_acc) G_acc[r] += g;
+    }
+  }
+}
+
+__global__ void k_argmax(const float* __restrict__ G, int n, int* __restrict__ pred) {
+  const int i = blockIdx.x * blockDim.x + threadIdx.x;
+  if (i >= n) return;
+  const float* g = G + (size_t)i * 10;
+  int best = 0;
+  float bv = g[0];
+#pragma unroll
+  for (int c = 1; c < 10; ++c)
+    if (g[c] > bv) {
+      bv = g[c];
+      best = c;
+    }
+  pred[i] = best;
+}
+
+int grid_for(long long work, int per_block, int cap) {
+  long long b = (work + per_block - 1) / per_block;
+  if (b < 1) b = 1;
+  return (int)(b > cap ? cap : b);
+}
+
+}  // namespace
+
+cudaError_t launch_overlay(const float* x, const int* labels, int rows, int F, void* out, int ldo, bool out_bf16,
+                           float* s_out, int mode, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  const int grid = cdiv(rows, 8);
+  if (out_bf16)
+    k_overlay<bf16><<<grid, 256, 0, st>>>(x, labels, rows, F, (bf16*)out, ldo, s_out, mode);
+  else
+    k_overlay<float><<<grid, 256, 0, st>>>(x, labels, rows, F, (float*)out, ldo, s_out, mode);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_row_scale(const void* x, int ldx, bool x_bf16, int rows, int F, float* s_out, cudaStream_t st) {
+  if (rows <= 0) return cudaSuccess;
+  const int grid = cdiv(rows, 8);
+  if (x_bf16)
+    k_row_scale<bf16><<<grid, 256, 0, st>>>((const bf16*)x, ldx, rows, F, s_out);
+  else
+    k_row_scale<float><<<grid, 256, 0, st>>>((const float*)x, ldx, rows, F, s_out);
+  return cudaGetLastError();
+}
+
+int finalize_grid(int M) { return cdiv(M, 256); }
+
+cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st) {
+  if (a.M <= 0) return cudaSuccess;
+  k_finalize<<<finalize_grid(a.M), 256, 0, st>>>(a);
+  return cudaGetLastError();
+}
+
+int local_grad_row_blocks(int M) { return cdiv(M, kGradRows); }
+
+cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, void* dZ, cudaStream_t st) {
+  dim3 grid(cdiv(a.ld, 256), local_grad_row_blocks(a.M));
+  dim3 block(32, 8);
+  if (b16)
+    k_grad_prep<bf16><<<grid, block, 0, st>>>(a, (const bf16*)H, (bf16*)dZ);
+  else
+    k_grad_prep<float><<<grid, block, 0, st>>>(a, (const float*)H, (float*)dZ);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st) {
+  const long long total = (long long)a.N * a.K;
+  const int w_blocks = grid_for((a.K & 3) == 0 ? total / 4 : total, 256, 152 * 16);
+  const int b_blocks = cdiv(a.N, 256);
+  k_adam<<<w_blocks + b_blocks, 256, 0, st>>>(a, w_blocks);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st) {
+  const long long total = (long long)N * K;
+  const unsigned long long key = ((seed & ((1ull << 56) - 1)) << 8) | kStreamWeights;
+  const unsigned long long s0 = sm64_mix(key);
+  const double bound = std::sqrt(6.0 / (double)K);
+  k_init_weights<<<grid_for(total, 256, 152 * 32), 256, 0, st>>>(W, total, s0, bound);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cudaStream_t st) {
+  k_to_bf16<<<grid_for((long long)N * ldb, 256, 152 * 32), 256, 0, st>>>(W, N, K, Wb, ldb);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols, cudaStream_t st) {
+  if (w_bf16)
+    k_label_columns<bf16><<<cdiv(N, 256), 256, 0, st>>>((const bf16*)W, ldw, N, cols);
+  else
+    k_label_columns<float><<<cdiv(N, 256), 256, 0, st>>>((const float*)W, ldw, N, cols);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_expand(const float* base, int ldbase, const float* cols, const float* s1, const float* bias, int n,
+                          int N, void* H, int ldh, bool h_bf16, float* s_next, float* G_acc, int* err,
+                          cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  if (h_bf16)
+    k_expand<bf16><<<n, 256, 0, st>>>(base, ldbase, cols, s1, bias, N, (bf16*)H, ldh, s_next, G_acc, err);
+  else
+    k_expand<float><<<n, 256, 0, st>>>(base, ldbase, cols, s1, bias, N, (float*)H, ldh, s_next, G_acc, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_argmax(const float* G, int n, int* pred, float* /*unused*/, cudaStream_t st) {
+  if (n <= 0) return cudaSuccess;
+  k_argmax<<<cdiv(n, 256), 256, 0, st>>>(G, n, pred);
+  return cudaGetLastError();
+}
+
+}  // namespace ff

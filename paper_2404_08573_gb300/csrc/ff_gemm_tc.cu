@@ -1,0 +1,433 @@
+// Tensor-core GEMMs of the FF layer step (bf16 operands, fp32 accumulate in
+// TMEM), written for sm_103a with tcgen05 + TMA:
+//
+//   forward  Z = diag(s) X W^T + b, H = ReLU(Z), per-tile goodness partials
+//            (the linear+ReLU of §3 on the concatenated batch of §4, and the
+//            sum of squared activities of Eq. 1 taken from the fp32
+//            accumulator);
+//   store    C = X W^T in fp32 (the label-free part of layer 1 in predict);
+//   wgrad    dW = G^T X with G = diag(s) dZ, contracting over the batch rows
+//            (both operands are read MN-major straight from their row-major
+//            buffers: no transposed copies).
+//
+// One CTA computes one BM x BN output tile with three warp roles:
+//   warp 0      TMA producer: 128-byte-swizzled tiles into a STAGES-deep ring
+//   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
+//               N=BN, K=16) and commits each stage back to the producer
+//   warps 2..5  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).. -> registers,
+//               fused scale/bias/ReLU/goodness or plain store
+// Every mbarrier wait is bounded (kWaitTimeoutNs); a timeout latches
+// DEVERR_TIMEOUT in *err, tells the other roles to stop, waits for copies and
+// MMAs already in flight and frees TMEM before the CTA exits.
+#include <cudaTypedefs.h>
+
+#include <mutex>
+
+#include "ff_internal.cuh"
+#include "ff_ptx.cuh"
+
+namespace ff {
+namespace {
+
+constexpr int BM = 128;
+constexpr int BK = 64;  // one 128-byte swizzle row of bf16
+constexpr int NTHREADS = 192;
+constexpr int MODE_FWD = 0;
+constexpr int MODE_STORE = 1;
+
+template <int BN>
+struct TcCfg {
+  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int RAW_STAGES = (220 * 1024 - 2048) / STAGE;
+  static constexpr int STAGES = RAW_STAGES > 8 ? 8 : RAW_STAGES;
+  static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
+  static constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static_assert(BN % 64 == 0 && BN <= 256, "BN must be a multiple of 64, at most 256");
+  static_assert(4 * 32 * BN * 4 <= STAGES * STAGE, "epilogue staging must fit in the operand ring");
+  static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
+};
+
+__device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
+  *abort_flag = 1;
+  atomicOr(err, DEVERR_TIMEOUT);
+}
+
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM>
+__global__ void __launch_bounds__(NTHREADS, 1)
+    k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
+              const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
+  using C = TcCfg<BN>;
+  extern __shared__ uint8_t smem_raw[];
+  // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
+  const uint32_t raw_s = ptx::smem_u32(smem_raw);
+  uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
+  uint8_t* sA = smem;
+  uint8_t* sB = smem + C::STAGES * C::A_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  uint64_t* empty = full + C::STAGES;
+  uint64_t* tfull = empty + C::STAGES;
+  uint32_t* tslot = reinterpret_cast<uint32_t*>(tfull + 1);
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(tslot + 1);
+  volatile int* never_set = reinterpret_cast<volatile int*>(tslot + 2);  // drain waits ignore the abort
+  float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [BN] bias of this tile
+
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const int m0 = blockIdx.y * BM;
+  const int n0 = blockIdx.x * BN;
+  const int num_kb = (K + BK - 1) / BK;
+
+  // CM > 1: the CM CTAs of a cluster (consecutive tile rows, same columns)
+  // share the B tile; CTA `crank` loads B rows [crank*BN/CM, (crank+1)*BN/CM)
+  // and multicasts them, and a stage is refilled only after all CM CTAs have
+  // consumed it (their MMA warps arrive on every CTA's `empty`).
+  const uint32_t crank = CM > 1 ? ptx::cluster_ctarank() : 0u;
+  constexpr uint16_t cmask = (uint16_t)((1u << CM) - 1u);
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < C::STAGES; ++s) {
+      ptx::mbar_init(&full[s], 1);
+      ptx::mbar_init(&empty[s], CM);
+    }
+    ptx::mbar_init(tfull, 1);
+    *abort_flag = 0;
+    *never_set = 0;
+    ptx::fence_mbar_init();
+    ptx::prefetch_tmap(&tmA);
+    ptx::prefetch_tmap(&tmB);
+    if (MODE == MODE_FWD || tma_store) ptx::prefetch_tmap(&tmC);
+  }
+  if (warp == 1) {
+    ptx::tmem_alloc(tslot, C::TMEM_COLS);
+    ptx::tmem_relinquish();
+  }
+  ptx::tc_fence_before();
+  __syncthreads();
+  if (CM > 1) ptx::cluster_sync();  // every CTA's barriers exist before any multicast
+  ptx::tc_fence_after();
+  const uint32_t tmem = *tslot;
+
+  if (warp == 0) {
+    // ------------------------------------------------------------ producer
+    if (lane == 0) {
+      int issued = 0;
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % C::STAGES;
+        const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
+        if (!ptx::mbar_wait(&empty[s], ph ^ 1u, kWaitTimeoutNs, abort_flag)) {
+          latch(err, abort_flag);
+          break;
+        }
+        ptx::mbar_arrive_expect_tx(&full[s], C::STAGE);
+        uint8_t* a = sA + s * C::A_BYTES;
+        uint8_t* b = sB + s * C::B_BYTES;
+        const int k0 = kb * BK;
+        if (!A_MN) {
+          ptx::tma_load_2d(a, &tmA, &full[s], k0, m0);
+        } else {
+#pragma unroll
+          for (int j = 0; j < BM / 64; ++j) ptx::tma_load_2d(a + j * 64 * BK * 2, &tmA, &full[s], m0 + 64 * j, k0);
+        }
+        if (CM == 1) {
+          if (!B_MN) {
+            ptx::tma_load_2d(b, &tmB, &full[s], k0, n0);
+          } else {
+#pragma unroll
+            for (int j = 0; j < BN / 64; ++j) ptx::tma_load_2d(b + j * 64 * BK * 2, &tmB, &full[s], n0 + 64 * j, k0);
+          }
+        } else {
+          // this CTA's slice of B: BN/CM rows (K-major) or BN/CM columns (MN-major)
+          constexpr int SL = BN / CM;
+          if (!B_MN) {
+            ptx::tma_load_2d_mc(b + crank * SL * 128, &tmB, &full[s], k0, n0 + (int)crank * SL, cmask);
+          } else {
+#pragma unroll
+            for (int j = 0; j < SL / 64; ++j) {
+              const int jj = (int)crank * (SL / 64) + j;
+              ptx::tma_load_2d_mc(b + jj * 64 * BK * 2, &tmB, &full[s], n0 + 64 * jj, k0, cmask);
+            }
+          }
+        }
+        issued = kb + 1;
+      }
+      if (CM > 1 && !*abort_flag) {
+        // Producer tail: wait until every CTA of the cluster has released every
+        // stage, so no remote arrival targets this CTA after it exits.
+        for (int kb = num_kb; kb < num_kb + C::STAGES; ++kb) {
+          if (!ptx::mbar_wait(&empty[kb % C::STAGES], ((uint32_t)(kb / C::STAGES) & 1u) ^ 1u, kWaitTimeoutNs,
+                              abort_flag)) {
+            latch(err, abort_flag);
+            break;
+          }
+        }
+      }
+      if (*abort_flag) {
+        // let copies already issued land before the CTA's shared memory goes away
+        int lo = issued - C::STAGES;
+        if (lo < 0) lo = 0;
+        for (int kb = lo; kb < issued; ++kb)
+          ptx::mbar_wait(&full[kb % C::STAGES], (uint32_t)(kb / C::STAGES) & 1u, 10000000ull, never_set);
+      }
+    }
+  } else if (warp == 1) {
+    // ----------------------------------------------------------------- MMA
+    if (lane == 0) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % C::STAGES;
+        const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
+        if (!ptx::mbar_wait(&full[s], ph, kWaitTimeoutNs, abort_flag)) {
+          latch(err, abort_flag);
+          break;
+        }
+        ptx::tc_fence_after();
+        const uint32_t a_base = ptx::smem_u32(sA + s * C::A_BYTES);
+        const uint32_t b_base = ptx::smem_u32(sB + s * C::B_BYTES);
+#pragma unroll
+        for (int k = 0; k < BK / 16; ++k) {
+          // K-major: the 16-element K slice sits 32 bytes further along each
+          // swizzled 128-byte row (SBO = 1024 between 8-row groups).
+          // MN-major: 16 K rows further = 2 x 1024 bytes; LBO = 8192 between
+          // the 64-element MN chunks, SBO = 1024 between 8-row K groups.
+          const uint64_t ad = A_MN ? ptx::sdesc_sw128(a_base + k * 2048, 64 * BK * 2, 1024)
+                                   : ptx::sdesc_sw128(a_base + k * 32, 16, 1024);
+          const uint64_t bd = B_MN ? ptx::sdesc_sw128(b_base + k * 2048, 64 * BK * 2, 1024)
+                                   : ptx::sdesc_sw128(b_base + k * 32, 16, 1024);
+          ptx::umma_f16(tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+        }
+        if (CM == 1)
+          ptx::umma_commit(&empty[s]);
+        else
+          ptx::umma_commit_mc(&empty[s], cmask);
+      }
+      ptx::umma_commit(tfull);  // always: the epilogue and the teardown wait on it
+    }
+  } else {
+    // ------------------------------------------------------------ epilogue
+    // Thread t of warp q owns TMEM lane / tile row 32q + t.  The operand ring
+    // is idle once the accumulator is complete, so each warp stages its 32
+    // rows there in the 128-byte-swizzled layout (conflict-free for
+    // row-per-thread 16-byte writes) and one lane writes them out with TMA.
+    const int q = warp & 3;
+    const int row = q * 32 + lane;
+    const int gi = m0 + row;
+    float s = 0.f;
+    if (MODE == MODE_FWD) {
+      // While the mainloop runs: the tile's bias (zero past N or without bias)
+      // into shared memory and this thread's row scale into a register.
+      for (int c = (int)threadIdx.x - 64; c < BN; c += 128)
+        sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
+      if (gi < M) s = __ldg(ep.row_scale + gi);
+      ptx::named_bar(1, 128);
+    }
+    const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
+    if (!ok) latch(err, abort_flag);
+    ptx::tc_fence_after();
+    // tcgen05.ld is warp-collective: decide for the whole warp at once
+    if (__all_sync(0xffffffffu, ok && !*abort_flag)) {
+      constexpr int ES = MODE == MODE_FWD ? 2 : 4;      // staged element size
+      constexpr int CW = 128 / ES;                       // columns per 128-byte swizzle row
+      uint8_t* stage = smem + q * (32 * BN * ES);
+      const uint32_t sw = (uint32_t)(lane & 7);
+      const bool staged = MODE == MODE_FWD || tma_store;
+      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
+      float g = 0.f;
+      // Columns past N and rows past M hold zero products (their operand rows
+      // were zero-filled); the TMA store clips them and gpart skips them.
+      auto process = [&](const uint32_t (&r)[32], int c0) {
+        const int col0 = n0 + c0;
+        if (MODE == MODE_FWD) {
+          uint32_t packed[16];
+          const float4* b4 = reinterpret_cast<const float4*>(sbias + c0);
+#pragma unroll
+          for (int v = 0; v < 8; ++v) {
+            const float4 bb = b4[v];
+            const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+            float h[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              const float z = fmaf(s, __uint_as_float(r[4 * v + e]), bv[e]);
+              h[e] = z != z ? z : fmaxf(z, 0.f);  // ReLU, NaN kept for the non-finite check
+              g = fmaf(h[e], h[e], g);
+            }
+            __nv_bfloat162 p0 = __floats2bfloat162_rn(h[0], h[1]);
+            __nv_bfloat162 p1 = __floats2bfloat162_rn(h[2], h[3]);
+            packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
+            packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
+          }
+          uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
+#pragma unroll
+          for (int v = 0; v < 4; ++v) {
+            const uint32_t j = (uint32_t)((c0 % CW) / 8 + v);
+            *reinterpret_cast<uint4*>(base + ((j ^ sw) << 4)) =
+                make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2], packed[4 * v + 3]);
+          }
+        } else if (staged) {
+          uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
+#pragma unroll
+          for (int v = 0; v < 8; ++v)
+            *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
+                make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+        } else if (gi < M) {
+          float* out = reinterpret_cast<float*>(ep.out) + (size_t)gi * ep.ldo;
+#pragma unroll
+          for (int j = 0; j < 32; ++j)
+            if (col0 + j < N) out[col0 + j] = __uint_as_float(r[j]);
+        }
+      };
+      // TMEM loads double-buffered: the next 32 columns load while these are processed.
+      uint32_t ra[32], rb[32];
+      ptx::tmem_ld32(trow, ra);
+      ptx::tmem_ld_wait();
+#pragma unroll 1
+      for (int c0 = 0; c0 < BN; c0 += 64) {
+        ptx::tmem_ld32(trow + (uint32_t)(c0 + 32), rb);
+        process(ra, c0);
+        ptx::tmem_ld_wait();
+        if (c0 + 64 < BN) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
+        process(rb, c0 + 32);
+        ptx::tmem_ld_wait();
+      }
+      if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)blockIdx.x * M + gi] = g;
+      if (staged) {
+        ptx::fence_async_smem();
+        __syncwarp();
+        const int r0 = m0 + q * 32;
+        if (lane == 0 && r0 < M) {
+#pragma unroll 1
+          for (int ch = 0; ch < BN / CW; ++ch) {
+            const int col = n0 + ch * CW;
+            if (col < ep.ldo) ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, r0);
+          }
+          ptx::bulk_commit();
+          ptx::bulk_wait_read0();
+        }
+        __syncwarp();
+      }
+    }
+  }
+
+  ptx::tc_fence_before();
+  __syncthreads();
+  ptx::tc_fence_after();
+  if (warp == 1) {
+    if (*abort_flag) {
+      // MMAs issued before the abort must finish before TMEM is released
+      ptx::mbar_wait(tfull, 0, 10000000ull, never_set);
+    }
+    ptx::tmem_dealloc(tmem, C::TMEM_COLS);
+  }
+  if (CM > 1) ptx::cluster_sync();  // no CTA leaves while a peer may still address it
+}
+
+PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
+  static PFN_cuTensorMapEncodeTiled_v12000 fn = nullptr;
+  static std::once_flag once;
+  std::call_once(once, [] {
+    void* p = nullptr;
+    cudaDriverEntryPointQueryResult q;
+    if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &p, 12000, cudaEnableDefault, &q) ==
+            cudaSuccess &&
+        q == cudaDriverEntryPointSuccess)
+      fn = reinterpret_cast<PFN_cuTensorMapEncodeTiled_v12000>(p);
+  });
+  return fn;
+}
+
+// Row-major matrix [rows, cols] of bf16 (esize 2) or fp32 (esize 4) with row
+// stride ld (elements), tiled in boxes of box_rows x box_cols with 128-byte
+// swizzle; out-of-range elements of a box read as zero and are not written.
+bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols, int box_rows) {
+  auto enc = encode_fn();
+  if (!enc) return false;
+  if ((reinterpret_cast<uintptr_t>(ptr) & 15u) || ((size_t)ld * esize) % 16 != 0) return false;
+  cuuint64_t dims[2] = {(cuuint64_t)cols, (cuuint64_t)rows};
+  cuuint64_t strides[1] = {(cuuint64_t)ld * esize};
+  cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
+             const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
+             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
+             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM>
+cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
+                      int K, const EpiArgs& ep, int* err, cudaStream_t st) {
+  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM>;
+  static cudaError_t attr =
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+  if (attr != cudaSuccess) return attr;
+  cudaLaunchConfig_t cfg = {};
+  // tile rows padded to a whole number of clusters; padding CTAs load zeros,
+  // share their B slice and write nothing
+  cfg.gridDim = dim3(cdiv(N, BN), cdiv(cdiv(M, BM), CM) * CM, 1);
+  cfg.blockDim = dim3(NTHREADS, 1, 1);
+  cfg.dynamicSmemBytes = TcCfg<BN>::SMEM;
+  cfg.stream = st;
+  cudaLaunchAttribute at[1];
+  at[0].id = cudaLaunchAttributeClusterDimension;
+  at[0].val.clusterDim.x = 1;
+  at[0].val.clusterDim.y = CM;
+  at[0].val.clusterDim.z = 1;
+  cfg.attrs = at;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, tma_store, M, N, K, ep, err);
+}
+
+constexpr int FWD_BN = 256;
+constexpr int WGRAD_BN = 256;
+constexpr int CLUSTER_M = 4;  // CTAs per cluster along M sharing one B tile
+
+}  // namespace
+
+bool tc_supported() {
+  int dev = 0, major = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess) return false;
+  if (cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess) return false;
+  return major == 10 && encode_fn() != nullptr;
+}
+
+int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN); }
+
+cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
+                        int* err, cudaStream_t st) {
+  CUtensorMap ta, tb, tc;
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M) ||
+      !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
+    return cudaErrorInvalidValue;
+  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M>(ta, tb, tc, 1, M, N, K, ep, err, st);
+}
+
+// fp32 C written through shared memory and TMA when its rows are 16-byte
+// aligned, directly otherwise.
+static bool store_map(CUtensorMap* tc, float* C, int ldc, int rows, int cols) {
+  return make_map(tc, C, 4, ldc, rows, ldc, 32, 32) && cols <= ldc;
+}
+
+cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, float* Cm,
+                          int ldc, int* err, cudaStream_t st) {
+  CUtensorMap ta, tb, tc;
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M))
+    return cudaErrorInvalidValue;
+  const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
+  if (!tma) tc = ta;  // unused
+  EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
+  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M>(ta, tb, tc, tma, M, N, K, ep, err, st);
+}
+
+cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K, float* Cm, int ldc,
+                          int* err, cudaStream_t st) {
+  // C[N, K] = sum_r G[r, n] X[r, k]: the GEMM's M is N (rows of dW), its N is
+  // K (columns of dW), its contraction is R; both operands MN-major.
+  CUtensorMap ta, tb, tc;
+  if (!make_map(&ta, G, 2, N, R, ldg, 64, BK) || !make_map(&tb, X, 2, K, R, ldx, 64, BK))
+    return cudaErrorInvalidValue;
+  const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
+  if (!tma) tc = ta;
+  EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
+  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M>(ta, tb, tc, tma, N, K, R, ep, err, st);
+}
+
+}  // namespace ff

@@ -1,0 +1,159 @@
+// Internal declarations shared by the libff translation units.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+
+#include <cstddef>
+#include <cstdint>
+
+#include "ff.h"
+
+typedef __nv_bfloat16 bf16;
+
+namespace ff {
+
+// Device-side error bits latched in ff_dev_state::err.
+enum : int { DEVERR_TIMEOUT = 1, DEVERR_NONFINITE = 2 };
+
+// Bound on every spin-wait in a kernel: after this many nanoseconds of
+// %globaltimer the wait gives up, latches DEVERR_TIMEOUT and the kernel
+// winds down.
+constexpr unsigned long long kWaitTimeoutNs = 1000000000ull;  // 1 s
+
+// Per-layer scalars that kernels read and write on the device, so that a
+// captured CUDA graph replays correctly (no per-step host arguments).
+struct ff_dev_state {
+  long long t;        // Adam step counter (number of completed updates)
+  double pow1, pow2;  // beta1^t, beta2^t
+  float bc1, bc2;     // 1 - beta1^t, 1 - beta2^t of the current update
+  int err;            // latched DEVERR_* bits
+  unsigned counter;   // last-block-done counter of the goodness/loss kernel
+  float loss;         // loss of the last train step when the caller passed none
+  int pad;
+};
+
+inline int row_stride(int features) { return (features + 7) & ~7; }
+inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
+
+// ------------------------------------------------------------------ kernels
+// All launchers return the launch status (cudaGetLastError after the launch).
+
+// Overlay (train/forward) or label-area zeroing (predict), cast, row scale.
+//   mode 0: out[:,0..9] = one-hot(labels[r]); mode 1: out[:,0..9] = 0 and the
+//   norm counts one extra 1.0 (the one-hot every predict overlay adds).
+cudaError_t launch_overlay(const float* x, const int* labels, int rows, int F, void* out,
+                           int ldo, bool out_bf16, float* s_out, int mode, cudaStream_t st);
+// s_r = 1 / max(||x_r||, 1e-12) of an activation buffer.
+cudaError_t launch_row_scale(const void* x, int ldx, bool x_bf16, int rows, int F,
+                             float* s_out, cudaStream_t st);
+// Goodness from the forward GEMM's per-tile partials (forward and predict).
+struct FinalizeArgs {
+  const float* gpart; int ntiles; int M;
+  float* g_out;        // [M] or null
+  float* s_next;       // [M] or null
+  float* G_acc;        // [M] predict goodness accumulator or null
+  int* err;            // error word
+};
+int finalize_grid(int M);
+cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st);
+// Train step after the forward GEMM: goodness, loss, dL/dg, next-layer scale,
+// dZ' = (s * 2 dL/dg) * H in the operand type, db partials per 32 rows, and
+// the Adam step counter / bias-correction terms.
+struct GradPrepArgs {
+  const float* gpart; int ntiles; int M; int N; int ld;  // ld: row stride of H and dZ
+  int B; float theta;
+  const float* s;      // [M] row scale of this layer's input
+  float* g_out;        // [M] or null
+  float* s_next;       // [M] or null
+  float* dbpart;       // [row blocks, N]
+  float* loss_part;    // [row blocks]
+  float* loss_out;     // [1]
+  ff_dev_state* ds;
+  double beta1, beta2;
+  int* err;
+};
+cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, void* dZ, cudaStream_t st);
+int local_grad_row_blocks(int M);
+struct AdamArgs {
+  float* W; float* mW; float* vW; const float* dW; int N; int K;
+  bf16* Wb; int ldb;      // bf16 copy of W or null
+  float* b; float* mb; float* vb; const float* dbpart; int nrb; float* db_out;
+  int has_bias;
+  float lr, beta1, beta2, eps;
+  const ff_dev_state* ds;
+};
+cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
+cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
+cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cudaStream_t st);
+// predict helpers
+cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols /*[10,N]*/,
+                                 cudaStream_t st);
+cudaError_t launch_expand(const float* base, int ldbase, const float* cols, const float* s1,
+                          const float* bias, int n, int N, void* H, int ldh, bool h_bf16,
+                          float* s_next, float* G_acc /*null unless single layer*/, int* err,
+                          cudaStream_t st);
+cudaError_t launch_argmax(const float* G, int n, int* pred, float* goodness_out, cudaStream_t st);
+
+// ------------------------------------------------------------------- GEMMs
+// Forward epilogue: H = ReLU(s_r * acc + b) (bf16 or fp32), per-tile goodness
+// partials gpart[tile_n * M + r].  Store epilogue: C = acc (fp32).
+struct EpiArgs {
+  const float* row_scale;
+  const float* bias;   // null: no bias
+  void* out; int ldo;
+  float* gpart;        // forward only
+};
+
+// Tensor-core (tcgen05) bf16 GEMMs, fp32 accumulate.
+//   fwd/store: C[M,N] = A[M,K] B[N,K]^T  (A, B row-major, K contiguous)
+//   wgrad:     C[N,K] = G[R,N]^T X[R,K]  (contraction over R rows)
+int tc_fwd_ntiles(int N);
+cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
+                        const EpiArgs& ep, int* err, cudaStream_t st);
+cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
+                          float* C, int ldc, int* err, cudaStream_t st);
+cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K,
+                          float* C, int ldc, int* err, cudaStream_t st);
+bool tc_supported();
+
+// SIMT fp32 GEMMs with the same contracts.
+int simt_fwd_ntiles(int N);
+cudaError_t simt_gemm_fwd(const float* A, int lda, const float* B, int ldb, int M, int N, int K,
+                          const EpiArgs& ep, cudaStream_t st);
+cudaError_t simt_gemm_store(const float* A, int lda, const float* B, int ldb, int M, int N, int K,
+                            float* C, int ldc, cudaStream_t st);
+cudaError_t simt_gemm_wgrad(const float* G, int ldg, const float* X, int ldx, int R, int N, int K,
+                            float* C, int ldc, cudaStream_t st);
+
+}  // namespace ff
+
+// The layer object behind the opaque handle.
+struct ff_layer {
+  ff_layer_config cfg;
+  int K, N, ldK, ldN;
+  int device;
+  bool is_bf16;
+  cudaStream_t last_stream;
+  // parameters and Adam moments (fp32, dense [N,K] / [N])
+  float *W, *b, *mW, *vW, *mb, *vb;
+  bf16* Wb;          // [N, ldK] bf16 copy (bf16 mode)
+  float* db;         // [N] reduced bias gradient of the last step
+  float* dW;         // [N, K] weight gradient of the last step
+  ff::ff_dev_state* ds;
+  // workspace, capacity cap rows
+  int cap;
+  void* X;           // [cap, ldK] overlay output
+  float* s_in;       // [cap]
+  void* H;           // [cap, ldN] activity when the caller passes no h_out
+  void* dZ;          // [cap, ldN] weight-gradient operand s*dZ
+  float* gpart;      // [ntiles, cap]
+  float* g;          // [cap]
+  float* c;          // [cap]
+  float* s_next;     // [cap]
+  float* dbpart;     // [row blocks, N]
+  float* loss_part;  // [max(finalize blocks, row blocks)]
+  // predict scratch (owned here when this layer is layers[0] of ff_predict)
+  void* pws; size_t pws_bytes;
+};

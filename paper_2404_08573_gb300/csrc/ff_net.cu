@@ -1,0 +1,190 @@
+// A net of FF layers trained concurrently on one GPU, one CUDA stream per
+// layer: the single-GPU analogue of Single-Layer PFF (§4.1, Algorithm 1),
+// where node i trains L_i on the output of L_{i-1} while node i-1 already
+// trains further.  Here the hand-off is per batch through ring buffers of
+// `depth` activation slots per layer boundary:
+//   layer k, batch t: waits ready[k-1][t % depth] (layer k-1's forward of
+//   batch t is written) and, before overwriting its own output slot,
+//   consumed[k][t % depth] (layer k+1 has finished batch t - depth).
+// Each layer's own steps stay in order on its stream, so every kernel sees
+// exactly the inputs it would see in a one-stream run: results are bitwise
+// identical to the sequential schedule.
+#include <vector>
+
+#include "ff_api_internal.h"
+
+struct ff_net {
+  std::vector<ff_layer*> layers;
+  int L = 0, max_B = 0, depth = 0;
+  std::vector<cudaStream_t> streams;
+  std::vector<std::vector<void*>> hbuf;
+  std::vector<std::vector<float*>> sbuf;
+  std::vector<std::vector<cudaEvent_t>> ready, consumed;
+  std::vector<cudaEvent_t> tail;
+  cudaEvent_t ev_x_in = nullptr, ev_x_done = nullptr;
+  long long step = 0;
+  long long since_sync = 0;  // steps enqueued since the last ff_net_sync
+  void* mem = nullptr;
+};
+
+namespace {
+
+void release(ff_net* n) {
+  if (!n) return;
+  for (auto st : n->streams)
+    if (st) cudaStreamSynchronize(st);
+  // the layers outlive the net: they must not keep a stream that is about to go away
+  for (auto* l : n->layers)
+    for (auto st : n->streams)
+      if (l && st && l->last_stream == st) l->last_stream = nullptr;
+  for (auto& v : n->ready)
+    for (auto e : v)
+      if (e) cudaEventDestroy(e);
+  for (auto& v : n->consumed)
+    for (auto e : v)
+      if (e) cudaEventDestroy(e);
+  for (auto e : n->tail)
+    if (e) cudaEventDestroy(e);
+  if (n->ev_x_in) cudaEventDestroy(n->ev_x_in);
+  if (n->ev_x_done) cudaEventDestroy(n->ev_x_done);
+  for (auto st : n->streams)
+    if (st) cudaStreamDestroy(st);
+  ff::dev_free(n->mem);
+  delete n;
+}
+
+}  // namespace
+
+extern "C" {
+
+ff_status ff_net_create(ff_layer* const* layers, int n_layers, int max_B, int depth, ff_net** out) {
+  if (!out) return FF_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!layers || n_layers < 1 || max_B < 1 || depth < 1 || depth > 64) return FF_ERR_INVALID_ARG;
+  for (int k = 0; k < n_layers; ++k) {
+    if (!layers[k]) return FF_ERR_INVALID_ARG;
+    if (k > 0 && (layers[k]->K != layers[k - 1]->N || layers[k]->is_bf16 != layers[0]->is_bf16)) return FF_ERR_INVALID_ARG;
+    for (int j = 0; j < k; ++j)
+      if (layers[j] == layers[k]) return FF_ERR_INVALID_ARG;
+  }
+  if (layers[0]->K < 10) return FF_ERR_INVALID_ARG;
+  ff_net* n = new (std::nothrow) ff_net();
+  if (!n) return FF_ERR_OOM;
+  n->layers.assign(layers, layers + n_layers);
+  n->L = n_layers;
+  n->max_B = max_B;
+  n->depth = depth;
+  const size_t M = 2 * (size_t)max_B;
+  const size_t es = layers[0]->is_bf16 ? 2 : 4;
+  size_t total = 0;
+  for (int k = 0; k + 1 < n_layers; ++k)
+    total += (size_t)depth * (((M * layers[k]->ldN * es + 255) & ~(size_t)255) + ((M * 4 + 255) & ~(size_t)255));
+  ff_status s = FF_OK;
+  if (total) s = ff::cuda_status(ff::dev_alloc(&n->mem, total), "net activation buffers");
+  if (s != FF_OK) {
+    release(n);
+    return s;
+  }
+  char* p = static_cast<char*>(n->mem);
+  n->hbuf.resize(n_layers > 1 ? n_layers - 1 : 0);
+  n->sbuf.resize(n->hbuf.size());
+  n->ready.resize(n->hbuf.size());
+  n->consumed.resize(n->hbuf.size());
+  for (int k = 0; k + 1 < n_layers; ++k) {
+    for (int d = 0; d < depth; ++d) {
+      n->hbuf[k].push_back(p);
+      p += (M * layers[k]->ldN * es + 255) & ~(size_t)255;
+      n->sbuf[k].push_back(reinterpret_cast<float*>(p));
+      p += (M * 4 + 255) & ~(size_t)255;
+      cudaEvent_t e1 = nullptr, e2 = nullptr;
+      cudaError_t e = cudaEventCreateWithFlags(&e1, cudaEventDisableTiming);
+      if (e == cudaSuccess) e = cudaEventCreateWithFlags(&e2, cudaEventDisableTiming);
+      n->ready[k].push_back(e1);
+      n->consumed[k].push_back(e2);
+      if (e != cudaSuccess) {
+        release(n);
+        return ff::cuda_status(e, "net events");
+      }
+    }
+  }
+  for (int k = 0; k < n_layers; ++k) {
+    cudaStream_t st = nullptr;
+    cudaEvent_t ev = nullptr;
+    cudaError_t e = cudaStreamCreateWithFlags(&st, cudaStreamNonBlocking);
+    n->streams.push_back(st);
+    if (e == cudaSuccess) e = cudaEventCreateWithFlags(&ev, cudaEventDisableTiming);
+    n->tail.push_back(ev);
+    if (e != cudaSuccess) {
+      release(n);
+      return ff::cuda_status(e, "net streams");
+    }
+  }
+  cudaError_t e = cudaEventCreateWithFlags(&n->ev_x_in, cudaEventDisableTiming);
+  if (e == cudaSuccess) e = cudaEventCreateWithFlags(&n->ev_x_done, cudaEventDisableTiming);
+  if (e != cudaSuccess) {
+    release(n);
+    return ff::cuda_status(e, "net events");
+  }
+  *out = n;
+  return FF_OK;
+}
+
+ff_status ff_net_destroy(ff_net* n) {
+  release(n);
+  return FF_OK;
+}
+
+ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
+  if (!n || !x || !labels || B < 0 || B > n->max_B) return FF_ERR_INVALID_ARG;
+  if (B == 0) return FF_OK;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  const int slot = (int)(n->step % n->depth);
+  ff_status s = ff::cuda_status(cudaEventRecord(n->ev_x_in, cs), "record input event");
+  if (s != FF_OK) return s;
+  for (int k = 0; k < n->L; ++k) {
+    cudaStream_t st = n->streams[k];
+    cudaError_t e = cudaStreamWaitEvent(st, k == 0 ? n->ev_x_in : n->ready[k - 1][slot], 0);
+    // Before overwriting its output slot, layer k waits until layer k+1 has
+    // read what batch t - depth left there.  Within `depth` steps after an
+    // ff_net_sync that read is already ordered before this point (every
+    // stream joined the caller's stream, which this step's input event
+    // follows), so no wait is issued: a synced run of steps is self-contained
+    // and can be captured in a CUDA graph.
+    if (e == cudaSuccess && k + 1 < n->L && n->since_sync >= n->depth)
+      e = cudaStreamWaitEvent(st, n->consumed[k][slot], 0);
+    s = ff::cuda_status(e, "stream wait");
+    if (s != FF_OK) return s;
+    const void* xin = k == 0 ? static_cast<const void*>(x) : n->hbuf[k - 1][slot];
+    const float* scale = k == 0 ? nullptr : n->sbuf[k - 1][slot];
+    void* hout = k + 1 < n->L ? n->hbuf[k][slot] : nullptr;
+    float* sn = k + 1 < n->L ? n->sbuf[k][slot] : nullptr;
+    s = ff::train_step_impl(n->layers[k], xin, k == 0 ? labels : nullptr, scale, B, hout, sn, nullptr,
+                            loss ? loss + k : nullptr, st, k == 0 ? n->ev_x_done : nullptr,
+                            k + 1 < n->L ? n->ready[k][slot] : nullptr);
+    if (s != FF_OK) return s;
+    if (k > 0) {
+      s = ff::cuda_status(cudaEventRecord(n->consumed[k - 1][slot], st), "record consumed event");
+      if (s != FF_OK) return s;
+    }
+  }
+  s = ff::cuda_status(cudaStreamWaitEvent(cs, n->ev_x_done, 0), "input hand-back");
+  if (s != FF_OK) return s;
+  ++n->step;
+  ++n->since_sync;
+  return FF_OK;
+}
+
+ff_status ff_net_sync(ff_net* n, void* stream) {
+  if (!n) return FF_ERR_INVALID_ARG;
+  cudaStream_t cs = static_cast<cudaStream_t>(stream);
+  for (int k = 0; k < n->L; ++k) {
+    cudaError_t e = cudaEventRecord(n->tail[k], n->streams[k]);
+    if (e == cudaSuccess) e = cudaStreamWaitEvent(cs, n->tail[k], 0);
+    ff_status s = ff::cuda_status(e, "net sync");
+    if (s != FF_OK) return s;
+  }
+  n->since_sync = 0;
+  return FF_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,274 @@
+"""Python binding of libff (ctypes).  Argument marshalling only.
+
+Every computation runs in libff's CUDA kernels; PyTorch supplies device
+memory (tensors whose data pointers are passed through) and streams.  There
+is no fallback: if libff.so is missing or the GPU cannot run it, calls raise.
+
+Names follow the C ABI in include/ff.h:
+``Layer`` (ff_layer_*), ``overlay_label``, ``predict``, ``Net`` (ff_net_*).
+"""
+
+from __future__ import annotations
+
+import ctypes
+import os
+from ctypes import POINTER, c_float, c_int, c_longlong, c_ulonglong, c_void_p
+
+import numpy as np
+import torch
+
+FF_FP32, FF_BF16 = 0, 1
+_STATUS = {
+    0: "FF_OK", 1: "FF_ERR_INVALID_ARG", 2: "FF_ERR_CUDA", 3: "FF_ERR_OOM",
+    4: "FF_ERR_TIMEOUT", 5: "FF_ERR_NONFINITE", 6: "FF_ERR_UNSUPPORTED",
+}
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libff.so")
+
+
+class FFError(RuntimeError):
+    def __init__(self, status: int, what: str):
+        self.status = status
+        super().__init__(f"{what}: {_STATUS.get(status, status)}")
+
+
+class LayerConfig(ctypes.Structure):
+    _fields_ = [
+        ("in_features", c_int), ("out_features", c_int), ("has_bias", c_int),
+        ("theta", c_float), ("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
+        ("prec", c_int), ("init_seed", c_ulonglong), ("max_rows", c_int), ("keep_grad", c_int),
+    ]
+
+
+_lib = None
+
+
+def lib():
+    """Loads libff.so (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(LIB_PATH):
+            raise RuntimeError(
+                "libff.so is not built; run `python -c 'import __graft_entry__ as g; g.build()'`")
+        L = ctypes.CDLL(LIB_PATH)
+        L.ff_status_string.restype = ctypes.c_char_p
+        L.ff_status_string.argtypes = [c_int]
+        L.ff_row_stride.restype = c_int
+        L.ff_row_stride.argtypes = [c_int]
+        sig = {
+            "ff_layer_create": [POINTER(LayerConfig), c_void_p, POINTER(c_void_p)],
+            "ff_layer_destroy": [c_void_p],
+            "ff_overlay_label": [c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p, c_int, c_void_p],
+            "ff_layer_forward": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p,
+                                 c_void_p],
+            "ff_layer_train_step": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p,
+                                    c_void_p, c_void_p],
+            "ff_predict": [c_void_p, c_int, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
+            "ff_layer_get_state": [c_void_p] + [c_void_p] * 6 + [POINTER(c_longlong)],
+            "ff_layer_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
+            "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
+            "ff_layer_check": [c_void_p],
+            "ff_net_create": [c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
+            "ff_net_destroy": [c_void_p],
+            "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
+            "ff_net_sync": [c_void_p, c_void_p],
+        }
+        for name, args in sig.items():
+            f = getattr(L, name)
+            f.restype = c_int
+            f.argtypes = args
+        _lib = L
+    return _lib
+
+
+def _check(status: int, what: str):
+    if status != 0:
+        raise FFError(status, what)
+
+
+def row_stride(features: int) -> int:
+    return lib().ff_row_stride(int(features))
+
+
+def _stream(stream) -> int:
+    if stream is None:
+        return torch.cuda.current_stream().cuda_stream
+    if isinstance(stream, torch.cuda.Stream):
+        return stream.cuda_stream
+    return int(stream)
+
+
+def _ptr(t, dtype=None, what="tensor", need_cuda=True):
+    if t is None:
+        return None
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{what} must be a torch.Tensor")
+    if need_cuda and not t.is_cuda:
+        raise ValueError(f"{what} must be a CUDA tensor")
+    if dtype is not None and t.dtype != dtype:
+        raise TypeError(f"{what} must be {dtype}, got {t.dtype}")
+    if not t.is_contiguous():
+        raise ValueError(f"{what} must be contiguous")
+    return t.data_ptr()
+
+
+def act_dtype(prec: str):
+    return torch.bfloat16 if prec == "bf16" else torch.float32
+
+
+class Layer:
+    """One FF layer (``ff_layer``): parameters, Adam moments and workspace on the GPU."""
+
+    def __init__(self, in_features: int, out_features: int, prec: str = "bf16", theta: float = 2.0,
+                 lr: float = 0.03, beta1: float = 0.9, beta2: float = 0.999, eps: float = 1e-8,
+                 has_bias: bool = True, init_seed: int = 0, max_rows: int = 0, keep_grad: bool = False,
+                 stream=None):
+        if prec not in ("bf16", "fp32"):
+            raise ValueError("prec must be 'bf16' or 'fp32'")
+        self.in_features, self.out_features, self.prec = int(in_features), int(out_features), prec
+        self.dtype = act_dtype(prec)
+        self.cfg = LayerConfig(self.in_features, self.out_features, int(bool(has_bias)), theta, lr, beta1, beta2,
+                               eps, FF_BF16 if prec == "bf16" else FF_FP32, int(init_seed), int(max_rows),
+                               int(bool(keep_grad)))
+        h = c_void_p()
+        _check(lib().ff_layer_create(ctypes.byref(self.cfg), c_void_p(_stream(stream)), ctypes.byref(h)),
+               "ff_layer_create")
+        self._h = h
+
+    @property
+    def handle(self):
+        return self._h
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(lib().ff_layer_destroy(self._h), "ff_layer_destroy")
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    # buffers in the layer's activation format
+    def new_activation(self, rows: int, features: int | None = None, device="cuda"):
+        f = self.out_features if features is None else features
+        return torch.zeros(rows, row_stride(f), dtype=self.dtype, device=device)
+
+    def _x_args(self, x, labels, row_scale):
+        if labels is not None:
+            xp = _ptr(x, torch.float32, "x (raw input)")
+            if x.shape[-1] != self.in_features:
+                raise ValueError("raw x must have in_features columns")
+            return xp, _ptr(labels, torch.int32, "labels"), None
+        xp = _ptr(x, self.dtype, "x (activation)")
+        if x.shape[-1] != row_stride(self.in_features):
+            raise ValueError("activation x must have ff_row_stride(in_features) columns")
+        return xp, None, _ptr(row_scale, torch.float32, "row_scale")
+
+    def train_step(self, x, labels=None, row_scale=None, B=None, h_out=None, next_scale=None, goodness=None,
+                   loss=None, stream=None):
+        """ff_layer_train_step: rows 0..B-1 positive, B..2B-1 negative."""
+        if B is None:
+            B = x.shape[0] // 2
+        xp, lp, sp = self._x_args(x, labels, row_scale)
+        _check(lib().ff_layer_train_step(
+            self._h, xp, lp, sp, int(B), _ptr(h_out, self.dtype, "h_out"),
+            _ptr(next_scale, torch.float32, "next_scale"), _ptr(goodness, torch.float32, "goodness"),
+            _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))), "ff_layer_train_step")
+
+    def forward(self, x, labels=None, row_scale=None, rows=None, h_out=None, next_scale=None, goodness=None,
+                stream=None):
+        """ff_layer_forward (L_i(x)) without an update."""
+        if rows is None:
+            rows = x.shape[0]
+        xp, lp, sp = self._x_args(x, labels, row_scale)
+        _check(lib().ff_layer_forward(
+            self._h, xp, lp, sp, int(rows), _ptr(h_out, self.dtype, "h_out"),
+            _ptr(next_scale, torch.float32, "next_scale"), _ptr(goodness, torch.float32, "goodness"),
+            c_void_p(_stream(stream))), "ff_layer_forward")
+
+    def get_state(self):
+        N, K = self.out_features, self.in_features
+        W = np.empty((N, K), np.float32); mW = np.empty_like(W); vW = np.empty_like(W)
+        b = np.empty(N, np.float32); mb = np.empty_like(b); vb = np.empty_like(b)
+        step = c_longlong()
+        _check(lib().ff_layer_get_state(self._h, W.ctypes.data, b.ctypes.data, mW.ctypes.data, vW.ctypes.data,
+                                        mb.ctypes.data, vb.ctypes.data, ctypes.byref(step)), "ff_layer_get_state")
+        return dict(W=W, b=b, mW=mW, vW=vW, mb=mb, vb=vb, t=step.value)
+
+    def set_state(self, W=None, b=None, mW=None, vW=None, mb=None, vb=None, t=0):
+        N, K = self.out_features, self.in_features
+
+        def host(a, shape):
+            if a is None:
+                return None, None
+            a = np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+            if a.shape != shape:
+                raise ValueError(f"expected shape {shape}, got {a.shape}")
+            return a, a.ctypes.data
+        keep = [host(W, (N, K)), host(b, (N,)), host(mW, (N, K)), host(vW, (N, K)), host(mb, (N,)), host(vb, (N,))]
+        _check(lib().ff_layer_set_state(self._h, *[k[1] for k in keep], int(t)), "ff_layer_set_state")
+
+    def get_grad(self):
+        N, K = self.out_features, self.in_features
+        dW = np.empty((N, K), np.float32); db = np.empty(N, np.float32)
+        _check(lib().ff_layer_get_grad(self._h, dW.ctypes.data, db.ctypes.data), "ff_layer_get_grad")
+        return dW, db
+
+    def check(self):
+        _check(lib().ff_layer_check(self._h), "ff_layer_check")
+
+
+def overlay_label(x, labels, prec="bf16", out=None, row_scale=None, stream=None):
+    """ff_overlay_label: returns the overlaid activation buffer."""
+    rows, F = x.shape
+    if out is None:
+        out = torch.empty(rows, row_stride(F), dtype=act_dtype(prec), device=x.device)
+    _check(lib().ff_overlay_label(_ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"), rows, F,
+                                  _ptr(out, act_dtype(prec), "out"), _ptr(row_scale, torch.float32, "row_scale"),
+                                  FF_BF16 if prec == "bf16" else FF_FP32, c_void_p(_stream(stream))),
+           "ff_overlay_label")
+    return out
+
+
+def predict(layers, x, pred=None, goodness=None, stream=None):
+    """ff_predict: goodness prediction over the 10 label overlays.  Returns (pred, goodness)."""
+    n = x.shape[0]
+    if pred is None:
+        pred = torch.empty(n, dtype=torch.int32, device=x.device)
+    arr = (c_void_p * len(layers))(*[l.handle.value for l in layers])
+    _check(lib().ff_predict(arr, len(layers), _ptr(x, torch.float32, "x"), n, _ptr(pred, torch.int32, "pred"),
+                            _ptr(goodness, torch.float32, "goodness"), c_void_p(_stream(stream))), "ff_predict")
+    return pred, goodness
+
+
+class Net:
+    """ff_net: the layers of a net trained concurrently, one CUDA stream per layer."""
+
+    def __init__(self, layers, max_B: int, depth: int = 2):
+        self.layers = list(layers)
+        arr = (c_void_p * len(self.layers))(*[l.handle.value for l in self.layers])
+        h = c_void_p()
+        _check(lib().ff_net_create(arr, len(self.layers), int(max_B), int(depth), ctypes.byref(h)), "ff_net_create")
+        self._h = h
+
+    def train_step(self, x, labels, B=None, loss=None, stream=None):
+        if B is None:
+            B = x.shape[0] // 2
+        _check(lib().ff_net_train_step(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
+                                       int(B), _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
+               "ff_net_train_step")
+
+    def sync(self, stream=None):
+        _check(lib().ff_net_sync(self._h, c_void_p(_stream(stream))), "ff_net_sync")
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            lib().ff_net_destroy(self._h)
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass

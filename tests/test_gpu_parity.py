@@ -1,0 +1,395 @@
+"""GPU parity: the CUDA path through the C ABI against the CPU oracle on the
+same seeded inputs.
+
+Tolerances.  fp32 mode: 1e-4 relative on goodness, loss and weights after
+each step.  bf16-operand mode: 2e-2 relative per step; the oracle is run with
+the bf16 rounding of the stored operands emulated, which lets most checks use
+tighter bounds (they are stated per assertion).  Adam's first steps move a
+weight by about lr*sign(g): where a gradient element is within its own
+rounding bound of zero or of eps, the update is steep in g, so weights are
+held to 1e-4 plus the spread of the oracle's Adam over that bound (derived in
+tests/gpu_common.py), and the Adam kernel itself is checked tightly against
+the GPU's own gradient.
+"""
+
+import numpy as np
+import pytest
+
+from oracle import ff_oracle as fo
+from paper_2404_08573_gb300 import synth
+from tests.gpu_common import (assert_adam_state, assert_close, grad_uncertainty, lib_ready, oracle_state, pair_inputs,
+                              rel_norm, torch_cuda)
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module")
+def env():
+    torch = torch_cuda()
+    ff = lib_ready()
+    return torch, ff
+
+
+def _rand_layer_state(N, K, seed, bias_scale=0.05):
+    rng = np.random.default_rng(seed)
+    W = synth.he_uniform(seed, N, K)
+    b = (rng.standard_normal(N) * bias_scale).astype(np.float32)
+    return W, b
+
+
+# ------------------------------------------------------------------ init
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_created_weights_equal_the_generator(env, prec):
+    torch, ff = env
+    layer = ff.Layer(784, 500, prec=prec, init_seed=5)
+    st = layer.get_state()
+    assert np.array_equal(st["W"], synth.he_uniform(5, 500, 784))
+    for k in ("b", "mW", "vW", "mb", "vb"):
+        assert not st[k].any()
+    assert st["t"] == 0
+
+
+# --------------------------------------------------------------- overlay
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_overlay_kernel(env, prec):
+    torch, ff = env
+    rows, F = 37, 794
+    x = synth.mnist_like(rows, seed=3, features=F)
+    x[:, :10] = 0.5
+    lab = synth.labels(rows, seed=3)
+    lab[0], lab[1] = 0, 9
+    xg = torch.from_numpy(x).cuda()
+    s = torch.empty(rows, device="cuda")
+    out = ff.overlay_label(xg, torch.from_numpy(lab).cuda(), prec=prec, row_scale=s)
+    torch.cuda.synchronize()
+    ref = fo.overlay_label(x, lab)
+    got = out.float().cpu().numpy()
+    assert got.shape == (rows, ff.row_stride(F))
+    exp = ref if prec == "fp32" else fo.bf16_round(ref)
+    assert np.array_equal(got[:, :F], exp.astype(np.float32))
+    assert not got[:, F:].any()
+    assert_close(s.cpu().numpy(), 1.0 / fo.row_norm(ref), 1e-6, 0, "row scale")
+
+
+# --------------------------------------------------------------- forward
+FWD_CASES = [
+    ("fp32", 300, 784, 600), ("bf16", 300, 784, 600), ("bf16", 1, 11, 5), ("fp32", 1, 11, 5),
+    ("bf16", 130, 2003, 777), ("fp32", 130, 2003, 777), ("bf16", 257, 64, 256), ("bf16", 2048, 2000, 2000),
+]
+
+
+@pytest.mark.parametrize("prec,M,K,N", FWD_CASES)
+def test_forward_hidden_layer(env, prec, M, K, N):
+    torch, ff = env
+    rng = np.random.default_rng(M + K + N)
+    xin = np.maximum(rng.standard_normal((M, K)), 0.0).astype(np.float32)
+    xin[M // 2] = 0.0                                   # a dead row: s = 1/1e-12 path, g = ReLU(b)^2
+    if prec == "bf16":
+        xin = fo.bf16_round(xin).astype(np.float32)     # the stored activity is bf16
+    W, b = _rand_layer_state(N, K, seed=K)
+    layer = ff.Layer(K, N, prec=prec, init_seed=1)
+    layer.set_state(W=W, b=b)
+    xa = layer.new_activation(M, K)
+    xa[:, :K] = torch.from_numpy(xin).to(xa.dtype)
+    h = layer.new_activation(M)
+    g = torch.empty(M, device="cuda")
+    sn = torch.empty(M, device="cuda")
+    layer.forward(xa, h_out=h, goodness=g, next_scale=sn)
+    torch.cuda.synchronize()
+    layer.check()
+    ref = fo.layer_forward_full(fo.LayerState(W, b), xin, emulate_bf16=(prec == "bf16"))
+    tol = 1e-5 if prec == "fp32" else 1e-3
+    assert_close(g.cpu().numpy(), ref["g"], tol, 1e-6, "goodness")
+    hg = h.float().cpu().numpy()
+    assert not hg[:, N:].any()
+    hrt = 1e-5 if prec == "fp32" else 2.0 ** -8 + 1e-3
+    assert_close(hg[:, :N], ref["H"], hrt, 1e-5, "activity")
+    assert_close(sn.cpu().numpy(), 1.0 / np.maximum(np.sqrt(ref["g"]), 1e-12), tol, 0, "next scale")
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_forward_first_layer_with_labels(env, prec):
+    torch, ff = env
+    B = 70
+    x2, l2 = pair_inputs(B, seed=4)
+    W, b = _rand_layer_state(500, 784, seed=9)
+    layer = ff.Layer(784, 500, prec=prec)
+    layer.set_state(W=W, b=b)
+    g = torch.empty(2 * B, device="cuda")
+    layer.forward(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), goodness=g)
+    torch.cuda.synchronize()
+    ref = fo.layer_forward_full(fo.LayerState(W, b), fo.overlay_label(x2, l2), emulate_bf16=(prec == "bf16"))
+    assert_close(g.cpu().numpy(), ref["g"], 1e-5 if prec == "fp32" else 1e-3, 1e-6, "goodness")
+    plain = fo.layer_forward_full(fo.LayerState(W, b), fo.overlay_label(x2, l2))
+    assert_close(g.cpu().numpy(), plain["g"], 1e-4 if prec == "fp32" else 2e-2, 1e-4, "goodness vs fp64")
+
+
+# ------------------------------------------------------------ train step
+STEP_CASES = [
+    ("fp32", 64, 784, 500, True), ("bf16", 64, 784, 500, True), ("bf16", 3, 11, 5, True), ("fp32", 1, 11, 5, True),
+    ("bf16", 1024, 784, 2000, True), ("bf16", 1024, 2000, 2000, False), ("fp32", 150, 2000, 300, False),
+    ("bf16", 608, 2000, 2000, False),
+]
+
+
+@pytest.mark.parametrize("prec,B,K,N,first", STEP_CASES)
+def test_train_step(env, prec, B, K, N, first):
+    torch, ff = env
+    M = 2 * B
+    theta, lr = 2.0, 0.03
+    W, b = _rand_layer_state(N, K, seed=B + K)
+    layer = ff.Layer(K, N, prec=prec, theta=theta, lr=lr, keep_grad=True)
+    layer.set_state(W=W, b=b)
+    if first:
+        x2, l2 = pair_inputs(B, seed=B, features=K) if K >= 784 else pair_inputs(B, seed=B, features=K)
+        xin = fo.overlay_label(x2, l2)
+        xg, lg = torch.from_numpy(x2).cuda(), torch.from_numpy(l2).cuda()
+    else:
+        rng = np.random.default_rng(B)
+        xin = np.maximum(rng.standard_normal((M, K)), 0).astype(np.float32)
+        if prec == "bf16":
+            xin = fo.bf16_round(xin).astype(np.float32)
+        xg = layer.new_activation(M, K)
+        xg[:, :K] = torch.from_numpy(xin).to(xg.dtype)
+        lg = None
+    g = torch.empty(M, device="cuda")
+    loss = torch.empty(1, device="cuda")
+    h = layer.new_activation(M)
+    sn = torch.empty(M, device="cuda")
+    layer.train_step(xg, labels=lg, B=B, h_out=h, next_scale=sn, goodness=g, loss=loss)
+    torch.cuda.synchronize()
+    layer.check()
+    emul = prec == "bf16"
+    st = fo.LayerState(W, b)
+    ref = fo.layer_train_step(st, xin, B, theta, fo.AdamHyper(lr=lr), emulate_bf16=emul)
+    gtol = 1e-5 if not emul else 1e-3
+    assert_close(g.cpu().numpy(), ref["g"], gtol, 1e-6, "goodness")
+    assert abs(loss.item() - ref["loss"]) <= (1e-5 if not emul else 1e-3) * abs(ref["loss"]) + 1e-7
+    dW, db = layer.get_grad()
+    assert rel_norm(dW, ref["dW"]) < (1e-5 if not emul else 1e-3), rel_norm(dW, ref["dW"])
+    assert rel_norm(db, ref["db"]) < (1e-5 if not emul else 1e-3), rel_norm(db, ref["db"])
+    s2 = layer.get_state()
+    assert s2["t"] == 1
+    dgW, dgb = grad_uncertainty(ref, W, b, xin, B, emul, tensor_cores=emul)
+    assert np.all(np.abs(dW - ref["dW"]) <= dgW + 1e-6 * np.abs(ref["dW"])), "dW outside its rounding bound"
+    assert np.all(np.abs(db - ref["db"]) <= dgb + 1e-6 * np.abs(ref["db"])), "db outside its rounding bound"
+    hp = fo.AdamHyper(lr=lr)
+    z = np.zeros_like(W, dtype=np.float64)
+    zb = np.zeros_like(b, dtype=np.float64)
+    # the Adam kernel applied to the GPU's own gradient, with the float32 hyper-parameters: tight
+    hp32 = fo.AdamHyper(*[float(np.float32(v)) for v in (lr, 0.9, 0.999, 1e-8)])
+    assert_adam_state(s2["W"], s2["mW"], s2["vW"], W, z, z, 1, dW.astype(np.float64), 0 * z, hp32, "W (own grad)",
+                      rtol=1e-5, w_floor=0.05, max_band_frac=0.0)
+    # against the oracle's gradient: 1e-4 plus Adam's spread over the rounding bound
+    assert_adam_state(s2["W"], s2["mW"], s2["vW"], W, z, z, 1, ref["dW"], dgW, hp, "W")
+    assert_adam_state(s2["b"], s2["mb"], s2["vb"], b, zb, zb, 1, ref["db"], dgb, hp, "b")
+    assert rel_norm(s2["W"], st.W) <= (1e-4 if not emul else 2e-2)
+    # the activity handed to the next layer and its scale
+    assert_close(h.float().cpu().numpy()[:, :N], ref["H"], 1e-5 if not emul else 2.0 ** -8 + 1e-3, 1e-5, "activity")
+    assert_close(sn.cpu().numpy(), 1.0 / np.maximum(np.sqrt(ref["g"]), 1e-12), gtol, 0, "next scale")
+    # against the plain fp64 definition, at the benchmark spec's tolerances
+    plain = fo.layer_train_step(fo.LayerState(W, b), xin, B, theta, fo.AdamHyper(lr=lr))
+    assert_close(g.cpu().numpy(), plain["g"], 1e-4 if not emul else 2e-2, 1e-4, "goodness vs fp64")
+    assert abs(loss.item() - plain["loss"]) <= (1e-4 if not emul else 2e-2) * abs(plain["loss"])
+
+
+def test_config0_sixteen_steps_fp32(env):
+    """784->500->500, fp32, 16 steps of B=64: each step is compared with the
+    oracle started from the GPU's state before that step."""
+    torch, ff = env
+    theta, lr, B = 2.0, 0.03, 64
+    layers = [ff.Layer(784, 500, prec="fp32", theta=theta, lr=lr, init_seed=0, keep_grad=True),
+              ff.Layer(500, 500, prec="fp32", theta=theta, lr=lr, init_seed=1, keep_grad=True)]
+    h = layers[0].new_activation(2 * B)
+    s1 = torch.empty(2 * B, device="cuda")
+    loss = torch.empty(2, device="cuda")
+    g = torch.empty(2, 2 * B, device="cuda")
+    for step in range(16):
+        x = synth.mnist_like(B, seed=0, start_row=step * B)
+        y = synth.labels(B, seed=0, start=step * B)
+        yn = synth.negative_labels(y, seed=0, start=step * B)
+        x2, l2 = synth.pair_batch(x, y, yn)
+        pre = [oracle_state(l.get_state()) for l in layers]
+        layers[0].train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=B, h_out=h,
+                             next_scale=s1, goodness=g[0], loss=loss[0:1])
+        layers[1].train_step(h, row_scale=s1, B=B, goodness=g[1], loss=loss[1:2])
+        torch.cuda.synchronize()
+        refs = fo.net_train_step([p.copy() for p in pre], x2, l2, B, theta, fo.AdamHyper(lr=lr))
+        xins = [fo.overlay_label(x2, l2), refs[0]["H"]]
+        for k in range(2):
+            assert_close(g[k].cpu().numpy(), refs[k]["g"], 1e-4, 1e-6, f"step {step} layer {k} goodness")
+            assert abs(loss[k].item() - refs[k]["loss"]) <= 1e-4 * abs(refs[k]["loss"])
+            st = layers[k].get_state()
+            dgW, dgb = grad_uncertainty(refs[k], pre[k].W, pre[k].b, xins[k], B, False, tensor_cores=False)
+            hp = fo.AdamHyper(lr=lr)
+            p = pre[k]
+            assert_adam_state(st["W"], st["mW"], st["vW"], p.W, p.mW, p.vW, step + 1, refs[k]["dW"], dgW, hp,
+                              f"step {step} layer {k} W")
+            assert_adam_state(st["b"], st["mb"], st["vb"], p.b, p.mb, p.vb, step + 1, refs[k]["db"], dgb, hp,
+                              f"step {step} layer {k} b")
+            assert st["t"] == step + 1
+
+
+# ---------------------------------------------------------------- predict
+@pytest.mark.parametrize("prec,dims,n", [("fp32", (784, 256, 256, 128), 300), ("bf16", (784, 256, 256, 128), 300),
+                                         ("bf16", (784, 96), 40), ("bf16", (784, 200, 128), 9000)])
+def test_predict(env, prec, dims, n):
+    torch, ff = env
+    layers, states = [], []
+    for i in range(len(dims) - 1):
+        W, b = _rand_layer_state(dims[i + 1], dims[i], seed=30 + i, bias_scale=0.02)
+        l = ff.Layer(dims[i], dims[i + 1], prec=prec)
+        l.set_state(W=W, b=b)
+        layers.append(l)
+        states.append(fo.LayerState(W, b))
+    x = synth.mnist_like(n, seed=31)
+    G = torch.empty(n, 10, device="cuda")
+    pred, _ = ff.predict(layers, torch.from_numpy(x).cuda(), goodness=G)
+    torch.cuda.synchronize()
+    layers[0].check()
+    emul = prec == "bf16"
+    rp, rG = fo.predict(states, x, emulate_bf16=emul)
+    assert_close(G.cpu().numpy(), rG, 1e-4 if not emul else 2e-3, 1e-6, "predict goodness")
+    p = pred.cpu().numpy()
+    agree = np.mean(p == rp)
+    assert agree >= 0.995, agree
+    for i in np.nonzero(p != rp)[0]:   # disagreements only at near ties
+        gap = abs(rG[i, p[i]] - rG[i, rp[i]])
+        assert gap <= (1e-4 if not emul else 1e-2) * abs(rG[i, rp[i]]), (i, gap)
+    plain_p, plain_G = fo.predict(states, x)
+    assert_close(G.cpu().numpy(), plain_G, 1e-4 if not emul else 2e-2, 1e-4, "predict goodness vs fp64")
+
+
+# ----------------------------------------------- multi-stream net == sequential
+def test_net_on_streams_is_bitwise_sequential(env):
+    torch, ff = env
+    dims, B, steps = (784, 256, 256, 192), 128, 6
+    mk = lambda: [ff.Layer(dims[i], dims[i + 1], prec="bf16", init_seed=40 + i) for i in range(3)]
+    par, seq = mk(), mk()
+    net = ff.Net(par, max_B=B, depth=2)
+    hs = [seq[0].new_activation(2 * B), seq[1].new_activation(2 * B)]
+    ss = [torch.empty(2 * B, device="cuda") for _ in range(2)]
+    lp = torch.empty(steps, 3, device="cuda")
+    ls = torch.empty(steps, 3, device="cuda")
+    xs = []
+    for t in range(steps):
+        x2, l2 = pair_inputs(B, seed=100 + t)
+        xs.append((torch.from_numpy(x2).cuda(), torch.from_numpy(l2).cuda()))
+    for t in range(steps):
+        net.train_step(xs[t][0], xs[t][1], B=B, loss=lp[t])
+    net.sync()
+    for t in range(steps):
+        seq[0].train_step(xs[t][0], labels=xs[t][1], B=B, h_out=hs[0], next_scale=ss[0], loss=ls[t, 0:1])
+        seq[1].train_step(hs[0], row_scale=ss[0], B=B, h_out=hs[1], next_scale=ss[1], loss=ls[t, 1:2])
+        seq[2].train_step(hs[1], row_scale=ss[1], B=B, loss=ls[t, 2:3])
+    torch.cuda.synchronize()
+    assert torch.equal(lp, ls)
+    for a, b in zip(par, seq):
+        sa, sb = a.get_state(), b.get_state()
+        for k in ("W", "b", "mW", "vW"):
+            assert np.array_equal(sa[k], sb[k]), k
+
+
+def test_repeat_runs_are_bitwise_equal(env):
+    torch, ff = env
+    B = 256
+    x2, l2 = pair_inputs(B, seed=77)
+    outs = []
+    for _ in range(2):
+        l = ff.Layer(784, 2000, prec="bf16", init_seed=3)
+        loss = torch.empty(3, device="cuda")
+        for t in range(3):
+            l.train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=B, loss=loss[t:t + 1])
+        torch.cuda.synchronize()
+        outs.append((loss.cpu().numpy(), l.get_state()["W"]))
+    assert np.array_equal(outs[0][0], outs[1][0]) and np.array_equal(outs[0][1], outs[1][1])
+
+
+# ---------------------------------------------------------------- edges
+def test_edge_cases(env):
+    torch, ff = env
+    l = ff.Layer(784, 300, prec="bf16", init_seed=2)
+    before = l.get_state()
+    x2, l2 = pair_inputs(4, seed=1)
+    l.train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=0)  # empty batch: no-op
+    after = l.get_state()
+    assert after["t"] == 0 and np.array_equal(before["W"], after["W"])
+    # misaligned activation pointer is rejected before anything runs
+    buf = torch.zeros(2 * 4 * 784 + 8, dtype=torch.bfloat16, device="cuda")
+    with pytest.raises(ff.FFError) as ei:
+        l.forward(buf[1:1 + 8 * 784].view(8, 784), goodness=torch.empty(8, device="cuda"))
+    assert ei.value.status == 1
+    # a non-finite input is latched and reported by check()
+    bad = x2.copy()
+    bad[0, 20] = np.nan
+    l.train_step(torch.from_numpy(bad).cuda(), labels=torch.from_numpy(l2).cuda(), B=4)
+    with pytest.raises(ff.FFError) as ei:
+        l.check()
+    assert ei.value.status == 5
+    l.check()  # cleared
+    # a batch larger than the workspace grows it
+    big = ff.Layer(784, 64, prec="bf16", max_rows=16)
+    x3, l3 = pair_inputs(300, seed=2)
+    loss = torch.empty(1, device="cuda")
+    big.train_step(torch.from_numpy(x3).cuda(), labels=torch.from_numpy(l3).cuda(), B=300, loss=loss)
+    torch.cuda.synchronize()
+    assert np.isfinite(loss.item())
+
+
+def test_state_round_trip_resumes_bitwise(env):
+    """8 steps, save, load into a fresh layer, 8 more == 16 steps."""
+    torch, ff = env
+    B = 64
+    batches = [pair_inputs(B, seed=200 + t) for t in range(16)]
+    a = ff.Layer(784, 500, prec="bf16", init_seed=9)
+    for t in range(16):
+        a.train_step(torch.from_numpy(batches[t][0]).cuda(), labels=torch.from_numpy(batches[t][1]).cuda(), B=B)
+    b = ff.Layer(784, 500, prec="bf16", init_seed=9)
+    for t in range(8):
+        b.train_step(torch.from_numpy(batches[t][0]).cuda(), labels=torch.from_numpy(batches[t][1]).cuda(), B=B)
+    saved = b.get_state()
+    c = ff.Layer(784, 500, prec="bf16", init_seed=123)
+    c.set_state(**saved)
+    for t in range(8, 16):
+        c.train_step(torch.from_numpy(batches[t][0]).cuda(), labels=torch.from_numpy(batches[t][1]).cuda(), B=B)
+    sa, sc = a.get_state(), c.get_state()
+    for k in ("W", "b", "mW", "vW", "mb", "vb"):
+        assert np.array_equal(sa[k], sc[k]), k
+    assert sa["t"] == sc["t"] == 16
+
+
+def test_net_steps_captured_in_a_cuda_graph_match_eager(env):
+    """A synced run of ff_net steps replayed from a CUDA graph gives the same
+    bits as the same steps called eagerly."""
+    torch, ff = env
+    dims, B = (784, 256, 128), 64
+    mk = lambda: [ff.Layer(dims[i], dims[i + 1], prec="bf16", init_seed=60 + i, max_rows=2 * B) for i in range(2)]
+    ga, gb = mk(), mk()
+    na, nb = ff.Net(ga, max_B=B, depth=2), ff.Net(gb, max_B=B, depth=2)
+    xs = [pair_inputs(B, seed=300 + t) for t in range(3)]
+    X = torch.from_numpy(np.concatenate([x for x, _ in xs])).cuda()
+    L = torch.from_numpy(np.concatenate([l for _, l in xs])).cuda()
+    la = torch.zeros(3, 2, device="cuda")
+    lb = torch.zeros(3, 2, device="cuda")
+    s = torch.cuda.Stream()
+
+    def run(net, loss):
+        for t in range(3):
+            net.train_step(X[2 * B * t:2 * B * (t + 1)], L[2 * B * t:2 * B * (t + 1)], B=B, loss=loss[t], stream=s)
+        net.sync(s)
+
+    g = torch.cuda.CUDAGraph()
+    with torch.cuda.graph(g, stream=s):
+        run(na, la)
+    for _ in range(2):
+        g.replay()
+    with torch.cuda.stream(s):
+        for _ in range(2):
+            run(nb, lb)
+    torch.cuda.synchronize()
+    assert torch.equal(la, lb)
+    for a, b in zip(ga, gb):
+        sa, sb = a.get_state(), b.get_state()
+        assert sa["t"] == sb["t"] == 6
+        for k in ("W", "b", "mW", "vW"):
+            assert np.array_equal(sa[k], sb[k]), k
