@@ -193,6 +193,36 @@ FF_API ff_status ff_net_train_step(ff_net* net, const float* x, const int* label
 FF_API ff_status ff_net_sync(ff_net* net, void* stream);
 
 /* ---------------------------------------------------------------------------
+ * Allocation-free forward pass.  The paper has no counterpart: this is a
+ * service for callers that cannot call cudaMalloc -- code embedded in a host
+ * application that owns all device memory through its own pool, or that must
+ * keep the device's memory footprint fixed after start-up -- and therefore
+ * cannot create an ff_layer (which allocates its parameters and workspace).
+ *
+ * Computes what ff_layer_forward computes in FF_BF16 mode, from caller
+ * buffers only: x [rows, ff_row_stride(in_features)] bf16 (16-byte aligned),
+ * row_scale [rows] (required), W_bf16 [out_features, ff_row_stride(in_features)]
+ * bf16, bias [out_features] fp32 or NULL, h_out [rows, ff_row_stride(out_features)]
+ * bf16, goodness and next_scale [rows] or NULL, device_status [1] int or NULL
+ * (set to 0 by the call, then OR-ed with 1 if a kernel wait timed out, 2 if a
+ * goodness was not finite).  It allocates nothing: the per-tile goodness
+ * partials live in a fixed 4 MiB array in the library's device image, which
+ * every GPU that loads libff holds until the process exits.
+ *   - Limit: rows * ceil(out_features / 256) <= 1048512; larger requests
+ *     return FF_ERR_INVALID_ARG before anything is enqueued.
+ *   - The first call on a device looks up that array's device address (once
+ *     per device, with that device current); make that first call before any
+ *     stream capture.
+ *   - Every call shares the array and it keeps the last call's contents:
+ *     calls whose work overlaps on the GPU (other streams, other threads)
+ *     race; order them on one stream.
+ *   - Needs an sm_100-family GPU (FF_ERR_UNSUPPORTED otherwise). */
+FF_API ff_status ff_forward_noalloc(const void* x, const float* row_scale, const void* W_bf16,
+                                    const float* bias, int rows, int in_features, int out_features,
+                                    void* h_out, float* goodness, float* next_scale,
+                                    int* device_status, void* stream);
+
+/* ---------------------------------------------------------------------------
  * Instrumentation (not part of the method).
  * Every kernel launch libff makes is counted; ff_kernel_launches returns the
  * process-wide total so far.  ff_profile_enable(1) clears earlier records and

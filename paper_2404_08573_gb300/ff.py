@@ -71,6 +71,8 @@ def lib():
             "ff_net_destroy": [c_void_p],
             "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_sync": [c_void_p, c_void_p],
+            "ff_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
+                                   c_void_p, c_void_p, c_void_p],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -272,3 +274,16 @@ class Net:
             self.close()
         except Exception:
             pass
+
+
+def forward_noalloc(x, row_scale, W_bf16, in_features, out_features, h_out, bias=None, goodness=None,
+                    next_scale=None, device_status=None, stream=None):
+    """ff_forward_noalloc: the bf16 forward pass from caller buffers only (no
+    device allocation inside the library); see include/ff.h."""
+    rows = x.shape[0]
+    _check(lib().ff_forward_noalloc(
+        _ptr(x, torch.bfloat16, "x"), _ptr(row_scale, torch.float32, "row_scale"),
+        _ptr(W_bf16, torch.bfloat16, "W_bf16"), _ptr(bias, torch.float32, "bias"), int(rows), int(in_features),
+        int(out_features), _ptr(h_out, torch.bfloat16, "h_out"), _ptr(goodness, torch.float32, "goodness"),
+        _ptr(next_scale, torch.float32, "next_scale"), _ptr(device_status, torch.int32, "device_status"),
+        c_void_p(_stream(stream))), "ff_forward_noalloc")
