@@ -57,7 +57,36 @@ __device__ __forceinline__ float block_sum_256(float v, float* red /*[8]*/) {
   return t;
 }
 
+// g = sum over t of gpart[t * M + i], t = 0..ntiles-1, in that order; the
+// loads are issued together (8 at a time) rather than one per dependent add.
+__device__ __forceinline__ float sum_partials(const float* __restrict__ gpart, int ntiles, int M, int i) {
+  float g = 0.f;
+  for (int t0 = 0; t0 < ntiles; t0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = (t0 + u < ntiles) ? __ldg(gpart + (size_t)(t0 + u) * M + i) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (t0 + u < ntiles) g += v[u];
+  }
+  return g;
+}
+
 // ------------------------------------------------------------------ overlay
+template <typename T>
+__device__ __forceinline__ void store4(T* p, float a, float b, float c, float d);
+template <>
+__device__ __forceinline__ void store4<float>(float* p, float a, float b, float c, float d) {
+  *reinterpret_cast<float4*>(p) = make_float4(a, b, c, d);
+}
+template <>
+__device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c, float d) {
+  __nv_bfloat162 p0 = __floats2bfloat162_rn(a, b), p1 = __floats2bfloat162_rn(c, d);
+  *reinterpret_cast<uint2*>(p) = make_uint2(*reinterpret_cast<uint32_t*>(&p0), *reinterpret_cast<uint32_t*>(&p1));
+}
+
+// One warp per row.  Rows whose length is a multiple of 4 (16-byte aligned
+// when x is) move as float4; others element by element.
 template <typename T>
 __global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ labels, int rows, int F,
                           T* __restrict__ out, int ldo, float* __restrict__ s_out, int mode) {
@@ -68,11 +97,28 @@ __global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ l
   T* orow = out + (size_t)row * ldo;
   const int lab = (mode == 0 && labels) ? labels[row] : -1;
   float ss = 0.f;
-  for (int f = lane; f < ldo; f += 32) {
-    float v = 0.f;
-    if (f < F) v = (f < 10) ? (f == lab ? 1.f : 0.f) : __ldg(xr + f);
-    orow[f] = from_f<T>(v);
-    ss = fmaf(v, v, ss);
+  const bool vec = (F & 3) == 0 && (reinterpret_cast<uintptr_t>(x) & 15u) == 0;
+  if (vec) {
+    for (int f = 4 * lane; f < ldo; f += 128) {
+      float v[4] = {0.f, 0.f, 0.f, 0.f};
+      if (f < F) {
+        const float4 q = __ldg(reinterpret_cast<const float4*>(xr + f));
+        v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        if (f + u < 10) v[u] = (f + u == lab) ? 1.f : 0.f;
+        ss = fmaf(v[u], v[u], ss);
+      }
+      store4<T>(orow + f, v[0], v[1], v[2], v[3]);
+    }
+  } else {
+    for (int f = lane; f < ldo; f += 32) {
+      float v = 0.f;
+      if (f < F) v = (f < 10) ? (f == lab ? 1.f : 0.f) : __ldg(xr + f);
+      orow[f] = from_f<T>(v);
+      ss = fmaf(v, v, ss);
+    }
   }
   ss = warp_sum(ss);
   if (lane == 0 && s_out) s_out[row] = inv_norm(ss + (mode == 1 ? 1.f : 0.f));
@@ -104,8 +150,7 @@ __device__ __forceinline__ float sigmoid_f(float t) {
 __global__ void __launch_bounds__(256) k_finalize(FinalizeArgs a) {
   const int i = blockIdx.x * 256 + threadIdx.x;
   if (i >= a.M) return;
-  float g = 0.f;
-  for (int t = 0; t < a.ntiles; ++t) g += a.gpart[(size_t)t * a.M + i];
+  const float g = sum_partials(a.gpart, a.ntiles, a.M, i);
   if (!isfinite(g)) atomicOr(a.err, DEVERR_NONFINITE);
   if (a.g_out) a.g_out[i] = g;
   if (a.s_next) a.s_next[i] = inv_norm(g);
@@ -187,8 +232,7 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
     const int i = r0 + threadIdx.x;
     float cc = 0.f, sc = 0.f, lv = 0.f;
     if (i < a.M) {
-      float g = 0.f;
-      for (int t = 0; t < a.ntiles; ++t) g += a.gpart[(size_t)t * a.M + i];
+      const float g = sum_partials(a.gpart, a.ntiles, a.M, i);
       const bool pos = i < a.B;
       const float tt = pos ? a.theta - g : g - a.theta;  // the pair member's margin error
       const float sg = sigmoid_f(tt);
@@ -311,10 +355,31 @@ __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
       }
     }
   } else {
-    const int j = (blockIdx.x - w_blocks) * 256 + threadIdx.x;
-    if (j >= a.N) return;
+    // 32 bias elements per block: warp w sums row blocks w, w+8, ... for the
+    // block's 32 columns (lane = column), then warp 0 adds the 8 warp sums in
+    // order -- a fixed reduction order, with the loads batched.
+    __shared__ float part[8][33];
+    const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+    const int j = (blockIdx.x - w_blocks) * 32 + lane;
+    float acc = 0.f;
+    if (j < a.N) {
+      for (int rb0 = w; rb0 < a.nrb; rb0 += 64) {
+        float v[8];
+#pragma unroll
+        for (int u = 0; u < 8; ++u) {
+          const int rb = rb0 + 8 * u;
+          v[u] = rb < a.nrb ? __ldg(a.dbpart + (size_t)rb * a.N + j) : 0.f;
+        }
+#pragma unroll
+        for (int u = 0; u < 8; ++u) acc += v[u];
+      }
+    }
+    part[w][lane] = acc;
+    __syncthreads();
+    if (w != 0 || j >= a.N) return;
     float db = 0.f;
-    for (int rb = 0; rb < a.nrb; ++rb) db += a.dbpart[(size_t)rb * a.N + j];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) db += part[u][lane];
     if (a.db_out) a.db_out[j] = db;
     if (a.has_bias) {
       float b = a.b[j], m = a.mb[j], v = a.vb[j];
@@ -468,7 +533,7 @@ cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, voi
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st) {
   const long long total = (long long)a.N * a.K;
   const int w_blocks = grid_for((a.K & 3) == 0 ? total / 4 : total, 256, 152 * 16);
-  const int b_blocks = cdiv(a.N, 256);
+  const int b_blocks = cdiv(a.N, 32);
   k_adam<<<w_blocks + b_blocks, 256, 0, st>>>(a, w_blocks);
   return cudaGetLastError();
 }

@@ -10,7 +10,8 @@
 //            (both operands are read MN-major straight from their row-major
 //            buffers: no transposed copies).
 //
-// One CTA computes one BM x BN output tile with three warp roles:
+// One CTA computes one BM x BN output tile with three warp roles (two CTAs fit
+// on one SM, so GEMMs of different layer streams overlap):
 //   warp 0      TMA producer: 128-byte-swizzled tiles into a STAGES-deep ring
 //   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
 //               N=BN, K=16) and commits each stage back to the producer
@@ -35,17 +36,18 @@ constexpr int NTHREADS = 192;
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
 
-template <int BN>
+template <int BN, int NSTAGE>
 struct TcCfg {
   static constexpr int A_BYTES = BM * BK * 2;
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
-  static constexpr int RAW_STAGES = (220 * 1024 - 2048) / STAGE;
-  static constexpr int STAGES = RAW_STAGES > 8 ? 8 : RAW_STAGES;
+  static constexpr int STAGES = NSTAGE;
   static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
   static constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
   static_assert(BN % 64 == 0 && BN <= 256, "BN must be a multiple of 64, at most 256");
-  static_assert(4 * 32 * BN * 4 <= STAGES * STAGE, "epilogue staging must fit in the operand ring");
+  static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+  static_assert(4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
+  static_assert(4 * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
   static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
 };
 
@@ -54,11 +56,11 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
   atomicOr(err, DEVERR_TIMEOUT);
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM>
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
-  using C = TcCfg<BN>;
+  using C = TcCfg<BN, NSTAGE>;
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -228,7 +230,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (__all_sync(0xffffffffu, ok && !*abort_flag)) {
       constexpr int ES = MODE == MODE_FWD ? 2 : 4;      // staged element size
       constexpr int CW = 128 / ES;                       // columns per 128-byte swizzle row
-      uint8_t* stage = smem + q * (32 * BN * ES);
+      // bf16: the warp's whole 32 x BN slab; fp32: two 32 x 32 slots, streamed
+      uint8_t* stage = smem + q * (MODE == MODE_FWD ? 32 * BN * 2 : 8192);
       const uint32_t sw = (uint32_t)(lane & 7);
       const bool staged = MODE == MODE_FWD || tma_store;
       const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
@@ -264,11 +267,24 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                 make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2], packed[4 * v + 3]);
           }
         } else if (staged) {
-          uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
+          // fp32: chunk c0 goes through slot (c0/32)&1; before refilling a slot
+          // the store issued from it two chunks ago must have read it
+          const int slot = (c0 / 32) & 1;
+          uint8_t* sbuf = stage + slot * 4096;
+          if (lane == 0 && c0 >= 64) ptx::bulk_wait_read1();
+          __syncwarp();
+          uint8_t* base = sbuf + lane * 128;
 #pragma unroll
           for (int v = 0; v < 8; ++v)
             *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
                 make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+          ptx::fence_async_smem();
+          __syncwarp();
+          const int r0 = m0 + q * 32;
+          if (lane == 0 && r0 < M && col0 < ep.ldo) {
+            ptx::tma_store_2d(&tmC, sbuf, col0, r0);
+          }
+          if (lane == 0) ptx::bulk_commit();
         } else if (gi < M) {
           float* out = reinterpret_cast<float*>(ep.out) + (size_t)gi * ep.ldo;
 #pragma unroll
@@ -290,7 +306,11 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         ptx::tmem_ld_wait();
       }
       if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)blockIdx.x * M + gi] = g;
-      if (staged) {
+      if (MODE != MODE_FWD && staged) {
+        if (lane == 0) ptx::bulk_wait_read0();
+        __syncwarp();
+      }
+      if (MODE == MODE_FWD) {
         ptx::fence_async_smem();
         __syncwarp();
         const int r0 = m0 + q * 32;
@@ -352,19 +372,19 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM>
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st) {
-  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM>;
+  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM, NSTAGE>;
   static cudaError_t attr =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN>::SMEM);
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN, NSTAGE>::SMEM);
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg = {};
   // tile rows padded to a whole number of clusters; padding CTAs load zeros,
   // share their B slice and write nothing
   cfg.gridDim = dim3(cdiv(N, BN), cdiv(cdiv(M, BM), CM) * CM, 1);
   cfg.blockDim = dim3(NTHREADS, 1, 1);
-  cfg.dynamicSmemBytes = TcCfg<BN>::SMEM;
+  cfg.dynamicSmemBytes = TcCfg<BN, NSTAGE>::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeClusterDimension;
@@ -378,7 +398,14 @@ cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtens
 
 constexpr int FWD_BN = 256;
 constexpr int WGRAD_BN = 256;
-constexpr int CLUSTER_M = 4;  // CTAs per cluster along M sharing one B tile
+// Measured on the 784-2000x4 train step with the layers on 4 streams: a
+// 2-deep ring (98 KB of shared memory, so two GEMM CTAs share an SM and one's
+// prologue/epilogue overlaps the other's mainloop) without clusters gave the
+// shortest epoch (9.8 ms vs 11.1 ms for 4 stages with 4-CTA multicast
+// clusters, which also constrain co-scheduling).  Cluster multicast of the B
+// tile stays available through CLUSTER_M.
+constexpr int CLUSTER_M = 1;  // CTAs per cluster along M sharing one B tile
+constexpr int NSTAGES = 2;    // operand ring depth
 
 }  // namespace
 
@@ -397,7 +424,7 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
   if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
-  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M>(ta, tb, tc, 1, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M, NSTAGES>(ta, tb, tc, 1, M, N, K, ep, err, st);
 }
 
 // fp32 C written through shared memory and TMA when its rows are 16-byte
@@ -414,7 +441,7 @@ cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M,
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M>(ta, tb, tc, tma, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M, NSTAGES>(ta, tb, tc, tma, M, N, K, ep, err, st);
 }
 
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K, float* Cm, int ldc,
@@ -427,7 +454,7 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M>(ta, tb, tc, tma, N, K, R, ep, err, st);
+  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M, NSTAGES>(ta, tb, tc, tma, N, K, R, ep, err, st);
 }
 
 }  // namespace ff
