@@ -218,7 +218,6 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   ga.s_next = next_scale;
   ga.dbpart = L->dbpart;
   ga.loss_part = L->loss_part;
-  ga.loss_out = loss ? loss : &L->ds->loss;
   ga.ds = L->ds;
   ga.beta1 = L->cfg.beta1;
   ga.beta2 = L->cfg.beta2;
@@ -260,6 +259,9 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   aa.beta2 = L->cfg.beta2;
   aa.eps = L->cfg.eps;
   aa.ds = L->ds;
+  aa.loss_part = L->loss_part;
+  aa.loss_out = loss ? loss : &L->ds->loss;
+  aa.B = B;
   FF_LAUNCH(K_ADAM, (double)L->N * L->K * (28.0 + (L->is_bf16 ? 2.0 : 0.0)) + (double)L->N * (aa.nrb * 4.0 + 28), st,
             launch_adam(aa, st),
             "Adam");
@@ -338,7 +340,7 @@ ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** o
   if (e == cudaSuccess) e = cudaMemsetAsync(L->dW, 0, nk * 4, st);
   if (e == cudaSuccess) e = cudaMemsetAsync(L->b, 0, (size_t)L->N * 4 * 4, st);
   if (e == cudaSuccess) {
-    static const ff_dev_state fresh = {0, 1.0, 1.0, 0.f, 0.f, 0, 0u, 0.f, 0};
+    static const ff_dev_state fresh = {0, 1.0, 1.0, 0.f, 0.f, 0, 0.f};
     e = cudaMemcpyAsync(L->ds, &fresh, sizeof(ff_dev_state), cudaMemcpyHostToDevice, st);
     if (e == cudaSuccess) e = cudaStreamSynchronize(st);  // `fresh` is pageable host memory
   }

@@ -196,26 +196,26 @@ struct Vec8<float> {
 };
 
 // Train-step epilogue of the forward GEMM, one block per 32 rows x 256
-// columns (block 32 x 8; thread (x, y) owns columns 8x..8x+7 of rows y,
-// y+8, y+16, y+24, whose activities it loads first so that the loads
-// overlap the per-row work):
-//   warp 0: g_i from the per-tile partials (fixed order) and dL/dg_i; in the
-//     blocks of column 0 also g, the next layer's scale 1/max(sqrt g, 1e-12)
-//     and the loss terms of the rows; the last of those blocks to finish
-//     reduces the loss in block order and sets the Adam step t and the
-//     bias-correction terms for the update that follows;
-//   all: dZ'_ij = s_i * 2 dL/dg_i * h_ij (h = 0 where z <= 0) in the operand
-//     type, and the block's column sums of dZ for db.
+// columns (block 32 x 8).  Thread (x, y) owns columns 8x..8x+7 of rows
+// y, y+8, y+16, y+24: it issues those activity loads first; meanwhile lanes
+// 0..3 of its warp reduce the per-tile goodness partials of the warp's four
+// rows and form dL/dg, broadcast to the warp by shuffles.  Then
+//   dZ'_ij = s_i * 2 dL/dg_i * h_ij (h = 0 where z <= 0) in the operand type,
+//   and the block's column sums of dZ for db.
+// Blocks of column 0 also write g, the next layer's scale
+// 1/max(sqrt g, 1e-12) and the block's loss partial (reduced by the Adam
+// kernel that follows on the same stream); block (0, 0) advances the Adam
+// step t and its bias-correction terms.
 constexpr int kGradRows = 32;
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __restrict__ H, T* __restrict__ dZ) {
   __shared__ float red[8][256 + 8];
-  __shared__ float c2s[kGradRows], c2[kGradRows];
-  __shared__ int is_last;
+  __shared__ float lred[8];
   const int r0 = blockIdx.y * kGradRows;
   const bool lead = blockIdx.x == 0;
-  const int cg = blockIdx.x * 256 + threadIdx.x * 8;
+  const int lane = threadIdx.x;
+  const int cg = blockIdx.x * 256 + lane * 8;
   const bool cols_ok = cg < a.ld;
   float h[4][8];
 #pragma unroll
@@ -228,9 +228,10 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
       for (int e = 0; e < 8; ++e) h[k][e] = 0.f;
     }
   }
-  if (threadIdx.y == 0) {
-    const int i = r0 + threadIdx.x;
-    float cc = 0.f, sc = 0.f, lv = 0.f;
+  // lanes 0..3: row r0 + y + 8 * lane
+  float cc = 0.f, sc = 0.f, lv = 0.f;
+  if (lane < 4) {
+    const int i = r0 + threadIdx.y + 8 * lane;
     if (i < a.M) {
       const float g = sum_partials(a.gpart, a.ntiles, a.M, i);
       const bool pos = i < a.B;
@@ -245,37 +246,28 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
         lv = softplus_f(tt);
       }
     }
-    c2[threadIdx.x] = cc;
-    c2s[threadIdx.x] = sc;
-    if (lead) {
-      lv = warp_sum(lv);
-      if (threadIdx.x == 0) {
-        a.loss_part[blockIdx.y] = lv;
-        __threadfence();
-        const unsigned prev = atomicAdd(&a.ds->counter, 1u);
-        is_last = (prev == gridDim.y - 1);
-      }
-    }
   }
-  __syncthreads();
   float db[8];
 #pragma unroll
   for (int e = 0; e < 8; ++e) db[e] = 0.f;
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    const int rr = threadIdx.y + 8 * k;
-    const int i = r0 + rr;
-    const float cc = c2[rr], sc = c2s[rr];
+    const float ck = __shfl_sync(0xffffffffu, cc, k), sk = __shfl_sync(0xffffffffu, sc, k);
+    const int i = r0 + threadIdx.y + 8 * k;
     float z[8];
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
-      z[e] = sc * h[k][e];
-      db[e] = fmaf(cc, h[k][e], db[e]);
+      z[e] = sk * h[k][e];
+      db[e] = fmaf(ck, h[k][e], db[e]);
     }
     if (cols_ok && i < a.M) Vec8<T>::store(dZ + (size_t)i * a.ld + cg, z);
   }
+  if (lead) {
+    lv = warp_sum(lv);  // lanes 4..31 contribute 0
+    if (lane == 0) lred[threadIdx.y] = lv;
+  }
 #pragma unroll
-  for (int e = 0; e < 8; ++e) red[threadIdx.y][threadIdx.x * 8 + e] = db[e];
+  for (int e = 0; e < 8; ++e) red[threadIdx.y][lane * 8 + e] = db[e];
   __syncthreads();
   if (threadIdx.y == 0) {
 #pragma unroll
@@ -283,21 +275,16 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
       const int j = cg + e;
       float t = 0.f;
 #pragma unroll
-      for (int y = 0; y < 8; ++y) t += red[y][threadIdx.x * 8 + e];
+      for (int y = 0; y < 8; ++y) t += red[y][lane * 8 + e];
       if (j < a.N) a.dbpart[(size_t)blockIdx.y * a.N + j] = t;
     }
-  }
-  if (lead && is_last && threadIdx.y == 0) {
-    // warp 0 of the last block: loss partials summed lane-strided, then a
-    // fixed-order warp tree (the same order every run)
-    __threadfence();
-    const volatile float* lp = a.loss_part;
-    float tot = 0.f;
-    for (unsigned b = threadIdx.x; b < gridDim.y; b += 32) tot += lp[b];
-    tot = warp_sum(tot);
-    if (threadIdx.x == 0) {
-      a.loss_out[0] = tot / (float)a.B;
-      a.ds->counter = 0;
+    if (lead && lane == 0) {
+      float t = 0.f;
+#pragma unroll
+      for (int y = 0; y < 8; ++y) t += lred[y];
+      a.loss_part[blockIdx.y] = t;
+    }
+    if (lead && blockIdx.y == 0 && lane == 0) {
       // the Adam update that follows is step t; beta^t kept as running products
       a.ds->t += 1;
       a.ds->pow1 *= a.beta1;
@@ -376,6 +363,14 @@ __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
     }
     part[w][lane] = acc;
     __syncthreads();
+    if (blockIdx.x == w_blocks && w == 1 && a.loss_part) {
+      // the step's loss: grad_prep's per-row-block partials, lane-strided then
+      // a fixed-order warp tree
+      float tot = 0.f;
+      for (int rb = lane; rb < a.nrb; rb += 32) tot += a.loss_part[rb];
+      tot = warp_sum(tot);
+      if (lane == 0) a.loss_out[0] = tot / (float)a.B;
+    }
     if (w != 0 || j >= a.N) return;
     float db = 0.f;
 #pragma unroll

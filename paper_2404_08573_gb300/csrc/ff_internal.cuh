@@ -29,9 +29,7 @@ struct ff_dev_state {
   double pow1, pow2;  // beta1^t, beta2^t
   float bc1, bc2;     // 1 - beta1^t, 1 - beta2^t of the current update
   int err;            // latched DEVERR_* bits
-  unsigned counter;   // last-block-done counter of the goodness/loss kernel
   float loss;         // loss of the last train step when the caller passed none
-  int pad;
 };
 
 inline int row_stride(int features) { return (features + 7) & ~7; }
@@ -68,8 +66,7 @@ struct GradPrepArgs {
   float* g_out;        // [M] or null
   float* s_next;       // [M] or null
   float* dbpart;       // [row blocks, N]
-  float* loss_part;    // [row blocks]
-  float* loss_out;     // [1]
+  float* loss_part;    // [row blocks]; the Adam kernel reduces them into the loss
   ff_dev_state* ds;
   double beta1, beta2;
   int* err;
@@ -83,6 +80,9 @@ struct AdamArgs {
   int has_bias;
   float lr, beta1, beta2, eps;
   const ff_dev_state* ds;
+  const float* loss_part;  // [nrb] grad_prep's loss partials of this step, or null
+  float* loss_out;         // [1] receives their sum / B
+  int B;
 };
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
