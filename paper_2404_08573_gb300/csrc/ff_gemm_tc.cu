@@ -10,11 +10,11 @@
 //            (both operands are read MN-major straight from their row-major
 //            buffers: no transposed copies).
 //
-// One CTA computes one BM x BN output tile with three warp roles (two CTAs fit
-// on one SM, so GEMMs of different layer streams overlap):
+// One CTA computes one (ROW_SUBTILES*BM) x BN output tile with three warp roles:
 //   warp 0      TMA producer: 128-byte-swizzled tiles into a STAGES-deep ring
 //   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
-//               N=BN, K=16) and commits each stage back to the producer
+//               N=BN, K=16; one per row subtile, sharing the B stage) and
+//               commits each stage back to the producer
 //   warps 2..5  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).. -> registers,
 //               fused scale/bias/ReLU/goodness or plain store
 // Every mbarrier wait is bounded (kWaitTimeoutNs); a timeout latches
@@ -36,17 +36,19 @@ constexpr int NTHREADS = 192;
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
 
-template <int BN, int NSTAGE>
+template <int BN, int NSTAGE, int MT>
 struct TcCfg {
-  static constexpr int A_BYTES = BM * BK * 2;
+  static constexpr int A_BYTES = MT * BM * BK * 2;  // MT row subtiles of BM rows
   static constexpr int B_BYTES = BN * BK * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int STAGES = NSTAGE;
   static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
-  static constexpr uint32_t TMEM_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
+  static constexpr uint32_t TMEM_COLS = MT * ACC_COLS;  // one accumulator per row subtile
   static_assert(BN % 64 == 0 && BN <= 256, "BN must be a multiple of 64, at most 256");
+  static_assert(MT >= 1 && MT * ACC_COLS <= 512, "accumulators must fit in TMEM");
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-  static_assert(4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
+  static_assert(MT * 4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
   static_assert(4 * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
   static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
 };
@@ -56,11 +58,11 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
   atomicOr(err, DEVERR_TIMEOUT);
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE>
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE, int MT>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
-  using C = TcCfg<BN, NSTAGE>;
+  using C = TcCfg<BN, NSTAGE, MT>;
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -77,7 +79,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int m0 = blockIdx.y * BM;
+  const int m0 = blockIdx.y * (BM * MT);
   const int n0 = blockIdx.x * BN;
   const int num_kb = (K + BK - 1) / BK;
 
@@ -126,10 +128,12 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         uint8_t* b = sB + s * C::B_BYTES;
         const int k0 = kb * BK;
         if (!A_MN) {
-          ptx::tma_load_2d(a, &tmA, &full[s], k0, m0);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) ptx::tma_load_2d(a + mt * BM * BK * 2, &tmA, &full[s], k0, m0 + BM * mt);
         } else {
 #pragma unroll
-          for (int j = 0; j < BM / 64; ++j) ptx::tma_load_2d(a + j * 64 * BK * 2, &tmA, &full[s], m0 + 64 * j, k0);
+          for (int j = 0; j < MT * BM / 64; ++j)
+            ptx::tma_load_2d(a + j * 64 * BK * 2, &tmA, &full[s], m0 + 64 * j, k0);
         }
         if (CM == 1) {
           if (!B_MN) {
@@ -192,11 +196,16 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           // swizzled 128-byte row (SBO = 1024 between 8-row groups).
           // MN-major: 16 K rows further = 2 x 1024 bytes; LBO = 8192 between
           // the 64-element MN chunks, SBO = 1024 between 8-row K groups.
-          const uint64_t ad = A_MN ? ptx::sdesc_sw128(a_base + k * 2048, 64 * BK * 2, 1024)
-                                   : ptx::sdesc_sw128(a_base + k * 32, 16, 1024);
           const uint64_t bd = B_MN ? ptx::sdesc_sw128(b_base + k * 2048, 64 * BK * 2, 1024)
                                    : ptx::sdesc_sw128(b_base + k * 32, 16, 1024);
-          ptx::umma_f16(tmem, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+#pragma unroll
+          for (int mt = 0; mt < MT; ++mt) {
+            // row subtile mt: BM rows further in the A stage, its own accumulator
+            const uint32_t as = a_base + mt * BM * BK * 2;
+            const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
+                                     : ptx::sdesc_sw128(as + k * 32, 16, 1024);
+            ptx::umma_f16(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          }
         }
         if (CM == 1)
           ptx::umma_commit(&empty[s]);
@@ -207,20 +216,20 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    // Thread t of warp q owns TMEM lane / tile row 32q + t.  The operand ring
-    // is idle once the accumulator is complete, so each warp stages its 32
-    // rows there in the 128-byte-swizzled layout (conflict-free for
-    // row-per-thread 16-byte writes) and one lane writes them out with TMA.
+    // Thread t of warp q owns TMEM lane 32q + t, i.e. row 32q + t of each of
+    // the MT row subtiles.  The operand ring is idle once the accumulators
+    // are complete, so each warp stages its rows there in the 128-byte-
+    // swizzled layout (conflict-free for row-per-thread 16-byte writes) and
+    // one lane writes them out with TMA.
     const int q = warp & 3;
-    const int row = q * 32 + lane;
-    const int gi = m0 + row;
-    float s = 0.f;
+    float s0 = 0.f;
     if (MODE == MODE_FWD) {
       // While the mainloop runs: the tile's bias (zero past N or without bias)
-      // into shared memory and this thread's row scale into a register.
+      // into shared memory and this thread's first row scale into a register.
       for (int c = (int)threadIdx.x - 64; c < BN; c += 128)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
-      if (gi < M) s = __ldg(ep.row_scale + gi);
+      const int gi0 = m0 + q * 32 + lane;
+      if (gi0 < M) s0 = __ldg(ep.row_scale + gi0);
       ptx::named_bar(1, 128);
     }
     const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
@@ -230,99 +239,101 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (__all_sync(0xffffffffu, ok && !*abort_flag)) {
       constexpr int ES = MODE == MODE_FWD ? 2 : 4;      // staged element size
       constexpr int CW = 128 / ES;                       // columns per 128-byte swizzle row
-      // bf16: the warp's whole 32 x BN slab; fp32: two 32 x 32 slots, streamed
-      uint8_t* stage = smem + q * (MODE == MODE_FWD ? 32 * BN * 2 : 8192);
       const uint32_t sw = (uint32_t)(lane & 7);
       const bool staged = MODE == MODE_FWD || tma_store;
-      const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16);
-      float g = 0.f;
-      // Columns past N and rows past M hold zero products (their operand rows
-      // were zero-filled); the TMA store clips them and gpart skips them.
-      auto process = [&](const uint32_t (&r)[32], int c0) {
-        const int col0 = n0 + c0;
-        if (MODE == MODE_FWD) {
-          uint32_t packed[16];
-          const float4* b4 = reinterpret_cast<const float4*>(sbias + c0);
+      int fchunk = 0;  // fp32 chunks streamed so far (slot parity)
+#pragma unroll 1
+      for (int mt = 0; mt < MT; ++mt) {
+        const int rbase = m0 + mt * BM + q * 32;  // this warp's first row in subtile mt
+        const int gi = rbase + lane;
+        // bf16: the warp's whole 32 x BN slab per subtile; fp32: two 32 x 32 slots, streamed
+        uint8_t* stage = smem + (MODE == MODE_FWD ? (q * MT + mt) * (32 * BN * 2) : q * 8192);
+        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS);
+        float s = s0;
+        if (MODE == MODE_FWD && mt > 0) s = gi < M ? __ldg(ep.row_scale + gi) : 0.f;
+        float g = 0.f;
+        // Columns past N and rows past M hold zero products (their operand rows
+        // were zero-filled); the TMA store clips them and gpart skips them.
+        auto process = [&](const uint32_t (&r)[32], int c0) {
+          const int col0 = n0 + c0;
+          if (MODE == MODE_FWD) {
+            uint32_t packed[16];
+            const float4* b4 = reinterpret_cast<const float4*>(sbias + c0);
 #pragma unroll
-          for (int v = 0; v < 8; ++v) {
-            const float4 bb = b4[v];
-            const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
-            float h[4];
+            for (int v = 0; v < 8; ++v) {
+              const float4 bb = b4[v];
+              const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
+              float h[4];
 #pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              const float z = fmaf(s, __uint_as_float(r[4 * v + e]), bv[e]);
-              h[e] = z != z ? z : fmaxf(z, 0.f);  // ReLU, NaN kept for the non-finite check
-              g = fmaf(h[e], h[e], g);
+              for (int e = 0; e < 4; ++e) {
+                const float z = fmaf(s, __uint_as_float(r[4 * v + e]), bv[e]);
+                h[e] = z != z ? z : fmaxf(z, 0.f);  // ReLU, NaN kept for the non-finite check
+                g = fmaf(h[e], h[e], g);
+              }
+              __nv_bfloat162 p0 = __floats2bfloat162_rn(h[0], h[1]);
+              __nv_bfloat162 p1 = __floats2bfloat162_rn(h[2], h[3]);
+              packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
+              packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
             }
-            __nv_bfloat162 p0 = __floats2bfloat162_rn(h[0], h[1]);
-            __nv_bfloat162 p1 = __floats2bfloat162_rn(h[2], h[3]);
-            packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
-            packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
-          }
-          uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
+            uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
 #pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            const uint32_t j = (uint32_t)((c0 % CW) / 8 + v);
-            *reinterpret_cast<uint4*>(base + ((j ^ sw) << 4)) =
-                make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2], packed[4 * v + 3]);
-          }
-        } else if (staged) {
-          // fp32: chunk c0 goes through slot (c0/32)&1; before refilling a slot
-          // the store issued from it two chunks ago must have read it
-          const int slot = (c0 / 32) & 1;
-          uint8_t* sbuf = stage + slot * 4096;
-          if (lane == 0 && c0 >= 64) ptx::bulk_wait_read1();
-          __syncwarp();
-          uint8_t* base = sbuf + lane * 128;
+            for (int v = 0; v < 4; ++v) {
+              const uint32_t j = (uint32_t)((c0 % CW) / 8 + v);
+              *reinterpret_cast<uint4*>(base + ((j ^ sw) << 4)) =
+                  make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2], packed[4 * v + 3]);
+            }
+          } else if (staged) {
+            // fp32: chunk n goes through slot n&1; before refilling a slot the
+            // store issued from it two chunks ago must have read it
+            uint8_t* sbuf = stage + (fchunk & 1) * 4096;
+            if (lane == 0 && fchunk >= 2) ptx::bulk_wait_read1();
+            __syncwarp();
+            uint8_t* base = sbuf + lane * 128;
 #pragma unroll
-          for (int v = 0; v < 8; ++v)
-            *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
-                make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+            for (int v = 0; v < 8; ++v)
+              *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
+                  make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+            ptx::fence_async_smem();
+            __syncwarp();
+            if (lane == 0 && rbase < M && col0 < ep.ldo) ptx::tma_store_2d(&tmC, sbuf, col0, rbase);
+            if (lane == 0) ptx::bulk_commit();
+            ++fchunk;
+          } else if (gi < M) {
+            float* out = reinterpret_cast<float*>(ep.out) + (size_t)gi * ep.ldo;
+#pragma unroll
+            for (int j = 0; j < 32; ++j)
+              if (col0 + j < N) out[col0 + j] = __uint_as_float(r[j]);
+          }
+        };
+        // TMEM loads double-buffered: the next 32 columns load while these are processed.
+        uint32_t ra[32], rb[32];
+        ptx::tmem_ld32(trow, ra);
+        ptx::tmem_ld_wait();
+#pragma unroll 1
+        for (int c0 = 0; c0 < BN; c0 += 64) {
+          ptx::tmem_ld32(trow + (uint32_t)(c0 + 32), rb);
+          process(ra, c0);
+          ptx::tmem_ld_wait();
+          if (c0 + 64 < BN) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
+          process(rb, c0 + 32);
+          ptx::tmem_ld_wait();
+        }
+        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)blockIdx.x * M + gi] = g;
+        if (MODE == MODE_FWD) {
           ptx::fence_async_smem();
           __syncwarp();
-          const int r0 = m0 + q * 32;
-          if (lane == 0 && r0 < M && col0 < ep.ldo) {
-            ptx::tma_store_2d(&tmC, sbuf, col0, r0);
-          }
-          if (lane == 0) ptx::bulk_commit();
-        } else if (gi < M) {
-          float* out = reinterpret_cast<float*>(ep.out) + (size_t)gi * ep.ldo;
-#pragma unroll
-          for (int j = 0; j < 32; ++j)
-            if (col0 + j < N) out[col0 + j] = __uint_as_float(r[j]);
-        }
-      };
-      // TMEM loads double-buffered: the next 32 columns load while these are processed.
-      uint32_t ra[32], rb[32];
-      ptx::tmem_ld32(trow, ra);
-      ptx::tmem_ld_wait();
+          if (lane == 0 && rbase < M) {
 #pragma unroll 1
-      for (int c0 = 0; c0 < BN; c0 += 64) {
-        ptx::tmem_ld32(trow + (uint32_t)(c0 + 32), rb);
-        process(ra, c0);
-        ptx::tmem_ld_wait();
-        if (c0 + 64 < BN) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
-        process(rb, c0 + 32);
-        ptx::tmem_ld_wait();
+            for (int ch = 0; ch < BN / CW; ++ch) {
+              const int col = n0 + ch * CW;
+              if (col < ep.ldo) ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
+            }
+            ptx::bulk_commit();
+          }
+        }
       }
-      if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)blockIdx.x * M + gi] = g;
-      if (MODE != MODE_FWD && staged) {
+      if (staged) {
         if (lane == 0) ptx::bulk_wait_read0();
-        __syncwarp();
-      }
-      if (MODE == MODE_FWD) {
-        ptx::fence_async_smem();
-        __syncwarp();
-        const int r0 = m0 + q * 32;
-        if (lane == 0 && r0 < M) {
-#pragma unroll 1
-          for (int ch = 0; ch < BN / CW; ++ch) {
-            const int col = n0 + ch * CW;
-            if (col < ep.ldo) ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, r0);
-          }
-          ptx::bulk_commit();
-          ptx::bulk_wait_read0();
-        }
         __syncwarp();
       }
     }
@@ -372,19 +383,19 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE>
+template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE, int MT>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st) {
-  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM, NSTAGE>;
+  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM, NSTAGE, MT>;
   static cudaError_t attr =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN, NSTAGE>::SMEM);
+      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN, NSTAGE, MT>::SMEM);
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg = {};
   // tile rows padded to a whole number of clusters; padding CTAs load zeros,
   // share their B slice and write nothing
-  cfg.gridDim = dim3(cdiv(N, BN), cdiv(cdiv(M, BM), CM) * CM, 1);
+  cfg.gridDim = dim3(cdiv(N, BN), cdiv(cdiv(M, BM * MT), CM) * CM, 1);
   cfg.blockDim = dim3(NTHREADS, 1, 1);
-  cfg.dynamicSmemBytes = TcCfg<BN, NSTAGE>::SMEM;
+  cfg.dynamicSmemBytes = TcCfg<BN, NSTAGE, MT>::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeClusterDimension;
@@ -398,14 +409,17 @@ cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtens
 
 constexpr int FWD_BN = 256;
 constexpr int WGRAD_BN = 256;
-// Measured on the 784-2000x4 train step with the layers on 4 streams: a
-// 2-deep ring (98 KB of shared memory, so two GEMM CTAs share an SM and one's
-// prologue/epilogue overlaps the other's mainloop) without clusters gave the
-// shortest epoch (9.8 ms vs 11.1 ms for 4 stages with 4-CTA multicast
-// clusters, which also constrain co-scheduling).  Cluster multicast of the B
-// tile stays available through CLUSTER_M.
-constexpr int CLUSTER_M = 1;  // CTAs per cluster along M sharing one B tile
-constexpr int NSTAGES = 2;    // operand ring depth
+// Measured on the 784-2000x4 train step with the layers on 4 streams (epoch):
+//   128x256 tile, 4-stage ring, 4-CTA multicast clusters ....... 11.1 ms
+//   128x256 tile, 2-stage ring (two CTAs per SM), no clusters ..  9.8 ms
+//   256x256 tile (two 128-row accumulators sharing each B stage),
+//   3-stage ring (192 KB, one CTA per SM), no clusters .........  9.1 ms
+// The step is bound by moving operand tiles into shared memory, so the
+// 256x256 tile's third fewer bytes per FLOP wins; clusters constrain
+// co-scheduling with the other layers' kernels and did not pay.
+constexpr int CLUSTER_M = 1;     // CTAs per cluster along M sharing one B tile
+constexpr int NSTAGES = 3;       // operand ring depth
+constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
 
 }  // namespace
 
@@ -424,7 +438,7 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
   if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
-  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M, NSTAGES>(ta, tb, tc, 1, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
 }
 
 // fp32 C written through shared memory and TMA when its rows are 16-byte
@@ -441,7 +455,7 @@ cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M,
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M, NSTAGES>(ta, tb, tc, tma, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
 }
 
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K, float* Cm, int ldc,
@@ -454,7 +468,7 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M, NSTAGES>(ta, tb, tc, tma, N, K, R, ep, err, st);
+  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
 }
 
 }  // namespace ff
