@@ -389,6 +389,138 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
+# ----------------------------------------------------- other workloads
+def _timed_loop(torch, stream, fn, k):
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        e0.record(stream)
+        for _ in range(k):
+            fn()
+        e1.record(stream)
+    torch.cuda.synchronize()
+    return e0.elapsed_time(e1)
+
+
+def run_other(args):
+    """Single-GPU measurements of the other workloads (one JSON line each)."""
+    import numpy as np
+    import torch
+
+    from paper_2404_08573_gb300 import build, ff, synth
+    build.build()
+    lib = ff.lib()
+    dev = torch.device("cuda", 0)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.Stream(device=dev)
+    pk = peaks()
+    out = {"n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "data": "synthetic",
+           "scaling": "weak", "vs_baseline": None, "higher_is_better": True}
+    w = args.workload
+    if w.startswith("predict"):
+        # 10 000 samples x 10 label overlays through 784-2000x4, goodness of layers 2..4
+        prec = "fp32" if w.endswith("fp32") else "bf16"
+        n = 10000
+        layers = [ff.Layer(NET[k], NET[k + 1], prec=prec, init_seed=1000 + k) for k in range(len(NET) - 1)]
+        x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
+        pred = torch.empty(n, dtype=torch.int32, device=dev)
+        G = torch.empty(n, 10, device=dev)
+        fn = lambda: ff.predict(layers, x, pred=pred, goodness=G, stream=stream)
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        flops = 2.0 * n * NET[1] * NET[0] + 3 * 2.0 * 10 * n * NET[2] * NET[1]
+        tf = flops / (ms / 1e3) / 1e12
+        out.update({"metric": "FF goodness predict samples/s (10 label overlays) on 4x2000 net", "value": round(n / (ms / 1e3), 1),
+                    "unit": "samples/s", "ms_per_step": round(ms, 4), "dtype": prec, "tflops": round(tf, 2),
+                    "frac_of_bf16_peak": round(tf / pk["bf16"], 4) if prec == "bf16" else None,
+                    "config": {"workload": f"ff_predict_784-2000x4_{prec}_n10000", "algorithmic_tflop": flops / 1e12}})
+    elif w == "pipeline_5x2000":
+        # 784-2000x5, 60 chunks of 1000 pairs; 5 layer streams vs the same steps on one stream
+        net5 = [784] + [2000] * 5
+        B, chunks = 1000, 60
+        x = synth.mnist_like(B * chunks, seed=9)
+        y = synth.labels(B * chunks, seed=9)
+        yn = synth.negative_labels(y, seed=9)
+        xs = [torch.from_numpy(np.concatenate([x[c * B:(c + 1) * B]] * 2)).to(dev) for c in range(chunks)]
+        ls = [torch.from_numpy(np.concatenate([y[c * B:(c + 1) * B], yn[c * B:(c + 1) * B]])).to(dev)
+              for c in range(chunks)]
+
+        def mk():
+            return [ff.Layer(net5[k], net5[k + 1], prec="bf16", init_seed=2000 + k, max_rows=2 * B) for k in range(5)]
+        la, lb = mk(), mk()
+        net = ff.Net(la, max_B=B, depth=2)
+        hs = [lb[k].new_activation(2 * B) for k in range(4)]
+        ss = [torch.empty(2 * B, device=dev) for _ in range(4)]
+
+        def streams_run():
+            for c in range(chunks):
+                net.train_step(xs[c], ls[c], B=B, stream=stream)
+            net.sync(stream)
+
+        def single_run():
+            for c in range(chunks):
+                for k in range(5):
+                    lb[k].train_step(xs[c] if k == 0 else hs[k - 1], labels=ls[c] if k == 0 else None,
+                                     row_scale=None if k == 0 else ss[k - 1], B=B,
+                                     h_out=hs[k] if k < 4 else None, next_scale=ss[k] if k < 4 else None,
+                                     stream=stream)
+        _timed_loop(torch, stream, streams_run, args.warmup)
+        _timed_loop(torch, stream, single_run, args.warmup)
+        ms_p = _timed_loop(torch, stream, streams_run, args.steps) / args.steps
+        ms_s = _timed_loop(torch, stream, single_run, args.steps) / args.steps
+        flops = 4.0 * 2 * B * sum(net5[i] * net5[i + 1] for i in range(5)) * chunks
+        out.update({"metric": "FF train pairs/s, 784-2000x5 on 5 CUDA streams (60 chunks of 1000 pairs)",
+                    "value": round(B * chunks / (ms_p / 1e3), 1), "unit": "pairs/s", "ms_per_step": round(ms_p, 4),
+                    "dtype": "bf16", "tflops": round(flops / (ms_p / 1e3) / 1e12, 2),
+                    "single_stream_ms_per_step": round(ms_s, 4), "speedup_vs_single_stream": round(ms_s / ms_p, 3),
+                    "config": {"workload": "ff_train_784-2000x5_bf16_5streams_60x1000"}})
+        net.close()
+    elif w == "wide_4x8192":
+        # 3072-8192x4, B = 4096 pairs, theta = 8; one step = one batch through all layers
+        netw = [3072] + [8192] * 4
+        B = 4096
+        x = synth.cifar_like(B, seed=11)
+        y = synth.labels(B, seed=11)
+        x2, l2 = synth.pair_batch(x, y, synth.negative_labels(y, seed=11))
+        xg, lg = torch.from_numpy(x2).to(dev), torch.from_numpy(l2).to(dev)
+        layers = [ff.Layer(netw[k], netw[k + 1], prec="bf16", theta=8.0, lr=LR, init_seed=3000 + k, max_rows=2 * B)
+                  for k in range(4)]
+        net = ff.Net(layers, max_B=B, depth=2)
+        fn = lambda: (net.train_step(xg, lg, B=B, stream=stream), net.sync(stream))
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        flops = 4.0 * 2 * B * sum(netw[i] * netw[i + 1] for i in range(4))
+        tf = flops / (ms / 1e3) / 1e12
+        out.update({"metric": "FF train pairs/s on 3072-8192x4 (B=4096 pairs)", "value": round(B / (ms / 1e3), 1),
+                    "unit": "pairs/s", "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
+                    "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
+                    "config": {"workload": "ff_train_3072-8192x4_bf16_B4096_theta8"}})
+        net.close()
+    elif w == "tiny_fp32":
+        # 784-500-500 fp32, 16 steps of 64 pairs (latency-bound)
+        B = 64
+        layers = [ff.Layer(784, 500, prec="fp32", init_seed=0), ff.Layer(500, 500, prec="fp32", init_seed=1)]
+        h = layers[0].new_activation(2 * B)
+        sc = torch.empty(2 * B, device=dev)
+        batches16 = []
+        for t in range(16):
+            x = synth.mnist_like(B, seed=0, start_row=t * B)
+            y = synth.labels(B, seed=0, start=t * B)
+            x2, l2 = synth.pair_batch(x, y, synth.negative_labels(y, seed=0, start=t * B))
+            batches16.append((torch.from_numpy(x2).to(dev), torch.from_numpy(l2).to(dev)))
+
+        def run16():
+            for xb, lb in batches16:
+                layers[0].train_step(xb, labels=lb, B=B, h_out=h, next_scale=sc, stream=stream)
+                layers[1].train_step(h, row_scale=sc, B=B, stream=stream)
+        _timed_loop(torch, stream, run16, args.warmup)
+        ms = _timed_loop(torch, stream, run16, args.steps) / args.steps
+        out.update({"metric": "FF train step latency, 784-500-500 fp32, B=64 pairs", "value": round(1e3 * ms / 16, 2),
+                    "unit": "us/step", "higher_is_better": False, "ms_per_step": round(ms, 4), "dtype": "f32",
+                    "config": {"workload": "ff_train_784-500-500_fp32_B64_16steps"}})
+    print(json.dumps(out), flush=True)
+
+
 # -------------------------------------------------------------- reference
 def run_reference(args):
     rank = int(os.environ.get("RANK", "0"))
@@ -420,6 +552,9 @@ def main():
     ap.add_argument("--steps", type=int, default=10)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", default="train_4x2000",
+                    choices=["train_4x2000", "predict_bf16", "predict_fp32", "pipeline_5x2000", "wide_4x8192",
+                             "tiny_fp32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")
@@ -435,6 +570,8 @@ def main():
         print("warning: fewer than 3 warm-up steps", file=sys.stderr)
     if args.impl == "reference":
         run_reference(args)
+    elif args.workload != "train_4x2000":
+        run_other(args)
     else:
         run_ours(args)
 
