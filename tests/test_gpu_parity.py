@@ -393,3 +393,50 @@ def test_net_steps_captured_in_a_cuda_graph_match_eager(env):
         assert sa["t"] == sb["t"] == 6
         for k in ("W", "b", "mW", "vW"):
             assert np.array_equal(sa[k], sb[k]), k
+
+
+# ------------------------------------------------ wide net (3072-8192x4)
+def test_wide_first_layer_train_step_full_size(env):
+    """3072 -> 8192, B = 4096 pairs, theta = 8: the wide workload's first layer
+    at full size against the bf16-emulating oracle."""
+    torch, ff = env
+    B, K, N, theta, lr = 4096, 3072, 8192, 8.0, 0.03
+    x = synth.cifar_like(B, seed=41)
+    y = synth.labels(B, seed=41)
+    x2, l2 = synth.pair_batch(x, y, synth.negative_labels(y, seed=41))
+    layer = ff.Layer(K, N, prec="bf16", theta=theta, lr=lr, init_seed=3000, keep_grad=True, max_rows=2 * B)
+    W = layer.get_state()["W"]
+    g = torch.empty(2 * B, device="cuda")
+    loss = torch.empty(1, device="cuda")
+    layer.train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=B, goodness=g, loss=loss)
+    torch.cuda.synchronize()
+    layer.check()
+    st = fo.LayerState(W, np.zeros(N))
+    ref = fo.layer_train_step(st, fo.overlay_label(x2, l2), B, theta, fo.AdamHyper(lr=lr), emulate_bf16=True)
+    assert_close(g.cpu().numpy(), ref["g"], 1e-3, 1e-6, "goodness")
+    assert abs(loss.item() - ref["loss"]) <= 1e-3 * abs(ref["loss"]) + 1e-7
+    dW, db = layer.get_grad()
+    assert rel_norm(dW, ref["dW"]) < 1e-3 and rel_norm(db, ref["db"]) < 1e-3
+    assert rel_norm(layer.get_state()["W"], st.W) < 2e-2
+
+
+def test_wide_hidden_layer_forward_sampled_rows(env):
+    """8192 -> 8192 over 8192 rows (the wide workload's hidden layer, as the
+    bench launches it); the oracle checks 256 sampled rows one by one."""
+    torch, ff = env
+    M, K, N = 8192, 8192, 8192
+    layer = ff.Layer(K, N, prec="bf16", init_seed=3001, max_rows=M)
+    st = layer.get_state()
+    xin = torch.relu(torch.randn(M, K, device="cuda", generator=torch.Generator("cuda").manual_seed(3))).to(
+        torch.bfloat16)
+    xa = layer.new_activation(M, K)
+    xa[:, :K] = xin
+    g = torch.empty(M, device="cuda")
+    h = layer.new_activation(M)
+    layer.forward(xa, h_out=h, goodness=g)
+    torch.cuda.synchronize()
+    rows = np.sort(np.random.default_rng(4).choice(M, 256, replace=False))
+    xs = xin[rows].float().cpu().numpy().astype(np.float64)
+    ref = fo.layer_forward_full(fo.LayerState(st["W"], st["b"]), xs, emulate_bf16=True)
+    assert_close(g.cpu().numpy()[rows], ref["g"], 1e-3, 1e-6, "sampled goodness")
+    assert_close(h[rows].float().cpu().numpy()[:, :N], ref["H"], 2.0 ** -8 + 1e-3, 1e-5, "sampled activity")
