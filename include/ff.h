@@ -208,8 +208,9 @@ FF_API ff_status ff_net_sync(ff_net* net, void* stream);
  * goodness was not finite).  It allocates nothing: the per-tile goodness
  * partials live in a fixed 4 MiB array in the library's device image, which
  * every GPU that loads libff holds until the process exits.
- *   - Limit: rows * ceil(out_features / 256) <= 1048512; larger requests
- *     return FF_ERR_INVALID_ARG before anything is enqueued.
+ *   - Limit: rows * 2 * ceil(out_features / 256) <= 1048512 (two goodness
+ *     partials per 256-column tile and row); larger requests return
+ *     FF_ERR_INVALID_ARG before anything is enqueued.
  *   - The first call on a device looks up that array's device address (once
  *     per device, with that device current); make that first call before any
  *     stream capture.

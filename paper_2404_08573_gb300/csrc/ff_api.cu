@@ -69,7 +69,11 @@ void dev_free(void* p) {
 
 static size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
-static int gpart_tiles_max(int N) { return cdiv(N, 128); }
+// goodness partials per row: the most either forward GEMM writes
+static int gpart_tiles_max(int N) {
+  const int a = tc_fwd_ntiles(N), b = simt_fwd_ntiles(N);
+  return a > b ? a : b;
+}
 
 // Grows the per-row workspace to at least `rows` rows (one allocation).
 static ff_status ensure_capacity(ff_layer* L, int rows) {
@@ -113,8 +117,7 @@ static ff_status ensure_capacity(ff_layer* L, int rows) {
 static void free_layer(ff_layer* L) {
   if (!L) return;
   dev_free(L->W);
-  dev_free(L->mW);
-  dev_free(L->vW);
+  dev_free(L->mW);  // also holds v_W
   dev_free(L->dW);
   dev_free(L->b);
   dev_free(L->Wb);
@@ -324,8 +327,8 @@ ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** o
     }                                                                             \
   } while (0)
   FF_ALLOC(L->W, nk * 4);
-  FF_ALLOC(L->mW, nk * 4);
-  FF_ALLOC(L->vW, nk * 4);
+  FF_ALLOC(L->mW, nk * 4 * 2);  // m_W then v_W, one range
+  L->vW = L->mW + nk;
   FF_ALLOC(L->dW, nk * 4);
   FF_ALLOC(L->b, (size_t)L->N * 4 * 4);  // b, mb, vb, db
   if (L->is_bf16) FF_ALLOC(L->Wb, (size_t)L->N * L->ldK * 2);

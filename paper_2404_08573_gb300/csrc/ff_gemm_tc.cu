@@ -15,8 +15,9 @@
 //   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
 //               N=BN, K=16; one per row subtile, sharing the B stage) and
 //               commits each stage back to the producer
-//   warps 2..5  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).. -> registers,
-//               fused scale/bias/ReLU/goodness or plain store
+//   warps 2..9  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).., one half of
+//               the columns each -> registers, fused scale/bias/ReLU/goodness
+//               (partials per 128-column half) or plain store
 // Every mbarrier wait is bounded (kWaitTimeoutNs); a timeout latches
 // DEVERR_TIMEOUT in *err, tells the other roles to stop, waits for copies and
 // MMAs already in flight and frees TMEM before the CTA exits.
@@ -32,7 +33,8 @@ namespace {
 
 constexpr int BM = 128;
 constexpr int BK = 64;  // one 128-byte swizzle row of bf16
-constexpr int NTHREADS = 192;
+constexpr int EPI_WARPS = 8;                 // two per TMEM lane quarter, each on half the columns
+constexpr int NTHREADS = 64 + 32 * EPI_WARPS;  // producer warp, MMA warp, epilogue warps
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
 
@@ -49,7 +51,8 @@ struct TcCfg {
   static_assert(MT >= 1 && MT * ACC_COLS <= 512, "accumulators must fit in TMEM");
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
   static_assert(MT * 4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
-  static_assert(4 * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
+  static_assert(EPI_WARPS * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
+  static_assert(BN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
   static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
 };
 
@@ -216,21 +219,27 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     }
   } else {
     // ------------------------------------------------------------ epilogue
-    // Thread t of warp q owns TMEM lane 32q + t, i.e. row 32q + t of each of
-    // the MT row subtiles.  The operand ring is idle once the accumulators
-    // are complete, so each warp stages its rows there in the 128-byte-
-    // swizzled layout (conflict-free for row-per-thread 16-byte writes) and
-    // one lane writes them out with TMA.
+    // Warp w (2..9) reads TMEM lane quarter q = w % 4 -- row 32q + t of each
+    // of the MT row subtiles for its thread t -- and the columns of half
+    // (w - 2) / 4 of the tile.  The operand ring is idle once the
+    // accumulators are complete, so each warp stages its block there in the
+    // 128-byte-swizzled layout (conflict-free for row-per-thread 16-byte
+    // writes) and one lane writes it out with TMA.
+    constexpr int HALVES = EPI_WARPS / 4;
+    constexpr int CPW = BN / HALVES;  // columns per epilogue warp
     const int q = warp & 3;
+    const int ew = warp - 2;          // 0 .. EPI_WARPS-1
+    const int half = ew / 4;
+    const int cbase = half * CPW;     // this warp's first column within the tile
     float s0 = 0.f;
     if (MODE == MODE_FWD) {
       // While the mainloop runs: the tile's bias (zero past N or without bias)
       // into shared memory and this thread's first row scale into a register.
-      for (int c = (int)threadIdx.x - 64; c < BN; c += 128)
+      for (int c = (int)threadIdx.x - 64; c < BN; c += 32 * EPI_WARPS)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
       const int gi0 = m0 + q * 32 + lane;
       if (gi0 < M) s0 = __ldg(ep.row_scale + gi0);
-      ptx::named_bar(1, 128);
+      ptx::named_bar(1, 32 * EPI_WARPS);
     }
     const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
     if (!ok) latch(err, abort_flag);
@@ -246,19 +255,20 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       for (int mt = 0; mt < MT; ++mt) {
         const int rbase = m0 + mt * BM + q * 32;  // this warp's first row in subtile mt
         const int gi = rbase + lane;
-        // bf16: the warp's whole 32 x BN slab per subtile; fp32: two 32 x 32 slots, streamed
-        uint8_t* stage = smem + (MODE == MODE_FWD ? (q * MT + mt) * (32 * BN * 2) : q * 8192);
-        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS);
+        // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
+        uint8_t* stage = smem + (MODE == MODE_FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
+        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS + cbase);
         float s = s0;
         if (MODE == MODE_FWD && mt > 0) s = gi < M ? __ldg(ep.row_scale + gi) : 0.f;
         float g = 0.f;
         // Columns past N and rows past M hold zero products (their operand rows
         // were zero-filled); the TMA store clips them and gpart skips them.
+        // c0 counts columns within this warp's half.
         auto process = [&](const uint32_t (&r)[32], int c0) {
-          const int col0 = n0 + c0;
+          const int col0 = n0 + cbase + c0;
           if (MODE == MODE_FWD) {
             uint32_t packed[16];
-            const float4* b4 = reinterpret_cast<const float4*>(sbias + c0);
+            const float4* b4 = reinterpret_cast<const float4*>(sbias + cbase + c0);
 #pragma unroll
             for (int v = 0; v < 8; ++v) {
               const float4 bb = b4[v];
@@ -310,22 +320,22 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         ptx::tmem_ld32(trow, ra);
         ptx::tmem_ld_wait();
 #pragma unroll 1
-        for (int c0 = 0; c0 < BN; c0 += 64) {
+        for (int c0 = 0; c0 < CPW; c0 += 64) {
           ptx::tmem_ld32(trow + (uint32_t)(c0 + 32), rb);
           process(ra, c0);
           ptx::tmem_ld_wait();
-          if (c0 + 64 < BN) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
+          if (c0 + 64 < CPW) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
           process(rb, c0 + 32);
           ptx::tmem_ld_wait();
         }
-        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)blockIdx.x * M + gi] = g;
+        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)(blockIdx.x * HALVES + half) * M + gi] = g;
         if (MODE == MODE_FWD) {
           ptx::fence_async_smem();
           __syncwarp();
           if (lane == 0 && rbase < M) {
 #pragma unroll 1
-            for (int ch = 0; ch < BN / CW; ++ch) {
-              const int col = n0 + ch * CW;
+            for (int ch = 0; ch < CPW / CW; ++ch) {
+              const int col = n0 + cbase + ch * CW;
               if (col < ep.ldo) ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
             }
             ptx::bulk_commit();
@@ -430,7 +440,7 @@ bool tc_supported() {
   return major == 10 && encode_fn() != nullptr;
 }
 
-int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN); }
+int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN) * (EPI_WARPS / 4); }  // goodness partials per row
 
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
                         int* err, cudaStream_t st) {

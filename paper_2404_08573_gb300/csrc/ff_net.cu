@@ -9,6 +9,8 @@
 // Each layer's own steps stay in order on its stream, so every kernel sees
 // exactly the inputs it would see in a one-stream run: results are bitwise
 // identical to the sequential schedule.
+#include <cstdio>
+#include <cstdlib>
 #include <vector>
 
 #include "ff_api_internal.h"
