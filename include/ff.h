@@ -223,6 +223,13 @@ FF_API ff_status ff_forward_noalloc(const void* x, const float* row_scale, const
                                     void* h_out, float* goodness, float* next_scale,
                                     int* device_status, void* stream);
 
+/* Self-test of failure detection (the paper has no counterpart): enqueues on
+ * `stream` one kernel that waits, through the same bounded mbarrier wait the
+ * GEMM kernels use, on a barrier nothing arrives on.  After timeout_us
+ * (1 .. 10 000 000) the wait gives up and latches the timeout in the layer;
+ * ff_layer_check then returns FF_ERR_TIMEOUT and the context stays usable. */
+FF_API ff_status ff_layer_selftest_wait(ff_layer* layer, unsigned int timeout_us, void* stream);
+
 /* ---------------------------------------------------------------------------
  * Instrumentation (not part of the method).
  * Every kernel launch libff makes is counted; ff_kernel_launches returns the

@@ -585,6 +585,14 @@ ff_status ff_layer_get_grad(const ff_layer* Lc, float* dW, float* db) {
   return FF_OK;
 }
 
+ff_status ff_layer_selftest_wait(ff_layer* L, unsigned int timeout_us, void* stream) {
+  if (!L || timeout_us == 0 || timeout_us > 10000000u) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  L->last_stream = st;
+  FF_TRY(launch_wait_selftest(&L->ds->err, 1000ull * timeout_us, st), "bounded-wait self-test");
+  return FF_OK;
+}
+
 ff_status ff_layer_check(ff_layer* L) {
   if (!L) return FF_ERR_INVALID_ARG;
   cudaError_t e = cudaStreamSynchronize(L->last_stream);

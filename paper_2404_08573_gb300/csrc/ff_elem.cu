@@ -14,6 +14,7 @@
 // Reductions use fixed orders (no floating-point atomics), so results do not
 // depend on scheduling.
 #include "ff_internal.cuh"
+#include "ff_ptx.cuh"
 
 namespace ff {
 namespace {
@@ -476,6 +477,21 @@ __global__ void k_argmax(const float* __restrict__ G, int n, int* __restrict__ p
   pred[i] = best;
 }
 
+// Self-test of the bounded waits: one thread waits on an mbarrier that
+// nothing arrives on, through the same bounded wait the GEMMs use, and
+// latches DEVERR_TIMEOUT when it gives up.
+__global__ void k_wait_selftest(int* err, unsigned long long timeout_ns) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    ptx::mbar_init(&bar, 1);
+    abort_flag = 0;
+    ptx::fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0 && !ptx::mbar_wait(&bar, 0, timeout_ns, &abort_flag)) atomicOr(err, DEVERR_TIMEOUT);
+}
+
 int grid_for(long long work, int per_block, int cap) {
   long long b = (work + per_block - 1) / per_block;
   if (b < 1) b = 1;
@@ -569,6 +585,11 @@ cudaError_t launch_expand(const float* base, int ldbase, const float* cols, cons
 cudaError_t launch_argmax(const float* G, int n, int* pred, float* /*unused*/, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
   k_argmax<<<cdiv(n, 256), 256, 0, st>>>(G, n, pred);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_wait_selftest(int* err, unsigned long long timeout_ns, cudaStream_t st) {
+  k_wait_selftest<<<1, 32, 0, st>>>(err, timeout_ns);
   return cudaGetLastError();
 }
 

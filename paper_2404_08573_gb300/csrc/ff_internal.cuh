@@ -95,6 +95,8 @@ cudaError_t launch_expand(const float* base, int ldbase, const float* cols, cons
                           float* s_next, float* G_acc /*null unless single layer*/, int* err,
                           cudaStream_t st);
 cudaError_t launch_argmax(const float* G, int n, int* pred, float* goodness_out, cudaStream_t st);
+// one bounded wait on an mbarrier nothing arrives on (latches DEVERR_TIMEOUT)
+cudaError_t launch_wait_selftest(int* err, unsigned long long timeout_ns, cudaStream_t st);
 
 // ------------------------------------------------------------------- GEMMs
 // Forward epilogue: H = ReLU(s_r * acc + b) (bf16 or fp32), per-tile goodness

@@ -67,6 +67,7 @@ def lib():
             "ff_layer_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
             "ff_layer_check": [c_void_p],
+            "ff_layer_selftest_wait": [c_void_p, ctypes.c_uint, c_void_p],
             "ff_net_create": [c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_destroy": [c_void_p],
             "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
@@ -219,6 +220,11 @@ class Layer:
 
     def check(self):
         _check(lib().ff_layer_check(self._h), "ff_layer_check")
+
+    def selftest_wait(self, timeout_us: int, stream=None):
+        """ff_layer_selftest_wait: a bounded wait that is made to run out."""
+        _check(lib().ff_layer_selftest_wait(self._h, int(timeout_us), c_void_p(_stream(stream))),
+               "ff_layer_selftest_wait")
 
 
 def overlay_label(x, labels, prec="bf16", out=None, row_scale=None, stream=None):
