@@ -30,6 +30,9 @@ What each function follows:
 * ``predict``         -- §3 "Prediction", Goodness method: run the input with
   each of the 10 labels, accumulate goodness over all but the first hidden
   layer, pick the label with the largest total.
+* ``adaptive_negatives`` -- AdaptiveNEG of §5: the negative label of a sample
+  is the incorrect label the network currently predicts most strongly, i.e.
+  the goodness-prediction argmax over the 9 wrong labels.
 
 Readings of points the paper leaves open (the paper states none of them):
 
@@ -273,3 +276,15 @@ def predict(states, x_raw, emulate_bf16: bool = False, n_classes: int = N_CLASSE
                 G[:, c] += f["g"]
             a = f["H"]
     return np.argmax(G, axis=1), G
+
+
+def adaptive_negatives(states, x_raw, labels, emulate_bf16: bool = False, n_classes: int = N_CLASSES):
+    """AdaptiveNEG (§5): for each sample, the wrong label with the largest
+    accumulated goodness (the lowest such label on ties).  Returns
+    (neg [n] int64, G [n, n_classes])."""
+    labels = np.asarray(labels, dtype=np.int64)
+    _, G = predict(states, x_raw, emulate_bf16=emulate_bf16, n_classes=n_classes)
+    masked = G.copy()
+    masked[np.arange(G.shape[0]), labels] = -np.inf
+    return np.argmax(masked, axis=1), G
+

@@ -332,3 +332,30 @@ def test_negative_labels_are_wrong_and_cover_all_offsets():
     off = (yn - y - 1) % 10
     assert set(np.unique(off)) == set(range(9))
     assert np.all(np.abs(np.bincount(y, minlength=10) / 20000 - 0.1) < 0.01)
+
+
+def test_adaptive_negatives_are_the_strongest_wrong_label():
+    """Brute force: for each sample the strongest of the 9 wrong labels, never
+    the true one; with hand-built nets the dominated label is chosen."""
+    rng = np.random.default_rng(13)
+    dims = (12, 5, 4)
+    Ws = [rng.standard_normal((dims[i + 1], dims[i])) for i in range(2)]
+    bs = [rng.standard_normal(dims[i + 1]) * 0.2 for i in range(2)]
+    x = rng.random((40, 12))
+    y = rng.integers(0, 10, 40)
+    states = [fo.LayerState(W, b) for W, b in zip(Ws, bs)]
+    neg, G = fo.adaptive_negatives(states, x, y)
+    _, bG = _brute_predict([W.tolist() for W in Ws], [b.tolist() for b in bs], x)
+    for i in range(40):
+        assert neg[i] != y[i]
+        best = max((c for c in range(10) if c != y[i]), key=lambda c: (bG[i][c], -c))
+        assert neg[i] == best
+    # the true label dominates: the negative is the runner-up
+    K = 14
+    W1 = np.zeros((10, K)); W1[np.arange(10), np.arange(10)] = 1.0
+    W2 = np.eye(10); W2[3, 3] = 5.0; W2[7, 7] = 3.0
+    xx = np.random.default_rng(0).random((6, K))
+    st = [fo.LayerState(W1, np.zeros(10)), fo.LayerState(W2, np.zeros(10))]
+    neg, _ = fo.adaptive_negatives(st, xx, np.full(6, 3))
+    assert np.all(neg == 7)
+
