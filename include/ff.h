@@ -145,6 +145,19 @@ FF_API ff_status ff_layer_train_step(ff_layer* layer, const void* x, const int* 
 FF_API ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n,
                      int* pred, float* goodness, void* stream);
 
+/* AdaptiveNEG negative labels of §5: the negative label of a sample is the
+ * wrong label the network currently predicts most strongly.  Runs the
+ * goodness prediction of ff_predict on x [n, in] (raw float32) and writes
+ * neg[r] (int32) = the label c != labels[r] with the largest goodness sum,
+ * the lowest such label on ties; goodness [n, 10] (or NULL) as in ff_predict.
+ * labels [n] int32 (device) are the true labels; a label outside 0..9 leaves
+ * no label out, so neg[r] is then the plain prediction.  Layers, scratch,
+ * stream and n == 0 behave as in ff_predict; labels == NULL with n > 0 is
+ * FF_ERR_INVALID_ARG. */
+FF_API ff_status ff_adaptive_negatives(ff_layer* const* layers, int n_layers, const float* x,
+                                       const int* labels, int n, int* neg, float* goodness,
+                                       void* stream);
+
 /* Copies the layer state to/from caller buffers, which may be host or device
  * memory: W [N,K] and its Adam moments m_W, v_W [N,K]; b, m_b, v_b [N]; the
  * Adam step counter.  Any pointer may be NULL to skip that tensor.  Both calls

@@ -417,8 +417,10 @@ ff_status ff_layer_train_step(ff_layer* L, const void* x, const int* labels, con
                          static_cast<cudaStream_t>(stream), nullptr, nullptr);
 }
 
-ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n, int* pred, float* goodness,
-                     void* stream) {
+// Goodness prediction over the 10 label overlays (§3 "Prediction"); with
+// `labels`, the argmax leaves each sample's own label out (AdaptiveNEG, §5).
+static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float* x, const int* labels, int n,
+                              int* pred, float* goodness, cudaStream_t st) {
   if (!layers || n_layers < 1 || n < 0) return FF_ERR_INVALID_ARG;
   for (int k = 0; k < n_layers; ++k) {
     if (!layers[k]) return FF_ERR_INVALID_ARG;
@@ -431,7 +433,6 @@ ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int 
   if (L0->K < 10) return FF_ERR_INVALID_ARG;
   const bool b16 = L0->is_bf16;
   const size_t es = b16 ? 2 : 4;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   int ldmax = 0, ntmax = 0;
   for (int k = 0; k < n_layers; ++k) {
     if (layers[k]->ldN > ldmax) ldmax = layers[k]->ldN;
@@ -531,8 +532,19 @@ ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int 
       cur ^= 1;
     }
   }
-  FF_LAUNCH(K_ARGMAX, (double)n * 44, st, launch_argmax(G, n, pred, nullptr, st), "argmax");
+  FF_LAUNCH(K_ARGMAX, (double)n * (labels ? 48 : 44), st, launch_argmax(G, n, labels, pred, st), "argmax");
   return FF_OK;
+}
+
+ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n, int* pred, float* goodness,
+                     void* stream) {
+  return predict_impl(layers, n_layers, x, nullptr, n, pred, goodness, static_cast<cudaStream_t>(stream));
+}
+
+ff_status ff_adaptive_negatives(ff_layer* const* layers, int n_layers, const float* x, const int* labels, int n,
+                                int* neg, float* goodness, void* stream) {
+  if (n > 0 && !labels) return FF_ERR_INVALID_ARG;
+  return predict_impl(layers, n_layers, x, labels, n, neg, goodness, static_cast<cudaStream_t>(stream));
 }
 
 static cudaMemcpyKind kind_default() { return cudaMemcpyDefault; }

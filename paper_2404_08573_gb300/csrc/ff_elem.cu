@@ -10,7 +10,8 @@
 //   adam         Adam (§5.1) on W and b, refreshing the bf16 copy of W
 //   init         He-uniform W from a counter-based SplitMix64 stream
 //   predict      label columns of W1, per-label expansion of layer 1,
-//                argmax over the 10 labels (§3 "Prediction")
+//                argmax over the 10 labels (§3 "Prediction"), and over
+//                the 9 wrong labels for AdaptiveNEG negatives (§5)
 // Reductions use fixed orders (no floating-point atomics), so results do not
 // depend on scheduling.
 #include "ff_internal.cuh"
@@ -462,18 +463,26 @@ __global__ void __launch_bounds__(256) k_expand(const float* __restrict__ base, 
   }
 }
 
-__global__ void k_argmax(const float* __restrict__ G, int n, int* __restrict__ pred) {
+// pred[i] = the label with the largest G[i, c], the lowest on ties.  With
+// labels (AdaptiveNEG, §5) the sample's own label is left out, so pred[i] is
+// its strongest wrong label; a label outside 0..9 leaves nothing out.
+__global__ void k_argmax(const float* __restrict__ G, int n, const int* __restrict__ labels,
+                         int* __restrict__ pred) {
   const int i = blockIdx.x * blockDim.x + threadIdx.x;
   if (i >= n) return;
   const float* g = G + (size_t)i * 10;
-  int best = 0;
-  float bv = g[0];
+  const int skip = labels ? labels[i] : -1;
+  int best = -1;
+  float bv = 0.f;
 #pragma unroll
-  for (int c = 1; c < 10; ++c)
-    if (g[c] > bv) {
-      bv = g[c];
+  for (int c = 0; c < 10; ++c) {
+    if (c == skip) continue;
+    const float v = g[c];
+    if (best < 0 || v > bv) {
+      bv = v;
       best = c;
     }
+  }
   pred[i] = best;
 }
 
@@ -582,9 +591,9 @@ cudaError_t launch_expand(const float* base, int ldbase, const float* cols, cons
   return cudaGetLastError();
 }
 
-cudaError_t launch_argmax(const float* G, int n, int* pred, float* /*unused*/, cudaStream_t st) {
+cudaError_t launch_argmax(const float* G, int n, const int* labels, int* pred, cudaStream_t st) {
   if (n <= 0) return cudaSuccess;
-  k_argmax<<<cdiv(n, 256), 256, 0, st>>>(G, n, pred);
+  k_argmax<<<cdiv(n, 256), 256, 0, st>>>(G, n, labels, pred);
   return cudaGetLastError();
 }
 

@@ -94,7 +94,7 @@ cudaError_t launch_expand(const float* base, int ldbase, const float* cols, cons
                           const float* bias, int n, int N, void* H, int ldh, bool h_bf16,
                           float* s_next, float* G_acc /*null unless single layer*/, int* err,
                           cudaStream_t st);
-cudaError_t launch_argmax(const float* G, int n, int* pred, float* goodness_out, cudaStream_t st);
+cudaError_t launch_argmax(const float* G, int n, const int* labels, int* pred, cudaStream_t st);
 // one bounded wait on an mbarrier nothing arrives on (latches DEVERR_TIMEOUT)
 cudaError_t launch_wait_selftest(int* err, unsigned long long timeout_ns, cudaStream_t st);
 

@@ -63,6 +63,7 @@ def lib():
             "ff_layer_train_step": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p,
                                     c_void_p, c_void_p],
             "ff_predict": [c_void_p, c_int, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
+            "ff_adaptive_negatives": [c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
             "ff_layer_get_state": [c_void_p] + [c_void_p] * 6 + [POINTER(c_longlong)],
             "ff_layer_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
@@ -248,6 +249,22 @@ def predict(layers, x, pred=None, goodness=None, stream=None):
     _check(lib().ff_predict(arr, len(layers), _ptr(x, torch.float32, "x"), n, _ptr(pred, torch.int32, "pred"),
                             _ptr(goodness, torch.float32, "goodness"), c_void_p(_stream(stream))), "ff_predict")
     return pred, goodness
+
+
+def adaptive_negatives(layers, x, labels, neg=None, goodness=None, stream=None):
+    """ff_adaptive_negatives: AdaptiveNEG negative labels (§5), each sample's
+    strongest wrong label under goodness prediction.  Returns (neg, goodness)."""
+    n = x.shape[0]
+    if labels.shape[0] != n:
+        raise ValueError("labels must have one entry per row of x")
+    if neg is None:
+        neg = torch.empty(n, dtype=torch.int32, device=x.device)
+    arr = (c_void_p * len(layers))(*[l.handle.value for l in layers])
+    _check(lib().ff_adaptive_negatives(arr, len(layers), _ptr(x, torch.float32, "x"),
+                                       _ptr(labels, torch.int32, "labels"), n, _ptr(neg, torch.int32, "neg"),
+                                       _ptr(goodness, torch.float32, "goodness"), c_void_p(_stream(stream))),
+           "ff_adaptive_negatives")
+    return neg, goodness
 
 
 class Net:

@@ -260,6 +260,54 @@ def test_predict(env, prec, dims, n):
     assert_close(G.cpu().numpy(), plain_G, 1e-4 if not emul else 2e-2, 1e-4, "predict goodness vs fp64")
 
 
+# ------------------------------------------------ AdaptiveNEG negatives (§5)
+@pytest.mark.parametrize("prec,dims,n", [("fp32", (784, 256, 256, 128), 300), ("bf16", (784, 256, 256, 128), 300),
+                                         ("bf16", (784, 96), 40), ("bf16", (784, 200, 128), 9000)])
+def test_adaptive_negatives(env, prec, dims, n):
+    torch, ff = env
+    layers, states = [], []
+    for i in range(len(dims) - 1):
+        W, b = _rand_layer_state(dims[i + 1], dims[i], seed=50 + i, bias_scale=0.02)
+        l = ff.Layer(dims[i], dims[i + 1], prec=prec)
+        l.set_state(W=W, b=b)
+        layers.append(l)
+        states.append(fo.LayerState(W, b))
+    x = synth.mnist_like(n, seed=51)
+    y = synth.labels(n, seed=52)
+    G = torch.empty(n, 10, device="cuda")
+    neg, _ = ff.adaptive_negatives(layers, torch.from_numpy(x).cuda(), torch.from_numpy(y).cuda(), goodness=G)
+    torch.cuda.synchronize()
+    layers[0].check()
+    g = G.cpu().numpy()
+    p = neg.cpu().numpy()
+    # the kernel's choice is exactly the masked argmax of its own goodness
+    own = g.copy()
+    own[np.arange(n), y] = -np.inf
+    assert np.array_equal(p, np.argmax(own, axis=1))
+    assert not np.any(p == y)
+    emul = prec == "bf16"
+    rn, rG = fo.adaptive_negatives(states, x, y, emulate_bf16=emul)
+    assert_close(g, rG, 1e-4 if not emul else 2e-3, 1e-6, "adaptive-negative goodness")
+    assert np.mean(p == rn) >= 0.995
+    for i in np.nonzero(p != rn)[0]:   # disagreements only at near ties
+        gap = abs(rG[i, p[i]] - rG[i, rn[i]])
+        assert gap <= (1e-4 if not emul else 1e-2) * abs(rG[i, rn[i]]), (i, gap)
+
+
+def test_adaptive_negatives_label_outside_range_is_plain_prediction(env):
+    torch, ff = env
+    layers = [ff.Layer(784, 128, prec="bf16", init_seed=60), ff.Layer(128, 128, prec="bf16", init_seed=61)]
+    x = torch.from_numpy(synth.mnist_like(64, seed=62)).cuda()
+    y = torch.full((64,), -1, dtype=torch.int32, device="cuda")
+    y[::2] = 10
+    neg, _ = ff.adaptive_negatives(layers, x, y)
+    pred, _ = ff.predict(layers, x)
+    torch.cuda.synchronize()
+    assert torch.equal(neg, pred)
+    empty = torch.empty(0, 784, device="cuda")
+    ff.adaptive_negatives(layers, empty, torch.empty(0, dtype=torch.int32, device="cuda"))
+
+
 # ----------------------------------------------- multi-stream net == sequential
 def test_net_on_streams_is_bitwise_sequential(env):
     torch, ff = env
