@@ -448,6 +448,24 @@ def run_other(args):
                     "unit": "samples/s", "ms_per_step": round(ms, 4), "dtype": prec, "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4) if prec == "bf16" else None,
                     "config": {"workload": f"ff_predict_784-2000x4_{prec}_n10000", "algorithmic_tflop": flops / 1e12}})
+    elif w == "adaptive_neg":
+        # AdaptiveNEG refresh of one chapter: the strongest wrong label of all
+        # 60 000 training samples under goodness prediction through 784-2000x4
+        n = PAIRS_PER_EPOCH
+        layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", init_seed=1000 + k) for k in range(len(NET) - 1)]
+        x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
+        y = torch.from_numpy(synth.labels(n, seed=7)).to(dev)
+        neg = torch.empty(n, dtype=torch.int32, device=dev)
+        fn = lambda: ff.adaptive_negatives(layers, x, y, neg=neg, stream=stream)
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        flops = 2.0 * n * NET[1] * NET[0] + 3 * 2.0 * 10 * n * NET[2] * NET[1]
+        tf = flops / (ms / 1e3) / 1e12
+        out.update({"metric": "AdaptiveNEG negative labels/s (10 label overlays) on 4x2000 net",
+                    "value": round(n / (ms / 1e3), 1), "unit": "samples/s", "ms_per_step": round(ms, 4),
+                    "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
+                    "config": {"workload": f"ff_adaptive_neg_784-2000x4_bf16_n{n}",
+                               "algorithmic_tflop": flops / 1e12}})
     elif w == "pipeline_5x2000":
         # 784-2000x5, 60 chunks of 1000 pairs; 5 layer streams vs the same steps on one stream
         net5 = [784] + [2000] * 5
@@ -567,8 +585,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="train_4x2000",
-                    choices=["train_4x2000", "predict_bf16", "predict_fp32", "pipeline_5x2000", "wide_4x8192",
-                             "tiny_fp32"])
+                    choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "pipeline_5x2000",
+                             "wide_4x8192", "tiny_fp32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")

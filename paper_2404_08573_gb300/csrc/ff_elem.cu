@@ -298,45 +298,50 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
 }
 
 // --------------------------------------------------------------------- Adam
-__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float lr, float b1, float b2, float eps,
-                                      float bc1, float bc2) {
+// One Adam step of one parameter.  a1 = lr / (1 - beta1^t) and
+// r2 = 1 / (1 - beta2^t) are formed once per thread, so the update
+// lr * (m / bc1) / (sqrt(v / bc2) + eps) costs one division per parameter
+// instead of three (the kernel is otherwise limited by those divisions, not
+// by HBM).
+__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float a1, float b1, float b2, float eps,
+                                      float r2) {
   m = b1 * m + (1.f - b1) * g;
   v = b2 * v + (1.f - b2) * g * g;
-  const float mh = m / bc1;
-  const float vh = v / bc2;
-  w -= lr * mh / (sqrtf(vh) + eps);
+  w -= a1 * m / (sqrtf(v * r2) + eps);
 }
 
 __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
-  const float bc1 = a.ds->bc1, bc2 = a.ds->bc2;
+  const float a1 = a.lr / a.ds->bc1, r2 = 1.f / a.ds->bc2;
   if ((int)blockIdx.x < w_blocks) {
     const long long total = (long long)a.N * a.K;
     const long long stride = (long long)w_blocks * 256;
     if ((a.K & 3) == 0) {
+      // bf16 copy addressed like W when its rows are not padded
+      const bool dense_b = a.ldb == a.K;
       for (long long q = (long long)blockIdx.x * 256 + threadIdx.x; q * 4 < total; q += stride) {
         const long long idx = q * 4;
         float4 w = *reinterpret_cast<float4*>(a.W + idx);
         float4 m = *reinterpret_cast<float4*>(a.mW + idx);
         float4 v = *reinterpret_cast<float4*>(a.vW + idx);
         const float4 g = *reinterpret_cast<const float4*>(a.dW + idx);
-        adam1(w.x, m.x, v.x, g.x, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
-        adam1(w.y, m.y, v.y, g.y, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
-        adam1(w.z, m.z, v.z, g.z, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
-        adam1(w.w, m.w, v.w, g.w, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        adam1(w.x, m.x, v.x, g.x, a1, a.beta1, a.beta2, a.eps, r2);
+        adam1(w.y, m.y, v.y, g.y, a1, a.beta1, a.beta2, a.eps, r2);
+        adam1(w.z, m.z, v.z, g.z, a1, a.beta1, a.beta2, a.eps, r2);
+        adam1(w.w, m.w, v.w, g.w, a1, a.beta1, a.beta2, a.eps, r2);
         *reinterpret_cast<float4*>(a.W + idx) = w;
         *reinterpret_cast<float4*>(a.mW + idx) = m;
         *reinterpret_cast<float4*>(a.vW + idx) = v;
         if (a.Wb) {
-          const long long n = idx / a.K, k = idx % a.K;
+          const long long o = dense_b ? idx : (idx / a.K) * a.ldb + idx % a.K;
           __nv_bfloat162 p0 = __floats2bfloat162_rn(w.x, w.y), p1 = __floats2bfloat162_rn(w.z, w.w);
           uint2 u = make_uint2(*reinterpret_cast<uint32_t*>(&p0), *reinterpret_cast<uint32_t*>(&p1));
-          *reinterpret_cast<uint2*>(a.Wb + n * a.ldb + k) = u;
+          *reinterpret_cast<uint2*>(a.Wb + o) = u;
         }
       }
     } else {
       for (long long idx = (long long)blockIdx.x * 256 + threadIdx.x; idx < total; idx += stride) {
         float w = a.W[idx], m = a.mW[idx], v = a.vW[idx];
-        adam1(w, m, v, a.dW[idx], a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+        adam1(w, m, v, a.dW[idx], a1, a.beta1, a.beta2, a.eps, r2);
         a.W[idx] = w;
         a.mW[idx] = m;
         a.vW[idx] = v;
@@ -380,7 +385,7 @@ __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
     if (a.db_out) a.db_out[j] = db;
     if (a.has_bias) {
       float b = a.b[j], m = a.mb[j], v = a.vb[j];
-      adam1(b, m, v, db, a.lr, a.beta1, a.beta2, a.eps, bc1, bc2);
+      adam1(b, m, v, db, a1, a.beta1, a.beta2, a.eps, r2);
       a.b[j] = b;
       a.mb[j] = m;
       a.vb[j] = v;
