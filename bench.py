@@ -279,33 +279,55 @@ def run_ours(args):
     final_loss = loss[-1].cpu().numpy().tolist()
     value, ms = replica_throughput(ms, PAIRS_PER_EPOCH * args.steps, world, dist)
 
-    # end to end through the public API: pinned host batches copied in per batch
+    # end to end through the public API: pinned host batches copied in per
+    # batch on a copy stream, RING batches ahead of the layer that reads them
     e2e = None
     if not args.no_e2e:
         Xp = torch.from_numpy(X_h).pin_memory()
         Lp = torch.from_numpy(L_h).pin_memory()
-        xbuf = [torch.empty(2 * BATCH, NET[0], device=dev) for _ in range(2)]
-        lbuf = [torch.empty(2 * BATCH, dtype=torch.int32, device=dev) for _ in range(2)]
+        RING = 3
+        xbuf = [torch.empty(2 * BATCH, NET[0], device=dev) for _ in range(RING)]
+        lbuf = [torch.empty(2 * BATCH, dtype=torch.int32, device=dev) for _ in range(RING)]
+        copied = [torch.cuda.Event() for _ in range(RING)]
+        freed = [torch.cuda.Event() for _ in range(RING)]
+        cstream = torch.cuda.Stream(device=dev)
         loss_h = torch.empty(len(layers), pin_memory=True)
 
-        def xsrc(t, r0, b):
-            xbuf[t % 2][:2 * b].copy_(Xp[r0:r0 + 2 * b], non_blocking=True)
-            return xbuf[t % 2][:2 * b]
-
-        def lsrc(t, r0, b):
-            lbuf[t % 2][:2 * b].copy_(Lp[r0:r0 + 2 * b], non_blocking=True)
-            return lbuf[t % 2][:2 * b]
-
-        with torch.cuda.stream(stream):
-            epoch(xsrc, lsrc)
+        def epoch_e2e():
+            def fetch(t):
+                start, b = bl[t]
+                r0 = 2 * start
+                j = t % RING
+                with torch.cuda.stream(cstream):
+                    cstream.wait_event(freed[j])      # the step that last read slot j is past layer 1
+                    xbuf[j][:2 * b].copy_(Xp[r0:r0 + 2 * b], non_blocking=True)
+                    lbuf[j][:2 * b].copy_(Lp[r0:r0 + 2 * b], non_blocking=True)
+                    copied[j].record(cstream)
+            begin = torch.cuda.Event()
+            begin.record(stream)
+            cstream.wait_event(begin)             # no copy starts before the step does
+            for t in range(min(RING - 1, len(bl))):
+                fetch(t)
+            for t, (start, b) in enumerate(bl):
+                if t + RING - 1 < len(bl):
+                    fetch(t + RING - 1)
+                j = t % RING
+                stream.wait_event(copied[j])
+                net.train_step(xbuf[j][:2 * b], lbuf[j][:2 * b], B=b, loss=loss[t], stream=stream)
+                freed[j].record(stream)  # ff_net_train_step returns with `stream` ordered after layer 1 read x
+            net.sync(stream)
             loss_h.copy_(loss[-1], non_blocking=True)
+
+        for j in range(RING):
+            freed[j].record(stream)
+        with torch.cuda.stream(stream):
+            epoch_e2e()
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
             e0.record(stream)
             for _ in range(args.steps):
-                epoch(xsrc, lsrc)
-                loss_h.copy_(loss[-1], non_blocking=True)
+                epoch_e2e()
             e1.record(stream)
         barrier()
         e2e_value, ems = replica_throughput(e0.elapsed_time(e1), PAIRS_PER_EPOCH * args.steps, world, dist)

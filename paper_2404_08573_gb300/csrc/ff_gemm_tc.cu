@@ -15,6 +15,9 @@
 //   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
 //               N=BN, K=16; one per row subtile, sharing the B stage) and
 //               commits each stage back to the producer
+// In pair mode two CTAs (a cluster of 2 along x) run as one cta_group::2
+// unit: each loads its own A rows and half of B, the even CTA's MMA warp
+// issues M=256 MMAs over both, and each CTA's epilogue reads its own TMEM.
 //   warps 2..9  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).., one half of
 //               the columns each -> registers, fused scale/bias/ReLU/goodness
 //               (partials per 128-column half) or plain store
@@ -38,10 +41,11 @@ constexpr int NTHREADS = 64 + 32 * EPI_WARPS;  // producer warp, MMA warp, epilo
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
 
-template <int BN, int NSTAGE, int MT>
+template <int BN, int NSTAGE, int MT, bool PAIR>
 struct TcCfg {
   static constexpr int A_BYTES = MT * BM * BK * 2;  // MT row subtiles of BM rows
-  static constexpr int B_BYTES = BN * BK * 2;
+  static constexpr int BH = PAIR ? BN / 2 : BN;     // B columns this CTA loads
+  static constexpr int B_BYTES = BH * BK * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int STAGES = NSTAGE;
   static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
@@ -53,6 +57,7 @@ struct TcCfg {
   static_assert(MT * 4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
   static_assert(EPI_WARPS * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
   static_assert(BN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
+  static_assert(!PAIR || BH % 64 == 0, "each CTA of a pair loads whole 64-column B groups");
   static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
 };
 
@@ -61,11 +66,11 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
   atomicOr(err, DEVERR_TIMEOUT);
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE, int MT>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
 __global__ void __launch_bounds__(NTHREADS, 1)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
-  using C = TcCfg<BN, NSTAGE, MT>;
+  using C = TcCfg<BN, NSTAGE, MT, PAIR>;
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -82,20 +87,28 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
-  const int m0 = blockIdx.y * (BM * MT);
-  const int n0 = blockIdx.x * BN;
+  // blockIdx.x: row tile (the two CTAs of a pair are consecutive in x, as
+  // cta_group::2 requires); blockIdx.y: column tile
+  const int m0 = blockIdx.x * (BM * MT);
+  const int n0 = blockIdx.y * BN;
   const int num_kb = (K + BK - 1) / BK;
 
-  // CM > 1: the CM CTAs of a cluster (consecutive tile rows, same columns)
-  // share the B tile; CTA `crank` loads B rows [crank*BN/CM, (crank+1)*BN/CM)
-  // and multicasts them, and a stage is refilled only after all CM CTAs have
-  // consumed it (their MMA warps arrive on every CTA's `empty`).
-  const uint32_t crank = CM > 1 ? ptx::cluster_ctarank() : 0u;
-  constexpr uint16_t cmask = (uint16_t)((1u << CM) - 1u);
+  // PAIR: the two CTAs of a cluster (consecutive tile rows, same columns)
+  // compute their 2 x MT x BM rows with cta_group::2 MMAs (M = 256).  Each
+  // CTA loads its own A rows and half of the B tile (columns crank*BN/2 ..);
+  // with one 128-row subtile a CTA moves 32 KB per 64-deep K step for
+  // 4.2 MFLOP instead of 48 KB for the same tile alone.  The
+  // even CTA issues the MMAs once both halves of a stage have landed (the odd
+  // CTA's copies complete on the even CTA's `full` barrier) and its commits
+  // arrive on both CTAs' `empty` and `tfull` barriers.
+  uint32_t crank = 0;
+  if constexpr (PAIR) crank = ptx::cluster_ctarank();
+  const bool issuer = !PAIR || crank == 0;
+  constexpr uint16_t pmask = 3;
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       ptx::mbar_init(&full[s], 1);
-      ptx::mbar_init(&empty[s], CM);
+      ptx::mbar_init(&empty[s], 1);
     }
     ptx::mbar_init(tfull, 1);
     *abort_flag = 0;
@@ -106,18 +119,33 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     if (MODE == MODE_FWD || tma_store) ptx::prefetch_tmap(&tmC);
   }
   if (warp == 1) {
-    ptx::tmem_alloc(tslot, C::TMEM_COLS);
-    ptx::tmem_relinquish();
+    if constexpr (PAIR) {
+      ptx::tmem_alloc_pair(tslot, C::TMEM_COLS);
+      ptx::tmem_relinquish_pair();
+    } else {
+      ptx::tmem_alloc(tslot, C::TMEM_COLS);
+      ptx::tmem_relinquish();
+    }
   }
   ptx::tc_fence_before();
   __syncthreads();
-  if (CM > 1) ptx::cluster_sync();  // every CTA's barriers exist before any multicast
+  if constexpr (PAIR) ptx::cluster_sync();  // both CTAs' barriers and TMEM exist before any cross-CTA use
   ptx::tc_fence_after();
   const uint32_t tmem = *tslot;
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
     if (lane == 0) {
+      // the stage barriers the copies complete on: the issuing CTA's
+      uint32_t full0 = ptx::smem_u32(&full[0]);
+      if constexpr (PAIR) full0 = ptx::mapa_shared(full0, 0u);
+      auto load = [&](void* dst, const CUtensorMap* map, int s, int c0, int c1) {
+        if constexpr (PAIR)
+          ptx::tma_load_2d_pair(dst, map, full0 + 8u * (uint32_t)s, c0, c1);
+        else
+          ptx::tma_load_2d(dst, map, &full[s], c0, c1);
+      };
+      const int nb = n0 + (int)crank * C::BH;  // first B column this CTA loads
       int issued = 0;
       for (int kb = 0; kb < num_kb; ++kb) {
         const int s = kb % C::STAGES;
@@ -126,43 +154,28 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           latch(err, abort_flag);
           break;
         }
-        ptx::mbar_arrive_expect_tx(&full[s], C::STAGE);
+        if (issuer) ptx::mbar_arrive_expect_tx(&full[s], PAIR ? 2 * C::STAGE : C::STAGE);
         uint8_t* a = sA + s * C::A_BYTES;
         uint8_t* b = sB + s * C::B_BYTES;
         const int k0 = kb * BK;
         if (!A_MN) {
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt) ptx::tma_load_2d(a + mt * BM * BK * 2, &tmA, &full[s], k0, m0 + BM * mt);
+          for (int mt = 0; mt < MT; ++mt) load(a + mt * BM * BK * 2, &tmA, s, k0, m0 + BM * mt);
         } else {
 #pragma unroll
-          for (int j = 0; j < MT * BM / 64; ++j)
-            ptx::tma_load_2d(a + j * 64 * BK * 2, &tmA, &full[s], m0 + 64 * j, k0);
+          for (int j = 0; j < MT * BM / 64; ++j) load(a + j * 64 * BK * 2, &tmA, s, m0 + 64 * j, k0);
         }
-        if (CM == 1) {
-          if (!B_MN) {
-            ptx::tma_load_2d(b, &tmB, &full[s], k0, n0);
-          } else {
-#pragma unroll
-            for (int j = 0; j < BN / 64; ++j) ptx::tma_load_2d(b + j * 64 * BK * 2, &tmB, &full[s], n0 + 64 * j, k0);
-          }
+        if (!B_MN) {
+          load(b, &tmB, s, k0, nb);
         } else {
-          // this CTA's slice of B: BN/CM rows (K-major) or BN/CM columns (MN-major)
-          constexpr int SL = BN / CM;
-          if (!B_MN) {
-            ptx::tma_load_2d_mc(b + crank * SL * 128, &tmB, &full[s], k0, n0 + (int)crank * SL, cmask);
-          } else {
 #pragma unroll
-            for (int j = 0; j < SL / 64; ++j) {
-              const int jj = (int)crank * (SL / 64) + j;
-              ptx::tma_load_2d_mc(b + jj * 64 * BK * 2, &tmB, &full[s], n0 + 64 * jj, k0, cmask);
-            }
-          }
+          for (int j = 0; j < C::BH / 64; ++j) load(b + j * 64 * BK * 2, &tmB, s, nb + 64 * j, k0);
         }
         issued = kb + 1;
       }
-      if (CM > 1 && !*abort_flag) {
-        // Producer tail: wait until every CTA of the cluster has released every
-        // stage, so no remote arrival targets this CTA after it exits.
+      if (PAIR && !*abort_flag) {
+        // Producer tail: wait for the commits of the last stages, so that no
+        // arrival from the other CTA targets this one after it exits.
         for (int kb = num_kb; kb < num_kb + C::STAGES; ++kb) {
           if (!ptx::mbar_wait(&empty[kb % C::STAGES], ((uint32_t)(kb / C::STAGES) & 1u) ^ 1u, kWaitTimeoutNs,
                               abort_flag)) {
@@ -172,17 +185,25 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         }
       }
       if (*abort_flag) {
-        // let copies already issued land before the CTA's shared memory goes away
-        int lo = issued - C::STAGES;
-        if (lo < 0) lo = 0;
-        for (int kb = lo; kb < issued; ++kb)
-          ptx::mbar_wait(&full[kb % C::STAGES], (uint32_t)(kb / C::STAGES) & 1u, 10000000ull, never_set);
+        if (issuer) {
+          // let copies already issued land before the CTA's shared memory goes away
+          int lo = issued - C::STAGES;
+          if (lo < 0) lo = 0;
+          for (int kb = lo; kb < issued; ++kb)
+            ptx::mbar_wait(&full[kb % C::STAGES], (uint32_t)(kb / C::STAGES) & 1u, 10000000ull, never_set);
+        } else {
+          // this CTA's copies complete on the other CTA's barrier: give them
+          // time to land
+          const uint64_t t0 = ptx::globaltimer();
+          while (ptx::globaltimer() - t0 < 1000000ull) {
+          }
+        }
       }
     }
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
-    if (lane == 0) {
-      constexpr uint32_t idesc = ptx::idesc_bf16_f32(BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+    if (lane == 0 && issuer) {
+      constexpr uint32_t idesc = ptx::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
       for (int kb = 0; kb < num_kb; ++kb) {
         const int s = kb % C::STAGES;
         const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
@@ -207,15 +228,22 @@ __global__ void __launch_bounds__(NTHREADS, 1)
             const uint32_t as = a_base + mt * BM * BK * 2;
             const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
                                      : ptx::sdesc_sw128(as + k * 32, 16, 1024);
-            ptx::umma_f16(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            if constexpr (PAIR)
+              ptx::umma_f16_pair(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            else
+              ptx::umma_f16(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
           }
         }
-        if (CM == 1)
-          ptx::umma_commit(&empty[s]);
+        if constexpr (PAIR)
+          ptx::umma_commit_pair(&empty[s], pmask);
         else
-          ptx::umma_commit_mc(&empty[s], cmask);
+          ptx::umma_commit(&empty[s]);
       }
-      ptx::umma_commit(tfull);  // always: the epilogue and the teardown wait on it
+      // always: the epilogues and the teardown wait on it
+      if constexpr (PAIR)
+        ptx::umma_commit_pair(tfull, pmask);
+      else
+        ptx::umma_commit(tfull);
     }
   } else {
     // ------------------------------------------------------------ epilogue
@@ -328,7 +356,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
           process(rb, c0 + 32);
           ptx::tmem_ld_wait();
         }
-        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)(blockIdx.x * HALVES + half) * M + gi] = g;
+        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
         if (MODE == MODE_FWD) {
           ptx::fence_async_smem();
           __syncwarp();
@@ -351,15 +379,18 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 
   ptx::tc_fence_before();
   __syncthreads();
+  if constexpr (PAIR) ptx::cluster_sync();  // both CTAs are done with the pair's TMEM and barriers
   ptx::tc_fence_after();
   if (warp == 1) {
     if (*abort_flag) {
       // MMAs issued before the abort must finish before TMEM is released
       ptx::mbar_wait(tfull, 0, 10000000ull, never_set);
     }
-    ptx::tmem_dealloc(tmem, C::TMEM_COLS);
+    if constexpr (PAIR)
+      ptx::tmem_dealloc_pair(tmem, C::TMEM_COLS);
+    else
+      ptx::tmem_dealloc(tmem, C::TMEM_COLS);
   }
-  if (CM > 1) ptx::cluster_sync();  // no CTA leaves while a peer may still address it
 }
 
 PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
@@ -393,24 +424,25 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
              CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, int CM, int NSTAGE, int MT>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st) {
-  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, CM, NSTAGE, MT>;
-  static cudaError_t attr =
-      cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, TcCfg<BN, NSTAGE, MT>::SMEM);
+  using C = TcCfg<BN, NSTAGE, MT, PAIR>;
+  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT>;
+  static cudaError_t attr = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg = {};
-  // tile rows padded to a whole number of clusters; padding CTAs load zeros,
-  // share their B slice and write nothing
-  cfg.gridDim = dim3(cdiv(N, BN), cdiv(cdiv(M, BM * MT), CM) * CM, 1);
+  // tile rows padded to whole pairs; a padding CTA loads zeros, supplies its
+  // half of B and writes nothing
+  constexpr int CM = PAIR ? 2 : 1;
+  cfg.gridDim = dim3(cdiv(cdiv(M, BM * MT), CM) * CM, cdiv(N, BN), 1);
   cfg.blockDim = dim3(NTHREADS, 1, 1);
-  cfg.dynamicSmemBytes = TcCfg<BN, NSTAGE, MT>::SMEM;
+  cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[1];
   at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = 1;
-  at[0].val.clusterDim.y = CM;
+  at[0].val.clusterDim.x = CM;
+  at[0].val.clusterDim.y = 1;
   at[0].val.clusterDim.z = 1;
   cfg.attrs = at;
   cfg.numAttrs = 1;
@@ -419,17 +451,20 @@ cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtens
 
 constexpr int FWD_BN = 256;
 constexpr int WGRAD_BN = 256;
-// Measured on the 784-2000x4 train step with the layers on 4 streams (epoch):
-//   128x256 tile, 4-stage ring, 4-CTA multicast clusters ....... 11.1 ms
-//   128x256 tile, 2-stage ring (two CTAs per SM), no clusters ..  9.8 ms
-//   256x256 tile (two 128-row accumulators sharing each B stage),
-//   3-stage ring (192 KB, one CTA per SM), no clusters .........  9.1 ms
-// The step is bound by moving operand tiles into shared memory, so the
-// 256x256 tile's third fewer bytes per FLOP wins; clusters constrain
-// co-scheduling with the other layers' kernels and did not pay.
-constexpr int CLUSTER_M = 1;     // CTAs per cluster along M sharing one B tile
+// Tile configuration: CTA pairs (cta_group::2) with two 128-row subtiles per
+// CTA, so a pair computes a 512 x 256 tile; per 64-deep K step a CTA loads
+// 48 KB of operands (its 256 A rows, half of B) for 8.4 MFLOP.  Measured on
+// the 784-2000x4 train step with the layers on 4 streams (epoch, ms):
+//   single CTA 256 x 256 (two subtiles), 3-stage ring ........... 9.30
+//   pairs, one subtile per CTA (128 CTAs per GEMM), 6 / 4 stages  9.90 / 10.52
+//   pairs, two subtiles per CTA (64 CTAs per GEMM), 4 / 3 stages  9.05 / 8.78
+// With 128 CTAs a GEMM alone is faster (20 vs 29 us for 2048x2000x2000) but
+// two layers' GEMMs no longer fit on the GPU side by side; earlier 128 x 256
+// tiles and 4-CTA multicast clusters measured 9.8 and 11.1 ms.
+constexpr bool USE_PAIR = true;
 constexpr int NSTAGES = 3;       // operand ring depth
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
+constexpr int B_BOX_ROWS = USE_PAIR ? FWD_BN / 2 : FWD_BN;
 
 }  // namespace
 
@@ -445,10 +480,10 @@ int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN) * (EPI_WARPS / 4); }  // goodn
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
                         int* err, cudaStream_t st) {
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M) ||
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, B_BOX_ROWS) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
-  return launch_tc<FWD_BN, false, false, MODE_FWD, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
 }
 
 // fp32 C written through shared memory and TMA when its rows are 16-byte
@@ -460,12 +495,12 @@ static bool store_map(CUtensorMap* tc, float* C, int ldc, int rows, int cols) {
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, float* Cm,
                           int ldc, int* err, cudaStream_t st) {
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, FWD_BN / CLUSTER_M))
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, B_BOX_ROWS))
     return cudaErrorInvalidValue;
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<FWD_BN, false, false, MODE_STORE, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
 }
 
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K, float* Cm, int ldc,
@@ -478,7 +513,7 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  return launch_tc<WGRAD_BN, true, true, MODE_STORE, CLUSTER_M, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
+  return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
 }
 
 }  // namespace ff
