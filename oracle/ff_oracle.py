@@ -33,6 +33,12 @@ What each function follows:
 * ``adaptive_negatives`` -- AdaptiveNEG of §5: the negative label of a sample
   is the incorrect label the network currently predicts most strongly, i.e.
   the goodness-prediction argmax over the 9 wrong labels.
+* ``overlay_neutral``/``softmax_features``/``head_*`` -- §3 "Prediction",
+  Softmax method: the input carries a neutral label (0.1 in each of the 10
+  label features), the activities of all but the first hidden layer feed a
+  linear softmax layer trained by backpropagation through that layer only
+  (cross-entropy, Adam with the head's own learning rate, §5.1); the
+  prediction is the class with the largest logit.
 
 Readings of points the paper leaves open (the paper states none of them):
 
@@ -46,6 +52,10 @@ Readings of points the paper leaves open (the paper states none of them):
    the lowest label.
 7. The layer input fed to the next layer is the ReLU activity computed with
    the pre-update weights of the same step.
+8. Softmax head: its input is the concatenation, over layers 2..L (layer 1
+   when L == 1), of each layer's activity normalised like a layer input,
+   h / max(||h||, 1e-12); cross-entropy averaged over the rows; weights and
+   biases start at zero; ties of the logits go to the lowest class.
 
 ``emulate_bf16=True`` rounds (round-to-nearest-even) the operands that the
 bf16-operand mode stores in bfloat16 -- the layer's input activity, W, the
@@ -287,4 +297,102 @@ def adaptive_negatives(states, x_raw, labels, emulate_bf16: bool = False, n_clas
     masked = G.copy()
     masked[np.arange(G.shape[0]), labels] = -np.inf
     return np.argmax(masked, axis=1), G
+
+
+# --------------------------------------------------------- softmax head (§3)
+NEUTRAL_LABEL = 0.1
+
+
+def overlay_neutral(x, n_classes: int = N_CLASSES, value: float = NEUTRAL_LABEL):
+    """§3 Softmax prediction: the unlabelled input gets the neutral label,
+    ``value`` (0.1) in each of the 10 label features (written, as the overlay)."""
+    out = np.array(x, dtype=np.float64, copy=True)
+    out[:, :n_classes] = value
+    return out
+
+
+def softmax_features(states, x_raw, emulate_bf16: bool = False):
+    """§3 Softmax prediction: run the neutral-labelled input through every
+    layer and concatenate the normalised activities of layers 2..L (layer 1
+    when L == 1).  In bf16 mode the stored activity is rounded and its scale
+    comes from the unrounded goodness, as the layers hand it on."""
+    a = overlay_neutral(x_raw)
+    L = len(states)
+    feats = []
+    for k, st in enumerate(states):
+        f = layer_forward_full(st, a, emulate_bf16=emulate_bf16)
+        if k >= 1 or L == 1:
+            h = bf16_round(f["H"]) if emulate_bf16 else f["H"]
+            scale = 1.0 / np.maximum(np.sqrt(f["g"]), NORM_EPS)
+            feats.append(scale[:, None] * h)
+        a = f["H"]
+    return np.concatenate(feats, axis=1)
+
+
+@dataclass
+class HeadState:
+    V: np.ndarray          # [classes, features]
+    c: np.ndarray          # [classes]
+    mV: np.ndarray = None
+    vV: np.ndarray = None
+    mc: np.ndarray = None
+    vc: np.ndarray = None
+    t: int = 0
+
+    def __post_init__(self):
+        self.V = np.array(self.V, dtype=np.float64)
+        self.c = np.array(self.c, dtype=np.float64)
+        for name, like in (("mV", self.V), ("vV", self.V), ("mc", self.c), ("vc", self.c)):
+            v = getattr(self, name)
+            setattr(self, name, np.zeros_like(like) if v is None else np.array(v, dtype=np.float64))
+
+
+def head_logits(A, V, c):
+    """z = A V^T + c."""
+    return np.asarray(A, dtype=np.float64) @ np.asarray(V, dtype=np.float64).T + np.asarray(c, dtype=np.float64)
+
+
+def softmax(z):
+    z = np.asarray(z, dtype=np.float64)
+    e = np.exp(z - np.max(z, axis=1, keepdims=True))
+    return e / np.sum(e, axis=1, keepdims=True)
+
+
+def cross_entropy(z, labels):
+    """Mean over rows of -log softmax(z)[label] = logsumexp(z) - z[label]."""
+    z = np.asarray(z, dtype=np.float64)
+    labels = np.asarray(labels, dtype=np.int64)
+    m = np.max(z, axis=1)
+    lse = m + np.log(np.sum(np.exp(z - m[:, None]), axis=1))
+    return float(np.mean(lse - z[np.arange(z.shape[0]), labels]))
+
+
+def dce_dz(z, labels):
+    """d(cross_entropy)/dz = (softmax(z) - onehot(label)) / n."""
+    p = softmax(z)
+    n = p.shape[0]
+    p[np.arange(n), np.asarray(labels, dtype=np.int64)] -= 1.0
+    return p / n
+
+
+def head_train_step(head: HeadState, A, labels, hp: AdamHyper):
+    """One backpropagation step of the softmax layer alone (the gradient does
+    not reach the FF layers); Adam on V and c.  Mutates ``head``."""
+    A = np.asarray(A, dtype=np.float64)
+    z = head_logits(A, head.V, head.c)
+    loss = cross_entropy(z, labels)
+    dz = dce_dz(z, labels)
+    dV = dz.T @ A
+    dc = np.sum(dz, axis=0)
+    head.t += 1
+    head.V, head.mV, head.vV = adam_update(head.V, dV, head.mV, head.vV, head.t, hp)
+    head.c, head.mc, head.vc = adam_update(head.c, dc, head.mc, head.vc, head.t, hp)
+    return dict(z=z, loss=loss, dz=dz, dV=dV, dc=dc)
+
+
+def head_predict(head: HeadState, A):
+    """The class with the largest logit (the lowest class on ties).
+    Returns (pred [n] int64, z [n, classes])."""
+    z = head_logits(A, head.V, head.c)
+    return np.argmax(z, axis=1), z
 

@@ -359,3 +359,131 @@ def test_adaptive_negatives_are_the_strongest_wrong_label():
     neg, _ = fo.adaptive_negatives(st, xx, np.full(6, 3))
     assert np.all(neg == 7)
 
+
+
+# ------------------------------------------------------- softmax head (§3)
+def _brute_features(Ws, bs, x, n_classes=10):
+    """Pure-Python loops: neutral label (0.1 in each label feature), normalise,
+    ReLU layers; each of layers 2..L (layer 1 if L == 1) contributes its
+    activity divided by its own norm."""
+    out = []
+    L = len(Ws)
+    for row in x:
+        a = [0.1] * n_classes + [float(v) for v in row[n_classes:]]
+        feats = []
+        for k in range(L):
+            nrm = max(math.sqrt(sum(v * v for v in a)), 1e-12)
+            xh = [v / nrm for v in a]
+            W, b = Ws[k], bs[k]
+            h = []
+            for i in range(len(b)):
+                z = b[i]
+                for j in range(len(xh)):
+                    z += W[i][j] * xh[j]
+                h.append(z if z > 0 else 0.0)
+            if k >= 1 or L == 1:
+                hn = max(math.sqrt(sum(v * v for v in h)), 1e-12)
+                feats += [v / hn for v in h]
+            a = h
+        out.append(feats)
+    return np.array(out)
+
+
+@pytest.mark.parametrize("dims", [(12, 5), (12, 6, 4), (14, 7, 5, 3)])
+def test_softmax_features_match_brute_force(dims):
+    rng = np.random.default_rng(len(dims))
+    Ws = [rng.standard_normal((dims[i + 1], dims[i])) for i in range(len(dims) - 1)]
+    bs = [rng.standard_normal(dims[i + 1]) * 0.3 for i in range(len(dims) - 1)]
+    x = rng.random((9, dims[0]))
+    x[3] = 0.0                                    # a zero image still carries the neutral label
+    A = fo.softmax_features([fo.LayerState(W, b) for W, b in zip(Ws, bs)], x)
+    ref = _brute_features([W.tolist() for W in Ws], [b.tolist() for b in bs], x)
+    assert A.shape == ref.shape == (9, sum(dims[2:]) if len(dims) > 2 else dims[1])
+    np.testing.assert_allclose(A, ref, rtol=1e-12, atol=1e-14)
+
+
+def test_neutral_overlay_writes_point_one():
+    x = np.arange(24, dtype=np.float64).reshape(2, 12)
+    o = fo.overlay_neutral(x)
+    assert np.all(o[:, :10] == 0.1) and np.array_equal(o[:, 10:], x[:, 10:])
+    assert x[0, 0] == 0.0                          # the input is not modified
+
+
+def test_cross_entropy_closed_forms():
+    y = np.array([0, 3, 9, 9])
+    z0 = np.zeros((4, 10))
+    assert fo.cross_entropy(z0, y) == pytest.approx(math.log(10.0), rel=0, abs=1e-15)
+    dz = fo.dce_dz(z0, y)
+    exp = np.full((4, 10), 0.1 / 4)
+    exp[np.arange(4), y] -= 1.0 / 4
+    np.testing.assert_allclose(dz, exp, rtol=0, atol=1e-17)
+    # a logit margin m on the right class: -log(e^m / (e^m + 9))
+    z = np.zeros((4, 10))
+    z[np.arange(4), y] = 3.0
+    assert fo.cross_entropy(z, y) == pytest.approx(math.log(1.0 + 9.0 * math.exp(-3.0)), rel=1e-14)
+    # shift invariance, probabilities sum to one, gradient rows sum to zero
+    rng = np.random.default_rng(3)
+    z = rng.standard_normal((6, 10)) * 4
+    yy = rng.integers(0, 10, 6)
+    assert fo.cross_entropy(z + 7.5, yy) == pytest.approx(fo.cross_entropy(z, yy), rel=1e-13)
+    np.testing.assert_allclose(fo.softmax(z).sum(axis=1), 1.0, rtol=1e-15)
+    np.testing.assert_allclose(fo.dce_dz(z, yy).sum(axis=1), 0.0, atol=1e-16)
+    # huge logits stay finite (no overflow in the exponent)
+    assert np.isfinite(fo.cross_entropy(z * 1e3, yy))
+
+
+def test_head_gradient_matches_finite_differences():
+    rng = np.random.default_rng(5)
+    n, F = 7, 6
+    A = rng.standard_normal((n, F))
+    y = rng.integers(0, 10, n)
+    V = rng.standard_normal((10, F)) * 0.5
+    c = rng.standard_normal(10) * 0.1
+    z = fo.head_logits(A, V, c)
+    dz = fo.dce_dz(z, y)
+    dV, dc = dz.T @ A, dz.sum(axis=0)
+    h = 1e-6
+    for (i, j) in [(0, 0), (3, 2), (9, 5), (5, 1)]:
+        Vp, Vm = V.copy(), V.copy()
+        Vp[i, j] += h
+        Vm[i, j] -= h
+        fd = (fo.cross_entropy(fo.head_logits(A, Vp, c), y) - fo.cross_entropy(fo.head_logits(A, Vm, c), y)) / (2 * h)
+        assert fd == pytest.approx(dV[i, j], rel=1e-6, abs=1e-9)
+    for i in (0, 4, 9):
+        cp, cm = c.copy(), c.copy()
+        cp[i] += h
+        cm[i] -= h
+        fd = (fo.cross_entropy(fo.head_logits(A, V, cp), y) - fo.cross_entropy(fo.head_logits(A, V, cm), y)) / (2 * h)
+        assert fd == pytest.approx(dc[i], rel=1e-6, abs=1e-9)
+
+
+def test_head_train_step_first_adam_step_and_prediction():
+    rng = np.random.default_rng(8)
+    n, F = 20, 9
+    A = rng.standard_normal((n, F))
+    y = rng.integers(0, 10, n)
+    head = fo.HeadState(np.zeros((10, F)), np.zeros(10))
+    hp = fo.AdamHyper(lr=1e-4)
+    out = fo.head_train_step(head, A, y, hp)
+    assert out["loss"] == pytest.approx(math.log(10.0), abs=1e-15)   # zero start: uniform softmax
+    # first Adam step: -lr * g / (|g| + eps) elementwise
+    np.testing.assert_allclose(head.V, -1e-4 * out["dV"] / (np.abs(out["dV"]) + 1e-8), rtol=1e-12, atol=1e-20)
+    np.testing.assert_allclose(head.c, -1e-4 * out["dc"] / (np.abs(out["dc"]) + 1e-8), rtol=1e-12, atol=1e-20)
+    assert head.t == 1
+    # prediction = first maximum of the logits (brute force)
+    V = rng.standard_normal((10, F))
+    c = rng.standard_normal(10)
+    hs = fo.HeadState(V, c)
+    pred, z = fo.head_predict(hs, A)
+    for i in range(n):
+        zi = [float(c[k] + sum(V[k][j] * A[i][j] for j in range(F))) for k in range(10)]
+        best = 0
+        for k in range(1, 10):
+            if zi[k] > zi[best]:
+                best = k
+        assert pred[i] == best
+    # a selector head predicts the class whose feature is largest
+    Fs = 10
+    A2 = rng.random((5, Fs))
+    hsel = fo.HeadState(np.eye(10), np.zeros(10))
+    assert np.array_equal(fo.head_predict(hsel, A2)[0], np.argmax(A2, axis=1))
