@@ -488,6 +488,41 @@ def run_other(args):
                     "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
                     "config": {"workload": f"ff_adaptive_neg_784-2000x4_bf16_n{n}",
                                "algorithmic_tflop": flops / 1e12}})
+    elif w in ("softmax_predict", "softmax_train"):
+        # the softmax head of §3 over layers 2..4 of 784-2000x4 (6000 features):
+        # one neutral-label pass per sample (predict, 10 000 samples), or one
+        # epoch of head training (58 x 1024 + 608 samples)
+        layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", init_seed=1000 + k) for k in range(len(NET) - 1)]
+        F = ff.Head.features_of(layers)
+        head = ff.Head(F, lr=1e-4, max_rows=4096)
+        fwd_flops = 2.0 * sum(NET[k] * NET[k + 1] for k in range(len(NET) - 1))
+        if w == "softmax_predict":
+            n = 10000
+            x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
+            pred = torch.empty(n, dtype=torch.int32, device=dev)
+            fn = lambda: head.predict(layers, x, pred=pred, stream=stream)
+            flops = n * (fwd_flops + 2.0 * 10 * F)
+            label = f"ff_softmax_predict_784-2000x4_bf16_n{n}"
+            metric = "FF softmax-head predict samples/s (one neutral-label pass) on 4x2000 net"
+        else:
+            n = PAIRS_PER_EPOCH
+            x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
+            y = torch.from_numpy(synth.labels(n, seed=7)).to(dev)
+            steps = [(r, min(BATCH, n - r)) for r in range(0, n, BATCH)]
+
+            def fn():
+                for r, b in steps:
+                    head.train_step(layers, x[r:r + b], y[r:r + b], stream=stream)
+            flops = n * (fwd_flops + 4.0 * 10 * F)
+            label = f"ff_softmax_train_784-2000x4_bf16_epoch{n}_B{BATCH}"
+            metric = "FF softmax-head train samples/s (neutral pass, CE backprop through the head, Adam) on 4x2000 net"
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        tf = flops / (ms / 1e3) / 1e12
+        out.update({"metric": metric, "value": round(n / (ms / 1e3), 1), "unit": "samples/s",
+                    "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
+                    "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
+                    "config": {"workload": label, "features": F, "algorithmic_tflop": flops / 1e12}})
     elif w == "pipeline_5x2000":
         # 784-2000x5, 60 chunks of 1000 pairs; 5 layer streams vs the same steps on one stream
         net5 = [784] + [2000] * 5
@@ -607,8 +642,8 @@ def main():
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="train_4x2000",
-                    choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "pipeline_5x2000",
-                             "wide_4x8192", "tiny_fp32"])
+                    choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "softmax_predict",
+                             "softmax_train", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")

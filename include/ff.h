@@ -158,6 +158,62 @@ FF_API ff_status ff_adaptive_negatives(ff_layer* const* layers, int n_layers, co
                                        const int* labels, int n, int* neg, float* goodness,
                                        void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Softmax prediction head of §3 "Prediction" (Softmax method).  The input,
+ * labelled with the neutral label (0.1 in each of the 10 label features),
+ * runs once through the layers; the activities of layers 2..L (layer 1 when
+ * L == 1), each divided by its own norm max(||h||, 1e-12), form the features
+ * A [n, n_features] of a linear softmax layer z = A V^T + c with 10 classes.
+ * The head is trained by backpropagation through itself only (mean
+ * cross-entropy over the rows, Adam): no gradient reaches the FF layers, which
+ * it reads but never changes.  V [10, n_features] and c [10] start at zero.
+ * ------------------------------------------------------------------------- */
+typedef struct ff_head ff_head;
+
+typedef struct {
+  int n_features;    /* sum of out_features of layers 2..L (of layer 1 when L == 1) */
+  float lr;          /* Adam learning rate (the paper uses 1e-4 for the softmax layer) */
+  float beta1, beta2, eps;
+  int max_rows;      /* rows per train step (and per predict chunk); 0 = 4096 */
+} ff_head_config;
+
+/* Allocates the head on the current device.  FF_ERR_INVALID_ARG on a bad
+ * config, FF_ERR_OOM / FF_ERR_CUDA on allocation failure (nothing leaks). */
+FF_API ff_status ff_head_create(const ff_head_config* cfg, ff_head** out);
+/* Waits for the head's last stream and frees it.  NULL is a no-op. */
+FF_API ff_status ff_head_destroy(ff_head* head);
+
+/* One training step of the head on n (<= max_rows) raw float32 input rows x
+ * [n, in_features of layer 1] with true labels [n] int32 (0..9), through
+ * layers[0..n_layers-1] (chained, one precision, read only): the neutral
+ * forward, logits, softmax, cross-entropy, dV = dz^T A, dc = sum dz and one
+ * Adam step on V and c.  loss [1] (device) or NULL receives the mean
+ * cross-entropy.  The layers must not be updated concurrently on another
+ * stream (order them before `stream`, e.g. with ff_net_sync).  The layer set
+ * must match n_features, else FF_ERR_INVALID_ARG. */
+FF_API ff_status ff_head_train_step(ff_head* head, ff_layer* const* layers, int n_layers,
+                                    const float* x, const int* labels, int n, float* loss,
+                                    void* stream);
+
+/* Softmax prediction of n raw input rows (any n; processed in chunks of
+ * max_rows): pred [n] int32 = the class with the largest logit (the lowest
+ * on ties) and/or logits [n, 10] float32; either may be NULL, not both. */
+FF_API ff_status ff_head_predict(ff_head* head, ff_layer* const* layers, int n_layers,
+                                 const float* x, int n, int* pred, float* logits, void* stream);
+
+/* Head state to/from host or device buffers (any NULL skipped): V, m_V, v_V
+ * [10, n_features]; c, m_c, v_c [10]; the Adam step.  Synchronous. */
+FF_API ff_status ff_head_get_state(const ff_head* head, float* V, float* c, float* m_V,
+                                   float* v_V, float* m_c, float* v_c, long long* step);
+FF_API ff_status ff_head_set_state(ff_head* head, const float* V, const float* c,
+                                   const float* m_V, const float* v_V, const float* m_c,
+                                   const float* v_c, long long step);
+/* The gradient (dV [10, n_features], dc [10]) of the last train step. */
+FF_API ff_status ff_head_get_grad(const ff_head* head, float* dV, float* dc);
+/* Waits for the head's stream; reports and clears latched device errors
+ * (FF_ERR_NONFINITE for non-finite logits or activities). */
+FF_API ff_status ff_head_check(ff_head* head);
+
 /* Copies the layer state to/from caller buffers, which may be host or device
  * memory: W [N,K] and its Adam moments m_W, v_W [N,K]; b, m_b, v_b [N]; the
  * Adam step counter.  Any pointer may be NULL to skip that tensor.  Both calls

@@ -29,22 +29,6 @@ ff_status cuda_status(cudaError_t e, const char* what) {
   return FF_ERR_CUDA;
 }
 
-#define FF_TRY(call, what)                                 \
-  do {                                                     \
-    ff_status s_ = ::ff::cuda_status((call), (what));      \
-    if (s_ != FF_OK) return s_;                            \
-  } while (0)
-
-// A kernel launch: counted, and timed on its stream while profiling is on.
-#define FF_LAUNCH(kind, work, st, call, what)                          \
-  do {                                                                 \
-    ff_status s_;                                                      \
-    {                                                                  \
-      ::ff::ProfScope p_((kind), (double)(work), (st));                \
-      s_ = ::ff::cuda_status((call), (what));                          \
-    }                                                                  \
-    if (s_ != FF_OK) return s_;                                        \
-  } while (0)
 
 // Host-side fault injection: FF_FAULT_ALLOC_FAIL_AT=n makes the n-th device
 // allocation (1-based, counted over the process) fail as out-of-memory.

@@ -2,6 +2,7 @@
 #pragma once
 
 #include "ff_internal.cuh"
+#include "ff_prof.h"
 
 namespace ff {
 
@@ -18,3 +19,20 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
                           cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done);
 
 }  // namespace ff
+
+#define FF_TRY(call, what)                                 \
+  do {                                                     \
+    ff_status s_ = ::ff::cuda_status((call), (what));      \
+    if (s_ != FF_OK) return s_;                            \
+  } while (0)
+
+// A kernel launch: counted, and timed on its stream while profiling is on.
+#define FF_LAUNCH(kind, work, st, call, what)                          \
+  do {                                                                 \
+    ff_status s_;                                                      \
+    {                                                                  \
+      ::ff::ProfScope p_((kind), (double)(work), (st));                \
+      s_ = ::ff::cuda_status((call), (what));                          \
+    }                                                                  \
+    if (s_ != FF_OK) return s_;                                        \
+  } while (0)

@@ -109,7 +109,7 @@ __global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ l
       }
 #pragma unroll
       for (int u = 0; u < 4; ++u) {
-        if (f + u < 10) v[u] = (f + u == lab) ? 1.f : 0.f;
+        if (f + u < 10) v[u] = mode == 2 ? 0.1f : (f + u == lab) ? 1.f : 0.f;
         ss = fmaf(v[u], v[u], ss);
       }
       store4<T>(orow + f, v[0], v[1], v[2], v[3]);
@@ -117,7 +117,7 @@ __global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ l
   } else {
     for (int f = lane; f < ldo; f += 32) {
       float v = 0.f;
-      if (f < F) v = (f < 10) ? (f == lab ? 1.f : 0.f) : __ldg(xr + f);
+      if (f < F) v = (f < 10) ? (mode == 2 ? 0.1f : f == lab ? 1.f : 0.f) : __ldg(xr + f);
       orow[f] = from_f<T>(v);
       ss = fmaf(v, v, ss);
     }

@@ -1,0 +1,754 @@
+// Softmax prediction head of §3 "Prediction" (Softmax method).
+//
+// The unlabelled input carries the neutral label (0.1 in each of the 10
+// label features) and runs once through every FF layer; the activities of
+// all but the first hidden layer, each normalised like a layer input
+// (h / max(||h||, 1e-12)), are the features A of a linear softmax layer
+// z = A V^T + c.  The head is trained by backpropagation through itself only
+// (cross-entropy averaged over the rows, Adam with its own learning rate,
+// §5.1): no gradient reaches the FF layers.  Prediction is the class with the
+// largest logit.
+//
+// Kernels (all fixed-order reductions, no floating-point atomics):
+//   k_head_logits  one pass over A: z, softmax, per-row loss and dz =
+//                  (softmax(z) - onehot(y)) / n, per-block partials of dc and
+//                  of the loss; A is never materialised -- it is read as the
+//                  stored activities H_k with their row scales s_k
+//   k_head_wgrad   dV partials per 128-row block: dz^T (s_k H_k)
+//   k_head_adam    reduces the partials in a fixed order, Adam on V and c,
+//                  the step's loss
+#include <cmath>
+#include <cstring>
+#include <new>
+
+#include "ff_api_internal.h"
+#include "ff_internal.cuh"
+#include "ff_prof.h"
+
+namespace ff {
+namespace {
+
+constexpr int kClasses = 10;
+constexpr int kMaxSegs = 16;
+constexpr int kLogitRows = 16;   // rows per block of k_head_logits (two per warp)
+constexpr int kLogitChunk = 256; // features per V chunk staged in shared memory (8 per lane)
+constexpr int kWgRows = 128;     // rows per block of k_head_wgrad (16 per warp)
+constexpr int kWgChunk = 128;    // features per block of k_head_wgrad (4 per lane)
+constexpr int kPart = kClasses + 1;  // per-block partials: dc[10], loss
+
+// The feature segments: segment k is layer (k+2)'s activity (layer 1's when
+// there is one layer), features off[k] .. off[k] + F[k] of A.
+struct Segs {
+  const void* H[kMaxSegs];
+  const float* s[kMaxSegs];
+  int ld[kMaxSegs];
+  int F[kMaxSegs];
+  int off[kMaxSegs];
+  int nseg;
+  int F_total;
+};
+
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// h[0..W) = H[row, f .. f+W) as float, zero past the segment or the rows.
+template <typename T, int W>
+__device__ __forceinline__ void load_feats(const T* __restrict__ H, int ld, int row, int n, int f, int F, float* h);
+template <>
+__device__ __forceinline__ void load_feats<bf16, 8>(const bf16* __restrict__ H, int ld, int row, int n, int f, int F,
+                                                    float* h) {
+  if (row < n && f + 8 <= F) {
+    const uint4 q = __ldg(reinterpret_cast<const uint4*>(H + (size_t)row * ld + f));
+    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+      const __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
+      const float2 v = __bfloat1622float2(p);
+      h[2 * i] = v.x;
+      h[2 * i + 1] = v.y;
+    }
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i)
+      h[i] = (row < n && f + i < F) ? __bfloat162float(H[(size_t)row * ld + f + i]) : 0.f;
+  }
+}
+template <>
+__device__ __forceinline__ void load_feats<float, 8>(const float* __restrict__ H, int ld, int row, int n, int f, int F,
+                                                     float* h) {
+  if (row < n && f + 8 <= F) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(H + (size_t)row * ld + f));
+    const float4 b = __ldg(reinterpret_cast<const float4*>(H + (size_t)row * ld + f + 4));
+    h[0] = a.x; h[1] = a.y; h[2] = a.z; h[3] = a.w;
+    h[4] = b.x; h[5] = b.y; h[6] = b.z; h[7] = b.w;
+  } else {
+#pragma unroll
+    for (int i = 0; i < 8; ++i) h[i] = (row < n && f + i < F) ? H[(size_t)row * ld + f + i] : 0.f;
+  }
+}
+template <>
+__device__ __forceinline__ void load_feats<bf16, 4>(const bf16* __restrict__ H, int ld, int row, int n, int f, int F,
+                                                    float* h) {
+  if (row < n && f + 4 <= F) {
+    const uint2 q = __ldg(reinterpret_cast<const uint2*>(H + (size_t)row * ld + f));
+    const float2 a = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.x));
+    const float2 b = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&q.y));
+    h[0] = a.x; h[1] = a.y; h[2] = b.x; h[3] = b.y;
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+      h[i] = (row < n && f + i < F) ? __bfloat162float(H[(size_t)row * ld + f + i]) : 0.f;
+  }
+}
+template <>
+__device__ __forceinline__ void load_feats<float, 4>(const float* __restrict__ H, int ld, int row, int n, int f, int F,
+                                                     float* h) {
+  if (row < n && f + 4 <= F) {
+    const float4 a = __ldg(reinterpret_cast<const float4*>(H + (size_t)row * ld + f));
+    h[0] = a.x; h[1] = a.y; h[2] = a.z; h[3] = a.w;
+  } else {
+#pragma unroll
+    for (int i = 0; i < 4; ++i) h[i] = (row < n && f + i < F) ? H[(size_t)row * ld + f + i] : 0.f;
+  }
+}
+
+// Softmax, loss and dz of one row from its logits (z has the bias added).
+// Writes logits/dz when given; returns the row's loss (0 without a label).
+__device__ __forceinline__ float finish_row(const float (&z)[kClasses], int row, const int* __restrict__ labels,
+                                            float inv_n, float* __restrict__ logits, float* __restrict__ dz,
+                                            float (&dzr)[kClasses], int* err) {
+  bool finite = true;
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    if (logits) logits[(size_t)row * kClasses + c] = z[c];
+    finite = finite && isfinite(z[c]);
+    dzr[c] = 0.f;
+  }
+  if (!finite) atomicOr(err, DEVERR_NONFINITE);
+  if (!labels) return 0.f;
+  float m = z[0];
+#pragma unroll
+  for (int c = 1; c < kClasses; ++c) m = fmaxf(m, z[c]);
+  float e[kClasses], sum = 0.f;
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    e[c] = expf(z[c] - m);
+    sum += e[c];
+  }
+  const int y = labels[row];
+  const float inv = 1.f / sum;
+  float zy = 0.f;
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    const float p = e[c] * inv;
+    dzr[c] = (p - (c == y ? 1.f : 0.f)) * inv_n;
+    if (c == y) zy = z[c];
+    if (dz) dz[(size_t)row * kClasses + c] = dzr[c];
+  }
+  return (m + logf(sum)) - zy;
+}
+
+// One block per kLogitRows rows, two rows per warp.  Each lane takes 8
+// consecutive features of a 256-feature chunk; the chunk of V is staged in
+// shared memory interleaved (Vs[c][e*32 + lane] = V[c][chunk + 8*lane + e])
+// so the lanes read it without bank conflicts.  Segment sums are scaled by
+// the row's s_k before they join the total, so A = s_k H_k is never formed.
+template <typename T>
+__global__ void __launch_bounds__(256) k_head_logits(Segs sg, int n, const float* __restrict__ V,
+                                                     const float* __restrict__ cb, const int* __restrict__ labels,
+                                                     float inv_n, float* __restrict__ logits, float* __restrict__ dz,
+                                                     float* __restrict__ part, ff_dev_state* ds, float beta1,
+                                                     float beta2, int* err) {
+  __shared__ float Vs[kClasses][kLogitChunk];
+  __shared__ float rowpart[kLogitRows][kPart];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int r0 = blockIdx.x * kLogitRows + warp * 2;
+  if (blockIdx.x == 0 && threadIdx.x == 0 && labels && ds) {
+    // this step's Adam counter and bias corrections, read by k_head_adam
+    ds->t += 1;
+    ds->pow1 *= (double)beta1;
+    ds->pow2 *= (double)beta2;
+    ds->bc1 = (float)(1.0 - ds->pow1);
+    ds->bc2 = (float)(1.0 - ds->pow2);
+  }
+  float tot[2][kClasses];
+#pragma unroll
+  for (int r = 0; r < 2; ++r)
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) tot[r][c] = 0.f;
+  for (int k = 0; k < sg.nseg; ++k) {
+    const T* H = static_cast<const T*>(sg.H[k]);
+    const int ld = sg.ld[k], Fk = sg.F[k], off = sg.off[k];
+    float seg[2][kClasses];
+#pragma unroll
+    for (int r = 0; r < 2; ++r)
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) seg[r][c] = 0.f;
+    for (int f0 = 0; f0 < Fk; f0 += kLogitChunk) {
+      __syncthreads();  // the previous chunk is consumed
+      for (int idx = threadIdx.x; idx < kClasses * kLogitChunk; idx += 256) {
+        const int c = idx / kLogitChunk, j = idx % kLogitChunk;
+        Vs[c][(j & 7) * 32 + (j >> 3)] = (f0 + j < Fk) ? __ldg(V + (size_t)c * sg.F_total + off + f0 + j) : 0.f;
+      }
+      __syncthreads();
+#pragma unroll
+      for (int r = 0; r < 2; ++r) {
+        float h[8];
+        load_feats<T, 8>(H, ld, r0 + r, n, f0 + 8 * lane, Fk, h);
+#pragma unroll
+        for (int c = 0; c < kClasses; ++c)
+#pragma unroll
+          for (int e = 0; e < 8; ++e) seg[r][c] = fmaf(h[e], Vs[c][e * 32 + lane], seg[r][c]);
+      }
+    }
+#pragma unroll
+    for (int r = 0; r < 2; ++r) {
+      const float sr = (r0 + r < n) ? __ldg(sg.s[k] + r0 + r) : 0.f;
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) tot[r][c] = fmaf(sr, seg[r][c], tot[r][c]);
+    }
+  }
+#pragma unroll
+  for (int r = 0; r < 2; ++r)
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) tot[r][c] = warp_sum(tot[r][c]);
+  // lane r finishes row r0 + r
+  float dzr[kClasses];
+  float loss = 0.f;
+  bool mine = false;
+  if (lane < 2 && r0 + lane < n) {
+    float z[kClasses];
+    if (lane == 0) {
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) z[c] = tot[0][c] + __ldg(cb + c);
+    } else {
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) z[c] = tot[1][c] + __ldg(cb + c);
+    }
+    loss = finish_row(z, r0 + lane, labels, inv_n, logits, dz, dzr, err);
+    mine = true;
+  }
+  if (!part) return;
+  if (lane < 2) {
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) rowpart[warp * 2 + lane][c] = mine ? dzr[c] : 0.f;
+    rowpart[warp * 2 + lane][kClasses] = mine ? loss : 0.f;
+  }
+  __syncthreads();
+  if (threadIdx.x < kPart) {
+    float acc = 0.f;
+    for (int r = 0; r < kLogitRows; ++r) acc += rowpart[r][threadIdx.x];
+    part[(size_t)blockIdx.x * kPart + threadIdx.x] = acc;
+  }
+}
+
+// dV partials of one 128-row block for one 128-feature chunk of one segment:
+// dVpart[rb, c, f] = sum over the block's rows i of dz[i, c] s_k[i] H_k[i, f].
+// Eight warps take 16 rows each (lane = 4 features); the eight partial sums
+// are added in warp order.
+template <typename T>
+__global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float* __restrict__ dz,
+                                                    float* __restrict__ dVpart) {
+  __shared__ float dzs[kWgRows][kClasses];
+  __shared__ float red[8][kClasses][kWgChunk];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  // segment and chunk of this block
+  int k = 0, chunk = blockIdx.x;
+  while (k + 1 < sg.nseg && chunk >= (sg.F[k] + kWgChunk - 1) / kWgChunk) {
+    chunk -= (sg.F[k] + kWgChunk - 1) / kWgChunk;
+    ++k;
+  }
+  const T* H = static_cast<const T*>(sg.H[k]);
+  const int ld = sg.ld[k], Fk = sg.F[k], off = sg.off[k];
+  const int f0 = chunk * kWgChunk;
+  const int rb0 = blockIdx.y * kWgRows;
+  for (int idx = threadIdx.x; idx < kWgRows * kClasses; idx += 256) {
+    const int i = idx / kClasses, c = idx % kClasses;
+    const int row = rb0 + i;
+    dzs[i][c] = row < n ? __ldg(dz + (size_t)row * kClasses + c) * __ldg(sg.s[k] + row) : 0.f;
+  }
+  __syncthreads();
+  float acc[kClasses][4];
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) acc[c][e] = 0.f;
+  const int f = f0 + 4 * lane;
+#pragma unroll 4
+  for (int i = warp * (kWgRows / 8); i < (warp + 1) * (kWgRows / 8); ++i) {
+    float h[4];
+    load_feats<T, 4>(H, ld, rb0 + i, n, f, Fk, h);
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      const float d = dzs[i][c];
+#pragma unroll
+      for (int e = 0; e < 4; ++e) acc[c][e] = fmaf(d, h[e], acc[c][e]);
+    }
+  }
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c)
+#pragma unroll
+    for (int e = 0; e < 4; ++e) red[warp][c][4 * lane + e] = acc[c][e];
+  __syncthreads();
+  for (int idx = threadIdx.x; idx < kClasses * kWgChunk; idx += 256) {
+    const int c = idx / kWgChunk, j = idx % kWgChunk;
+    if (f0 + j >= Fk) continue;
+    float v = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) v += red[w][c][j];
+    dVpart[((size_t)blockIdx.y * kClasses + c) * sg.F_total + off + f0 + j] = v;
+  }
+}
+
+struct HeadAdamArgs {
+  float *V, *mV, *vV, *c, *mc, *vc;
+  const float* dVpart;  // [nrb, 10, F]
+  int nrb, F;
+  const float* part;    // [nlb, 11]
+  int nlb;
+  float inv_n;
+  float lr, beta1, beta2, eps;
+  const ff_dev_state* ds;
+  float* loss_out;
+  float* dV_out;        // [10, F] or null
+  float* dc_out;        // [10] or null
+};
+
+__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float a1, float b1, float b2, float eps,
+                                      float r2) {
+  m = b1 * m + (1.f - b1) * g;
+  v = b2 * v + (1.f - b2) * g * g;
+  w -= a1 * m / (sqrtf(v * r2) + eps);
+}
+
+// Threads 0 .. 10F-1 of the grid own one V element each; the last block owns
+// the 10 biases (warp w: columns w and w + 8 of the partials, column 10 being
+// the loss).
+__global__ void __launch_bounds__(256) k_head_adam(HeadAdamArgs a) {
+  const float a1 = a.lr / a.ds->bc1, r2 = 1.f / a.ds->bc2;
+  const int total = kClasses * a.F;
+  const int vblocks = (total + 255) / 256;
+  if ((int)blockIdx.x < vblocks) {
+    const int idx = blockIdx.x * 256 + threadIdx.x;
+    if (idx >= total) return;
+    float g = 0.f;
+    for (int rb = 0; rb < a.nrb; ++rb) g += __ldg(a.dVpart + (size_t)rb * total + idx);
+    if (a.dV_out) a.dV_out[idx] = g;
+    float w = a.V[idx], m = a.mV[idx], v = a.vV[idx];
+    adam1(w, m, v, g, a1, a.beta1, a.beta2, a.eps, r2);
+    a.V[idx] = w;
+    a.mV[idx] = m;
+    a.vV[idx] = v;
+    return;
+  }
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  for (int col = warp; col < kPart; col += 8) {
+    float t = 0.f;
+    for (int b = lane; b < a.nlb; b += 32) t += __ldg(a.part + (size_t)b * kPart + col);
+    t = warp_sum(t);
+    if (lane != 0) continue;
+    if (col == kClasses) {
+      if (a.loss_out) a.loss_out[0] = t * a.inv_n;
+      continue;
+    }
+    if (a.dc_out) a.dc_out[col] = t;
+    float w = a.c[col], m = a.mc[col], v = a.vc[col];
+    adam1(w, m, v, t, a1, a.beta1, a.beta2, a.eps, r2);
+    a.c[col] = w;
+    a.mc[col] = m;
+    a.vc[col] = v;
+  }
+}
+
+size_t align256(size_t b) { return (b + 255) & ~size_t(255); }
+
+}  // namespace
+}  // namespace ff
+
+// The head object behind the opaque handle.
+struct ff_head {
+  ff_head_config cfg;
+  int F;
+  int device;
+  cudaStream_t last_stream;
+  float *V, *c, *mV, *vV, *mc, *vc;  // one allocation: V, mV, vV [10, F]; c, mc, vc [10]
+  float *dV, *dc;                    // gradient of the last train step [10, F], [10]
+  ff::ff_dev_state* ds;
+  void* ws;
+  size_t ws_bytes;
+};
+
+namespace ff {
+namespace {
+
+// Validates the layer chain for the head and describes its feature segments
+// (without buffers).  Returns FF_OK or FF_ERR_INVALID_ARG.
+ff_status head_layers(const ff_head* hd, ff_layer* const* layers, int n_layers) {
+  if (!layers || n_layers < 1 || n_layers > kMaxSegs + 1) return FF_ERR_INVALID_ARG;
+  int F = 0;
+  for (int k = 0; k < n_layers; ++k) {
+    if (!layers[k]) return FF_ERR_INVALID_ARG;
+    if (layers[k]->is_bf16 != layers[0]->is_bf16) return FF_ERR_INVALID_ARG;
+    if (k > 0 && layers[k]->K != layers[k - 1]->N) return FF_ERR_INVALID_ARG;
+    if (k >= 1 || n_layers == 1) F += layers[k]->N;
+  }
+  if (layers[0]->K < kClasses) return FF_ERR_INVALID_ARG;
+  if (F != hd->F) return FF_ERR_INVALID_ARG;
+  return FF_OK;
+}
+
+struct HeadWork {
+  void* X0;
+  float* S[kMaxSegs + 2];   // S[k]: row scale of layer k's input (S[L]: of the last activity)
+  void* Hk[kMaxSegs + 1];
+  float* gpart;
+  float* logits;
+  float* dz;
+  float* part;
+  float* dVpart;
+};
+
+// Carves the head's workspace for `rows` rows (grown on demand).
+ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, bool train, HeadWork* w) {
+  const bool b16 = layers[0]->is_bf16;
+  const size_t es = b16 ? 2 : 4;
+  int ntmax = 0;
+  for (int k = 0; k < L; ++k) {
+    const int nt = b16 ? tc_fwd_ntiles(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
+    if (nt > ntmax) ntmax = nt;
+  }
+  size_t off = 0;
+  size_t oX = off; off += align256((size_t)rows * layers[0]->ldK * es);
+  size_t oS[kMaxSegs + 2];
+  for (int k = 0; k <= L; ++k) { oS[k] = off; off += align256((size_t)rows * 4); }
+  size_t oH[kMaxSegs + 1];
+  for (int k = 0; k < L; ++k) { oH[k] = off; off += align256((size_t)rows * layers[k]->ldN * es); }
+  size_t oG = off; off += align256((size_t)ntmax * rows * 4);
+  size_t oZ = off; off += align256((size_t)rows * kClasses * 4);
+  size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
+  size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kLogitRows) * kPart * 4 : 0);
+  size_t oV = off; off += align256(train ? (size_t)cdiv(rows, kWgRows) * kClasses * hd->F * 4 : 0);
+  if (off > hd->ws_bytes) {
+    FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before head workspace growth");
+    dev_free(hd->ws);
+    hd->ws = nullptr;
+    hd->ws_bytes = 0;
+    FF_TRY(dev_alloc(&hd->ws, off), "head workspace");
+    hd->ws_bytes = off;
+  }
+  char* base = static_cast<char*>(hd->ws);
+  w->X0 = base + oX;
+  for (int k = 0; k <= L; ++k) w->S[k] = reinterpret_cast<float*>(base + oS[k]);
+  for (int k = 0; k < L; ++k) w->Hk[k] = base + oH[k];
+  w->gpart = reinterpret_cast<float*>(base + oG);
+  w->logits = reinterpret_cast<float*>(base + oZ);
+  w->dz = train ? reinterpret_cast<float*>(base + oD) : nullptr;
+  w->part = train ? reinterpret_cast<float*>(base + oP) : nullptr;
+  w->dVpart = train ? reinterpret_cast<float*>(base + oV) : nullptr;
+  return FF_OK;
+}
+
+// Neutral-labelled forward of `rows` raw input rows through every layer:
+// H_k and the row scale of every activity.
+ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows, const HeadWork& w, int* err,
+                       cudaStream_t st) {
+  ff_layer* L0 = layers[0];
+  const bool b16 = L0->is_bf16;
+  const double es = b16 ? 2.0 : 4.0;
+  FF_LAUNCH(K_OVERLAY, (double)rows * (L0->K * 4.0 + L0->ldK * es + 4), st,
+            launch_overlay(x, nullptr, rows, L0->K, w.X0, L0->ldK, b16, w.S[0], 2, st), "neutral-label overlay");
+  const void* in = w.X0;
+  for (int k = 0; k < L; ++k) {
+    ff_layer* Lk = layers[k];
+    EpiArgs ep{w.S[k], Lk->cfg.has_bias ? Lk->b : nullptr, w.Hk[k], Lk->ldN, w.gpart};
+    int nt;
+    if (b16) {
+      nt = tc_fwd_ntiles(Lk->N);
+      FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
+                tc_gemm_fwd(static_cast<const bf16*>(in), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep, err, st),
+                "head forward GEMM (tcgen05)");
+    } else {
+      nt = simt_fwd_ntiles(Lk->N);
+      FF_LAUNCH(K_FWD_SIMT, 2.0 * rows * Lk->N * Lk->K, st,
+                simt_gemm_fwd(static_cast<const float*>(in), Lk->ldK, Lk->W, Lk->K, rows, Lk->N, Lk->K, ep, st),
+                "head forward GEMM (fp32)");
+    }
+    FinalizeArgs fa{};
+    fa.gpart = w.gpart;
+    fa.ntiles = nt;
+    fa.M = rows;
+    fa.s_next = w.S[k + 1];
+    fa.err = err;
+    FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 4), st, launch_finalize(fa, st), "head activity scale");
+    in = w.Hk[k];
+  }
+  return FF_OK;
+}
+
+Segs make_segs(ff_layer* const* layers, int L, const HeadWork& w, int F) {
+  Segs sg{};
+  int off = 0, j = 0;
+  for (int k = (L == 1 ? 0 : 1); k < L; ++k, ++j) {
+    sg.H[j] = w.Hk[k];
+    sg.s[j] = w.S[k + 1];
+    sg.ld[j] = layers[k]->ldN;
+    sg.F[j] = layers[k]->N;
+    sg.off[j] = off;
+    off += layers[k]->N;
+  }
+  sg.nseg = j;
+  sg.F_total = F;
+  return sg;
+}
+
+cudaError_t launch_head_logits(const Segs& sg, bool b16, int n, const float* V, const float* c, const int* labels,
+                               float* logits, float* dz, float* part, ff_dev_state* ds, float beta1, float beta2,
+                               int* err, cudaStream_t st) {
+  const float inv_n = 1.f / (float)n;
+  if (b16)
+    k_head_logits<bf16><<<cdiv(n, kLogitRows), 256, 0, st>>>(sg, n, V, c, labels, inv_n, logits, dz, part, ds, beta1,
+                                                            beta2, err);
+  else
+    k_head_logits<float><<<cdiv(n, kLogitRows), 256, 0, st>>>(sg, n, V, c, labels, inv_n, logits, dz, part, ds,
+                                                             beta1, beta2, err);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_head_wgrad(const Segs& sg, bool b16, int n, const float* dz, float* dVpart, cudaStream_t st) {
+  int chunks = 0;
+  for (int k = 0; k < sg.nseg; ++k) chunks += cdiv(sg.F[k], kWgChunk);
+  dim3 grid(chunks, cdiv(n, kWgRows));
+  if (b16)
+    k_head_wgrad<bf16><<<grid, 256, 0, st>>>(sg, n, dz, dVpart);
+  else
+    k_head_wgrad<float><<<grid, 256, 0, st>>>(sg, n, dz, dVpart);
+  return cudaGetLastError();
+}
+
+}  // namespace
+}  // namespace ff
+
+using namespace ff;
+
+extern "C" {
+
+ff_status ff_head_create(const ff_head_config* cfg, ff_head** out) {
+  if (!out) return FF_ERR_INVALID_ARG;
+  *out = nullptr;
+  if (!cfg || cfg->n_features < 1 || cfg->max_rows < 0) return FF_ERR_INVALID_ARG;
+  if (!std::isfinite(cfg->lr) || !(cfg->beta1 >= 0.f && cfg->beta1 < 1.f) || !(cfg->beta2 >= 0.f && cfg->beta2 < 1.f) ||
+      !(cfg->eps > 0.f))
+    return FF_ERR_INVALID_ARG;
+  ff_head* hd = new (std::nothrow) ff_head();
+  if (!hd) return FF_ERR_OOM;
+  hd->cfg = *cfg;
+  if (hd->cfg.max_rows == 0) hd->cfg.max_rows = 4096;
+  hd->F = cfg->n_features;
+  cudaGetDevice(&hd->device);
+  const size_t nv = (size_t)kClasses * hd->F;
+  const size_t total = 4 * nv + 5 * kClasses;  // V, mV, vV, dV; c, mc, vc, dc (+ pad)
+  void* p = nullptr;
+  ff_status s = cuda_status(dev_alloc(&p, total * 4), "head parameters");
+  if (s != FF_OK) {
+    delete hd;
+    return s;
+  }
+  float* f = static_cast<float*>(p);
+  hd->V = f;
+  hd->mV = f + nv;
+  hd->vV = f + 2 * nv;
+  hd->dV = f + 3 * nv;
+  hd->c = f + 4 * nv;
+  hd->mc = hd->c + kClasses;
+  hd->vc = hd->mc + kClasses;
+  hd->dc = hd->vc + kClasses;
+  void* dsp = nullptr;
+  s = cuda_status(dev_alloc(&dsp, sizeof(ff_dev_state)), "head device state");
+  if (s != FF_OK) {
+    dev_free(p);
+    delete hd;
+    return s;
+  }
+  hd->ds = static_cast<ff_dev_state*>(dsp);
+  const ff_dev_state init{0, 1.0, 1.0, 0.f, 0.f, 0, 0.f};
+  cudaError_t e = cudaMemcpy(hd->ds, &init, sizeof(init), cudaMemcpyHostToDevice);
+  if (e == cudaSuccess) e = cudaMemset(p, 0, total * 4);  // V and c start at zero (the head's reading)
+  if (e == cudaSuccess) e = cudaDeviceSynchronize();
+  if (e != cudaSuccess) {
+    dev_free(p);
+    dev_free(dsp);
+    delete hd;
+    return cuda_status(e, "head initialisation");
+  }
+  *out = hd;
+  return FF_OK;
+}
+
+ff_status ff_head_destroy(ff_head* hd) {
+  if (!hd) return FF_OK;
+  cudaStreamSynchronize(hd->last_stream);
+  dev_free(hd->ws);
+  dev_free(hd->V);
+  dev_free(hd->ds);
+  delete hd;
+  return FF_OK;
+}
+
+ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, const int* labels,
+                             int n, float* loss, void* stream) {
+  if (!hd || n < 0) return FF_ERR_INVALID_ARG;
+  ff_status s = head_layers(hd, layers, n_layers);
+  if (s != FF_OK) return s;
+  if (n == 0) return FF_OK;
+  if (!x || !labels || n > hd->cfg.max_rows) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  HeadWork w;
+  s = head_workspace(hd, layers, n_layers, n, true, &w);
+  if (s != FF_OK) return s;
+  hd->last_stream = st;
+  int* err = &hd->ds->err;
+  s = head_forward(layers, n_layers, x, n, w, err, st);
+  if (s != FF_OK) return s;
+  const Segs sg = make_segs(layers, n_layers, w, hd->F);
+  const bool b16 = layers[0]->is_bf16;
+  const double es = b16 ? 2.0 : 4.0;
+  FF_LAUNCH(K_HEAD_LOGITS, (double)n * hd->F * es + (double)n * kClasses * 8, st,
+            launch_head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.dz, w.part, hd->ds, hd->cfg.beta1,
+                               hd->cfg.beta2, err, st),
+            "head logits, softmax, cross-entropy");
+  FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
+            launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
+  HeadAdamArgs a{};
+  a.V = hd->V;
+  a.mV = hd->mV;
+  a.vV = hd->vV;
+  a.c = hd->c;
+  a.mc = hd->mc;
+  a.vc = hd->vc;
+  a.dVpart = w.dVpart;
+  a.nrb = cdiv(n, kWgRows);
+  a.F = hd->F;
+  a.part = w.part;
+  a.nlb = cdiv(n, kLogitRows);
+  a.inv_n = 1.f / (float)n;
+  a.lr = hd->cfg.lr;
+  a.beta1 = hd->cfg.beta1;
+  a.beta2 = hd->cfg.beta2;
+  a.eps = hd->cfg.eps;
+  a.ds = hd->ds;
+  a.loss_out = loss ? loss : &hd->ds->loss;
+  a.dV_out = hd->dV;
+  a.dc_out = hd->dc;
+  const int vblocks = cdiv((long long)kClasses * hd->F, 256);
+  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st,
+            (k_head_adam<<<vblocks + 1, 256, 0, st>>>(a), cudaGetLastError()), "head Adam");
+  return FF_OK;
+}
+
+ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, int n, int* pred,
+                          float* logits, void* stream) {
+  if (!hd || n < 0) return FF_ERR_INVALID_ARG;
+  ff_status s = head_layers(hd, layers, n_layers);
+  if (s != FF_OK) return s;
+  if (n == 0) return FF_OK;
+  if (!x || (!pred && !logits)) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int C = n < hd->cfg.max_rows ? n : hd->cfg.max_rows;
+  HeadWork w;
+  s = head_workspace(hd, layers, n_layers, C, false, &w);
+  if (s != FF_OK) return s;
+  hd->last_stream = st;
+  int* err = &hd->ds->err;
+  const bool b16 = layers[0]->is_bf16;
+  const double es = b16 ? 2.0 : 4.0;
+  const int K0 = layers[0]->K;
+  for (int r0 = 0; r0 < n; r0 += C) {
+    const int cn = (n - r0) < C ? (n - r0) : C;
+    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, cn, w, err, st);
+    if (s != FF_OK) return s;
+    const Segs sg = make_segs(layers, n_layers, w, hd->F);
+    float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
+    FF_LAUNCH(K_HEAD_LOGITS, (double)cn * hd->F * es + (double)cn * kClasses * 4, st,
+              launch_head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, nullptr, nullptr, nullptr, 0.f, 0.f, err, st),
+              "head logits");
+    if (pred)
+      FF_LAUNCH(K_ARGMAX, (double)cn * 44, st, launch_argmax(z, cn, nullptr, pred + r0, st), "head argmax");
+  }
+  return FF_OK;
+}
+
+static ff_status head_copy(void* dst, const void* src, size_t bytes) {
+  if (!dst || !src) return FF_OK;
+  FF_TRY(cudaMemcpy(dst, src, bytes, cudaMemcpyDefault), "head state copy");
+  return FF_OK;
+}
+
+ff_status ff_head_get_state(const ff_head* hdc, float* V, float* c, float* mV, float* vV, float* mc, float* vc,
+                            long long* step) {
+  if (!hdc) return FF_ERR_INVALID_ARG;
+  ff_head* hd = const_cast<ff_head*>(hdc);
+  FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync");
+  const size_t nv = (size_t)kClasses * hd->F * 4, nc = kClasses * 4;
+  ff_status s;
+  if ((s = head_copy(V, hd->V, nv)) != FF_OK) return s;
+  if ((s = head_copy(mV, hd->mV, nv)) != FF_OK) return s;
+  if ((s = head_copy(vV, hd->vV, nv)) != FF_OK) return s;
+  if ((s = head_copy(c, hd->c, nc)) != FF_OK) return s;
+  if ((s = head_copy(mc, hd->mc, nc)) != FF_OK) return s;
+  if ((s = head_copy(vc, hd->vc, nc)) != FF_OK) return s;
+  if (step) {
+    ff_dev_state d;
+    FF_TRY(cudaMemcpy(&d, hd->ds, sizeof(d), cudaMemcpyDeviceToHost), "head step counter");
+    *step = d.t;
+  }
+  return FF_OK;
+}
+
+ff_status ff_head_set_state(ff_head* hd, const float* V, const float* c, const float* mV, const float* vV,
+                            const float* mc, const float* vc, long long step) {
+  if (!hd || step < 0) return FF_ERR_INVALID_ARG;
+  FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync");
+  const size_t nv = (size_t)kClasses * hd->F * 4, nc = kClasses * 4;
+  ff_status s;
+  if ((s = head_copy(hd->V, V, nv)) != FF_OK) return s;
+  if ((s = head_copy(hd->mV, mV, nv)) != FF_OK) return s;
+  if ((s = head_copy(hd->vV, vV, nv)) != FF_OK) return s;
+  if ((s = head_copy(hd->c, c, nc)) != FF_OK) return s;
+  if ((s = head_copy(hd->mc, mc, nc)) != FF_OK) return s;
+  if ((s = head_copy(hd->vc, vc, nc)) != FF_OK) return s;
+  ff_dev_state d;
+  FF_TRY(cudaMemcpy(&d, hd->ds, sizeof(d), cudaMemcpyDeviceToHost), "head device state");
+  d.t = step;
+  d.pow1 = std::pow((double)hd->cfg.beta1, (double)step);
+  d.pow2 = std::pow((double)hd->cfg.beta2, (double)step);
+  FF_TRY(cudaMemcpy(hd->ds, &d, sizeof(d), cudaMemcpyHostToDevice), "head device state");
+  return FF_OK;
+}
+
+ff_status ff_head_get_grad(const ff_head* hdc, float* dV, float* dc) {
+  if (!hdc) return FF_ERR_INVALID_ARG;
+  ff_head* hd = const_cast<ff_head*>(hdc);
+  FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync");
+  ff_status s;
+  if ((s = head_copy(dV, hd->dV, (size_t)kClasses * hd->F * 4)) != FF_OK) return s;
+  return head_copy(dc, hd->dc, kClasses * 4);
+}
+
+ff_status ff_head_check(ff_head* hd) {
+  if (!hd) return FF_ERR_INVALID_ARG;
+  FF_TRY(cudaStreamSynchronize(hd->last_stream), "check sync");
+  int err = 0;
+  FF_TRY(cudaMemcpy(&err, &hd->ds->err, sizeof(int), cudaMemcpyDeviceToHost), "read error word");
+  if (err) {
+    const int zero = 0;
+    FF_TRY(cudaMemcpy(&hd->ds->err, &zero, sizeof(int), cudaMemcpyHostToDevice), "clear error word");
+  }
+  if (err & DEVERR_TIMEOUT) return FF_ERR_TIMEOUT;
+  if (err & DEVERR_NONFINITE) return FF_ERR_NONFINITE;
+  return FF_OK;
+}
+
+}  // extern "C"

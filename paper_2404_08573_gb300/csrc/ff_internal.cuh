@@ -40,7 +40,8 @@ inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
 
 // Overlay (train/forward) or label-area zeroing (predict), cast, row scale.
 //   mode 0: out[:,0..9] = one-hot(labels[r]); mode 1: out[:,0..9] = 0 and the
-//   norm counts one extra 1.0 (the one-hot every predict overlay adds).
+//   norm counts one extra 1.0 (the one-hot every predict overlay adds);
+//   mode 2: out[:,0..9] = 0.1, the neutral label of the softmax head (§3).
 cudaError_t launch_overlay(const float* x, const int* labels, int rows, int F, void* out,
                            int ldo, bool out_bf16, float* s_out, int mode, cudaStream_t st);
 // s_r = 1 / max(||x_r||, 1e-12) of an activation buffer.

@@ -5,7 +5,8 @@ memory (tensors whose data pointers are passed through) and streams.  There
 is no fallback: if libff.so is missing or the GPU cannot run it, calls raise.
 
 Names follow the C ABI in include/ff.h:
-``Layer`` (ff_layer_*), ``overlay_label``, ``predict``, ``Net`` (ff_net_*).
+``Layer`` (ff_layer_*), ``overlay_label``, ``predict``, ``adaptive_negatives``,
+``Net`` (ff_net_*), ``Head`` (ff_head_*), ``forward_noalloc``.
 """
 
 from __future__ import annotations
@@ -36,6 +37,13 @@ class LayerConfig(ctypes.Structure):
         ("in_features", c_int), ("out_features", c_int), ("has_bias", c_int),
         ("theta", c_float), ("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
         ("prec", c_int), ("init_seed", c_ulonglong), ("max_rows", c_int), ("keep_grad", c_int),
+    ]
+
+
+class HeadConfig(ctypes.Structure):
+    _fields_ = [
+        ("n_features", c_int), ("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
+        ("max_rows", c_int),
     ]
 
 
@@ -75,6 +83,14 @@ def lib():
             "ff_net_sync": [c_void_p, c_void_p],
             "ff_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
                                    c_void_p, c_void_p, c_void_p],
+            "ff_head_create": [POINTER(HeadConfig), POINTER(c_void_p)],
+            "ff_head_destroy": [c_void_p],
+            "ff_head_train_step": [c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
+            "ff_head_predict": [c_void_p, c_void_p, c_int, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
+            "ff_head_get_state": [c_void_p] + [c_void_p] * 6 + [POINTER(c_longlong)],
+            "ff_head_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
+            "ff_head_get_grad": [c_void_p, c_void_p, c_void_p],
+            "ff_head_check": [c_void_p],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -310,3 +326,86 @@ def forward_noalloc(x, row_scale, W_bf16, in_features, out_features, h_out, bias
         int(out_features), _ptr(h_out, torch.bfloat16, "h_out"), _ptr(goodness, torch.float32, "goodness"),
         _ptr(next_scale, torch.float32, "next_scale"), _ptr(device_status, torch.int32, "device_status"),
         c_void_p(_stream(stream))), "ff_forward_noalloc")
+
+
+def _layer_array(layers):
+    return (c_void_p * len(layers))(*[l.handle.value for l in layers])
+
+
+class Head:
+    """The softmax prediction head (``ff_head``) over layers 2..L of a net."""
+
+    N_CLASSES = 10
+
+    def __init__(self, n_features: int, lr: float = 1e-4, beta1: float = 0.9, beta2: float = 0.999,
+                 eps: float = 1e-8, max_rows: int = 0):
+        self.n_features = int(n_features)
+        self.cfg = HeadConfig(self.n_features, lr, beta1, beta2, eps, int(max_rows))
+        h = c_void_p()
+        _check(lib().ff_head_create(ctypes.byref(self.cfg), ctypes.byref(h)), "ff_head_create")
+        self._h = h
+
+    @staticmethod
+    def features_of(layers) -> int:
+        """n_features for a layer chain: out_features of layers 2..L (of layer 1 when L == 1)."""
+        return sum(l.out_features for l in (layers[1:] if len(layers) > 1 else layers))
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(lib().ff_head_destroy(self._h), "ff_head_destroy")
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def train_step(self, layers, x, labels, loss=None, stream=None):
+        n = x.shape[0]
+        if labels.shape[0] != n:
+            raise ValueError("labels must have one entry per row of x")
+        _check(lib().ff_head_train_step(self._h, _layer_array(layers), len(layers), _ptr(x, torch.float32, "x"),
+                                        _ptr(labels, torch.int32, "labels"), n, _ptr(loss, torch.float32, "loss"),
+                                        c_void_p(_stream(stream))), "ff_head_train_step")
+
+    def predict(self, layers, x, pred=None, logits=None, stream=None):
+        """Returns (pred, logits)."""
+        n = x.shape[0]
+        if pred is None:
+            pred = torch.empty(n, dtype=torch.int32, device=x.device)
+        _check(lib().ff_head_predict(self._h, _layer_array(layers), len(layers), _ptr(x, torch.float32, "x"), n,
+                                     _ptr(pred, torch.int32, "pred"), _ptr(logits, torch.float32, "logits"),
+                                     c_void_p(_stream(stream))), "ff_head_predict")
+        return pred, logits
+
+    def get_state(self):
+        C, F = self.N_CLASSES, self.n_features
+        V = np.empty((C, F), np.float32); mV = np.empty_like(V); vV = np.empty_like(V)
+        c = np.empty(C, np.float32); mc = np.empty_like(c); vc = np.empty_like(c)
+        step = c_longlong()
+        _check(lib().ff_head_get_state(self._h, V.ctypes.data, c.ctypes.data, mV.ctypes.data, vV.ctypes.data,
+                                       mc.ctypes.data, vc.ctypes.data, ctypes.byref(step)), "ff_head_get_state")
+        return dict(V=V, c=c, mV=mV, vV=vV, mc=mc, vc=vc, t=step.value)
+
+    def set_state(self, V=None, c=None, mV=None, vV=None, mc=None, vc=None, t=0):
+        C, F = self.N_CLASSES, self.n_features
+
+        def host(a, shape):
+            if a is None:
+                return None, None
+            a = np.ascontiguousarray(np.asarray(a, dtype=np.float32))
+            if a.shape != shape:
+                raise ValueError(f"expected shape {shape}, got {a.shape}")
+            return a, a.ctypes.data
+        keep = [host(V, (C, F)), host(c, (C,)), host(mV, (C, F)), host(vV, (C, F)), host(mc, (C,)), host(vc, (C,))]
+        _check(lib().ff_head_set_state(self._h, *[k[1] for k in keep], int(t)), "ff_head_set_state")
+
+    def get_grad(self):
+        dV = np.empty((self.N_CLASSES, self.n_features), np.float32); dc = np.empty(self.N_CLASSES, np.float32)
+        _check(lib().ff_head_get_grad(self._h, dV.ctypes.data, dc.ctypes.data), "ff_head_get_grad")
+        return dV, dc
+
+    def check(self):
+        _check(lib().ff_head_check(self._h), "ff_head_check")
+
