@@ -410,7 +410,8 @@ PFN_cuTensorMapEncodeTiled_v12000 encode_fn() {
 // Row-major matrix [rows, cols] of bf16 (esize 2) or fp32 (esize 4) with row
 // stride ld (elements), tiled in boxes of box_rows x box_cols with 128-byte
 // swizzle; out-of-range elements of a box read as zero and are not written.
-bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols, int box_rows) {
+bool encode_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols, int box_rows,
+                CUtensorMapSwizzle swz) {
   auto enc = encode_fn();
   if (!enc) return false;
   if ((reinterpret_cast<uintptr_t>(ptr) & 15u) || ((size_t)ld * esize) % 16 != 0) return false;
@@ -419,9 +420,11 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
   cuuint32_t box[2] = {(cuuint32_t)box_cols, (cuuint32_t)box_rows};
   cuuint32_t estr[2] = {1, 1};
   return enc(m, esize == 2 ? CU_TENSOR_MAP_DATA_TYPE_BFLOAT16 : CU_TENSOR_MAP_DATA_TYPE_FLOAT32, 2,
-             const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE,
-             CU_TENSOR_MAP_SWIZZLE_128B, CU_TENSOR_MAP_L2_PROMOTION_L2_256B,
-             CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+             const_cast<void*>(ptr), dims, strides, box, estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swz,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols, int box_rows) {
+  return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
 template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
@@ -465,8 +468,23 @@ constexpr bool USE_PAIR = true;
 constexpr int NSTAGES = 3;       // operand ring depth
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
 constexpr int B_BOX_ROWS = USE_PAIR ? FWD_BN / 2 : FWD_BN;
+// A GEMM that would get fewer than kSmallGridCtas CTAs with two subtiles per
+// CTA (at most a third of the GPU, e.g. 1024 batch rows of a 2000-wide
+// layer) runs with one subtile per CTA instead: twice the CTAs, each with a
+// 6-stage ring of 32 KB stages.
+constexpr int kSmallGridCtas = 64;
+constexpr int NSTAGES_SMALL = 6;
+bool small_grid(int M, int N, int bn) {
+  constexpr int CM = USE_PAIR ? 2 : 1;
+  return (long long)cdiv(cdiv(M, BM * ROW_SUBTILES), CM) * CM * cdiv(N, bn) < kSmallGridCtas;
+}
 
 }  // namespace
+
+bool make_plain_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
+                    int box_rows) {
+  return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_NONE);
+}
 
 bool tc_supported() {
   int dev = 0, major = 0;
@@ -483,6 +501,8 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
   if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, B_BOX_ROWS) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
+  if (small_grid(M, N, FWD_BN))
+    return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
   return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
 }
 
@@ -500,6 +520,9 @@ cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M,
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
+  if (small_grid(M, N, FWD_BN))
+    return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, M, N, K, ep, err,
+                                                                                   st);
   return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
 }
 
@@ -513,6 +536,9 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
+  if (small_grid(N, K, WGRAD_BN))
+    return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, N, K, R, ep, err,
+                                                                                   st);
   return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
 }
 

@@ -10,10 +10,12 @@
 // largest logit.
 //
 // Kernels (all fixed-order reductions, no floating-point atomics):
-//   k_head_logits  one pass over A: z, softmax, per-row loss and dz =
-//                  (softmax(z) - onehot(y)) / n, per-block partials of dc and
-//                  of the loss; A is never materialised -- it is read as the
-//                  stored activities H_k with their row scales s_k
+//   k_head_dot     partial logits A V^T over 1024-feature splits of the
+//                  segments; A is never materialised -- it is read as the
+//                  stored activities H_k times their row scales s_k
+//   k_head_finish  z = c + the splits' partials (in split order), softmax,
+//                  per-row loss and dz = (softmax(z) - onehot(y)) / n,
+//                  per-block partials of dc and of the loss
 //   k_head_wgrad   dV partials per 128-row block: dz^T (s_k H_k)
 //   k_head_adam    reduces the partials in a fixed order, Adam on V and c,
 //                  the step's loss
@@ -24,14 +26,16 @@
 #include "ff_api_internal.h"
 #include "ff_internal.cuh"
 #include "ff_prof.h"
+#include "ff_ptx.cuh"
 
 namespace ff {
 namespace {
 
 constexpr int kClasses = 10;
 constexpr int kMaxSegs = 16;
-constexpr int kLogitRows = 16;   // rows per block of k_head_logits (two per warp)
-constexpr int kLogitChunk = 256; // features per V chunk staged in shared memory (8 per lane)
+constexpr int kDotRows = 64;     // rows per block of k_head_dot (eight per warp)
+constexpr int kSplit = 1024;     // features of one segment per k_head_dot block
+constexpr int kFinRows = 256;    // rows per block of k_head_finish (one per thread)
 constexpr int kWgRows = 128;     // rows per block of k_head_wgrad (16 per warp)
 constexpr int kWgChunk = 128;    // features per block of k_head_wgrad (4 per lane)
 constexpr int kPart = kClasses + 1;  // per-block partials: dc[10], loss
@@ -57,38 +61,6 @@ __device__ __forceinline__ float warp_sum(float v) {
 // h[0..W) = H[row, f .. f+W) as float, zero past the segment or the rows.
 template <typename T, int W>
 __device__ __forceinline__ void load_feats(const T* __restrict__ H, int ld, int row, int n, int f, int F, float* h);
-template <>
-__device__ __forceinline__ void load_feats<bf16, 8>(const bf16* __restrict__ H, int ld, int row, int n, int f, int F,
-                                                    float* h) {
-  if (row < n && f + 8 <= F) {
-    const uint4 q = __ldg(reinterpret_cast<const uint4*>(H + (size_t)row * ld + f));
-    const uint32_t w[4] = {q.x, q.y, q.z, q.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i) {
-      const __nv_bfloat162 p = *reinterpret_cast<const __nv_bfloat162*>(&w[i]);
-      const float2 v = __bfloat1622float2(p);
-      h[2 * i] = v.x;
-      h[2 * i + 1] = v.y;
-    }
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i)
-      h[i] = (row < n && f + i < F) ? __bfloat162float(H[(size_t)row * ld + f + i]) : 0.f;
-  }
-}
-template <>
-__device__ __forceinline__ void load_feats<float, 8>(const float* __restrict__ H, int ld, int row, int n, int f, int F,
-                                                     float* h) {
-  if (row < n && f + 8 <= F) {
-    const float4 a = __ldg(reinterpret_cast<const float4*>(H + (size_t)row * ld + f));
-    const float4 b = __ldg(reinterpret_cast<const float4*>(H + (size_t)row * ld + f + 4));
-    h[0] = a.x; h[1] = a.y; h[2] = a.z; h[3] = a.w;
-    h[4] = b.x; h[5] = b.y; h[6] = b.z; h[7] = b.w;
-  } else {
-#pragma unroll
-    for (int i = 0; i < 8; ++i) h[i] = (row < n && f + i < F) ? H[(size_t)row * ld + f + i] : 0.f;
-  }
-}
 template <>
 __device__ __forceinline__ void load_feats<bf16, 4>(const bf16* __restrict__ H, int ld, int row, int n, int f, int F,
                                                     float* h) {
@@ -151,21 +123,178 @@ __device__ __forceinline__ float finish_row(const float (&z)[kClasses], int row,
   return (m + logf(sum)) - zy;
 }
 
-// One block per kLogitRows rows, two rows per warp.  Each lane takes 8
-// consecutive features of a 256-feature chunk; the chunk of V is staged in
-// shared memory interleaved (Vs[c][e*32 + lane] = V[c][chunk + 8*lane + e])
-// so the lanes read it without bank conflicts.  Segment sums are scaled by
-// the row's s_k before they join the total, so A = s_k H_k is never formed.
+// Number of feature splits: segment k has ceil(F_k / kSplit) of them.
+__host__ __device__ inline int head_splits(const Segs& sg) {
+  int S = 0;
+  for (int k = 0; k < sg.nseg; ++k) S += (sg.F[k] + kSplit - 1) / kSplit;
+  return S;
+}
+
+// One tensor map per segment: H_k as [n, ld_k] with 64-row boxes of 512
+// bytes (256 bf16 or 128 fp32 features), no swizzle.
+struct HeadMaps {
+  CUtensorMap m[kMaxSegs];
+};
+
+constexpr int kDotStages = 2;
+constexpr int kDotStageBytes = kDotRows * 512;
+constexpr int kDotSmem = kDotStages * kDotStageBytes + kSplit * kClasses * 4 + 64;
+
+// zpart[split, row, c] = sum over the split's features f of s_k[row] H_k[row, f] V[c, off_k + f].
+// One block per (split, 64 rows), eight rows per warp.  Thread 0 streams the
+// split's 512-byte-wide row tiles of H_k into a two-stage shared-memory ring
+// with TMA (mbarrier completion; a stage is refilled once all eight warps
+// have arrived on its `empty` barrier); the split's slice of V sits in shared
+// memory interleaved so that lane l's features (FPL consecutive ones per
+// chunk) are read without bank conflicts.  Every wait is bounded.
 template <typename T>
-__global__ void __launch_bounds__(256) k_head_logits(Segs sg, int n, const float* __restrict__ V,
-                                                     const float* __restrict__ cb, const int* __restrict__ labels,
-                                                     float inv_n, float* __restrict__ logits, float* __restrict__ dz,
-                                                     float* __restrict__ part, ff_dev_state* ds, float beta1,
-                                                     float beta2, int* err) {
-  __shared__ float Vs[kClasses][kLogitChunk];
-  __shared__ float rowpart[kLogitRows][kPart];
+__global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ HeadMaps maps, Segs sg, int n,
+                                                     const float* __restrict__ V, float* __restrict__ zpart,
+                                                     int* err) {
+  constexpr int CH = 512 / (int)sizeof(T);  // features per chunk
+  constexpr int FPL = CH / 32;              // features per lane
+  constexpr int NCH = kSplit / CH;          // chunks in a full split
+  extern __shared__ __align__(128) uint8_t dsm[];
+  uint8_t* ring = dsm;
+  float* Vs = reinterpret_cast<float*>(dsm + kDotStages * kDotStageBytes);
+  uint64_t* full = reinterpret_cast<uint64_t*>(Vs + NCH * kClasses * CH);
+  uint64_t* empty = full + kDotStages;
+  volatile int* abort_flag = reinterpret_cast<volatile int*>(empty + kDotStages);
+  volatile int* never_set = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int r0 = blockIdx.x * kLogitRows + warp * 2;
+  int k = 0, sp = blockIdx.x;
+  while (k + 1 < sg.nseg && sp >= (sg.F[k] + kSplit - 1) / kSplit) {
+    sp -= (sg.F[k] + kSplit - 1) / kSplit;
+    ++k;
+  }
+  const int off = sg.off[k];
+  const int fs = sp * kSplit;
+  const int fe = min(fs + kSplit, sg.F[k]);
+  const int nch = (fe - fs + CH - 1) / CH;
+  const int rblk = blockIdx.y * kDotRows;
+  const CUtensorMap* map = &maps.m[k];
+  int issued = 0;
+  if (threadIdx.x == 0) {
+    for (int i = 0; i < kDotStages; ++i) {
+      ptx::mbar_init(&full[i], 1);
+      ptx::mbar_init(&empty[i], 8);
+    }
+    *abort_flag = 0;
+    *never_set = 0;
+    ptx::fence_mbar_init();
+    ptx::prefetch_tmap(map);
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    for (; issued < kDotStages && issued < nch; ++issued) {
+      ptx::mbar_arrive_expect_tx(&full[issued], kDotStageBytes);
+      ptx::tma_load_2d(ring + issued * kDotStageBytes, map, &full[issued], fs + issued * CH, rblk);
+    }
+  }
+  // the split's slice of V, zero past the segment
+  for (int idx = threadIdx.x; idx < NCH * kClasses * CH; idx += 256) {
+    const int ch = idx / (kClasses * CH), rem = idx % (kClasses * CH);
+    const int c = rem / CH, j = rem % CH;
+    const int f = fs + ch * CH + j;
+    Vs[((ch * kClasses + c) * FPL + j % FPL) * 32 + j / FPL] = f < fe ? __ldg(V + (size_t)c * sg.F_total + off + f) : 0.f;
+  }
+  const int r0 = rblk + warp * 8;
+  float srow[8];
+#pragma unroll
+  for (int r = 0; r < 8; ++r) srow[r] = (r0 + r < n) ? __ldg(sg.s[k] + r0 + r) : 0.f;
+  __syncthreads();
+  float acc[8][kClasses];
+#pragma unroll
+  for (int r = 0; r < 8; ++r)
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) acc[r][c] = 0.f;
+  for (int ch = 0; ch < nch; ++ch) {
+    const int s = ch % kDotStages;
+    const uint32_t ph = (uint32_t)(ch / kDotStages) & 1u;
+    if (!ptx::mbar_wait(&full[s], ph, kWaitTimeoutNs, abort_flag)) {
+      *abort_flag = 1;
+      atomicOr(err, DEVERR_TIMEOUT);
+      break;
+    }
+    const uint8_t* tile = ring + s * kDotStageBytes;
+    const float* vch = Vs + ch * kClasses * FPL * 32;
+    // the warp's 8 rows of this chunk (scaled by s_k), then every V value
+    // read once from shared memory serves all 8 rows
+    float h[8][FPL];
+#pragma unroll
+    for (int r = 0; r < 8; ++r) {
+      const uint8_t* rowp = tile + (warp * 8 + r) * 512 + lane * 16;
+      if constexpr (sizeof(T) == 2) {
+        const uint4 q = *reinterpret_cast<const uint4*>(rowp);
+        const uint32_t w[4] = {q.x, q.y, q.z, q.w};
+#pragma unroll
+        for (int i = 0; i < 4; ++i) {
+          const float2 v = __bfloat1622float2(*reinterpret_cast<const __nv_bfloat162*>(&w[i]));
+          h[r][2 * i] = v.x * srow[r];
+          h[r][2 * i + 1] = v.y * srow[r];
+        }
+      } else {
+        const float4 q = *reinterpret_cast<const float4*>(rowp);
+        h[r][0] = q.x * srow[r];
+        h[r][1] = q.y * srow[r];
+        h[r][2] = q.z * srow[r];
+        h[r][3] = q.w * srow[r];
+      }
+    }
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c)
+#pragma unroll
+      for (int e = 0; e < FPL; ++e) {
+        const float v = vch[(c * FPL + e) * 32 + lane];
+#pragma unroll
+        for (int r = 0; r < 8; ++r) acc[r][c] = fmaf(h[r][e], v, acc[r][c]);
+      }
+    __syncwarp();
+    if (lane == 0) ptx::mbar_arrive(&empty[s]);
+    if (threadIdx.x == 0 && issued < nch) {
+      // stage s is refilled with chunk `issued` (= ch + kDotStages) once every warp is done with it
+      if (!ptx::mbar_wait(&empty[s], ph, kWaitTimeoutNs, abort_flag)) {
+        *abort_flag = 1;
+        atomicOr(err, DEVERR_TIMEOUT);
+        break;
+      }
+      ptx::mbar_arrive_expect_tx(&full[s], kDotStageBytes);
+      ptx::tma_load_2d(ring + s * kDotStageBytes, map, &full[s], fs + issued * CH, rblk);
+      ++issued;
+    }
+  }
+  if (*abort_flag) {
+    // copies already issued land before the block's shared memory goes away
+    if (threadIdx.x == 0)
+      for (int ch = issued - kDotStages < 0 ? 0 : issued - kDotStages; ch < issued; ++ch)
+        ptx::mbar_wait(&full[ch % kDotStages], (uint32_t)(ch / kDotStages) & 1u, 10000000ull, never_set);
+    return;
+  }
+#pragma unroll
+  for (int r = 0; r < 8; ++r)
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) acc[r][c] = warp_sum(acc[r][c]);
+  // lane c writes class c of the warp's rows
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) {
+    if (lane != c) continue;
+#pragma unroll
+    for (int r = 0; r < 8; ++r)
+      if (r0 + r < n) zpart[((size_t)blockIdx.x * n + r0 + r) * kClasses + c] = acc[r][c];
+  }
+}
+
+// One thread per row: z = c + sum of the splits' partials (split order),
+// then softmax, loss and dz (training) or the logits (predict).  Per block:
+// the partial sums of dz (for dc) and of the loss, in a fixed order.
+__global__ void __launch_bounds__(kFinRows) k_head_finish(int n, int S, const float* __restrict__ zpart,
+                                                          const float* __restrict__ cb, const int* __restrict__ labels,
+                                                          float inv_n, float* __restrict__ logits,
+                                                          float* __restrict__ dz, float* __restrict__ part,
+                                                          ff_dev_state* ds, float beta1, float beta2, int* err) {
+  __shared__ float red[kFinRows / 32][kPart];
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int row = blockIdx.x * kFinRows + threadIdx.x;
   if (blockIdx.x == 0 && threadIdx.x == 0 && labels && ds) {
     // this step's Adam counter and bias corrections, read by k_head_adam
     ds->t += 1;
@@ -174,73 +303,34 @@ __global__ void __launch_bounds__(256) k_head_logits(Segs sg, int n, const float
     ds->bc1 = (float)(1.0 - ds->pow1);
     ds->bc2 = (float)(1.0 - ds->pow2);
   }
-  float tot[2][kClasses];
-#pragma unroll
-  for (int r = 0; r < 2; ++r)
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) tot[r][c] = 0.f;
-  for (int k = 0; k < sg.nseg; ++k) {
-    const T* H = static_cast<const T*>(sg.H[k]);
-    const int ld = sg.ld[k], Fk = sg.F[k], off = sg.off[k];
-    float seg[2][kClasses];
-#pragma unroll
-    for (int r = 0; r < 2; ++r)
-#pragma unroll
-      for (int c = 0; c < kClasses; ++c) seg[r][c] = 0.f;
-    for (int f0 = 0; f0 < Fk; f0 += kLogitChunk) {
-      __syncthreads();  // the previous chunk is consumed
-      for (int idx = threadIdx.x; idx < kClasses * kLogitChunk; idx += 256) {
-        const int c = idx / kLogitChunk, j = idx % kLogitChunk;
-        Vs[c][(j & 7) * 32 + (j >> 3)] = (f0 + j < Fk) ? __ldg(V + (size_t)c * sg.F_total + off + f0 + j) : 0.f;
-      }
-      __syncthreads();
-#pragma unroll
-      for (int r = 0; r < 2; ++r) {
-        float h[8];
-        load_feats<T, 8>(H, ld, r0 + r, n, f0 + 8 * lane, Fk, h);
-#pragma unroll
-        for (int c = 0; c < kClasses; ++c)
-#pragma unroll
-          for (int e = 0; e < 8; ++e) seg[r][c] = fmaf(h[e], Vs[c][e * 32 + lane], seg[r][c]);
-      }
-    }
-#pragma unroll
-    for (int r = 0; r < 2; ++r) {
-      const float sr = (r0 + r < n) ? __ldg(sg.s[k] + r0 + r) : 0.f;
-#pragma unroll
-      for (int c = 0; c < kClasses; ++c) tot[r][c] = fmaf(sr, seg[r][c], tot[r][c]);
-    }
-  }
-#pragma unroll
-  for (int r = 0; r < 2; ++r)
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) tot[r][c] = warp_sum(tot[r][c]);
-  // lane r finishes row r0 + r
   float dzr[kClasses];
   float loss = 0.f;
-  bool mine = false;
-  if (lane < 2 && r0 + lane < n) {
+#pragma unroll
+  for (int c = 0; c < kClasses; ++c) dzr[c] = 0.f;
+  if (row < n) {
     float z[kClasses];
-    if (lane == 0) {
 #pragma unroll
-      for (int c = 0; c < kClasses; ++c) z[c] = tot[0][c] + __ldg(cb + c);
-    } else {
+    for (int c = 0; c < kClasses; ++c) z[c] = __ldg(cb + c);
+    for (int sp = 0; sp < S; ++sp) {
+      const float* zp = zpart + ((size_t)sp * n + row) * kClasses;
 #pragma unroll
-      for (int c = 0; c < kClasses; ++c) z[c] = tot[1][c] + __ldg(cb + c);
+      for (int c = 0; c < kClasses; ++c) z[c] += __ldg(zp + c);
     }
-    loss = finish_row(z, r0 + lane, labels, inv_n, logits, dz, dzr, err);
-    mine = true;
+    loss = finish_row(z, row, labels, inv_n, logits, dz, dzr, err);
   }
   if (!part) return;
-  if (lane < 2) {
 #pragma unroll
-    for (int c = 0; c < kClasses; ++c) rowpart[warp * 2 + lane][c] = mine ? dzr[c] : 0.f;
-    rowpart[warp * 2 + lane][kClasses] = mine ? loss : 0.f;
+  for (int c = 0; c < kClasses; ++c) dzr[c] = warp_sum(dzr[c]);
+  loss = warp_sum(loss);
+  if (lane == 0) {
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) red[warp][c] = dzr[c];
+    red[warp][kClasses] = loss;
   }
   __syncthreads();
   if (threadIdx.x < kPart) {
     float acc = 0.f;
-    for (int r = 0; r < kLogitRows; ++r) acc += rowpart[r][threadIdx.x];
+    for (int w = 0; w < kFinRows / 32; ++w) acc += red[w][threadIdx.x];
     part[(size_t)blockIdx.x * kPart + threadIdx.x] = acc;
   }
 }
@@ -406,10 +496,18 @@ struct HeadWork {
   void* Hk[kMaxSegs + 1];
   float* gpart;
   float* logits;
+  float* zpart;
   float* dz;
   float* part;
   float* dVpart;
 };
+
+// Feature splits of the layer chain's segments (see head_splits).
+int n_splits(ff_layer* const* layers, int L) {
+  int S = 0;
+  for (int k = (L == 1 ? 0 : 1); k < L; ++k) S += cdiv(layers[k]->N, kSplit);
+  return S;
+}
 
 // Carves the head's workspace for `rows` rows (grown on demand).
 ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, bool train, HeadWork* w) {
@@ -428,8 +526,9 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   for (int k = 0; k < L; ++k) { oH[k] = off; off += align256((size_t)rows * layers[k]->ldN * es); }
   size_t oG = off; off += align256((size_t)ntmax * rows * 4);
   size_t oZ = off; off += align256((size_t)rows * kClasses * 4);
+  size_t oZP = off; off += align256((size_t)n_splits(layers, L) * rows * kClasses * 4);
   size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
-  size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kLogitRows) * kPart * 4 : 0);
+  size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kFinRows) * kPart * 4 : 0);
   size_t oV = off; off += align256(train ? (size_t)cdiv(rows, kWgRows) * kClasses * hd->F * 4 : 0);
   if (off > hd->ws_bytes) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before head workspace growth");
@@ -445,6 +544,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   for (int k = 0; k < L; ++k) w->Hk[k] = base + oH[k];
   w->gpart = reinterpret_cast<float*>(base + oG);
   w->logits = reinterpret_cast<float*>(base + oZ);
+  w->zpart = reinterpret_cast<float*>(base + oZP);
   w->dz = train ? reinterpret_cast<float*>(base + oD) : nullptr;
   w->part = train ? reinterpret_cast<float*>(base + oP) : nullptr;
   w->dVpart = train ? reinterpret_cast<float*>(base + oV) : nullptr;
@@ -504,17 +604,35 @@ Segs make_segs(ff_layer* const* layers, int L, const HeadWork& w, int F) {
   return sg;
 }
 
-cudaError_t launch_head_logits(const Segs& sg, bool b16, int n, const float* V, const float* c, const int* labels,
-                               float* logits, float* dz, float* part, ff_dev_state* ds, float beta1, float beta2,
-                               int* err, cudaStream_t st) {
+// Logits (and, with labels, softmax, loss, dz and the per-block partials)
+// of n rows: k_head_dot over the feature splits, then k_head_finish.
+ff_status head_logits(const Segs& sg, bool b16, int n, const float* V, const float* c, const int* labels,
+                      float* logits, float* zpart, float* dz, float* part, ff_dev_state* ds, float beta1, float beta2,
+                      int* err, cudaStream_t st) {
+  const int S = head_splits(sg);
+  const int es = b16 ? 2 : 4;
+  HeadMaps maps;
+  std::memset(&maps, 0, sizeof(maps));
+  for (int k = 0; k < sg.nseg; ++k)
+    if (!make_plain_map(&maps.m[k], sg.H[k], es, sg.ld[k], n, sg.ld[k], 512 / es, kDotRows))
+      return FF_ERR_INVALID_ARG;
+  static const cudaError_t attr_b = cudaFuncSetAttribute(k_head_dot<bf16>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                                         kDotSmem);
+  static const cudaError_t attr_f = cudaFuncSetAttribute(k_head_dot<float>,
+                                                         cudaFuncAttributeMaxDynamicSharedMemorySize, kDotSmem);
+  FF_TRY(b16 ? attr_b : attr_f, "head kernel attributes");
+  dim3 grid(S, cdiv(n, kDotRows));
+  FF_LAUNCH(K_HEAD_LOGITS, (double)n * sg.F_total * es + (double)n * S * kClasses * 4, st,
+            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, n, V, zpart, err), cudaGetLastError())
+                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, n, V, zpart, err), cudaGetLastError())),
+            "head partial logits");
   const float inv_n = 1.f / (float)n;
-  if (b16)
-    k_head_logits<bf16><<<cdiv(n, kLogitRows), 256, 0, st>>>(sg, n, V, c, labels, inv_n, logits, dz, part, ds, beta1,
-                                                            beta2, err);
-  else
-    k_head_logits<float><<<cdiv(n, kLogitRows), 256, 0, st>>>(sg, n, V, c, labels, inv_n, logits, dz, part, ds,
-                                                             beta1, beta2, err);
-  return cudaGetLastError();
+  FF_LAUNCH(K_HEAD_FINISH, (double)n * (S + 2) * kClasses * 4, st,
+            (k_head_finish<<<cdiv(n, kFinRows), kFinRows, 0, st>>>(n, S, zpart, c, labels, inv_n, logits, dz, part,
+                                                                   ds, beta1, beta2, err),
+             cudaGetLastError()),
+            "head softmax and cross-entropy");
+  return FF_OK;
 }
 
 cudaError_t launch_head_wgrad(const Segs& sg, bool b16, int n, const float* dz, float* dVpart, cudaStream_t st) {
@@ -615,10 +733,9 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
   const Segs sg = make_segs(layers, n_layers, w, hd->F);
   const bool b16 = layers[0]->is_bf16;
   const double es = b16 ? 2.0 : 4.0;
-  FF_LAUNCH(K_HEAD_LOGITS, (double)n * hd->F * es + (double)n * kClasses * 8, st,
-            launch_head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.dz, w.part, hd->ds, hd->cfg.beta1,
-                               hd->cfg.beta2, err, st),
-            "head logits, softmax, cross-entropy");
+  s = head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.zpart, w.dz, w.part, hd->ds, hd->cfg.beta1,
+                  hd->cfg.beta2, err, st);
+  if (s != FF_OK) return s;
   FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
             launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
   HeadAdamArgs a{};
@@ -632,7 +749,7 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
   a.nrb = cdiv(n, kWgRows);
   a.F = hd->F;
   a.part = w.part;
-  a.nlb = cdiv(n, kLogitRows);
+  a.nlb = cdiv(n, kFinRows);
   a.inv_n = 1.f / (float)n;
   a.lr = hd->cfg.lr;
   a.beta1 = hd->cfg.beta1;
@@ -663,7 +780,6 @@ ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, co
   hd->last_stream = st;
   int* err = &hd->ds->err;
   const bool b16 = layers[0]->is_bf16;
-  const double es = b16 ? 2.0 : 4.0;
   const int K0 = layers[0]->K;
   for (int r0 = 0; r0 < n; r0 += C) {
     const int cn = (n - r0) < C ? (n - r0) : C;
@@ -671,9 +787,8 @@ ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, co
     if (s != FF_OK) return s;
     const Segs sg = make_segs(layers, n_layers, w, hd->F);
     float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
-    FF_LAUNCH(K_HEAD_LOGITS, (double)cn * hd->F * es + (double)cn * kClasses * 4, st,
-              launch_head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, nullptr, nullptr, nullptr, 0.f, 0.f, err, st),
-              "head logits");
+    s = head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, w.zpart, nullptr, nullptr, nullptr, 0.f, 0.f, err, st);
+    if (s != FF_OK) return s;
     if (pred)
       FF_LAUNCH(K_ARGMAX, (double)cn * 44, st, launch_argmax(z, cn, nullptr, pred + r0, st), "head argmax");
   }

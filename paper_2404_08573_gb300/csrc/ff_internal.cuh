@@ -120,6 +120,11 @@ cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M,
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K,
                           float* C, int ldc, int* err, cudaStream_t st);
 bool tc_supported();
+// Tensor map of a row-major [rows, cols] bf16 (esize 2) or fp32 (esize 4)
+// matrix with row stride ld, boxes of box_rows x box_cols, no swizzle; false
+// if the pointer or the stride is not 16-byte aligned.
+bool make_plain_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
+                    int box_rows);
 
 // SIMT fp32 GEMMs with the same contracts.
 int simt_fwd_ntiles(int N);
