@@ -33,6 +33,11 @@ What each function follows:
 * ``adaptive_negatives`` -- AdaptiveNEG of §5: the negative label of a sample
   is the incorrect label the network currently predicts most strongly, i.e.
   the goodness-prediction argmax over the 9 wrong labels.
+* ``lr_at``/``chapter_schedule`` -- §3 "Sequential Training" and §4
+  (Algorithm 1, Single-Layer PFF; Algorithm 2 runs the same dependency
+  order on other nodes): the E epochs are cut into S chapters of C = E/S
+  epochs; in chapter c layer i trains C epochs on the output of layer i-1
+  as it stands after that layer's chapter c, then publishes its own output.
 * ``overlay_neutral``/``softmax_features``/``head_*`` -- §3 "Prediction",
   Softmax method: the input carries a neutral label (0.1 in each of the 10
   label features), the activities of all but the first hidden layer feed a
@@ -56,6 +61,12 @@ Readings of points the paper leaves open (the paper states none of them):
    when L == 1), of each layer's activity normalised like a layer input,
    h / max(||h||, 1e-12); cross-entropy averaged over the rows; weights and
    biases start at zero; ties of the logits go to the lowest class.
+9. Learning-rate cooldown (named, not given, in §5.1): constant until epoch
+   f*E, then falling linearly to 0 at epoch E (f = 0.5: the "after the 50th
+   of 100 epochs" of §5.1); f >= 1 keeps it constant.  The epoch of a step is
+   the layer's own epoch count.  Batches run in dataset order every epoch;
+   the negative labels of a chapter are an input (Random/Fixed/AdaptiveNEG
+   choose them).
 
 ``emulate_bf16=True`` rounds (round-to-nearest-even) the operands that the
 bf16-operand mode stores in bfloat16 -- the layer's input activity, W, the
@@ -395,4 +406,55 @@ def head_predict(head: HeadState, A):
     Returns (pred [n] int64, z [n, classes])."""
     z = head_logits(A, head.V, head.c)
     return np.argmax(z, axis=1), z
+
+
+# ------------------------------------------------------ chapter schedule (§4)
+def lr_at(lr0: float, epoch: int, total_epochs: int, cooldown_start: float) -> float:
+    """The learning rate of (0-based) epoch ``epoch`` of ``total_epochs``:
+    lr0 until epoch cooldown_start*E, then linearly down to 0 at epoch E."""
+    if cooldown_start >= 1.0:
+        return lr0
+    e0 = cooldown_start * total_epochs
+    if epoch < e0:
+        return lr0
+    return lr0 * (total_epochs - epoch) / (total_epochs - e0)
+
+
+def pair_batches(n_pairs: int, B: int):
+    """(first row, pairs) of each batch of the batch-major pair layout:
+    batch j occupies rows 2*j*B .. 2*j*B + 2*b (b positive rows, then the
+    same b images with wrong labels)."""
+    out, done = [], 0
+    while done < n_pairs:
+        b = min(B, n_pairs - done)
+        out.append((2 * done, b))
+        done += b
+    return out
+
+
+def chapter_schedule(states, x_pairs, labels_per_chapter, B: int, C: int, theta: float, hp: AdamHyper,
+                     emulate_bf16: bool = False, cooldown_start: float = 1.0):
+    """Chapters c = 1..S of §4 (Single-Layer PFF, Algorithm 1): layer i trains
+    C epochs over the batches of the output of layer i-1 after its chapter c
+    (layer 1: the raw pairs overlaid with chapter c's labels), then its own
+    output with the updated weights is published for layer i+1.  Mutates the
+    states; returns losses [S, L, C * batches] (each train step's loss)."""
+    x_pairs = np.asarray(x_pairs, dtype=np.float64)
+    labels_per_chapter = np.asarray(labels_per_chapter)
+    S = labels_per_chapter.shape[0]
+    L = len(states)
+    bl = pair_batches(x_pairs.shape[0] // 2, B)
+    E = C * S
+    losses = np.zeros((S, L, C * len(bl)))
+    for c in range(S):
+        a = overlay_label(x_pairs, labels_per_chapter[c])
+        for i, st in enumerate(states):
+            for m in range(C):
+                e = c * C + m
+                hpe = AdamHyper(lr_at(hp.lr, e, E, cooldown_start), hp.beta1, hp.beta2, hp.eps)
+                for j, (r0, b) in enumerate(bl):
+                    o = layer_train_step(st, a[r0:r0 + 2 * b], b, theta, hpe, emulate_bf16=emulate_bf16)
+                    losses[c, i, m * len(bl) + j] = o["loss"]
+            a = layer_forward_full(st, a, emulate_bf16=emulate_bf16)["H"]
+    return losses
 

@@ -487,3 +487,107 @@ def test_head_train_step_first_adam_step_and_prediction():
     A2 = rng.random((5, Fs))
     hsel = fo.HeadState(np.eye(10), np.zeros(10))
     assert np.array_equal(fo.head_predict(hsel, A2)[0], np.argmax(A2, axis=1))
+
+
+# ------------------------------------------------- chapter schedule (§4)
+def test_lr_cooldown_closed_forms():
+    assert fo.lr_at(0.01, 0, 100, 0.5) == 0.01
+    assert fo.lr_at(0.01, 49, 100, 0.5) == 0.01
+    assert fo.lr_at(0.01, 50, 100, 0.5) == pytest.approx(0.01)
+    assert fo.lr_at(0.01, 75, 100, 0.5) == pytest.approx(0.005)
+    assert fo.lr_at(0.01, 99, 100, 0.5) == pytest.approx(0.0002)
+    assert fo.lr_at(0.01, 99, 100, 1.0) == 0.01
+    assert fo.lr_at(0.03, 3, 4, 0.0) == pytest.approx(0.0075)
+
+
+def test_pair_batches_cover_the_set_once():
+    bl = fo.pair_batches(10, 4)
+    assert bl == [(0, 4), (8, 4), (16, 2)]
+    assert sum(2 * b for _, b in bl) == 20
+
+
+def _schedule_inputs(P, seed):
+    x = synth.mnist_like(P, seed=seed, features=24)
+    y = synth.labels(P, seed=seed)
+    xs, ls = [], []
+    for r0, b in fo.pair_batches(P, 4):
+        s0 = r0 // 2
+        x2, l2 = synth.pair_batch(x[s0:s0 + b], y[s0:s0 + b], synth.negative_labels(y[s0:s0 + b], seed=seed, start=s0))
+        xs.append(x2)
+        ls.append(l2)
+    return np.concatenate(xs), np.concatenate(ls), y
+
+
+def _fresh_states(dims, seed):
+    rng = np.random.default_rng(seed)
+    return [fo.LayerState(rng.standard_normal((dims[i + 1], dims[i])) * 0.4, rng.standard_normal(dims[i + 1]) * 0.05)
+            for i in range(len(dims) - 1)]
+
+
+def test_chapter_schedule_matches_a_wavefront_replay():
+    """The schedule's dependency order (layer i, chapter c after layer i-1,
+    chapter c and layer i, chapter c-1), replayed along the diagonals
+    t = i + c with every layer's published output kept per chapter, gives
+    the same weights and losses as the chapter-major definition."""
+    dims = (24, 6, 5, 4)
+    P, B, C, S, theta = 10, 4, 2, 3, 0.5
+    x2, l2, y = _schedule_inputs(P, seed=3)
+    rng = np.random.default_rng(4)
+    labs = np.stack([np.concatenate([y, (y + 1 + rng.integers(0, 9, P)) % 10]).astype(np.int32) for _ in range(S)])
+    # the batch-major layout: rebuild per chapter from the per-chapter negatives
+    def chapter_labels(c):
+        out = np.empty(2 * P, np.int32)
+        for r0, b in fo.pair_batches(P, B):
+            s0 = r0 // 2
+            out[r0:r0 + b] = labs[c, s0:s0 + b]
+            out[r0 + b:r0 + 2 * b] = labs[c, P + s0:P + s0 + b]
+        return out
+    lab_pc = np.stack([chapter_labels(c) for c in range(S)])
+    hp = fo.AdamHyper(lr=0.02)
+    ref_states = _fresh_states(dims, 5)
+    losses = fo.chapter_schedule(ref_states, x2, lab_pc, B, C, theta, hp, cooldown_start=0.5)
+    # wavefront replay, written independently
+    st = _fresh_states(dims, 5)
+    L = len(st)
+    published = {}
+    wl = np.zeros_like(losses)
+    E = C * S
+    for t in range(L + S - 1):
+        for i in range(L):
+            c = t - i
+            if not (0 <= c < S):
+                continue
+            inp = fo.overlay_label(x2, lab_pc[c]) if i == 0 else published[(i - 1, c)]
+            k = 0
+            for m in range(C):
+                lr = hp.lr if c * C + m < 0.5 * E else hp.lr * (E - (c * C + m)) / (0.5 * E)
+                for r0, b in fo.pair_batches(P, B):
+                    o = fo.layer_train_step(st[i], inp[r0:r0 + 2 * b], b, theta, fo.AdamHyper(lr=lr))
+                    wl[c, i, k] = o["loss"]
+                    k += 1
+            published[(i, c)] = fo.layer_forward_full(st[i], inp)["H"]
+    np.testing.assert_allclose(wl, losses, rtol=0, atol=0)
+    for a, b in zip(st, ref_states):
+        np.testing.assert_array_equal(a.W, b.W)
+        np.testing.assert_array_equal(a.b, b.b)
+        assert a.t == b.t == S * C * len(fo.pair_batches(P, B))
+
+
+def test_chapter_schedule_without_updates_is_a_fixed_forward():
+    """lr = 0: no weight moves, so every step's loss is the loss of the fixed
+    net on its batch -- computed here from plain forwards."""
+    dims = (24, 6, 5)
+    P, B, theta = 8, 4, 0.3
+    x2, l2, _ = _schedule_inputs(P, seed=6)
+    st = _fresh_states(dims, 7)
+    W0 = [s.W.copy() for s in st]
+    losses = fo.chapter_schedule(st, x2, np.stack([l2, l2]), B, 1, theta, fo.AdamHyper(lr=0.0))
+    assert all(np.array_equal(s.W, w) for s, w in zip(st, W0))
+    a = fo.overlay_label(x2, l2)
+    for i, s in enumerate(st):
+        for j, (r0, b) in enumerate(fo.pair_batches(P, B)):
+            g = fo.goodness(fo.layer_forward(fo.normalise(a[r0:r0 + 2 * b]), s.W, s.b)[1])
+            exp = fo.ff_loss(g, theta, b)
+            assert losses[0, i, j] == pytest.approx(exp, rel=1e-12)
+            assert losses[1, i, j] == pytest.approx(exp, rel=1e-12)
+        a = fo.layer_forward(fo.normalise(a), s.W, s.b)[1]
