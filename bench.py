@@ -523,6 +523,35 @@ def run_other(args):
                     "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
                     "config": {"workload": label, "features": F, "algorithmic_tflop": flops / 1e12}})
+    elif w == "pff_4x2000":
+        # the chapter schedule of §4 on 784-2000x4: 6 chapters of 1 epoch
+        # (60 000 pairs, 1024 per step) per layer, each layer publishing its
+        # output for the next; Single-Layer PFF (one stream per layer)
+        # against the same schedule on one stream (All-Layers with 1 node)
+        P, S = PAIRS_PER_EPOCH, 6
+        X_h, L_h = epoch_inputs()
+        x = torch.from_numpy(X_h).to(dev)
+        labs = torch.from_numpy(np.stack([L_h] * S)).to(dev)
+
+        def one(mode, nodes):
+            layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", theta=THETA, lr=LR, init_seed=1000 + k,
+                               max_rows=2 * BATCH) for k in range(len(NET) - 1)]
+            pff = ff.Pff(layers, P, BATCH, 1, S, mode=mode, nodes=nodes)
+            pff.run(x, labs, 0, S, stream=stream)          # warm-up run (same work)
+            torch.cuda.synchronize()
+            ms = _timed_loop(torch, stream, lambda: pff.run(x, labs, 0, S, stream=stream), 1)
+            pff.close()
+            return ms
+        ms_par = min(one("single_layer", 1) for _ in range(max(1, args.steps // 5)))
+        ms_seq = min(one("all_layers", 1) for _ in range(max(1, args.steps // 5)))
+        pair_epochs = S * P
+        flops = pair_epochs * (train_flops_per_pair() + 2.0 * 2 * sum(NET[k] * NET[k + 1] for k in range(3)))
+        out.update({"metric": "FF chapter-schedule (Single-Layer PFF) pair-epochs/s on 4x2000 net, 4 streams",
+                    "value": round(pair_epochs / (ms_par / 1e3), 1), "unit": "pair-epochs/s",
+                    "ms_per_step": round(ms_par, 3), "dtype": "bf16",
+                    "tflops": round(flops / (ms_par / 1e3) / 1e12, 2),
+                    "one_stream_ms": round(ms_seq, 3), "speedup_vs_one_stream": round(ms_seq / ms_par, 3),
+                    "config": {"workload": f"ff_pff_784-2000x4_bf16_S{S}_C1_P{P}_B{BATCH}"}})
     elif w == "pipeline_5x2000":
         # 784-2000x5, 60 chunks of 1000 pairs; 5 layer streams vs the same steps on one stream
         net5 = [784] + [2000] * 5
@@ -643,7 +672,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="train_4x2000",
                     choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "softmax_predict",
-                             "softmax_train", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
+                             "softmax_train", "pff_4x2000", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")

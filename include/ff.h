@@ -214,6 +214,56 @@ FF_API ff_status ff_head_get_grad(const ff_head* head, float* dV, float* dc);
  * (FF_ERR_NONFINITE for non-finite logits or activities). */
 FF_API ff_status ff_head_check(ff_head* head);
 
+/* ---------------------------------------------------------------------------
+ * Chapter schedule of the pipelined FF algorithms (§4, Algorithms 1 and 2).
+ * The E = C * S training epochs are cut into S chapters of C epochs.  In
+ * chapter c, layer i trains C epochs over the output of layer i-1 as it
+ * stands after that layer's chapter c (layer 1: the raw pairs overlaid with
+ * the chapter's labels), then publishes its own output with the updated
+ * weights.  Single-Layer PFF runs each layer on its own CUDA stream (one
+ * "node" per layer); All-Layers PFF lets `nodes` streams take the chapters in
+ * turn, each training all layers.  Both follow the same dependencies and give
+ * the same weights bit for bit.  Learning-rate cooldown (§5.1 names one but
+ * gives no formula): each layer's lr is constant until epoch
+ * cooldown_start * E of its own epochs, then falls linearly to 0 at E.
+ * ------------------------------------------------------------------------- */
+typedef struct ff_pff ff_pff;
+
+typedef enum { FF_PFF_SINGLE_LAYER = 0, FF_PFF_ALL_LAYERS = 1 } ff_pff_mode;
+
+typedef struct {
+  int n_pairs;             /* P: positive/negative pairs in the training set */
+  int batch_pairs;         /* pairs per train step (the last batch takes the rest) */
+  int epochs_per_chapter;  /* C */
+  int chapters;            /* S, chapters of the whole run (E = C * S) */
+  ff_pff_mode mode;
+  int nodes;               /* FF_PFF_ALL_LAYERS: streams taking chapters in turn (>= 1) */
+  float cooldown_start;    /* fraction of E where the lr cooldown starts; >= 1: none */
+} ff_pff_config;
+
+/* Binds a chain of layers (one precision, out_features of layer k ==
+ * in_features of k+1, layer 1 in_features >= 10) to a schedule: creates its
+ * streams and two chapter slots of published output per layer below the top
+ * (2P rows each, in HBM), and sizes every layer's workspace for a batch.
+ * The layers must outlive the schedule and must not be used elsewhere while
+ * a run is in flight. */
+FF_API ff_status ff_pff_create(ff_layer* const* layers, int n_layers, const ff_pff_config* cfg,
+                               ff_pff** out);
+/* Waits for the schedule's streams and frees it (not the layers).  NULL: no-op. */
+FF_API ff_status ff_pff_destroy(ff_pff* pff);
+
+/* Enqueues chapters first .. first+count-1 (0-based, within 0..S-1; chapters
+ * must be run in order across calls).  x [2P, in_features of layer 1] raw
+ * float32 in the batch-major pair layout (batch j: its b positive rows, then
+ * the same b images as negative rows); labels [count, 2P] int32, chapter by
+ * chapter, in the same row order (the negative rows' labels are the
+ * chapter's negative labels: fixed, random or adaptive).  loss [count, L,
+ * C * batches] (device) or NULL receives every train step's loss.  Nothing
+ * starts before `stream` reaches this call, and `stream` waits for the whole
+ * run; the host returns after enqueueing. */
+FF_API ff_status ff_pff_run(ff_pff* pff, const float* x, const int* labels, int first, int count,
+                            float* loss, void* stream);
+
 /* Copies the layer state to/from caller buffers, which may be host or device
  * memory: W [N,K] and its Adam moments m_W, v_W [N,K]; b, m_b, v_b [N]; the
  * Adam step counter.  Any pointer may be NULL to skip that tensor.  Both calls

@@ -20,7 +20,7 @@ BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libff.so")
 
 SOURCES = ["ff_api.cu", "ff_net.cu", "ff_elem.cu", "ff_gemm_tc.cu", "ff_gemm_simt.cu", "ff_prof.cu", "ff_noalloc.cu",
-           "ff_head.cu"]
+           "ff_head.cu", "ff_pff.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
     "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-Xcompiler", "-fvisibility=hidden",

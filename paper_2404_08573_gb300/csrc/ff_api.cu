@@ -60,7 +60,7 @@ static int gpart_tiles_max(int N) {
 }
 
 // Grows the per-row workspace to at least `rows` rows (one allocation).
-static ff_status ensure_capacity(ff_layer* L, int rows) {
+ff_status ensure_capacity(ff_layer* L, int rows) {
   if (rows <= L->cap) return FF_OK;
   const int cap = ((rows + 127) / 128) * 128;
   const size_t es = L->is_bf16 ? 2 : 4;

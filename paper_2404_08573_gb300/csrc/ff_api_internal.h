@@ -10,6 +10,10 @@ ff_status cuda_status(cudaError_t e, const char* what);
 cudaError_t dev_alloc(void** p, size_t bytes);
 void dev_free(void* p);
 
+// Grows the layer's workspace to at least `rows` rows (waits for the layer's
+// last stream before replacing it).
+ff_status ensure_capacity(ff_layer* L, int rows);
+
 // One layer-local train step (see ff_layer_train_step).  ev_input_read, if
 // not null, is recorded once the raw input x has been consumed (after the
 // overlay; only meaningful when labels are given); ev_forward_done, if not

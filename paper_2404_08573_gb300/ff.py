@@ -6,7 +6,7 @@ is no fallback: if libff.so is missing or the GPU cannot run it, calls raise.
 
 Names follow the C ABI in include/ff.h:
 ``Layer`` (ff_layer_*), ``overlay_label``, ``predict``, ``adaptive_negatives``,
-``Net`` (ff_net_*), ``Head`` (ff_head_*), ``forward_noalloc``.
+``Net`` (ff_net_*), ``Head`` (ff_head_*), ``Pff`` (ff_pff_*), ``forward_noalloc``.
 """
 
 from __future__ import annotations
@@ -44,6 +44,13 @@ class HeadConfig(ctypes.Structure):
     _fields_ = [
         ("n_features", c_int), ("lr", c_float), ("beta1", c_float), ("beta2", c_float), ("eps", c_float),
         ("max_rows", c_int),
+    ]
+
+
+class PffConfig(ctypes.Structure):
+    _fields_ = [
+        ("n_pairs", c_int), ("batch_pairs", c_int), ("epochs_per_chapter", c_int), ("chapters", c_int),
+        ("mode", c_int), ("nodes", c_int), ("cooldown_start", c_float),
     ]
 
 
@@ -91,6 +98,9 @@ def lib():
             "ff_head_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_head_get_grad": [c_void_p, c_void_p, c_void_p],
             "ff_head_check": [c_void_p],
+            "ff_pff_create": [c_void_p, c_int, POINTER(PffConfig), POINTER(c_void_p)],
+            "ff_pff_destroy": [c_void_p],
+            "ff_pff_run": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p],
         }
         for name, args in sig.items():
             f = getattr(L, name)
@@ -408,4 +418,43 @@ class Head:
 
     def check(self):
         _check(lib().ff_head_check(self._h), "ff_head_check")
+
+
+class Pff:
+    """The chapter schedule (``ff_pff``) of a layer chain: Single-Layer PFF
+    (one stream per layer) or All-Layers PFF (``nodes`` streams taking the
+    chapters in turn)."""
+
+    def __init__(self, layers, n_pairs: int, batch_pairs: int, epochs_per_chapter: int, chapters: int,
+                 mode: str = "single_layer", nodes: int = 1, cooldown_start: float = 1.0):
+        if mode not in ("single_layer", "all_layers"):
+            raise ValueError("mode must be 'single_layer' or 'all_layers'")
+        self.layers = list(layers)
+        self.cfg = PffConfig(int(n_pairs), int(batch_pairs), int(epochs_per_chapter), int(chapters),
+                             0 if mode == "single_layer" else 1, int(nodes), float(cooldown_start))
+        h = c_void_p()
+        _check(lib().ff_pff_create(_layer_array(self.layers), len(self.layers), ctypes.byref(self.cfg),
+                                   ctypes.byref(h)), "ff_pff_create")
+        self._h = h
+
+    @property
+    def batches(self) -> int:
+        return (self.cfg.n_pairs + self.cfg.batch_pairs - 1) // self.cfg.batch_pairs
+
+    def close(self):
+        if getattr(self, "_h", None) is not None and self._h.value:
+            _check(lib().ff_pff_destroy(self._h), "ff_pff_destroy")
+            self._h = None
+
+    def __del__(self):
+        try:
+            self.close()
+        except Exception:
+            pass
+
+    def run(self, x, labels, first: int, count: int, loss=None, stream=None):
+        """Enqueues chapters first .. first+count-1; labels [count, 2P] int32."""
+        _check(lib().ff_pff_run(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
+                                int(first), int(count), _ptr(loss, torch.float32, "loss"),
+                                c_void_p(_stream(stream))), "ff_pff_run")
 
