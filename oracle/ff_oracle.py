@@ -38,6 +38,10 @@ What each function follows:
   order on other nodes): the E epochs are cut into S chapters of C = E/S
   epochs; in chapter c layer i trains C epochs on the output of layer i-1
   as it stands after that layer's chapter c, then publishes its own output.
+* ``po_layer_train_step``/``po_predict`` -- Performance-Optimized PFF (§4,
+  "PFF with a new goodness function"): each layer gets its own softmax block
+  and the two are trained together by backpropagation through these two
+  layers only, on the block's cross-entropy; no negative data.
 * ``overlay_neutral``/``softmax_features``/``head_*`` -- §3 "Prediction",
   Softmax method: the input carries a neutral label (0.1 in each of the 10
   label features), the activities of all but the first hidden layer feed a
@@ -67,6 +71,12 @@ Readings of points the paper leaves open (the paper states none of them):
    the layer's own epoch count.  Batches run in dataset order every epoch;
    the negative labels of a chapter are an input (Random/Fixed/AdaptiveNEG
    choose them).
+10. Performance-Optimized layer: the input of layer 1 carries the neutral
+   label; the layer's block reads its raw activity h (z = h V^T + c); the
+   gradient reaching the layer is dz V, masked by the ReLU; the layer and its
+   block each keep their own Adam state and learning rate; the input of the
+   next layer is h from the pre-update weights, as in FF; prediction is the
+   last layer's block's argmax.
 
 ``emulate_bf16=True`` rounds (round-to-nearest-even) the operands that the
 bf16-operand mode stores in bfloat16 -- the layer's input activity, W, the
@@ -457,4 +467,55 @@ def chapter_schedule(states, x_pairs, labels_per_chapter, B: int, C: int, theta:
                     losses[c, i, m * len(bl) + j] = o["loss"]
             a = layer_forward_full(st, a, emulate_bf16=emulate_bf16)["H"]
     return losses
+
+
+# ------------------------------------- Performance-Optimized PFF layer (§4)
+def po_layer_train_step(state: LayerState, head: HeadState, x_in, labels, hp_layer: AdamHyper, hp_head: AdamHyper,
+                        emulate_bf16: bool = False, rounding=None):
+    """One step of a Performance-Optimized PFF layer and its softmax block
+    (§4): z = h V^T + c on the layer's activity h = ReLU(x_hat W^T + b),
+    cross-entropy averaged over the n rows, backpropagation through the block
+    and the layer only, then Adam on W, b and on V, c.  x_in [n, in] is the
+    raw layer input (layer 1: the neutral-labelled image).  Mutates both
+    states; returns the forward quantities, the loss and the gradients."""
+    rnd = rounding if rounding is not None else (bf16_round if emulate_bf16 else _identity)
+    emul = emulate_bf16 or rounding is not None
+    x_in = np.asarray(x_in, dtype=np.float64)
+    s = 1.0 / np.maximum(row_norm(x_in), NORM_EPS)
+    A = rnd(x_in)
+    x_hat = s[:, None] * A
+    Z, H = layer_forward(x_hat, rnd(state.W), state.b)
+    Hs = rnd(H) if emul else H                   # the activity as stored, read by the block
+    z = head_logits(Hs, head.V, head.c)
+    loss = cross_entropy(z, labels)
+    dz = dce_dz(z, labels)
+    dV = dz.T @ Hs
+    dc = np.sum(dz, axis=0)
+    dZ = (dz @ head.V) * (Z > 0)                 # through the block (pre-update V) and the ReLU
+    if emul:
+        G = rnd(s[:, None] * dZ)
+        dW = G.T @ A
+    else:
+        dW = dZ.T @ x_hat
+    db = np.sum(dZ, axis=0)
+    state.t += 1
+    state.W, state.mW, state.vW = adam_update(state.W, dW, state.mW, state.vW, state.t, hp_layer)
+    state.b, state.mb, state.vb = adam_update(state.b, db, state.mb, state.vb, state.t, hp_layer)
+    head.t += 1
+    head.V, head.mV, head.vV = adam_update(head.V, dV, head.mV, head.vV, head.t, hp_head)
+    head.c, head.mc, head.vc = adam_update(head.c, dc, head.mc, head.vc, head.t, hp_head)
+    return dict(H=H, g=goodness(H), s=s, z=z, loss=loss, dz=dz, dW=dW, db=db, dV=dV, dc=dc, dZ=dZ)
+
+
+def po_predict(states, heads, x_raw, emulate_bf16: bool = False):
+    """The last layer's block's prediction on the neutral-labelled input.
+    Returns (pred [n] int64, z [n, classes])."""
+    a = overlay_neutral(x_raw)
+    H = None
+    for st in states:
+        f = layer_forward_full(st, a, emulate_bf16=emulate_bf16)
+        H = f["H"]
+        a = H
+    Hs = bf16_round(H) if emulate_bf16 else H
+    return head_predict(heads[-1], Hs)
 

@@ -591,3 +591,71 @@ def test_chapter_schedule_without_updates_is_a_fixed_forward():
             assert losses[0, i, j] == pytest.approx(exp, rel=1e-12)
             assert losses[1, i, j] == pytest.approx(exp, rel=1e-12)
         a = fo.layer_forward(fo.normalise(a), s.W, s.b)[1]
+
+
+# --------------------------------- Performance-Optimized PFF layer (§4)
+def _po_loss(W, b, V, c, x_in, y):
+    xh = fo.normalise(x_in)
+    H = np.maximum(xh @ W.T + b, 0.0)
+    return fo.cross_entropy(H @ V.T + c, y)
+
+
+def test_po_layer_gradients_match_finite_differences():
+    rng = np.random.default_rng(21)
+    n, K, N = 9, 14, 7
+    x = rng.random((n, K))
+    y = rng.integers(0, 10, n)
+    W = rng.standard_normal((N, K))
+    b = rng.standard_normal(N) * 0.2
+    V = rng.standard_normal((10, N))
+    c = rng.standard_normal(10) * 0.1
+    st, hd = fo.LayerState(W, b), fo.HeadState(V, c)
+    out = fo.po_layer_train_step(st, hd, x, y, fo.AdamHyper(lr=0.0), fo.AdamHyper(lr=0.0))
+    assert out["loss"] == pytest.approx(_po_loss(W, b, V, c, x, y), rel=1e-13)
+    h = 1e-6
+    for (i, j) in [(0, 0), (3, 5), (6, 13), (2, 7)]:
+        Wp, Wm = W.copy(), W.copy()
+        Wp[i, j] += h
+        Wm[i, j] -= h
+        fd = (_po_loss(Wp, b, V, c, x, y) - _po_loss(Wm, b, V, c, x, y)) / (2 * h)
+        assert fd == pytest.approx(out["dW"][i, j], rel=1e-5, abs=1e-9)
+    for i in (0, 3, 6):
+        bp, bm = b.copy(), b.copy()
+        bp[i] += h
+        bm[i] -= h
+        fd = (_po_loss(W, bp, V, c, x, y) - _po_loss(W, bm, V, c, x, y)) / (2 * h)
+        assert fd == pytest.approx(out["db"][i], rel=1e-5, abs=1e-9)
+    for (i, j) in [(0, 0), (9, 6), (4, 2)]:
+        Vp, Vm = V.copy(), V.copy()
+        Vp[i, j] += h
+        Vm[i, j] -= h
+        fd = (_po_loss(W, b, Vp, c, x, y) - _po_loss(W, b, Vm, c, x, y)) / (2 * h)
+        assert fd == pytest.approx(out["dV"][i, j], rel=1e-5, abs=1e-9)
+    np.testing.assert_allclose(out["dc"], fo.dce_dz(out["z"], y).sum(axis=0), rtol=1e-14)
+
+
+def test_po_layer_special_cases():
+    rng = np.random.default_rng(22)
+    n, K, N = 6, 12, 5
+    x = rng.random((n, K))
+    y = rng.integers(0, 10, n)
+    W = rng.standard_normal((N, K))
+    # a zero block: nothing reaches the layer, its Adam step is zero, the loss is log 10
+    st, hd = fo.LayerState(W, np.zeros(N)), fo.HeadState(np.zeros((10, N)), np.zeros(10))
+    out = fo.po_layer_train_step(st, hd, x, y, fo.AdamHyper(), fo.AdamHyper(lr=1e-4))
+    assert out["loss"] == pytest.approx(math.log(10.0), abs=1e-15)
+    assert not out["dW"].any() and not out["db"].any()
+    np.testing.assert_array_equal(st.W, W)
+    # identity rounding reproduces the plain definition
+    V = rng.standard_normal((10, N))
+    a = fo.po_layer_train_step(fo.LayerState(W, np.zeros(N)), fo.HeadState(V, np.zeros(10)), x, y,
+                               fo.AdamHyper(), fo.AdamHyper())
+    b = fo.po_layer_train_step(fo.LayerState(W, np.zeros(N)), fo.HeadState(V, np.zeros(10)), x, y,
+                               fo.AdamHyper(), fo.AdamHyper(), rounding=lambda v: np.asarray(v, np.float64))
+    np.testing.assert_allclose(b["dW"], a["dW"], rtol=1e-12, atol=1e-15)
+    # a dead unit (all pre-activations negative) gets no gradient
+    Wd = W.copy()
+    Wd[2] = -np.abs(Wd[2]) - 1.0
+    o = fo.po_layer_train_step(fo.LayerState(Wd, np.zeros(N)), fo.HeadState(V, np.zeros(10)), x, y,
+                               fo.AdamHyper(), fo.AdamHyper())
+    assert not o["dW"][2].any() and o["db"][2] == 0.0
