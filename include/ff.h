@@ -264,6 +264,37 @@ FF_API ff_status ff_pff_destroy(ff_pff* pff);
 FF_API ff_status ff_pff_run(ff_pff* pff, const float* x, const int* labels, int first, int count,
                             float* loss, void* stream);
 
+/* ---------------------------------------------------------------------------
+ * Performance-Optimized PFF (§4, "a new goodness function"): each layer has
+ * its own softmax block (an ff_head with n_features = the layer's
+ * out_features) and the two are trained together by backpropagation through
+ * these two layers only, on the block's cross-entropy; there is no negative
+ * data.  The block reads the layer's raw activity h: z = h V^T + c.
+ * ------------------------------------------------------------------------- */
+
+/* One step on n rows: the layer's forward pass (raw_input != 0: x is raw
+ * float32 [n, in_features], overlaid with the neutral label 0.1 in features
+ * 0..9; else x is an activation buffer [n, ff_row_stride(in)] with row_scale
+ * [n] or NULL as in ff_layer_forward), the block's logits, the mean
+ * cross-entropy over labels [n] (int32, 0..9), dV = dz^T h, dc = sum dz,
+ * dZ = (dz V) * [h > 0] with the block's weights before this step,
+ * dW = dZ^T x_hat, db = sum dZ, then one Adam step of the layer (its own lr)
+ * and one of the block (the block's lr).  h_out / next_scale (or NULL) take
+ * the activity and the next layer's row scale from the pre-update weights,
+ * as in ff_layer_train_step; loss [1] (device) or NULL.  `block` must have
+ * n_features == the layer's out_features, else FF_ERR_INVALID_ARG. */
+FF_API ff_status ff_po_train_step(ff_layer* layer, ff_head* block, const void* x, int raw_input,
+                                  const float* row_scale, const int* labels, int n, void* h_out,
+                                  float* next_scale, float* loss, void* stream);
+
+/* Prediction of a Performance-Optimized net: the neutral-labelled raw input
+ * x [n, in] runs through layers[0..n_layers-1]; pred [n] (int32) is the
+ * argmax of the last layer's block (`block`, n_features == the last layer's
+ * out_features) on its raw activity, logits [n, 10]; either may be NULL, not
+ * both.  Processed in chunks of the block's max_rows. */
+FF_API ff_status ff_po_predict(ff_layer* const* layers, int n_layers, ff_head* block, const float* x,
+                               int n, int* pred, float* logits, void* stream);
+
 /* Copies the layer state to/from caller buffers, which may be host or device
  * memory: W [N,K] and its Adam moments m_W, v_W [N,K]; b, m_b, v_b [N]; the
  * Adam step counter.  Any pointer may be NULL to skip that tensor.  Both calls

@@ -41,7 +41,8 @@ constexpr int kWgChunk = 128;    // features per block of k_head_wgrad (4 per la
 constexpr int kPart = kClasses + 1;  // per-block partials: dc[10], loss
 
 // The feature segments: segment k is layer (k+2)'s activity (layer 1's when
-// there is one layer), features off[k] .. off[k] + F[k] of A.
+// there is one layer), features off[k] .. off[k] + F[k] of A, scaled per row
+// by s[k] (a null s[k] reads the activity unscaled).
 struct Segs {
   const void* H[kMaxSegs];
   const float* s[kMaxSegs];
@@ -201,7 +202,7 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
   const int r0 = rblk + warp * 8;
   float srow[8];
 #pragma unroll
-  for (int r = 0; r < 8; ++r) srow[r] = (r0 + r < n) ? __ldg(sg.s[k] + r0 + r) : 0.f;
+  for (int r = 0; r < 8; ++r) srow[r] = (r0 + r < n) ? (sg.s[k] ? __ldg(sg.s[k] + r0 + r) : 1.f) : 0.f;
   __syncthreads();
   float acc[8][kClasses];
 #pragma unroll
@@ -358,7 +359,7 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
   for (int idx = threadIdx.x; idx < kWgRows * kClasses; idx += 256) {
     const int i = idx / kClasses, c = idx % kClasses;
     const int row = rb0 + i;
-    dzs[i][c] = row < n ? __ldg(dz + (size_t)row * kClasses + c) * __ldg(sg.s[k] + row) : 0.f;
+    dzs[i][c] = row < n ? __ldg(dz + (size_t)row * kClasses + c) * (sg.s[k] ? __ldg(sg.s[k] + row) : 1.f) : 0.f;
   }
   __syncthreads();
   float acc[kClasses][4];
@@ -390,6 +391,138 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
 #pragma unroll
     for (int w = 0; w < 8; ++w) v += red[w][c][j];
     dVpart[((size_t)blockIdx.y * kClasses + c) * sg.F_total + off + f0 + j] = v;
+  }
+}
+
+// ------------------------------------------ Performance-Optimized layer (§4)
+// The gradient that a layer's softmax block sends back into the layer, one
+// block per 32 rows x 256 columns (block 32 x 8; thread (x, y) owns columns
+// 8x..8x+7 of rows y, y+8, y+16, y+24):
+//   dZ_ij = (sum_c dz_ic V_cj) [h_ij > 0],  G_ij = s_i dZ_ij (weight-gradient
+//   operand, in the activity type),  db partials = sum over the block's rows.
+// V (before this step's update) and dz are staged in shared memory.  Lead
+// blocks (x == 0) also write the next layer's row scale from the forward's
+// goodness partials; block (0, 0) advances the layer's Adam step.
+template <typename T>
+struct V8;
+template <>
+struct V8<bf16> {
+  static __device__ __forceinline__ void load(const bf16* p, float (&v)[8]) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __bfloat1622float2(h[e]);
+      v[2 * e] = f.x;
+      v[2 * e + 1] = f.y;
+    }
+  }
+  static __device__ __forceinline__ void store(bf16* p, const float (&v)[8]) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+    *reinterpret_cast<uint4*>(p) = u;
+  }
+};
+template <>
+struct V8<float> {
+  static __device__ __forceinline__ void load(const float* p, float (&v)[8]) {
+    const float4 a = *reinterpret_cast<const float4*>(p);
+    const float4 b = *reinterpret_cast<const float4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+  static __device__ __forceinline__ void store(float* p, const float (&v)[8]) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+  }
+};
+
+struct PoGradArgs {
+  const float* dz;      // [n, 10]
+  const float* V;       // [10, N] (before this step's update)
+  const float* s;       // [n] row scale of the layer input
+  const float* gpart;   // forward goodness partials [ntiles, n]
+  int ntiles, n, N, ld;
+  float* s_next;        // [n] or null
+  float* dbpart;        // [row blocks, N]
+  ff_dev_state* ds;     // the layer's
+  float beta1, beta2;
+  int* err;
+};
+
+constexpr int kPoRows = 32;
+
+template <typename T>
+__global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restrict__ H, T* __restrict__ G) {
+  __shared__ float Vsh[kClasses][256];
+  __shared__ float dzs[kPoRows][kClasses];
+  __shared__ float red[8][256 + 8];
+  const int r0 = blockIdx.y * kPoRows;
+  const int lane = threadIdx.x, tid = threadIdx.y * 32 + threadIdx.x;
+  const int c0 = blockIdx.x * 256;
+  const int cg = c0 + lane * 8;
+  for (int idx = tid; idx < kClasses * 256; idx += 256) {
+    const int c = idx / 256, j = idx % 256;
+    Vsh[c][j] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
+  }
+  for (int idx = tid; idx < kPoRows * kClasses; idx += 256) {
+    const int i = idx / kClasses, c = idx % kClasses;
+    dzs[i][c] = (r0 + i < a.n) ? __ldg(a.dz + (size_t)(r0 + i) * kClasses + c) : 0.f;
+  }
+  if (blockIdx.x == 0 && tid < kPoRows && r0 + tid < a.n) {
+    float g = 0.f;
+    for (int t = 0; t < a.ntiles; ++t) g += __ldg(a.gpart + (size_t)t * a.n + r0 + tid);
+    if (!isfinite(g)) atomicOr(a.err, DEVERR_NONFINITE);
+    if (a.s_next) {
+      const float r = sqrtf(g);
+      a.s_next[r0 + tid] = r != r ? r : 1.f / fmaxf(r, 1e-12f);
+    }
+  }
+  if (blockIdx.x == 0 && blockIdx.y == 0 && tid == 0) {
+    a.ds->t += 1;
+    a.ds->pow1 *= a.beta1;
+    a.ds->pow2 *= a.beta2;
+    a.ds->bc1 = (float)(1.0 - a.ds->pow1);
+    a.ds->bc2 = (float)(1.0 - a.ds->pow2);
+  }
+  __syncthreads();
+  const bool cols_ok = cg < a.ld;
+  float db[8];
+#pragma unroll
+  for (int e = 0; e < 8; ++e) db[e] = 0.f;
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int li = threadIdx.y + 8 * k;
+    const int i = r0 + li;
+    if (!cols_ok || i >= a.n) continue;
+    float h[8], z[8];
+    V8<T>::load(H + (size_t)i * a.ld + cg, h);
+    const float si = __ldg(a.s + i);
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      float d = 0.f;
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) d = fmaf(dzs[li][c], Vsh[c][lane * 8 + e], d);
+      d = h[e] > 0.f ? d : 0.f;
+      db[e] += d;
+      z[e] = si * d;
+    }
+    V8<T>::store(G + (size_t)i * a.ld + cg, z);
+  }
+#pragma unroll
+  for (int e = 0; e < 8; ++e) red[threadIdx.y][lane * 8 + e] = db[e];
+  __syncthreads();
+  if (threadIdx.y == 0) {
+#pragma unroll
+    for (int e = 0; e < 8; ++e) {
+      const int j = cg + e;
+      float t = 0.f;
+#pragma unroll
+      for (int y = 0; y < 8; ++y) t += red[y][lane * 8 + e];
+      if (j < a.N) a.dbpart[(size_t)blockIdx.y * a.N + j] = t;
+    }
   }
 }
 
@@ -651,6 +784,67 @@ cudaError_t launch_head_wgrad(const Segs& sg, bool b16, int n, const float* dz, 
 
 using namespace ff;
 
+namespace ff {
+namespace {
+
+// Scratch of a softmax block for n rows of a layer of width N, carved from
+// the head's workspace (grown on demand).
+struct PoWork {
+  float *zpart, *dz, *part, *dVpart;
+};
+
+ff_status po_workspace(ff_head* hd, int n, int N, PoWork* w) {
+  size_t off = 0;
+  const size_t oZ = off; off += align256((size_t)cdiv(N, kSplit) * n * kClasses * 4);
+  const size_t oD = off; off += align256((size_t)n * kClasses * 4);
+  const size_t oP = off; off += align256((size_t)cdiv(n, kFinRows) * kPart * 4);
+  const size_t oV = off; off += align256((size_t)cdiv(n, kWgRows) * kClasses * N * 4);
+  if (off > hd->ws_bytes) {
+    FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before workspace growth");
+    dev_free(hd->ws);
+    hd->ws = nullptr;
+    hd->ws_bytes = 0;
+    FF_TRY(dev_alloc(&hd->ws, off), "block workspace");
+    hd->ws_bytes = off;
+  }
+  char* base = static_cast<char*>(hd->ws);
+  w->zpart = reinterpret_cast<float*>(base + oZ);
+  w->dz = reinterpret_cast<float*>(base + oD);
+  w->part = reinterpret_cast<float*>(base + oP);
+  w->dVpart = reinterpret_cast<float*>(base + oV);
+  return FF_OK;
+}
+
+// Adam arguments of the head / block from its state and this step's partials.
+HeadAdamArgs head_adam_args(ff_head* hd, const float* dVpart, int nrb, const float* part, int nlb, int n,
+                            float* loss) {
+  HeadAdamArgs a{};
+  a.V = hd->V;
+  a.mV = hd->mV;
+  a.vV = hd->vV;
+  a.c = hd->c;
+  a.mc = hd->mc;
+  a.vc = hd->vc;
+  a.dVpart = dVpart;
+  a.nrb = nrb;
+  a.F = hd->F;
+  a.part = part;
+  a.nlb = nlb;
+  a.inv_n = 1.f / (float)n;
+  a.lr = hd->cfg.lr;
+  a.beta1 = hd->cfg.beta1;
+  a.beta2 = hd->cfg.beta2;
+  a.eps = hd->cfg.eps;
+  a.ds = hd->ds;
+  a.loss_out = loss ? loss : &hd->ds->loss;
+  a.dV_out = hd->dV;
+  a.dc_out = hd->dc;
+  return a;
+}
+
+}  // namespace
+}  // namespace ff
+
 extern "C" {
 
 ff_status ff_head_create(const ff_head_config* cfg, ff_head** out) {
@@ -738,27 +932,7 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
   if (s != FF_OK) return s;
   FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
             launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
-  HeadAdamArgs a{};
-  a.V = hd->V;
-  a.mV = hd->mV;
-  a.vV = hd->vV;
-  a.c = hd->c;
-  a.mc = hd->mc;
-  a.vc = hd->vc;
-  a.dVpart = w.dVpart;
-  a.nrb = cdiv(n, kWgRows);
-  a.F = hd->F;
-  a.part = w.part;
-  a.nlb = cdiv(n, kFinRows);
-  a.inv_n = 1.f / (float)n;
-  a.lr = hd->cfg.lr;
-  a.beta1 = hd->cfg.beta1;
-  a.beta2 = hd->cfg.beta2;
-  a.eps = hd->cfg.eps;
-  a.ds = hd->ds;
-  a.loss_out = loss ? loss : &hd->ds->loss;
-  a.dV_out = hd->dV;
-  a.dc_out = hd->dc;
+  const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kFinRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
   FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st,
             (k_head_adam<<<vblocks + 1, 256, 0, st>>>(a), cudaGetLastError()), "head Adam");
@@ -863,6 +1037,179 @@ ff_status ff_head_check(ff_head* hd) {
   }
   if (err & DEVERR_TIMEOUT) return FF_ERR_TIMEOUT;
   if (err & DEVERR_NONFINITE) return FF_ERR_NONFINITE;
+  return FF_OK;
+}
+
+// ------------------------------------------ Performance-Optimized layer (§4)
+ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_input, const float* row_scale,
+                           const int* labels, int n, void* h_out, float* next_scale, float* loss, void* stream) {
+  if (!L || !hd || n < 0) return FF_ERR_INVALID_ARG;
+  if (hd->F != L->N) return FF_ERR_INVALID_ARG;
+  if (raw_input && L->K < kClasses) return FF_ERR_INVALID_ARG;
+  if (n == 0) return FF_OK;
+  if (!x || !labels) return FF_ERR_INVALID_ARG;
+  if (h_out && (reinterpret_cast<uintptr_t>(h_out) & 15u)) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  ff_status s = ensure_capacity(L, n);
+  if (s != FF_OK) return s;
+  PoWork w;
+  s = po_workspace(hd, n, L->N, &w);
+  if (s != FF_OK) return s;
+  L->last_stream = st;
+  hd->last_stream = st;
+  const bool b16 = L->is_bf16;
+  const double es = b16 ? 2.0 : 4.0;
+  const int K = L->K, N = L->N;
+  // the layer's forward pass (layer 1: the neutral-labelled raw input)
+  const void* X;
+  const float* sc;
+  if (raw_input) {
+    FF_LAUNCH(K_OVERLAY, (double)n * (K * 4.0 + L->ldK * es + 4), st,
+              launch_overlay(static_cast<const float*>(x), nullptr, n, K, L->X, L->ldK, b16, L->s_in, 2, st),
+              "neutral-label overlay");
+    X = L->X;
+    sc = L->s_in;
+  } else {
+    X = x;
+    if (row_scale) {
+      sc = row_scale;
+    } else {
+      FF_LAUNCH(K_ROW_SCALE, (double)n * (K * es + 4), st, launch_row_scale(x, L->ldK, b16, n, K, L->s_in, st),
+                "row scale");
+      sc = L->s_in;
+    }
+  }
+  void* H = h_out ? h_out : L->H;
+  EpiArgs ep{sc, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
+  int ntiles;
+  if (b16) {
+    ntiles = tc_fwd_ntiles(N);
+    FF_LAUNCH(K_FWD_TC, 2.0 * n * N * K, st,
+              tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, n, N, K, ep, &L->ds->err, st),
+              "forward GEMM (tcgen05)");
+  } else {
+    ntiles = simt_fwd_ntiles(N);
+    FF_LAUNCH(K_FWD_SIMT, 2.0 * n * N * K, st,
+              simt_gemm_fwd(static_cast<const float*>(X), L->ldK, L->W, K, n, N, K, ep, st), "forward GEMM (fp32)");
+  }
+  // the block on the raw activity: logits, cross-entropy, dz, dV partials
+  Segs sg{};
+  sg.H[0] = H;
+  sg.s[0] = nullptr;
+  sg.ld[0] = L->ldN;
+  sg.F[0] = N;
+  sg.off[0] = 0;
+  sg.nseg = 1;
+  sg.F_total = N;
+  s = head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.zpart, w.dz, w.part, hd->ds, hd->cfg.beta1,
+                  hd->cfg.beta2, &hd->ds->err, st);
+  if (s != FF_OK) return s;
+  FF_LAUNCH(K_HEAD_WGRAD, (double)n * N * es + (double)cdiv(n, kWgRows) * kClasses * N * 4, st,
+            launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "block weight gradient");
+  // the gradient reaching the layer, with the block's weights before its update
+  PoGradArgs pa{};
+  pa.dz = w.dz;
+  pa.V = hd->V;
+  pa.s = sc;
+  pa.gpart = L->gpart;
+  pa.ntiles = ntiles;
+  pa.n = n;
+  pa.N = N;
+  pa.ld = L->ldN;
+  pa.s_next = next_scale;
+  pa.dbpart = L->dbpart;
+  pa.ds = L->ds;
+  pa.beta1 = L->cfg.beta1;
+  pa.beta2 = L->cfg.beta2;
+  pa.err = &L->ds->err;
+  dim3 grid(cdiv(L->ldN, 256), cdiv(n, kPoRows)), block(32, 8);
+  FF_LAUNCH(K_GRAD_PREP, (double)n * L->ldN * es * 2 + (double)cdiv(n, kPoRows) * N * 4, st,
+            (b16 ? (k_po_grad<bf16><<<grid, block, 0, st>>>(pa, static_cast<const bf16*>(H), static_cast<bf16*>(L->dZ)),
+                    cudaGetLastError())
+                 : (k_po_grad<float><<<grid, block, 0, st>>>(pa, static_cast<const float*>(H),
+                                                            static_cast<float*>(L->dZ)),
+                    cudaGetLastError())),
+            "block gradient into the layer");
+  if (b16) {
+    FF_LAUNCH(K_WGRAD_TC, 2.0 * n * N * K, st,
+              tc_gemm_wgrad(static_cast<const bf16*>(L->dZ), L->ldN, static_cast<const bf16*>(X), L->ldK, n, N, K,
+                            L->dW, K, &L->ds->err, st),
+              "weight-gradient GEMM (tcgen05)");
+  } else {
+    FF_LAUNCH(K_WGRAD_SIMT, 2.0 * n * N * K, st,
+              simt_gemm_wgrad(static_cast<const float*>(L->dZ), L->ldN, static_cast<const float*>(X), L->ldK, n, N,
+                              K, L->dW, K, st),
+              "weight-gradient GEMM (fp32)");
+  }
+  AdamArgs aa{};
+  aa.W = L->W;
+  aa.mW = L->mW;
+  aa.vW = L->vW;
+  aa.dW = L->dW;
+  aa.N = N;
+  aa.K = K;
+  aa.Wb = b16 ? L->Wb : nullptr;
+  aa.ldb = L->ldK;
+  aa.b = L->b;
+  aa.mb = L->mb;
+  aa.vb = L->vb;
+  aa.dbpart = L->dbpart;
+  aa.nrb = cdiv(n, kPoRows);
+  aa.db_out = L->db;
+  aa.has_bias = L->cfg.has_bias;
+  aa.lr = L->cfg.lr;
+  aa.beta1 = L->cfg.beta1;
+  aa.beta2 = L->cfg.beta2;
+  aa.eps = L->cfg.eps;
+  aa.ds = L->ds;
+  aa.loss_part = nullptr;
+  aa.loss_out = nullptr;
+  aa.B = n;
+  FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
+  const HeadAdamArgs ha = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kFinRows), n, loss);
+  const int vblocks = cdiv((long long)kClasses * hd->F, 256);
+  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), st,
+            (k_head_adam<<<vblocks + 1, 256, 0, st>>>(ha), cudaGetLastError()), "block Adam");
+  return FF_OK;
+}
+
+ff_status ff_po_predict(ff_layer* const* layers, int n_layers, ff_head* hd, const float* x, int n, int* pred,
+                        float* logits, void* stream) {
+  if (!layers || n_layers < 1 || n_layers > kMaxSegs + 1 || !hd || n < 0) return FF_ERR_INVALID_ARG;
+  for (int k = 0; k < n_layers; ++k) {
+    if (!layers[k]) return FF_ERR_INVALID_ARG;
+    if (layers[k]->is_bf16 != layers[0]->is_bf16) return FF_ERR_INVALID_ARG;
+    if (k > 0 && layers[k]->K != layers[k - 1]->N) return FF_ERR_INVALID_ARG;
+  }
+  if (layers[0]->K < kClasses || hd->F != layers[n_layers - 1]->N) return FF_ERR_INVALID_ARG;
+  if (n == 0) return FF_OK;
+  if (!x || (!pred && !logits)) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  const int C = n < hd->cfg.max_rows ? n : hd->cfg.max_rows;
+  HeadWork w;
+  ff_status s = head_workspace(hd, layers, n_layers, C, false, &w);
+  if (s != FF_OK) return s;
+  hd->last_stream = st;
+  int* err = &hd->ds->err;
+  const bool b16 = layers[0]->is_bf16;
+  ff_layer* top = layers[n_layers - 1];
+  for (int r0 = 0; r0 < n; r0 += C) {
+    const int cn = (n - r0) < C ? (n - r0) : C;
+    s = head_forward(layers, n_layers, x + (size_t)r0 * layers[0]->K, cn, w, err, st);
+    if (s != FF_OK) return s;
+    Segs sg{};
+    sg.H[0] = w.Hk[n_layers - 1];
+    sg.s[0] = nullptr;
+    sg.ld[0] = top->ldN;
+    sg.F[0] = top->N;
+    sg.nseg = 1;
+    sg.F_total = top->N;
+    float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
+    s = head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, w.zpart, nullptr, nullptr, nullptr, 0.f, 0.f, err, st);
+    if (s != FF_OK) return s;
+    if (pred)
+      FF_LAUNCH(K_ARGMAX, (double)cn * 44, st, launch_argmax(z, cn, nullptr, pred + r0, st), "block argmax");
+  }
   return FF_OK;
 }
 

@@ -6,7 +6,8 @@ is no fallback: if libff.so is missing or the GPU cannot run it, calls raise.
 
 Names follow the C ABI in include/ff.h:
 ``Layer`` (ff_layer_*), ``overlay_label``, ``predict``, ``adaptive_negatives``,
-``Net`` (ff_net_*), ``Head`` (ff_head_*), ``Pff`` (ff_pff_*), ``forward_noalloc``.
+``Net`` (ff_net_*), ``Head`` (ff_head_*), ``Pff`` (ff_pff_*), ``po_train_step_raw``/
+``po_train_step_act``/``po_predict`` (ff_po_*), ``forward_noalloc``.
 """
 
 from __future__ import annotations
@@ -98,6 +99,9 @@ def lib():
             "ff_head_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_head_get_grad": [c_void_p, c_void_p, c_void_p],
             "ff_head_check": [c_void_p],
+            "ff_po_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p,
+                                 c_void_p, c_void_p],
+            "ff_po_predict": [c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
             "ff_pff_create": [c_void_p, c_int, POINTER(PffConfig), POINTER(c_void_p)],
             "ff_pff_destroy": [c_void_p],
             "ff_pff_run": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p],
@@ -457,4 +461,38 @@ class Pff:
         _check(lib().ff_pff_run(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
                                 int(first), int(count), _ptr(loss, torch.float32, "loss"),
                                 c_void_p(_stream(stream))), "ff_pff_run")
+
+
+def _po_step(layer, block, x, labels, raw, row_scale, h_out, next_scale, loss, stream):
+    n = x.shape[0]
+    if labels.shape[0] != n:
+        raise ValueError("labels must have one entry per row of x")
+    xp = _ptr(x, torch.float32 if raw else layer.dtype, "x")
+    _check(lib().ff_po_train_step(layer.handle, block._h, xp, int(bool(raw)),
+                                  _ptr(row_scale, torch.float32, "row_scale"), _ptr(labels, torch.int32, "labels"), n,
+                                  _ptr(h_out, layer.dtype, "h_out"), _ptr(next_scale, torch.float32, "next_scale"),
+                                  _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))), "ff_po_train_step")
+
+
+def po_train_step_raw(layer, block, x, labels, h_out=None, next_scale=None, loss=None, stream=None):
+    """ff_po_train_step on raw float32 input rows (the first layer, with the
+    neutral label): one Performance-Optimized step of ``layer`` and its
+    softmax ``block`` (a Head with n_features == layer.out_features)."""
+    _po_step(layer, block, x, labels, True, None, h_out, next_scale, loss, stream)
+
+
+def po_train_step_act(layer, block, x, labels, row_scale=None, h_out=None, next_scale=None, loss=None, stream=None):
+    """ff_po_train_step on an activation buffer of the layer (a hidden layer)."""
+    _po_step(layer, block, x, labels, False, row_scale, h_out, next_scale, loss, stream)
+
+
+def po_predict(layers, block, x, pred=None, logits=None, stream=None):
+    """ff_po_predict: the last layer's block's prediction.  Returns (pred, logits)."""
+    n = x.shape[0]
+    if pred is None:
+        pred = torch.empty(n, dtype=torch.int32, device=x.device)
+    _check(lib().ff_po_predict(_layer_array(layers), len(layers), block._h, _ptr(x, torch.float32, "x"), n,
+                               _ptr(pred, torch.int32, "pred"), _ptr(logits, torch.float32, "logits"),
+                               c_void_p(_stream(stream))), "ff_po_predict")
+    return pred, logits
 
