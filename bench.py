@@ -523,6 +523,40 @@ def run_other(args):
                     "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
                     "config": {"workload": label, "features": F, "algorithmic_tflop": flops / 1e12}})
+    elif w == "po_train":
+        # Performance-Optimized PFF on 784-2000x4: every layer with its own
+        # softmax block, one epoch of 60 000 samples (1024 per step), no
+        # negatives; layer k+1 trains on layer k's activity of the same step
+        n = PAIRS_PER_EPOCH
+        layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", lr=LR, init_seed=1000 + k, max_rows=BATCH)
+                  for k in range(len(NET) - 1)]
+        blocks = [ff.Head(NET[k + 1], lr=1e-4, max_rows=BATCH) for k in range(len(NET) - 1)]
+        x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
+        y = torch.from_numpy(synth.labels(n, seed=7)).to(dev)
+        hs = [layers[k].new_activation(BATCH) for k in range(len(NET) - 2)]
+        ss = [torch.empty(BATCH, device=dev) for _ in range(len(NET) - 2)]
+        steps = [(r, min(BATCH, n - r)) for r in range(0, n, BATCH)]
+
+        def fn():
+            for r, b in steps:
+                for k, (l, bk) in enumerate(zip(layers, blocks)):
+                    last = k == len(layers) - 1
+                    h = None if last else hs[k][:b]
+                    sn = None if last else ss[k][:b]
+                    if k == 0:
+                        ff.po_train_step_raw(l, bk, x[r:r + b], y[r:r + b], h_out=h, next_scale=sn, stream=stream)
+                    else:
+                        ff.po_train_step_act(l, bk, hs[k - 1][:b], y[r:r + b], row_scale=ss[k - 1][:b], h_out=h,
+                                             next_scale=sn, stream=stream)
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        flops = n * (2.0 * 2 * sum(NET[k] * NET[k + 1] for k in range(len(NET) - 1))
+                     + 3 * 2.0 * 10 * sum(NET[1:]))
+        tf = flops / (ms / 1e3) / 1e12
+        out.update({"metric": "FF Performance-Optimized PFF train samples/s (per-layer softmax blocks) on 4x2000 net",
+                    "value": round(n / (ms / 1e3), 1), "unit": "samples/s", "ms_per_step": round(ms, 4),
+                    "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
+                    "config": {"workload": f"ff_po_train_784-2000x4_bf16_epoch{n}_B{BATCH}"}})
     elif w == "pff_4x2000":
         # the chapter schedule of §4 on 784-2000x4: 6 chapters of 1 epoch
         # (60 000 pairs, 1024 per step) per layer, each layer publishing its
@@ -672,7 +706,7 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="train_4x2000",
                     choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "softmax_predict",
-                             "softmax_train", "pff_4x2000", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
+                             "softmax_train", "po_train", "pff_4x2000", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")
