@@ -264,6 +264,10 @@ FF_API ff_status ff_pff_destroy(ff_pff* pff);
 FF_API ff_status ff_pff_run(ff_pff* pff, const float* x, const int* labels, int first, int count,
                             float* loss, void* stream);
 
+/* Host-side bounded wait for everything the schedule has enqueued so far, as
+ * ff_net_wait: FF_OK, or FF_ERR_TIMEOUT after timeout_ms milliseconds. */
+FF_API ff_status ff_pff_wait(ff_pff* pff, unsigned int timeout_ms);
+
 /* ---------------------------------------------------------------------------
  * Performance-Optimized PFF (§4, "a new goodness function"): each layer has
  * its own softmax block (an ff_head with n_features = the layer's
@@ -341,6 +345,12 @@ FF_API ff_status ff_net_train_step(ff_net* net, const float* x, const int* label
  * outside them but that stream, so such a sequence can be captured into a
  * CUDA graph (the layers' workspaces must already be large enough). */
 FF_API ff_status ff_net_sync(ff_net* net, void* stream);
+
+/* Host-side bounded wait: blocks the calling thread until everything the net
+ * has enqueued so far has finished (FF_OK) or timeout_ms milliseconds have
+ * passed (FF_ERR_TIMEOUT; the work keeps running and a later wait can finish
+ * it).  Polls event completion; takes no GPU-side wait of its own. */
+FF_API ff_status ff_net_wait(ff_net* net, unsigned int timeout_ms);
 
 /* ---------------------------------------------------------------------------
  * Allocation-free forward pass.  The paper has no counterpart: this is a

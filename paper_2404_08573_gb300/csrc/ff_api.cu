@@ -6,7 +6,9 @@
 #include <cstdio>
 #include <cstdlib>
 #include <cstring>
+#include <chrono>
 #include <new>
+#include <thread>
 
 #include "ff_api_internal.h"
 #include "ff_internal.cuh"
@@ -57,6 +59,21 @@ static size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 static int gpart_tiles_max(int N) {
   const int a = tc_fwd_ntiles(N), b = simt_fwd_ntiles(N);
   return a > b ? a : b;
+}
+
+ff_status wait_events(const cudaEvent_t* ev, int n, unsigned timeout_ms) {
+  const auto deadline = std::chrono::steady_clock::now() + std::chrono::milliseconds(timeout_ms);
+  for (int k = 0; k < n;) {
+    const cudaError_t e = cudaEventQuery(ev[k]);
+    if (e == cudaSuccess) {
+      ++k;
+      continue;
+    }
+    if (e != cudaErrorNotReady) return cuda_status(e, "event query");
+    if (std::chrono::steady_clock::now() >= deadline) return FF_ERR_TIMEOUT;
+    std::this_thread::sleep_for(std::chrono::microseconds(50));
+  }
+  return FF_OK;
 }
 
 // Grows the per-row workspace to at least `rows` rows (one allocation).
@@ -333,11 +350,13 @@ ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** o
   }
   if (e == cudaSuccess) {
     ProfScope p(K_INIT, (double)nk * 4, st);
-    e = launch_init_weights(L->W, L->N, L->K, cfg->init_seed, st);
+    e = p.injected_failure() ? cudaErrorLaunchOutOfResources
+                             : launch_init_weights(L->W, L->N, L->K, cfg->init_seed, st);
   }
   if (e == cudaSuccess && L->is_bf16) {
     ProfScope p(K_TO_BF16, (double)nk * 4 + (double)L->N * L->ldK * 2, st);
-    e = launch_to_bf16(L->W, L->N, L->K, L->Wb, L->ldK, st);
+    e = p.injected_failure() ? cudaErrorLaunchOutOfResources
+                             : launch_to_bf16(L->W, L->N, L->K, L->Wb, L->ldK, st);
   }
   s = cuda_status(e, "layer initialisation");
   if (s == FF_OK) s = ensure_capacity(L, cfg->max_rows > 0 ? cfg->max_rows : 256);
@@ -359,6 +378,7 @@ ff_status ff_layer_destroy(ff_layer* L) {
 
 ff_status ff_overlay_label(const float* x, const int* labels, int rows, int features, void* out, float* row_scale,
                            ff_precision prec, void* stream) {
+  ff::NvtxRange nvtx_("ff_overlay_label");
   if (rows < 0 || features < 10 || (prec != FF_FP32 && prec != FF_BF16)) return FF_ERR_INVALID_ARG;
   if (rows == 0) return FF_OK;
   if (!x || !labels || !out) return FF_ERR_INVALID_ARG;
@@ -372,6 +392,7 @@ ff_status ff_overlay_label(const float* x, const int* labels, int rows, int feat
 
 ff_status ff_layer_forward(ff_layer* L, const void* x, const int* labels, const float* row_scale, int rows,
                            void* h_out, float* next_scale, float* goodness, void* stream) {
+  ff::NvtxRange nvtx_("ff_layer_forward");
   ff_status cs = check_call(L, x, labels, rows);
   if (cs != FF_OK) return cs;
   if (!h_out && !next_scale && !goodness) return FF_ERR_INVALID_ARG;
@@ -397,6 +418,7 @@ ff_status ff_layer_forward(ff_layer* L, const void* x, const int* labels, const 
 
 ff_status ff_layer_train_step(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B,
                               void* h_out, float* next_scale, float* goodness, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_layer_train_step");
   return train_step_impl(L, x, labels, row_scale, B, h_out, next_scale, goodness, loss,
                          static_cast<cudaStream_t>(stream), nullptr, nullptr);
 }
@@ -522,11 +544,13 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
 
 ff_status ff_predict(ff_layer* const* layers, int n_layers, const float* x, int n, int* pred, float* goodness,
                      void* stream) {
+  ff::NvtxRange nvtx_("ff_predict");
   return predict_impl(layers, n_layers, x, nullptr, n, pred, goodness, static_cast<cudaStream_t>(stream));
 }
 
 ff_status ff_adaptive_negatives(ff_layer* const* layers, int n_layers, const float* x, const int* labels, int n,
                                 int* neg, float* goodness, void* stream) {
+  ff::NvtxRange nvtx_("ff_adaptive_negatives");
   if (n > 0 && !labels) return FF_ERR_INVALID_ARG;
   return predict_impl(layers, n_layers, x, labels, n, neg, goodness, static_cast<cudaStream_t>(stream));
 }

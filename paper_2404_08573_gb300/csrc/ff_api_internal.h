@@ -10,6 +10,11 @@ ff_status cuda_status(cudaError_t e, const char* what);
 cudaError_t dev_alloc(void** p, size_t bytes);
 void dev_free(void* p);
 
+// Host-side bounded wait: polls the events until all have completed
+// (FF_OK) or timeout_ms has passed (FF_ERR_TIMEOUT); a failed event query is
+// reported as its CUDA status.
+ff_status wait_events(const cudaEvent_t* ev, int n, unsigned timeout_ms);
+
 // Grows the layer's workspace to at least `rows` rows (waits for the layer's
 // last stream before replacing it).
 ff_status ensure_capacity(ff_layer* L, int rows);
@@ -36,7 +41,8 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
     ff_status s_;                                                      \
     {                                                                  \
       ::ff::ProfScope p_((kind), (double)(work), (st));                \
-      s_ = ::ff::cuda_status((call), (what));                          \
+      s_ = p_.injected_failure() ? ::ff::injected_launch_failure(what) \
+                                 : ::ff::cuda_status((call), (what));  \
     }                                                                  \
     if (s_ != FF_OK) return s_;                                        \
   } while (0)

@@ -911,6 +911,7 @@ ff_status ff_head_destroy(ff_head* hd) {
 
 ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, const int* labels,
                              int n, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_head_train_step");
   if (!hd || n < 0) return FF_ERR_INVALID_ARG;
   ff_status s = head_layers(hd, layers, n_layers);
   if (s != FF_OK) return s;
@@ -941,6 +942,7 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
 
 ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, int n, int* pred,
                           float* logits, void* stream) {
+  ff::NvtxRange nvtx_("ff_head_predict");
   if (!hd || n < 0) return FF_ERR_INVALID_ARG;
   ff_status s = head_layers(hd, layers, n_layers);
   if (s != FF_OK) return s;
@@ -1043,6 +1045,7 @@ ff_status ff_head_check(ff_head* hd) {
 // ------------------------------------------ Performance-Optimized layer (§4)
 ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_input, const float* row_scale,
                            const int* labels, int n, void* h_out, float* next_scale, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_po_train_step");
   if (!L || !hd || n < 0) return FF_ERR_INVALID_ARG;
   if (hd->F != L->N) return FF_ERR_INVALID_ARG;
   if (raw_input && L->K < kClasses) return FF_ERR_INVALID_ARG;
@@ -1175,6 +1178,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
 
 ff_status ff_po_predict(ff_layer* const* layers, int n_layers, ff_head* hd, const float* x, int n, int* pred,
                         float* logits, void* stream) {
+  ff::NvtxRange nvtx_("ff_po_predict");
   if (!layers || n_layers < 1 || n_layers > kMaxSegs + 1 || !hd || n < 0) return FF_ERR_INVALID_ARG;
   for (int k = 0; k < n_layers; ++k) {
     if (!layers[k]) return FF_ERR_INVALID_ARG;

@@ -14,6 +14,7 @@
 #include <vector>
 
 #include "ff_api_internal.h"
+#include "ff_prof.h"
 
 struct ff_net {
   std::vector<ff_layer*> layers;
@@ -137,6 +138,7 @@ ff_status ff_net_destroy(ff_net* n) {
 }
 
 ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_net_train_step");
   if (!n || !x || !labels || B < 0 || B > n->max_B) return FF_ERR_INVALID_ARG;
   if (B == 0) return FF_OK;
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
@@ -187,6 +189,17 @@ ff_status ff_net_sync(ff_net* n, void* stream) {
   }
   n->since_sync = 0;
   return FF_OK;
+}
+
+ff_status ff_net_wait(ff_net* n, unsigned timeout_ms) {
+  if (!n) return FF_ERR_INVALID_ARG;
+  for (int k = 0; k < n->L; ++k) {
+    ff_status s = ff::cuda_status(cudaEventRecord(n->tail[k], n->streams[k]), "net wait");
+    if (s != FF_OK) return s;
+  }
+  ff_status s = ff::wait_events(n->tail.data(), n->L, timeout_ms);
+  if (s == FF_OK) n->since_sync = 0;  // everything enqueued so far has finished
+  return s;
 }
 
 }  // extern "C"

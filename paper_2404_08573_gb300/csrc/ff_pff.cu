@@ -23,6 +23,7 @@
 #include <vector>
 
 #include "ff_api_internal.h"
+#include "ff_prof.h"
 #include "ff_internal.cuh"
 
 struct ff_pff {
@@ -218,6 +219,7 @@ ff_status ff_pff_destroy(ff_pff* p) {
 }
 
 ff_status ff_pff_run(ff_pff* p, const float* x, const int* labels, int first, int count, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_pff_run");
   if (!p || first < 0 || count < 0 || first + count > p->cfg.chapters) return FF_ERR_INVALID_ARG;
   if (count == 0) return FF_OK;
   if (!x || !labels) return FF_ERR_INVALID_ARG;
@@ -240,6 +242,25 @@ ff_status ff_pff_run(ff_pff* p, const float* x, const int* labels, int first, in
   // the caller's stream waits for every layer's last chapter
   for (int i = 0; i < nl; ++i) FF_TRY(cudaStreamWaitEvent(cs, p->ev_done[i], 0), "run end");
   return FF_OK;
+}
+
+ff_status ff_pff_wait(ff_pff* p, unsigned timeout_ms) {
+  if (!p) return FF_ERR_INVALID_ARG;
+  std::vector<cudaEvent_t> evs;
+  for (size_t k = 0; k < p->streams.size(); ++k) {
+    cudaEvent_t e = nullptr;
+    ff_status s = cuda_status(cudaEventCreateWithFlags(&e, cudaEventDisableTiming), "pff wait");
+    if (s == FF_OK) s = cuda_status(cudaEventRecord(e, p->streams[k]), "pff wait");
+    if (s != FF_OK) {
+      if (e) cudaEventDestroy(e);
+      for (auto x : evs) cudaEventDestroy(x);
+      return s;
+    }
+    evs.push_back(e);
+  }
+  ff_status s = ff::wait_events(evs.data(), (int)evs.size(), timeout_ms);
+  for (auto x : evs) cudaEventDestroy(x);
+  return s;
 }
 
 }  // extern "C"

@@ -7,8 +7,12 @@
 // algorithm must move for the bandwidth-bound kernels).  ff_profile_read
 // waits for the recorded events and returns per-kind totals.
 #include <atomic>
+#include <cstdio>
+#include <cstdlib>
 #include <mutex>
 #include <vector>
+
+#include <nvtx3/nvToolsExt.h>
 
 #include "ff_prof.h"
 
@@ -47,8 +51,21 @@ cudaEvent_t take() {
 
 }  // namespace
 
+long long launch_fail_at() {
+  static const long long v = [] {
+    const char* e = std::getenv("FF_FAULT_LAUNCH_FAIL_AT");
+    return e ? std::atoll(e) : 0ll;
+  }();
+  return v;
+}
+
 ProfScope::ProfScope(KernelKind k, double work, cudaStream_t st) : kind_(k), work_(work), st_(st) {
-  launches.fetch_add(1, std::memory_order_relaxed);
+  const unsigned long long nth = launches.fetch_add(1, std::memory_order_relaxed) + 1;
+  const long long f = launch_fail_at();
+  if (f > 0 && nth == (unsigned long long)f) {
+    injected_ = true;
+    return;
+  }
   std::lock_guard<std::mutex> g(mu);
   if (!enabled) return;
   a_ = take();
@@ -68,6 +85,14 @@ ProfScope::~ProfScope() {
   cudaEventRecord(b_, st_);
   recs.push_back(Rec{kind_, work_, a_, b_, st_});
 }
+
+ff_status injected_launch_failure(const char* what) {
+  if (std::getenv("FF_DEBUG")) std::fprintf(stderr, "libff: %s: injected launch failure\n", what);
+  return FF_ERR_CUDA;
+}
+
+NvtxRange::NvtxRange(const char* name) { nvtxRangePushA(name); }
+NvtxRange::~NvtxRange() { nvtxRangePop(); }
 
 }  // namespace ff
 

@@ -17,6 +17,10 @@ class ProfScope {
  public:
   ProfScope(KernelKind k, double work, cudaStream_t st);
   ~ProfScope();
+  // Host-side fault injection: with FF_FAULT_LAUNCH_FAIL_AT=n in the
+  // environment, the n-th launch of the process (1-based) is not made and
+  // its call reports a launch failure.
+  bool injected_failure() const { return injected_; }
   ProfScope(const ProfScope&) = delete;
   ProfScope& operator=(const ProfScope&) = delete;
 
@@ -25,6 +29,20 @@ class ProfScope {
   double work_;
   cudaStream_t st_;
   cudaEvent_t a_ = nullptr, b_ = nullptr;
+  bool injected_ = false;
+};
+
+// The status a call returns for an injected launch failure.
+ff_status injected_launch_failure(const char* what);
+
+// NVTX range over the scope (shown by profilers that record NVTX; free
+// otherwise).
+class NvtxRange {
+ public:
+  explicit NvtxRange(const char* name);
+  ~NvtxRange();
+  NvtxRange(const NvtxRange&) = delete;
+  NvtxRange& operator=(const NvtxRange&) = delete;
 };
 
 }  // namespace ff

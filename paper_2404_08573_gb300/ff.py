@@ -104,6 +104,8 @@ def lib():
             "ff_po_predict": [c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
             "ff_pff_create": [c_void_p, c_int, POINTER(PffConfig), POINTER(c_void_p)],
             "ff_pff_destroy": [c_void_p],
+            "ff_pff_wait": [c_void_p, ctypes.c_uint],
+            "ff_net_wait": [c_void_p, ctypes.c_uint],
             "ff_pff_run": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p],
         }
         for name, args in sig.items():
@@ -317,6 +319,10 @@ class Net:
     def sync(self, stream=None):
         _check(lib().ff_net_sync(self._h, c_void_p(_stream(stream))), "ff_net_sync")
 
+    def wait(self, timeout_ms: int):
+        """ff_net_wait: host-side wait with a deadline (raises FFError FF_ERR_TIMEOUT)."""
+        _check(lib().ff_net_wait(self._h, int(timeout_ms)), "ff_net_wait")
+
     def close(self):
         if getattr(self, "_h", None) is not None and self._h.value:
             lib().ff_net_destroy(self._h)
@@ -456,6 +462,10 @@ class Pff:
         except Exception:
             pass
 
+    def wait(self, timeout_ms: int):
+        """ff_pff_wait: host-side wait with a deadline (raises FFError FF_ERR_TIMEOUT)."""
+        _check(lib().ff_pff_wait(self._h, int(timeout_ms)), "ff_pff_wait")
+
     def run(self, x, labels, first: int, count: int, loss=None, stream=None):
         """Enqueues chapters first .. first+count-1; labels [count, 2P] int32."""
         _check(lib().ff_pff_run(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
@@ -496,3 +506,35 @@ def po_predict(layers, block, x, pred=None, logits=None, stream=None):
                                c_void_p(_stream(stream))), "ff_po_predict")
     return pred, logits
 
+
+
+def save_checkpoint(path, layers, heads=()):
+    """Writes every layer's and head's full state (parameters, Adam moments
+    and step) to one .npz file, with the shapes needed to check a restore."""
+    arrays = {}
+    for k, l in enumerate(layers):
+        st = l.get_state()
+        for name, v in st.items():
+            arrays[f"layer{k}.{name}"] = np.asarray(v)
+        arrays[f"layer{k}.shape"] = np.array([l.in_features, l.out_features])
+    for k, h in enumerate(heads):
+        st = h.get_state()
+        for name, v in st.items():
+            arrays[f"head{k}.{name}"] = np.asarray(v)
+    np.savez(path, n_layers=np.array(len(layers)), n_heads=np.array(len(heads)), **arrays)
+
+
+def load_checkpoint(path, layers, heads=()):
+    """Restores states written by save_checkpoint into layers (and heads) of
+    the same shapes; raises ValueError on a mismatch."""
+    with np.load(path) as z:
+        if int(z["n_layers"]) != len(layers) or int(z["n_heads"]) != len(heads):
+            raise ValueError("checkpoint holds a different number of layers or heads")
+        for k, l in enumerate(layers):
+            if tuple(z[f"layer{k}.shape"]) != (l.in_features, l.out_features):
+                raise ValueError(f"layer {k}: checkpoint shape {tuple(z[f'layer{k}.shape'])}")
+            l.set_state(**{n: z[f"layer{k}.{n}"] for n in ("W", "b", "mW", "vW", "mb", "vb")},
+                        t=int(z[f"layer{k}.t"]))
+        for k, h in enumerate(heads):
+            h.set_state(**{n: z[f"head{k}.{n}"] for n in ("V", "c", "mV", "vV", "mc", "vc")},
+                        t=int(z[f"head{k}.t"]))
