@@ -310,6 +310,13 @@ FF_API ff_status ff_layer_set_state(ff_layer* layer, const float* W, const float
                              const float* m_W, const float* v_W, const float* m_b,
                              const float* v_b, long long step);
 
+/* Statistics of the last ff_layer_train_step (or ff_net step) of the layer,
+ * for logging: stats[0] = mean goodness of the B positive rows, stats[1] =
+ * mean goodness of the B negative rows, stats[2] = fraction of the 2B x out
+ * activities that are positive (active ReLUs).  Host or device pointer;
+ * waits for the layer's last stream.  Zero before the first step. */
+FF_API ff_status ff_layer_get_stats(const ff_layer* layer, float* stats);
+
 /* The gradient of the last ff_layer_train_step (dW [N,K], db [N], fp32, host
  * or device pointers; NULL skips).  Needs cfg.keep_grad = 1, else
  * FF_ERR_UNSUPPORTED.  Synchronous. */

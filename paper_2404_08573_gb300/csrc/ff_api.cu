@@ -92,6 +92,7 @@ ff_status ensure_capacity(ff_layer* L, int rows) {
   const size_t oN = off; off += align256((size_t)cap * 4);
   const size_t oD = off; off += align256((size_t)local_grad_row_blocks(cap) * L->N * 4);
   const size_t oL = off; off += align256((size_t)(finalize_grid(cap) > local_grad_row_blocks(cap) ? finalize_grid(cap) : local_grad_row_blocks(cap)) * 4);
+  const size_t oT = off; off += align256((size_t)local_grad_row_blocks(cap) * (2 + cdiv(L->ldN, 256)) * 4);
   if (L->cap > 0) {
     FF_TRY(cudaStreamSynchronize(L->last_stream), "sync before workspace growth");
     dev_free(L->X);
@@ -111,6 +112,7 @@ ff_status ensure_capacity(ff_layer* L, int rows) {
   L->s_next = reinterpret_cast<float*>(b + oN);
   L->dbpart = reinterpret_cast<float*>(b + oD);
   L->loss_part = reinterpret_cast<float*>(b + oL);
+  L->stat_part = reinterpret_cast<float*>(b + oT);
   L->cap = cap;
   return FF_OK;
 }
@@ -222,6 +224,8 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   ga.s_next = next_scale;
   ga.dbpart = L->dbpart;
   ga.loss_part = L->loss_part;
+  ga.stat_part = L->stat_part;
+  ga.ncb = cdiv(L->ldN, 256);
   ga.ds = L->ds;
   ga.beta1 = L->cfg.beta1;
   ga.beta2 = L->cfg.beta2;
@@ -264,6 +268,9 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   aa.eps = L->cfg.eps;
   aa.ds = L->ds;
   aa.loss_part = L->loss_part;
+  aa.stat_part = L->stat_part;
+  aa.ncb = cdiv(L->ldN, 256);
+  aa.stats_out = L->ds->stats;
   aa.loss_out = loss ? loss : &L->ds->loss;
   aa.B = B;
   FF_LAUNCH(K_ADAM, (double)L->N * L->K * (28.0 + (L->is_bf16 ? 2.0 : 0.0)) + (double)L->N * (aa.nrb * 4.0 + 28), st,
@@ -610,6 +617,14 @@ ff_status ff_layer_selftest_wait(ff_layer* L, unsigned int timeout_us, void* str
   cudaStream_t st = static_cast<cudaStream_t>(stream);
   L->last_stream = st;
   FF_TRY(launch_wait_selftest(&L->ds->err, 1000ull * timeout_us, st), "bounded-wait self-test");
+  return FF_OK;
+}
+
+ff_status ff_layer_get_stats(const ff_layer* Lc, float* stats) {
+  if (!Lc || !stats) return FF_ERR_INVALID_ARG;
+  ff_layer* L = const_cast<ff_layer*>(Lc);
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  FF_TRY(cudaMemcpy(stats, L->ds->stats, 3 * sizeof(float), cudaMemcpyDefault), "read statistics");
   return FF_OK;
 }
 

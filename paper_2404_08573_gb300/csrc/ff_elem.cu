@@ -213,7 +213,7 @@ constexpr int kGradRows = 32;
 template <typename T>
 __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __restrict__ H, T* __restrict__ dZ) {
   __shared__ float red[8][256 + 8];
-  __shared__ float lred[8];
+  __shared__ float lred[8], gpred[8], gnred[8], ared[8];
   const int r0 = blockIdx.y * kGradRows;
   const bool lead = blockIdx.x == 0;
   const int lane = threadIdx.x;
@@ -231,7 +231,7 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
     }
   }
   // lanes 0..3: row r0 + y + 8 * lane
-  float cc = 0.f, sc = 0.f, lv = 0.f;
+  float cc = 0.f, sc = 0.f, lv = 0.f, gp = 0.f, gn = 0.f;
   if (lane < 4) {
     const int i = r0 + threadIdx.y + 8 * lane;
     if (i < a.M) {
@@ -246,6 +246,7 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
         if (a.g_out) a.g_out[i] = g;
         if (a.s_next) a.s_next[i] = inv_norm(g);
         lv = softplus_f(tt);
+        (pos ? gp : gn) = g;
       }
     }
   }
@@ -266,7 +267,23 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
   }
   if (lead) {
     lv = warp_sum(lv);  // lanes 4..31 contribute 0
-    if (lane == 0) lred[threadIdx.y] = lv;
+    gp = warp_sum(gp);
+    gn = warp_sum(gn);
+    if (lane == 0) {
+      lred[threadIdx.y] = lv;
+      gpred[threadIdx.y] = gp;
+      gnred[threadIdx.y] = gn;
+    }
+  }
+  if (a.stat_part) {
+    // active ReLUs among this thread's values (zero past the rows and columns)
+    float act = 0.f;
+#pragma unroll
+    for (int k = 0; k < 4; ++k)
+#pragma unroll
+      for (int e = 0; e < 8; ++e) act += h[k][e] > 0.f ? 1.f : 0.f;
+    act = warp_sum(act);
+    if (lane == 0) ared[threadIdx.y] = act;
   }
 #pragma unroll
   for (int e = 0; e < 8; ++e) red[threadIdx.y][lane * 8 + e] = db[e];
@@ -280,11 +297,27 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
       for (int y = 0; y < 8; ++y) t += red[y][lane * 8 + e];
       if (j < a.N) a.dbpart[(size_t)blockIdx.y * a.N + j] = t;
     }
+    if (a.stat_part && lane == 0) {
+      float t = 0.f;
+#pragma unroll
+      for (int y = 0; y < 8; ++y) t += ared[y];
+      a.stat_part[2 * gridDim.y + (size_t)blockIdx.y * a.ncb + blockIdx.x] = t;
+    }
     if (lead && lane == 0) {
       float t = 0.f;
 #pragma unroll
       for (int y = 0; y < 8; ++y) t += lred[y];
       a.loss_part[blockIdx.y] = t;
+      if (a.stat_part) {
+        float tp = 0.f, tn = 0.f;
+#pragma unroll
+        for (int y = 0; y < 8; ++y) {
+          tp += gpred[y];
+          tn += gnred[y];
+        }
+        a.stat_part[blockIdx.y] = tp;
+        a.stat_part[gridDim.y + blockIdx.y] = tn;
+      }
     }
     if (lead && blockIdx.y == 0 && lane == 0) {
       // the Adam update that follows is step t; beta^t kept as running products
@@ -377,6 +410,16 @@ __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
       for (int rb = lane; rb < a.nrb; rb += 32) tot += a.loss_part[rb];
       tot = warp_sum(tot);
       if (lane == 0) a.loss_out[0] = tot / (float)a.B;
+    }
+    if (blockIdx.x == w_blocks && w >= 2 && w <= 4 && a.stat_part) {
+      // the step's statistics: mean goodness of the positive and of the
+      // negative rows, and the fraction of active ReLUs
+      const int n = w == 4 ? a.nrb * a.ncb : a.nrb;
+      const float* src = a.stat_part + (w == 2 ? 0 : w == 3 ? a.nrb : 2 * a.nrb);
+      float tot = 0.f;
+      for (int k = lane; k < n; k += 32) tot += src[k];
+      tot = warp_sum(tot);
+      if (lane == 0) a.stats_out[w - 2] = w == 4 ? tot / (2.f * (float)a.B * (float)a.N) : tot / (float)a.B;
     }
     if (w != 0 || j >= a.N) return;
     float db = 0.f;

@@ -30,6 +30,7 @@ struct ff_dev_state {
   float bc1, bc2;     // 1 - beta1^t, 1 - beta2^t of the current update
   int err;            // latched DEVERR_* bits
   float loss;         // loss of the last train step when the caller passed none
+  float stats[3];     // last train step: mean g of positive rows, of negative rows, active-ReLU fraction
 };
 
 inline int row_stride(int features) { return (features + 7) & ~7; }
@@ -68,6 +69,8 @@ struct GradPrepArgs {
   float* s_next;       // [M] or null
   float* dbpart;       // [row blocks, N]
   float* loss_part;    // [row blocks]; the Adam kernel reduces them into the loss
+  float* stat_part;    // [2 * row blocks + row blocks * ncb]: g sums of positive / negative rows, active counts
+  int ncb;             // column blocks (256 columns each)
   ff_dev_state* ds;
   double beta1, beta2;
   int* err;
@@ -84,6 +87,9 @@ struct AdamArgs {
   const float* loss_part;  // [nrb] grad_prep's loss partials of this step, or null
   float* loss_out;         // [1] receives their sum / B
   int B;
+  const float* stat_part;  // grad_prep's statistics partials, or null
+  int ncb;
+  float* stats_out;        // [3] receives the step's statistics
 };
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
@@ -162,6 +168,7 @@ struct ff_layer {
   float* s_next;     // [cap]
   float* dbpart;     // [row blocks, N]
   float* loss_part;  // [max(finalize blocks, row blocks)]
+  float* stat_part;  // [row blocks * (2 + column blocks)] step statistics partials
   // predict scratch (owned here when this layer is layers[0] of ff_predict)
   void* pws; size_t pws_bytes;
 };

@@ -84,6 +84,7 @@ def lib():
             "ff_layer_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
             "ff_layer_check": [c_void_p],
+            "ff_layer_get_stats": [c_void_p, c_void_p],
             "ff_layer_selftest_wait": [c_void_p, ctypes.c_uint, c_void_p],
             "ff_net_create": [c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_destroy": [c_void_p],
@@ -250,6 +251,13 @@ class Layer:
         dW = np.empty((N, K), np.float32); db = np.empty(N, np.float32)
         _check(lib().ff_layer_get_grad(self._h, dW.ctypes.data, db.ctypes.data), "ff_layer_get_grad")
         return dW, db
+
+    def stats(self):
+        """ff_layer_get_stats: (mean positive goodness, mean negative goodness,
+        active-ReLU fraction) of the last train step."""
+        out = np.zeros(3, np.float32)
+        _check(lib().ff_layer_get_stats(self._h, out.ctypes.data), "ff_layer_get_stats")
+        return tuple(float(v) for v in out)
 
     def check(self):
         _check(lib().ff_layer_check(self._h), "ff_layer_check")

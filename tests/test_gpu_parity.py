@@ -488,3 +488,24 @@ def test_wide_hidden_layer_forward_sampled_rows(env):
     ref = fo.layer_forward_full(fo.LayerState(st["W"], st["b"]), xs, emulate_bf16=True)
     assert_close(g.cpu().numpy()[rows], ref["g"], 1e-3, 1e-6, "sampled goodness")
     assert_close(h[rows].float().cpu().numpy()[:, :N], ref["H"], 2.0 ** -8 + 1e-3, 1e-5, "sampled activity")
+
+
+@pytest.mark.parametrize("prec", ["fp32", "bf16"])
+def test_step_statistics(env, prec):
+    """ff_layer_get_stats after a train step: the mean goodness of the
+    positive and of the negative rows and the active-ReLU fraction, against
+    the oracle's forward of the same step."""
+    torch, ff = env
+    B, K, N = 96, 784, 300
+    layer = ff.Layer(K, N, prec=prec, init_seed=3)
+    assert layer.stats() == (0.0, 0.0, 0.0)
+    W = layer.get_state()["W"]
+    x2, l2 = pair_inputs(B, seed=17)
+    layer.train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=B)
+    gp, gn, act = layer.stats()
+    emul = prec == "bf16"
+    ref = fo.layer_forward_full(fo.LayerState(W, np.zeros(N)), fo.overlay_label(x2, l2), emulate_bf16=emul)
+    tol = 1e-5 if not emul else 2e-3
+    assert gp == pytest.approx(ref["g"][:B].mean(), rel=tol)
+    assert gn == pytest.approx(ref["g"][B:].mean(), rel=tol)
+    assert act == pytest.approx(float(np.mean(ref["H"] > 0)), abs=1e-3)
