@@ -58,7 +58,8 @@ typedef enum {
   FF_ERR_OOM = 3,         /* device allocation failed */
   FF_ERR_TIMEOUT = 4,     /* a kernel's bounded wait gave up (latched, see ff_layer_check) */
   FF_ERR_NONFINITE = 5,   /* a goodness value was NaN or Inf (latched) */
-  FF_ERR_UNSUPPORTED = 6  /* valid request this build or device cannot serve */
+  FF_ERR_UNSUPPORTED = 6, /* valid request this build or device cannot serve */
+  FF_ERR_DEVICE_CHECK = 7 /* a device-side check of the checked build failed (see build.py) */
 } ff_status;
 
 typedef enum { FF_FP32 = 0, FF_BF16 = 1 } ff_precision;

@@ -4,6 +4,11 @@ Each translation unit is compiled by nvcc in parallel into ``_build/`` and
 linked into ``paper_2404_08573_gb300/libff.so`` with the CUDA runtime linked
 statically.  A rebuild happens only when a source or header is newer than the
 library (or ``force=True``).
+
+``build(checked=True)`` builds ``libff_checked.so`` instead (``_build_checked/``,
+``-DFF_DEVICE_CHECKS``): the kernels check every TMA coordinate they issue
+(alignment, sign) and latch an error the layer reports, in place of the
+sanitizers this toolchain cannot run here; the arithmetic is unchanged.
 """
 
 from __future__ import annotations
@@ -18,6 +23,8 @@ ROOT = os.path.dirname(HERE)
 CSRC = os.path.join(HERE, "csrc")
 BUILD_DIR = os.path.join(HERE, "_build")
 LIB_PATH = os.path.join(HERE, "libff.so")
+CHECKED_BUILD_DIR = os.path.join(HERE, "_build_checked")
+CHECKED_LIB_PATH = os.path.join(HERE, "libff_checked.so")
 
 SOURCES = ["ff_api.cu", "ff_net.cu", "ff_elem.cu", "ff_gemm_tc.cu", "ff_gemm_simt.cu", "ff_prof.cu", "ff_noalloc.cu",
            "ff_head.cu", "ff_pff.cu"]
@@ -42,23 +49,27 @@ def _deps():
     return files
 
 
-def needs_build() -> bool:
-    if not os.path.exists(LIB_PATH):
+def needs_build(checked: bool = False) -> bool:
+    lib = CHECKED_LIB_PATH if checked else LIB_PATH
+    if not os.path.exists(lib):
         return True
-    t = os.path.getmtime(LIB_PATH)
+    t = os.path.getmtime(lib)
     return any(os.path.getmtime(f) > t for f in _deps())
 
 
-def build(force: bool = False, verbose: bool = False, extra_flags=None) -> str:
-    """Compiles and links libff.so if needed; returns its path."""
-    if not force and not needs_build():
-        return LIB_PATH
+def build(force: bool = False, verbose: bool = False, extra_flags=None, checked: bool = False) -> str:
+    """Compiles and links libff.so (libff_checked.so with checked=True) if
+    needed; returns its path."""
+    lib_path = CHECKED_LIB_PATH if checked else LIB_PATH
+    build_dir = CHECKED_BUILD_DIR if checked else BUILD_DIR
+    if not force and not needs_build(checked):
+        return lib_path
     nvcc = _nvcc()
-    os.makedirs(BUILD_DIR, exist_ok=True)
-    flags = NVCC_FLAGS + list(extra_flags or [])
+    os.makedirs(build_dir, exist_ok=True)
+    flags = NVCC_FLAGS + list(extra_flags or []) + (["-DFF_DEVICE_CHECKS"] if checked else [])
 
     def compile_one(src):
-        obj = os.path.join(BUILD_DIR, os.path.splitext(src)[0] + ".o")
+        obj = os.path.join(build_dir, os.path.splitext(src)[0] + ".o")
         cmd = [nvcc, *flags, "-c", os.path.join(CSRC, src), "-o", obj]
         if verbose:
             print(" ".join(cmd), flush=True)
@@ -71,18 +82,18 @@ def build(force: bool = False, verbose: bool = False, extra_flags=None) -> str:
 
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB_PATH + ".tmp"
+    tmp = lib_path + ".tmp"
     cmd = [nvcc, *ARCH, "-shared", "-cudart", "static", "-o", tmp, *objs, "-lrt", "-ldl", "-lpthread"]
     if verbose:
         print(" ".join(cmd), flush=True)
     r = subprocess.run(cmd, capture_output=True, text=True)
     if r.returncode != 0:
         raise RuntimeError(f"link failed:\n{r.stdout}\n{r.stderr}")
-    os.replace(tmp, LIB_PATH)
-    return LIB_PATH
+    os.replace(tmp, lib_path)
+    return lib_path
 
 
 if __name__ == "__main__":
     import sys
 
-    print(build(force="--force" in sys.argv, verbose=True))
+    print(build(force="--force" in sys.argv, verbose=True, checked="--checked" in sys.argv))

@@ -294,6 +294,7 @@ const char* ff_status_string(ff_status s) {
     case FF_ERR_TIMEOUT: return "FF_ERR_TIMEOUT";
     case FF_ERR_NONFINITE: return "FF_ERR_NONFINITE";
     case FF_ERR_UNSUPPORTED: return "FF_ERR_UNSUPPORTED";
+    case FF_ERR_DEVICE_CHECK: return "FF_ERR_DEVICE_CHECK";
   }
   return "FF_ERR_UNKNOWN";
 }
@@ -638,6 +639,7 @@ ff_status ff_layer_check(ff_layer* L) {
     const int zero = 0;
     FF_TRY(cudaMemcpy(&L->ds->err, &zero, sizeof(int), cudaMemcpyHostToDevice), "clear error word");
   }
+  if (err & DEVERR_CHECK) return FF_ERR_DEVICE_CHECK;  // a skipped copy also runs waits out
   if (err & DEVERR_TIMEOUT) return FF_ERR_TIMEOUT;
   if (err & DEVERR_NONFINITE) return FF_ERR_NONFINITE;
   return FF_OK;

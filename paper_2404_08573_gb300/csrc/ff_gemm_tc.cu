@@ -140,6 +140,10 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       uint32_t full0 = ptx::smem_u32(&full[0]);
       if constexpr (PAIR) full0 = ptx::mapa_shared(full0, 0u);
       auto load = [&](void* dst, const CUtensorMap* map, int s, int c0, int c1) {
+        if (!ff_dcheck(tma_x_aligned(c0, 2), err)) {
+          *abort_flag = 1;
+          return;
+        }
         if constexpr (PAIR)
           ptx::tma_load_2d_pair(dst, map, full0 + 8u * (uint32_t)s, c0, c1);
         else
@@ -333,7 +337,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
                   make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
             ptx::fence_async_smem();
             __syncwarp();
-            if (lane == 0 && rbase < M && col0 < ep.ldo) ptx::tma_store_2d(&tmC, sbuf, col0, rbase);
+            if (lane == 0 && rbase < M && col0 < ep.ldo &&
+                ff_dcheck(col0 >= 0 && rbase >= 0 && tma_x_aligned(col0, 4), err))
+              ptx::tma_store_2d(&tmC, sbuf, col0, rbase);
             if (lane == 0) ptx::bulk_commit();
             ++fchunk;
           } else if (gi < M) {
@@ -364,7 +370,8 @@ __global__ void __launch_bounds__(NTHREADS, 1)
 #pragma unroll 1
             for (int ch = 0; ch < CPW / CW; ++ch) {
               const int col = n0 + cbase + ch * CW;
-              if (col < ep.ldo) ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
+              if (col < ep.ldo && ff_dcheck(col >= 0 && rbase >= 0 && tma_x_aligned(col, 2), err))
+                ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
             }
             ptx::bulk_commit();
           }

@@ -188,6 +188,10 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
   __syncthreads();
   if (threadIdx.x == 0) {
     for (; issued < kDotStages && issued < nch; ++issued) {
+      if (!ff_dcheck(tma_x_aligned(fs + issued * CH, (int)sizeof(T)), err)) {
+        *abort_flag = 1;
+        break;
+      }
       ptx::mbar_arrive_expect_tx(&full[issued], kDotStageBytes);
       ptx::tma_load_2d(ring + issued * kDotStageBytes, map, &full[issued], fs + issued * CH, rblk);
     }
@@ -257,6 +261,10 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
       if (!ptx::mbar_wait(&empty[s], ph, kWaitTimeoutNs, abort_flag)) {
         *abort_flag = 1;
         atomicOr(err, DEVERR_TIMEOUT);
+        break;
+      }
+      if (!ff_dcheck(tma_x_aligned(fs + issued * CH, (int)sizeof(T)), err)) {
+        *abort_flag = 1;
         break;
       }
       ptx::mbar_arrive_expect_tx(&full[s], kDotStageBytes);
@@ -1037,6 +1045,7 @@ ff_status ff_head_check(ff_head* hd) {
     const int zero = 0;
     FF_TRY(cudaMemcpy(&hd->ds->err, &zero, sizeof(int), cudaMemcpyHostToDevice), "clear error word");
   }
+  if (err & DEVERR_CHECK) return FF_ERR_DEVICE_CHECK;  // a skipped copy also runs waits out
   if (err & DEVERR_TIMEOUT) return FF_ERR_TIMEOUT;
   if (err & DEVERR_NONFINITE) return FF_ERR_NONFINITE;
   return FF_OK;

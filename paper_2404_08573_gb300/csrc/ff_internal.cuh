@@ -15,7 +15,22 @@ typedef __nv_bfloat16 bf16;
 namespace ff {
 
 // Device-side error bits latched in ff_dev_state::err.
-enum : int { DEVERR_TIMEOUT = 1, DEVERR_NONFINITE = 2 };
+enum : int { DEVERR_TIMEOUT = 1, DEVERR_NONFINITE = 2, DEVERR_CHECK = 4 };
+
+// Device-side checks of the checked build (-DFF_DEVICE_CHECKS): ff_dcheck(c, err)
+// is c, and latches DEVERR_CHECK in *err when c is false; in the normal build
+// it is true and costs nothing.  Kernels skip the guarded access on failure.
+#ifdef FF_DEVICE_CHECKS
+__device__ __forceinline__ bool ff_dcheck(bool c, int* err) {
+  if (!c) atomicOr(err, DEVERR_CHECK);
+  return c;
+}
+#else
+__device__ __forceinline__ bool ff_dcheck(bool, int*) { return true; }
+#endif
+// A tiled TMA copy must start on a 16-byte boundary of its row: the
+// innermost coordinate times the element size is a multiple of 16.
+__device__ __forceinline__ bool tma_x_aligned(int x, int esize) { return ((long long)x * esize) % 16 == 0; }
 
 // Bound on every spin-wait in a kernel: after this many nanoseconds of
 // %globaltimer the wait gives up, latches DEVERR_TIMEOUT and the kernel

@@ -22,9 +22,11 @@ import torch
 FF_FP32, FF_BF16 = 0, 1
 _STATUS = {
     0: "FF_OK", 1: "FF_ERR_INVALID_ARG", 2: "FF_ERR_CUDA", 3: "FF_ERR_OOM",
-    4: "FF_ERR_TIMEOUT", 5: "FF_ERR_NONFINITE", 6: "FF_ERR_UNSUPPORTED",
+    4: "FF_ERR_TIMEOUT", 5: "FF_ERR_NONFINITE", 6: "FF_ERR_UNSUPPORTED", 7: "FF_ERR_DEVICE_CHECK",
 }
-LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)), "libff.so")
+# FF_LIB_VARIANT=checked loads the build with device-side checks (build.py).
+LIB_PATH = os.path.join(os.path.dirname(os.path.abspath(__file__)),
+                        "libff_checked.so" if os.environ.get("FF_LIB_VARIANT") == "checked" else "libff.so")
 
 
 class FFError(RuntimeError):
