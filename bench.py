@@ -28,12 +28,15 @@ import time
 ROOT = os.path.dirname(os.path.abspath(__file__))
 sys.path.insert(0, ROOT)
 
+from paper_2404_08573_gb300.workloads import WORKLOADS  # noqa: E402  (plain data, no torch)
+
 METRIC = "FF train samples/s (pos+neg pairs) on 4x2000 net, 1 GB300; % of bf16 TC peak"
-NET = [784, 2000, 2000, 2000, 2000]
-PAIRS_PER_EPOCH = 60000
-BATCH = 1024
-THETA, LR = 2.0, 0.03
 WORKLOAD = "ff_train_784-2000x4_bf16_epoch60000_B1024"
+_W = WORKLOADS[WORKLOAD]
+NET = list(_W.net)
+PAIRS_PER_EPOCH = _W.pairs
+BATCH = _W.batch_pairs
+THETA, LR = _W.theta, _W.lr
 
 
 def batches():
