@@ -529,21 +529,35 @@ def run_other(args):
     elif w == "po_train":
         # Performance-Optimized PFF on 784-2000x4: every layer with its own
         # softmax block, one epoch of 60 000 samples (1024 per step), no
-        # negatives; layer k+1 trains on layer k's activity of the same step
+        # negatives; the layers on 4 streams (ff_net_create_po), and the same
+        # steps on one stream for the speed-up
         n = PAIRS_PER_EPOCH
-        layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", lr=LR, init_seed=1000 + k, max_rows=BATCH)
-                  for k in range(len(NET) - 1)]
-        blocks = [ff.Head(NET[k + 1], lr=1e-4, max_rows=BATCH) for k in range(len(NET) - 1)]
         x = torch.from_numpy(synth.mnist_like(n, seed=7)).to(dev)
         y = torch.from_numpy(synth.labels(n, seed=7)).to(dev)
-        hs = [layers[k].new_activation(BATCH) for k in range(len(NET) - 2)]
-        ss = [torch.empty(BATCH, device=dev) for _ in range(len(NET) - 2)]
         steps = [(r, min(BATCH, n - r)) for r in range(0, n, BATCH)]
+
+        def make():
+            ls = [ff.Layer(NET[k], NET[k + 1], prec="bf16", lr=LR, init_seed=1000 + k, max_rows=BATCH)
+                  for k in range(len(NET) - 1)]
+            bs = [ff.Head(NET[k + 1], lr=1e-4, max_rows=BATCH) for k in range(len(NET) - 1)]
+            return ls, bs
+        layers, blocks = make()
+        net = ff.PoNet(layers, blocks, max_rows=BATCH, depth=2)
 
         def fn():
             for r, b in steps:
-                for k, (l, bk) in enumerate(zip(layers, blocks)):
-                    last = k == len(layers) - 1
+                net.train_step(x[r:r + b], y[r:r + b], stream=stream)
+            net.sync(stream)
+        _timed_loop(torch, stream, fn, args.warmup)
+        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        sl, sb = make()
+        hs = [sl[k].new_activation(BATCH) for k in range(len(NET) - 2)]
+        ss = [torch.empty(BATCH, device=dev) for _ in range(len(NET) - 2)]
+
+        def seq():
+            for r, b in steps:
+                for k, (l, bk) in enumerate(zip(sl, sb)):
+                    last = k == len(sl) - 1
                     h = None if last else hs[k][:b]
                     sn = None if last else ss[k][:b]
                     if k == 0:
@@ -551,15 +565,16 @@ def run_other(args):
                     else:
                         ff.po_train_step_act(l, bk, hs[k - 1][:b], y[r:r + b], row_scale=ss[k - 1][:b], h_out=h,
                                              next_scale=sn, stream=stream)
-        _timed_loop(torch, stream, fn, args.warmup)
-        ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
+        _timed_loop(torch, stream, seq, 1)
+        ms_seq = _timed_loop(torch, stream, seq, max(1, args.steps // 2)) / max(1, args.steps // 2)
         flops = n * (2.0 * 2 * sum(NET[k] * NET[k + 1] for k in range(len(NET) - 1))
                      + 3 * 2.0 * 10 * sum(NET[1:]))
         tf = flops / (ms / 1e3) / 1e12
         out.update({"metric": "FF Performance-Optimized PFF train samples/s (per-layer softmax blocks) on 4x2000 net",
                     "value": round(n / (ms / 1e3), 1), "unit": "samples/s", "ms_per_step": round(ms, 4),
                     "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
-                    "config": {"workload": f"ff_po_train_784-2000x4_bf16_epoch{n}_B{BATCH}"}})
+                    "one_stream_ms": round(ms_seq, 4), "speedup_vs_one_stream": round(ms_seq / ms, 3),
+                    "config": {"workload": f"ff_po_train_784-2000x4_bf16_epoch{n}_B{BATCH}_4streams"}})
     elif w == "pff_4x2000":
         # the chapter schedule of §4 on 784-2000x4: 6 chapters of 1 epoch
         # (60 000 pairs, 1024 per step) per layer, each layer publishing its

@@ -292,6 +292,22 @@ FF_API ff_status ff_po_train_step(ff_layer* layer, ff_head* block, const void* x
                                   const float* row_scale, const int* labels, int n, void* h_out,
                                   float* next_scale, float* loss, void* stream);
 
+/* A Performance-Optimized net on one CUDA stream per layer, as ff_net: layer
+ * k and its block (blocks[k], n_features == layers[k] out_features) train
+ * batch t while layer k-1 trains batch t+1; bitwise the same as calling
+ * ff_po_train_step layer after layer.  max_rows: the largest batch (rows);
+ * depth: activation (and label) ring slots.  ff_net_sync, ff_net_wait and
+ * ff_net_destroy apply; ff_net_train_step does not (FF_ERR_INVALID_ARG). */
+FF_API ff_status ff_net_create_po(ff_layer* const* layers, ff_head* const* blocks, int n_layers,
+                                  int max_rows, int depth, ff_net** out);
+/* One batch: x [rows, in] raw float32 (neutral label on layer 1), labels
+ * [rows] int32 (0..9, read by every layer); loss [n_layers] (device) or
+ * NULL gets each layer's block cross-entropy.  The caller's stream waits
+ * until layer 1 has read x; labels are copied before the call returns on
+ * the GPU side of that wait. */
+FF_API ff_status ff_net_po_train_step(ff_net* net, const float* x, const int* labels, int rows,
+                                      float* loss, void* stream);
+
 /* Prediction of a Performance-Optimized net: the neutral-labelled raw input
  * x [n, in] runs through layers[0..n_layers-1]; pred [n] (int32) is the
  * argmax of the last layer's block (`block`, n_features == the last layer's

@@ -15,6 +15,11 @@ void dev_free(void* p);
 // reported as its CUDA status.
 ff_status wait_events(const cudaEvent_t* ev, int n, unsigned timeout_ms);
 
+// Softmax heads (ff_head.cu): the feature count, and dropping a stream that
+// is about to be destroyed from the head's bookkeeping.
+int head_features(const ff_head* h);
+void head_forget_stream(ff_head* h, cudaStream_t st);
+
 // Grows the layer's workspace to at least `rows` rows (waits for the layer's
 // last stream before replacing it).
 ff_status ensure_capacity(ff_layer* L, int rows);

@@ -793,6 +793,12 @@ cudaError_t launch_head_wgrad(const Segs& sg, bool b16, int n, const float* dz, 
 using namespace ff;
 
 namespace ff {
+
+int head_features(const ff_head* h) { return h->F; }
+void head_forget_stream(ff_head* h, cudaStream_t st) {
+  if (h->last_stream == st) h->last_stream = nullptr;
+}
+
 namespace {
 
 // Scratch of a softmax block for n rows of a layer of width N, carved from

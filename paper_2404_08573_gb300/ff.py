@@ -92,6 +92,8 @@ def lib():
             "ff_net_destroy": [c_void_p],
             "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_sync": [c_void_p, c_void_p],
+            "ff_net_create_po": [c_void_p, c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
+            "ff_net_po_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
                                    c_void_p, c_void_p, c_void_p],
             "ff_head_create": [POINTER(HeadConfig), POINTER(c_void_p)],
@@ -548,3 +550,26 @@ def load_checkpoint(path, layers, heads=()):
         for k, h in enumerate(heads):
             h.set_state(**{n: z[f"head{k}.{n}"] for n in ("V", "c", "mV", "vV", "mc", "vc")},
                         t=int(z[f"head{k}.t"]))
+
+
+class PoNet(Net):
+    """A Performance-Optimized net on one CUDA stream per layer
+    (ff_net_create_po): layer k with its softmax block blocks[k]."""
+
+    def __init__(self, layers, blocks, max_rows: int, depth: int = 2):
+        self.layers, self.blocks = list(layers), list(blocks)
+        h = c_void_p()
+        _check(lib().ff_net_create_po(_layer_array(self.layers),
+                                      (c_void_p * len(self.blocks))(*[b._h.value for b in self.blocks]),
+                                      len(self.layers), int(max_rows), int(depth), ctypes.byref(h)),
+               "ff_net_create_po")
+        self._h = h
+
+    def train_step(self, x, labels, loss=None, stream=None):
+        n = x.shape[0]
+        if labels.shape[0] != n:
+            raise ValueError("labels must have one entry per row of x")
+        _check(lib().ff_net_po_train_step(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
+                                          n, _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
+               "ff_net_po_train_step")
+

@@ -75,6 +75,8 @@ def test_invalid_arguments_are_rejected_on_the_host(libff):
     assert libff.ff_pff_wait(None, 10) == 1
     assert libff.ff_net_wait(None, 10) == 1
     assert libff.ff_layer_get_stats(None, None) == 1
+    assert libff.ff_net_create_po(None, None, 2, 8, 2, ctypes.byref(out)) == 1
+    assert libff.ff_net_po_train_step(None, None, None, 4, None, None) == 1
     assert libff.ff_po_train_step(None, None, None, 1, None, None, 4, None, None, None, None) == 1
     assert libff.ff_po_predict(None, 1, None, None, 4, None, None, None) == 1
     assert libff.ff_pff_create(None, 2, None, ctypes.byref(out)) == 1

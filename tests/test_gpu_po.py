@@ -171,3 +171,43 @@ def test_po_argument_errors(env):
     assert layer.get_state()["t"] == 0
     with pytest.raises(ff.FFError):
         ff.po_predict([layer], wrong, x)
+
+
+def test_po_net_on_streams_is_bitwise_sequential(env):
+    """ff_net_create_po: three Performance-Optimized layers on their own
+    streams over five batches (one ragged) give bit for bit the states and
+    losses of the same steps issued layer after layer on one stream."""
+    torch, ff = env
+    dims, rows = (784, 128, 96, 64), [200, 200, 173, 200, 200]
+
+    def make():
+        ls = [ff.Layer(dims[i], dims[i + 1], prec="bf16", init_seed=60 + i, lr=0.003) for i in range(3)]
+        bs = [ff.Head(dims[i + 1], lr=0.01, max_rows=256) for i in range(3)]
+        for i, b in enumerate(bs):
+            b.set_state(V=_block(ff, dims[i + 1], seed=70 + i)[1], c=np.zeros(10, np.float32))
+        return ls, bs
+    data = [(torch.from_numpy(synth.mnist_like(n, seed=80 + t)).cuda(), torch.from_numpy(synth.labels(n, seed=90 + t)).cuda())
+            for t, n in enumerate(rows)]
+    la, ba = make()
+    net = ff.PoNet(la, ba, max_rows=200, depth=2)
+    lp = torch.zeros(len(rows), 3, device="cuda")
+    for t, (x, y) in enumerate(data):
+        net.train_step(x, y, loss=lp[t])
+    net.sync()
+    lb, bb = make()
+    ls = torch.zeros(len(rows), 3, device="cuda")
+    for t, (x, y) in enumerate(data):
+        n = x.shape[0]
+        hs = [lb[k].new_activation(n) for k in range(2)]
+        ss = [torch.empty(n, device="cuda") for _ in range(2)]
+        ff.po_train_step_raw(lb[0], bb[0], x, y, h_out=hs[0], next_scale=ss[0], loss=ls[t, 0:1])
+        ff.po_train_step_act(lb[1], bb[1], hs[0], y, row_scale=ss[0], h_out=hs[1], next_scale=ss[1], loss=ls[t, 1:2])
+        ff.po_train_step_act(lb[2], bb[2], hs[1], y, row_scale=ss[1], loss=ls[t, 2:3])
+    torch.cuda.synchronize()
+    assert torch.equal(lp, ls)
+    for a, b in zip(la + ba, lb + bb):
+        sa, sb = a.get_state(), b.get_state()
+        for k in sa:
+            assert np.array_equal(np.asarray(sa[k]), np.asarray(sb[k])), k
+    with pytest.raises(ff.FFError):
+        net.train_step(data[0][0][:0].new_zeros(300, 784), torch.zeros(300, dtype=torch.int32, device="cuda"))
