@@ -457,6 +457,30 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   // chunk's two activation buffers stay resident in L2 between layers.
   long long per = (40ll << 20) / ((long long)10 * ldmax * es);
   int C = (int)(per < 64 ? 64 : per > 8192 ? 8192 : per);
+  if (b16 && n > C) {
+    // Each forward GEMM CTA holds a whole SM, so a chunk whose GEMMs end in a
+    // nearly empty last wave wastes most of that wave: among chunk sizes
+    // down to half the L2 budget, take the one whose widest hidden GEMM fills
+    // its waves best (the largest on ties).
+    int dev = 0, sms = 0;
+    if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) ==
+                                                   cudaSuccess && sms > 0 && n_layers > 1) {
+      int Nw = 0;
+      for (int k = 1; k < n_layers; ++k)
+        if (layers[k]->N > Nw) Nw = layers[k]->N;
+      double best = -1.0;
+      int bestC = C;
+      for (int c = C; c >= C / 2 && c >= 64; --c) {
+        const int ctas = tc_gemm_fwd_ctas(10 * c, Nw);
+        const double eff = (double)ctas / ((double)cdiv(ctas, sms) * sms);
+        if (eff > best + 1e-9) {
+          best = eff;
+          bestC = c;
+        }
+      }
+      C = bestC;
+    }
+  }
   if (C > n) C = n;
   const int R = 10 * C;
   const int N1 = L0->N;
@@ -464,7 +488,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   const size_t oX = off; off += align256((size_t)C * L0->ldK * es);
   const size_t oS1 = off; off += align256((size_t)C * 4);
   const size_t oBase = off; off += align256((size_t)C * L0->ldN * 4);
-  const size_t oCols = off; off += align256((size_t)10 * N1 * 4);
+  const size_t oCols = off; off += align256((size_t)10 * L0->ldN * 4);
   const size_t oH0 = off; off += align256((size_t)R * ldmax * es);
   const size_t oH1 = off; off += align256((size_t)R * ldmax * es);
   const size_t oSa = off; off += align256((size_t)R * 4);
@@ -494,7 +518,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   FF_TRY(cudaMemsetAsync(G, 0, (size_t)n * 10 * 4, st), "zero goodness");
   FF_LAUNCH(K_LABEL_COLS, (double)N1 * 10 * (es + 4), st,
             launch_label_columns(b16 ? (const void*)L0->Wb : (const void*)L0->W, b16 ? L0->ldK : L0->K, b16, N1,
-                                 cols, st),
+                                 cols, L0->ldN, st),
             "label columns");
   for (int c0 = 0; c0 < n; c0 += C) {
     const int cn = (n - c0) < C ? (n - c0) : C;

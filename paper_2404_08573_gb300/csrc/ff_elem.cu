@@ -468,46 +468,72 @@ __global__ void k_to_bf16(const float* __restrict__ W, int N, int K, bf16* __res
 
 // ------------------------------------------------------------------ predict
 template <typename T>
-__global__ void k_label_columns(const T* __restrict__ W, int ldw, int N, float* __restrict__ cols) {
+__global__ void k_label_columns(const T* __restrict__ W, int ldw, int N, float* __restrict__ cols, int ldc) {
   const int j = blockIdx.x * blockDim.x + threadIdx.x;
-  if (j >= N) return;
+  if (j >= ldc) return;
 #pragma unroll
-  for (int c = 0; c < 10; ++c) cols[c * N + j] = to_f(W[(size_t)j * ldw + c]);
+  for (int c = 0; c < 10; ++c) cols[(size_t)c * ldc + j] = j < N ? to_f(W[(size_t)j * ldw + c]) : 0.f;
 }
 
 // One block per sample: for each label c the layer-1 activity of the
 // overlaid input, h = ReLU(s * (base + W[:, c]) + b), using
 //   overlay(x, c) W^T = x0 W^T + W[:, c]   (x0: x with features 0..9 zeroed)
-// and the goodness/next scale of that row (row r = 10 * sample + c).
+// and the goodness/next scale of that row (row r = 10 * sample + c).  Each
+// thread takes 8 consecutive columns: the base row and the bias are read
+// once for all 10 labels, the 10 goodness sums stay in registers and are
+// reduced once at the end (warp, then the 8 warps in order).
 template <typename T>
 __global__ void __launch_bounds__(256) k_expand(const float* __restrict__ base, int ldbase,
                                                 const float* __restrict__ cols, const float* __restrict__ s1,
                                                 const float* __restrict__ bias, int N, T* __restrict__ H, int ldh,
                                                 float* __restrict__ s_next, float* __restrict__ G_acc, int* err) {
-  __shared__ float red[8];
+  __shared__ float red[8][10];
   const int n = blockIdx.x;
+  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const float s = s1[n];
   const float* brow = base + (size_t)n * ldbase;
-  for (int c = 0; c < 10; ++c) {
-    const size_t r = (size_t)n * 10 + c;
-    T* hrow = H + r * ldh;
-    float g = 0.f;
-    for (int j = threadIdx.x; j < ldh; j += 256) {
-      float h = 0.f;
-      if (j < N) {
-        float z = s * (brow[j] + cols[c * N + j]);
-        if (bias) z += bias[j];
-        h = relu_nan(z);
+  float g[10];
+#pragma unroll
+  for (int c = 0; c < 10; ++c) g[c] = 0.f;
+  for (int j = 8 * threadIdx.x; j < ldh; j += 8 * 256) {
+    float b8[8], bi[8];
+    const float4 p = *reinterpret_cast<const float4*>(brow + j);
+    const float4 q = *reinterpret_cast<const float4*>(brow + j + 4);
+    b8[0] = p.x; b8[1] = p.y; b8[2] = p.z; b8[3] = p.w;
+    b8[4] = q.x; b8[5] = q.y; b8[6] = q.z; b8[7] = q.w;
+#pragma unroll
+    for (int e = 0; e < 8; ++e) bi[e] = (bias && j + e < N) ? __ldg(bias + j + e) : 0.f;
+#pragma unroll
+    for (int c = 0; c < 10; ++c) {
+      const float* cr = cols + (size_t)c * ldh + j;
+      const float4 u = __ldg(reinterpret_cast<const float4*>(cr));
+      const float4 v = __ldg(reinterpret_cast<const float4*>(cr + 4));
+      const float cv[8] = {u.x, u.y, u.z, u.w, v.x, v.y, v.z, v.w};
+      float h[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) {
+        float z = s * (b8[e] + cv[e]);
+        if (bias) z += bi[e];
+        h[e] = j + e < N ? relu_nan(z) : 0.f;
+        g[c] = fmaf(h[e], h[e], g[c]);
       }
-      g = fmaf(h, h, g);
-      hrow[j] = from_f<T>(h);
+      Vec8<T>::store(H + ((size_t)n * 10 + c) * ldh + j, h);
     }
-    g = block_sum_256(g, red);
-    if (threadIdx.x == 0) {
-      if (!isfinite(g)) atomicOr(err, DEVERR_NONFINITE);
-      s_next[r] = inv_norm(g);
-      if (G_acc) G_acc[r] += g;
-    }
+  }
+#pragma unroll
+  for (int c = 0; c < 10; ++c) {
+    const float v = warp_sum(g[c]);
+    if (lane == 0) red[warp][c] = v;
+  }
+  __syncthreads();
+  if (threadIdx.x < 10) {
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) t += red[w][threadIdx.x];
+    const size_t r = (size_t)n * 10 + threadIdx.x;
+    if (!isfinite(t)) atomicOr(err, DEVERR_NONFINITE);
+    s_next[r] = inv_norm(t);
+    if (G_acc) G_acc[r] += t;
   }
 }
 
@@ -620,11 +646,11 @@ cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cuda
   return cudaGetLastError();
 }
 
-cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols, cudaStream_t st) {
+cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols, int ldc, cudaStream_t st) {
   if (w_bf16)
-    k_label_columns<bf16><<<cdiv(N, 256), 256, 0, st>>>((const bf16*)W, ldw, N, cols);
+    k_label_columns<bf16><<<cdiv(ldc, 256), 256, 0, st>>>((const bf16*)W, ldw, N, cols, ldc);
   else
-    k_label_columns<float><<<cdiv(N, 256), 256, 0, st>>>((const float*)W, ldw, N, cols);
+    k_label_columns<float><<<cdiv(ldc, 256), 256, 0, st>>>((const float*)W, ldw, N, cols, ldc);
   return cudaGetLastError();
 }
 

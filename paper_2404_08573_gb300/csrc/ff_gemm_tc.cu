@@ -502,6 +502,12 @@ bool tc_supported() {
 
 int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN) * (EPI_WARPS / 4); }  // goodness partials per row
 
+int tc_gemm_fwd_ctas(int M, int N) {
+  constexpr int CM = USE_PAIR ? 2 : 1;
+  const int mt = small_grid(M, N, FWD_BN) ? 1 : ROW_SUBTILES;
+  return cdiv(cdiv(M, BM * mt), CM) * CM * cdiv(N, FWD_BN);
+}
+
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
                         int* err, cudaStream_t st) {
   CUtensorMap ta, tb, tc;

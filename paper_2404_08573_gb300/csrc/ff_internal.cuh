@@ -110,8 +110,8 @@ cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
 cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cudaStream_t st);
 // predict helpers
-cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols /*[10,N]*/,
-                                 cudaStream_t st);
+cudaError_t launch_label_columns(const void* W, int ldw, bool w_bf16, int N, float* cols /*[10,ldc]*/,
+                                 int ldc, cudaStream_t st);
 cudaError_t launch_expand(const float* base, int ldbase, const float* cols, const float* s1,
                           const float* bias, int n, int N, void* H, int ldh, bool h_bf16,
                           float* s_next, float* G_acc /*null unless single layer*/, int* err,
@@ -141,6 +141,8 @@ cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M,
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K,
                           float* C, int ldc, int* err, cudaStream_t st);
 bool tc_supported();
+// CTAs of the forward GEMM for an M x N output (its tile configuration).
+int tc_gemm_fwd_ctas(int M, int N);
 // Tensor map of a row-major [rows, cols] bf16 (esize 2) or fp32 (esize 4)
 // matrix with row stride ld, boxes of box_rows x box_cols, no swizzle; false
 // if the pointer or the stride is not 16-byte aligned.
