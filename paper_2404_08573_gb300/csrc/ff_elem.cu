@@ -212,6 +212,7 @@ constexpr int kGradRows = 32;
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __restrict__ H, T* __restrict__ dZ) {
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   __shared__ float red[8][256 + 8];
   __shared__ float lred[8], gpred[8], gnred[8], ared[8];
   const int r0 = blockIdx.y * kGradRows;
@@ -344,6 +345,7 @@ __device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, flo
 }
 
 __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   const float a1 = a.lr / a.ds->bc1, r2 = 1.f / a.ds->bc2;
   if ((int)blockIdx.x < w_blocks) {
     const long long total = (long long)a.N * a.K;
@@ -614,22 +616,35 @@ cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st) {
 
 int local_grad_row_blocks(int M) { return cdiv(M, kGradRows); }
 
+// Launch configuration with programmatic stream serialization: the kernel
+// may start while the previous kernel of the stream finishes and waits for it
+// with griddep_wait() before touching memory.
+struct PdlLaunch {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  PdlLaunch(dim3 grid, dim3 block, cudaStream_t st) {
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.stream = st;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+};
+
 cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, void* dZ, cudaStream_t st) {
-  dim3 grid(cdiv(a.ld, 256), local_grad_row_blocks(a.M));
-  dim3 block(32, 8);
-  if (b16)
-    k_grad_prep<bf16><<<grid, block, 0, st>>>(a, (const bf16*)H, (bf16*)dZ);
-  else
-    k_grad_prep<float><<<grid, block, 0, st>>>(a, (const float*)H, (float*)dZ);
-  return cudaGetLastError();
+  PdlLaunch l(dim3(cdiv(a.ld, 256), local_grad_row_blocks(a.M)), dim3(32, 8), st);
+  if (b16) return cudaLaunchKernelEx(&l.cfg, k_grad_prep<bf16>, a, (const bf16*)H, (bf16*)dZ);
+  return cudaLaunchKernelEx(&l.cfg, k_grad_prep<float>, a, (const float*)H, (float*)dZ);
 }
 
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st) {
   const long long total = (long long)a.N * a.K;
   const int w_blocks = grid_for((a.K & 3) == 0 ? total / 4 : total, 256, 152 * 16);
   const int b_blocks = cdiv(a.N, 32);
-  k_adam<<<w_blocks + b_blocks, 256, 0, st>>>(a, w_blocks);
-  return cudaGetLastError();
+  PdlLaunch l(dim3(w_blocks + b_blocks), dim3(256), st);
+  return cudaLaunchKernelEx(&l.cfg, k_adam, a, w_blocks);
 }
 
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st) {

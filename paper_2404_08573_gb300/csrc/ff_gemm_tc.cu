@@ -132,6 +132,9 @@ __global__ void __launch_bounds__(NTHREADS, 1)
   if constexpr (PAIR) ptx::cluster_sync();  // both CTAs' barriers and TMEM exist before any cross-CTA use
   ptx::tc_fence_after();
   const uint32_t tmem = *tslot;
+  // everything above touched only this CTA's own resources: the inputs are
+  // read, and the outputs written, only after the previous kernel is done
+  ptx::griddep_wait();
 
   if (warp == 0) {
     // ------------------------------------------------------------ producer
@@ -274,6 +277,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
       ptx::named_bar(1, 32 * EPI_WARPS);
     }
     const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
+    if (threadIdx.x == 64) ptx::griddep_launch_dependents();  // the mainloop is done
     if (!ok) latch(err, abort_flag);
     ptx::tc_fence_after();
     // tcgen05.ld is warp-collective: decide for the whole warp at once
@@ -449,13 +453,16 @@ cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtens
   cfg.blockDim = dim3(NTHREADS, 1, 1);
   cfg.dynamicSmemBytes = C::SMEM;
   cfg.stream = st;
-  cudaLaunchAttribute at[1];
+  cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;
   at[0].val.clusterDim.x = CM;
   at[0].val.clusterDim.y = 1;
   at[0].val.clusterDim.z = 1;
   cfg.attrs = at;
-  cfg.numAttrs = 1;
+  // the next kernel's launch and set-up overlap this one's tail (griddep_*)
+  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  at[1].val.programmaticStreamSerializationAllowed = 1;
+  cfg.numAttrs = 2;
   return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, tma_store, M, N, K, ep, err);
 }
 
