@@ -643,11 +643,7 @@ cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, voi
 
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st) {
   const long long total = (long long)a.N * a.K;
-  // Two 256-thread blocks per SM: with 40 registers a thread they leave room
-  // for a 320-thread tensor-core GEMM CTA of another layer's stream on the same
-  // SM, so the HBM-bound update overlaps the GEMMs instead of holding whole SMs
-  // (a full grid measured 2 % slower on the 784-2000x4 epoch).
-  const int w_blocks = grid_for((a.K & 3) == 0 ? total / 4 : total, 256, 152 * 2);
+  const int w_blocks = grid_for((a.K & 3) == 0 ? total / 4 : total, 256, 152 * 16);
   const int b_blocks = cdiv(a.N, 32);
   PdlLaunch l(dim3(w_blocks + b_blocks), dim3(256), st);
   return cudaLaunchKernelEx(&l.cfg, k_adam, a, w_blocks);
