@@ -34,9 +34,10 @@ namespace {
 constexpr int kClasses = 10;
 constexpr int kMaxSegs = 16;
 constexpr int kDotRows = 64;     // rows per block of k_head_dot (eight per warp)
-constexpr int kSplit = 1024;     // features of one segment per k_head_dot block
+constexpr int kSplit = 1024;     // widest feature split of one segment per k_head_dot block
+constexpr int kDotMinBlocks = 152 / 2;  // k_head_dot grids narrower than this split features finer
 constexpr int kFinRows = 256;    // rows per block of k_head_finish (one per thread)
-constexpr int kWgRows = 128;     // rows per block of k_head_wgrad (16 per warp)
+constexpr int kWgRows = 64;      // rows per block of k_head_wgrad (8 per warp)
 constexpr int kWgChunk = 128;    // features per block of k_head_wgrad (4 per lane)
 constexpr int kPart = kClasses + 1;  // per-block partials: dc[10], loss
 
@@ -124,11 +125,36 @@ __device__ __forceinline__ float finish_row(const float (&z)[kClasses], int row,
   return (m + logf(sum)) - zy;
 }
 
-// Number of feature splits: segment k has ceil(F_k / kSplit) of them.
-__host__ __device__ inline int head_splits(const Segs& sg) {
+// Number of feature splits of width `split`: segment k has ceil(F_k / split).
+__host__ __device__ inline int head_splits(const int* F, int nseg, int split) {
   int S = 0;
-  for (int k = 0; k < sg.nseg; ++k) S += (sg.F[k] + kSplit - 1) / kSplit;
+  for (int k = 0; k < nseg; ++k) S += (F[k] + split - 1) / split;
   return S;
+}
+
+// Split width of k_head_dot for n rows: kSplit, halved (down to one 512-byte
+// chunk, 512 / es features) while the grid would cover less than half the
+// SMs, so that few rows are spread over the SMs by features.  (A block's
+// fixed costs -- its slice of V, the cross-lane sums -- make narrower splits
+// slower once the grid covers the GPU: 6000 features x 1024 rows run fastest
+// at 96 blocks of 1024 features, 2000 x 1024 at 128 blocks of 256.)
+int dot_split(const int* F, int nseg, int n, int es) {
+  const int ch = 512 / es;
+  const long long rb = (n + kDotRows - 1) / kDotRows;
+  int split = kSplit;
+  while (split > ch && head_splits(F, nseg, split) * rb < kDotMinBlocks) split /= 2;
+  return split;
+}
+
+// Floats of partial logits k_head_dot writes for any row count up to `rows`.
+size_t zpart_floats(const int* F, int nseg, int rows, int es) {
+  size_t mx = 0;
+  for (int rb = 1; (rb - 1) * kDotRows < rows; ++rb) {
+    const int n = rb * kDotRows < rows ? rb * kDotRows : rows;
+    const size_t z = (size_t)head_splits(F, nseg, dot_split(F, nseg, n, es)) * n * kClasses;
+    if (z > mx) mx = z;
+  }
+  return mx;
 }
 
 // One tensor map per segment: H_k as [n, ld_k] with 64-row boxes of 512
@@ -149,12 +175,12 @@ constexpr int kDotSmem = kDotStages * kDotStageBytes + kSplit * kClasses * 4 + 6
 // memory interleaved so that lane l's features (FPL consecutive ones per
 // chunk) are read without bank conflicts.  Every wait is bounded.
 template <typename T>
-__global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ HeadMaps maps, Segs sg, int n,
+__global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ HeadMaps maps, Segs sg, int split, int n,
                                                      const float* __restrict__ V, float* __restrict__ zpart,
                                                      int* err) {
   constexpr int CH = 512 / (int)sizeof(T);  // features per chunk
   constexpr int FPL = CH / 32;              // features per lane
-  constexpr int NCH = kSplit / CH;          // chunks in a full split
+  constexpr int NCH = kSplit / CH;          // chunks in the widest split
   extern __shared__ __align__(128) uint8_t dsm[];
   uint8_t* ring = dsm;
   float* Vs = reinterpret_cast<float*>(dsm + kDotStages * kDotStageBytes);
@@ -164,13 +190,13 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
   volatile int* never_set = abort_flag + 1;
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   int k = 0, sp = blockIdx.x;
-  while (k + 1 < sg.nseg && sp >= (sg.F[k] + kSplit - 1) / kSplit) {
-    sp -= (sg.F[k] + kSplit - 1) / kSplit;
+  while (k + 1 < sg.nseg && sp >= (sg.F[k] + split - 1) / split) {
+    sp -= (sg.F[k] + split - 1) / split;
     ++k;
   }
   const int off = sg.off[k];
-  const int fs = sp * kSplit;
-  const int fe = min(fs + kSplit, sg.F[k]);
+  const int fs = sp * split;
+  const int fe = min(fs + split, sg.F[k]);
   const int nch = (fe - fs + CH - 1) / CH;
   const int rblk = blockIdx.y * kDotRows;
   const CUtensorMap* map = &maps.m[k];
@@ -197,7 +223,7 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
     }
   }
   // the split's slice of V, zero past the segment
-  for (int idx = threadIdx.x; idx < NCH * kClasses * CH; idx += 256) {
+  for (int idx = threadIdx.x; idx < nch * kClasses * CH; idx += 256) {
     const int ch = idx / (kClasses * CH), rem = idx % (kClasses * CH);
     const int c = rem / CH, j = rem % CH;
     const int f = fs + ch * CH + j;
@@ -464,7 +490,7 @@ constexpr int kPoRows = 32;
 
 template <typename T>
 __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restrict__ H, T* __restrict__ G) {
-  __shared__ float Vsh[kClasses][256];
+  __shared__ float Vsh[kClasses][8][32];  // V[c][c0 + 8 l + e] at [c][e][l]: conflict-free reads
   __shared__ float dzs[kPoRows][kClasses];
   __shared__ float red[8][256 + 8];
   const int r0 = blockIdx.y * kPoRows;
@@ -473,7 +499,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   const int cg = c0 + lane * 8;
   for (int idx = tid; idx < kClasses * 256; idx += 256) {
     const int c = idx / 256, j = idx % 256;
-    Vsh[c][j] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
+    Vsh[c][j % 8][j / 8] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
   }
   for (int idx = tid; idx < kPoRows * kClasses; idx += 256) {
     const int i = idx / kClasses, c = idx % kClasses;
@@ -512,7 +538,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     for (int e = 0; e < 8; ++e) {
       float d = 0.f;
 #pragma unroll
-      for (int c = 0; c < kClasses; ++c) d = fmaf(dzs[li][c], Vsh[c][lane * 8 + e], d);
+      for (int c = 0; c < kClasses; ++c) d = fmaf(dzs[li][c], Vsh[c][e][lane], d);
       d = h[e] > 0.f ? d : 0.f;
       db[e] += d;
       z[e] = si * d;
@@ -643,11 +669,11 @@ struct HeadWork {
   float* dVpart;
 };
 
-// Feature splits of the layer chain's segments (see head_splits).
-int n_splits(ff_layer* const* layers, int L) {
-  int S = 0;
-  for (int k = (L == 1 ? 0 : 1); k < L; ++k) S += cdiv(layers[k]->N, kSplit);
-  return S;
+// Partial-logit floats for up to `rows` rows of the layer chain's segments.
+size_t chain_zpart_floats(ff_layer* const* layers, int L, int rows) {
+  int F[kMaxSegs + 1], nseg = 0;
+  for (int k = (L == 1 ? 0 : 1); k < L; ++k) F[nseg++] = layers[k]->N;
+  return zpart_floats(F, nseg, rows, layers[0]->is_bf16 ? 2 : 4);
 }
 
 // Carves the head's workspace for `rows` rows (grown on demand).
@@ -667,7 +693,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   for (int k = 0; k < L; ++k) { oH[k] = off; off += align256((size_t)rows * layers[k]->ldN * es); }
   size_t oG = off; off += align256((size_t)ntmax * rows * 4);
   size_t oZ = off; off += align256((size_t)rows * kClasses * 4);
-  size_t oZP = off; off += align256((size_t)n_splits(layers, L) * rows * kClasses * 4);
+  size_t oZP = off; off += align256(chain_zpart_floats(layers, L, rows) * 4);
   size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
   size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kFinRows) * kPart * 4 : 0);
   size_t oV = off; off += align256(train ? (size_t)cdiv(rows, kWgRows) * kClasses * hd->F * 4 : 0);
@@ -750,8 +776,9 @@ Segs make_segs(ff_layer* const* layers, int L, const HeadWork& w, int F) {
 ff_status head_logits(const Segs& sg, bool b16, int n, const float* V, const float* c, const int* labels,
                       float* logits, float* zpart, float* dz, float* part, ff_dev_state* ds, float beta1, float beta2,
                       int* err, cudaStream_t st) {
-  const int S = head_splits(sg);
   const int es = b16 ? 2 : 4;
+  const int split = dot_split(sg.F, sg.nseg, n, es);
+  const int S = head_splits(sg.F, sg.nseg, split);
   HeadMaps maps;
   std::memset(&maps, 0, sizeof(maps));
   for (int k = 0; k < sg.nseg; ++k)
@@ -764,8 +791,9 @@ ff_status head_logits(const Segs& sg, bool b16, int n, const float* V, const flo
   FF_TRY(b16 ? attr_b : attr_f, "head kernel attributes");
   dim3 grid(S, cdiv(n, kDotRows));
   FF_LAUNCH(K_HEAD_LOGITS, (double)n * sg.F_total * es + (double)n * S * kClasses * 4, st,
-            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, n, V, zpart, err), cudaGetLastError())
-                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, n, V, zpart, err), cudaGetLastError())),
+            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, err), cudaGetLastError())
+                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, err),
+                    cudaGetLastError())),
             "head partial logits");
   const float inv_n = 1.f / (float)n;
   FF_LAUNCH(K_HEAD_FINISH, (double)n * (S + 2) * kClasses * 4, st,
@@ -807,9 +835,9 @@ struct PoWork {
   float *zpart, *dz, *part, *dVpart;
 };
 
-ff_status po_workspace(ff_head* hd, int n, int N, PoWork* w) {
+ff_status po_workspace(ff_head* hd, int n, int N, int es, PoWork* w) {
   size_t off = 0;
-  const size_t oZ = off; off += align256((size_t)cdiv(N, kSplit) * n * kClasses * 4);
+  const size_t oZ = off; off += align256(zpart_floats(&N, 1, n, es) * 4);
   const size_t oD = off; off += align256((size_t)n * kClasses * 4);
   const size_t oP = off; off += align256((size_t)cdiv(n, kFinRows) * kPart * 4);
   const size_t oV = off; off += align256((size_t)cdiv(n, kWgRows) * kClasses * N * 4);
@@ -1071,7 +1099,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   ff_status s = ensure_capacity(L, n);
   if (s != FF_OK) return s;
   PoWork w;
-  s = po_workspace(hd, n, L->N, &w);
+  s = po_workspace(hd, n, L->N, L->is_bf16 ? 2 : 4, &w);
   if (s != FF_OK) return s;
   L->last_stream = st;
   hd->last_stream = st;
