@@ -429,6 +429,53 @@ def run_ours(args):
 
 
 # ----------------------------------------------------- other workloads
+# fp32 FMA peak of the SIMT kernels: 152 SMs x 128 fp32 lanes x 2 FLOP x 2.07 GHz
+FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
+
+
+def _kernel_profile(lib, torch, fn, pk):
+    """Per-kernel device time of one more call of `fn`, every launch bracketed
+    by CUDA events on its own stream by libff's profiler: the kernel table and
+    the roofline of the kernel with the most device time (tensor-core GEMMs
+    against the measured bf16 peak, fp32 SIMT GEMMs against the fp32 FMA peak,
+    the rest against the measured HBM copy bandwidth)."""
+    import ctypes
+    torch.cuda.synchronize()
+    lib.ff_profile_enable(1)
+    fn()
+    torch.cuda.synchronize()
+    lib.ff_profile_enable(0)
+    cap = 32
+    names = (ctypes.c_char_p * cap)()
+    cnt = (ctypes.c_longlong * cap)()
+    tms = (ctypes.c_double * cap)()
+    wk = (ctypes.c_double * cap)()
+    lib.ff_profile_read.restype = ctypes.c_int
+    n = lib.ff_profile_read(cap, names, cnt, tms, wk)
+    total = sum(tms[i] for i in range(max(n, 0)))
+    kernels = []
+    for i in range(max(n, 0)):
+        nm = names[i].decode()
+        flop = "gemm" in nm
+        rate = wk[i] / (tms[i] / 1e3) if tms[i] > 0 else 0.0
+        kernels.append({"kernel": nm, "launches": int(cnt[i]), "ms": round(tms[i], 3),
+                        "share": round(tms[i] / total, 4) if total else None,
+                        "achieved": round(rate / (1e12 if flop else 1e9), 2), "unit": "TFLOP/s" if flop else "GB/s"})
+    roof = None
+    if kernels:
+        top = max(kernels, key=lambda k: k["ms"])
+        if "simt" in top["kernel"]:
+            bound, peak, src = "alu", FP32_ALU_TFLOPS, "fp32 FMA peak from unit counts and clock (152 x 128 x 2 x 2.07 GHz)"
+        elif top["unit"] == "TFLOP/s":
+            bound, peak, src = "tensor", pk["bf16"], pk["src"] + " bf16 burst"
+        else:
+            bound, peak, src = "hbm", pk["hbm"], pk["src"] + " HBM copy"
+        roof = {"kernel": top["kernel"], "bound": bound, "achieved": top["achieved"], "peak": round(peak, 1),
+                "unit": top["unit"], "frac": round(top["achieved"] / peak, 4), "peak_source": src, "traffic": None,
+                "share": top["share"]}
+    return kernels, roof
+
+
 def _timed_loop(torch, stream, fn, k):
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     torch.cuda.synchronize()
@@ -456,6 +503,7 @@ def run_other(args):
     out = {"n_gpus": 1, "steps": args.steps, "warmup": args.warmup, "data": "synthetic",
            "scaling": "weak", "vs_baseline": None, "higher_is_better": True}
     w = args.workload
+    prof = None  # the workload's call, profiled once more after the timed calls
     if w.startswith("predict"):
         # 10 000 samples x 10 label overlays through 784-2000x4, goodness of layers 2..4
         prec = "fp32" if w.endswith("fp32") else "bf16"
@@ -469,6 +517,7 @@ def run_other(args):
         ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
         flops = 2.0 * n * NET[1] * NET[0] + 3 * 2.0 * 10 * n * NET[2] * NET[1]
         tf = flops / (ms / 1e3) / 1e12
+        prof = fn
         out.update({"metric": "FF goodness predict samples/s (10 label overlays) on 4x2000 net", "value": round(n / (ms / 1e3), 1),
                     "unit": "samples/s", "ms_per_step": round(ms, 4), "dtype": prec, "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4) if prec == "bf16" else None,
@@ -486,6 +535,7 @@ def run_other(args):
         ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
         flops = 2.0 * n * NET[1] * NET[0] + 3 * 2.0 * 10 * n * NET[2] * NET[1]
         tf = flops / (ms / 1e3) / 1e12
+        prof = fn
         out.update({"metric": "AdaptiveNEG negative labels/s (10 label overlays) on 4x2000 net",
                     "value": round(n / (ms / 1e3), 1), "unit": "samples/s", "ms_per_step": round(ms, 4),
                     "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
@@ -522,6 +572,7 @@ def run_other(args):
         _timed_loop(torch, stream, fn, args.warmup)
         ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
         tf = flops / (ms / 1e3) / 1e12
+        prof = fn
         out.update({"metric": metric, "value": round(n / (ms / 1e3), 1), "unit": "samples/s",
                     "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
@@ -570,6 +621,7 @@ def run_other(args):
         flops = n * (2.0 * 2 * sum(NET[k] * NET[k + 1] for k in range(len(NET) - 1))
                      + 3 * 2.0 * 10 * sum(NET[1:]))
         tf = flops / (ms / 1e3) / 1e12
+        prof = fn
         out.update({"metric": "FF Performance-Optimized PFF train samples/s (per-layer softmax blocks) on 4x2000 net",
                     "value": round(n / (ms / 1e3), 1), "unit": "samples/s", "ms_per_step": round(ms, 4),
                     "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
@@ -598,6 +650,7 @@ def run_other(args):
         ms_seq = min(one("all_layers", 1) for _ in range(max(1, args.steps // 5)))
         pair_epochs = S * P
         flops = pair_epochs * (train_flops_per_pair() + 2.0 * 2 * sum(NET[k] * NET[k + 1] for k in range(3)))
+        prof = lambda: one("single_layer", 1)
         out.update({"metric": "FF chapter-schedule (Single-Layer PFF) pair-epochs/s on 4x2000 net, 4 streams",
                     "value": round(pair_epochs / (ms_par / 1e3), 1), "unit": "pair-epochs/s",
                     "ms_per_step": round(ms_par, 3), "dtype": "bf16",
@@ -639,11 +692,14 @@ def run_other(args):
         ms_p = _timed_loop(torch, stream, streams_run, args.steps) / args.steps
         ms_s = _timed_loop(torch, stream, single_run, args.steps) / args.steps
         flops = 4.0 * 2 * B * sum(net5[i] * net5[i + 1] for i in range(5)) * chunks
+        prof = streams_run
         out.update({"metric": "FF train pairs/s, 784-2000x5 on 5 CUDA streams (60 chunks of 1000 pairs)",
                     "value": round(B * chunks / (ms_p / 1e3), 1), "unit": "pairs/s", "ms_per_step": round(ms_p, 4),
                     "dtype": "bf16", "tflops": round(flops / (ms_p / 1e3) / 1e12, 2),
                     "single_stream_ms_per_step": round(ms_s, 4), "speedup_vs_single_stream": round(ms_s / ms_p, 3),
                     "config": {"workload": "ff_train_784-2000x5_bf16_5streams_60x1000"}})
+        out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, prof, 1), pk)
+        prof = None
         net.close()
     elif w == "wide_4x8192":
         # 3072-8192x4, B = 4096 pairs, theta = 8; one step = one batch through all layers
@@ -661,6 +717,8 @@ def run_other(args):
         ms = _timed_loop(torch, stream, fn, args.steps) / args.steps
         flops = 4.0 * 2 * B * sum(netw[i] * netw[i + 1] for i in range(4))
         tf = flops / (ms / 1e3) / 1e12
+        out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, fn, 1), pk)
+        prof = None
         out.update({"metric": "FF train pairs/s on 3072-8192x4 (B=4096 pairs)", "value": round(B / (ms / 1e3), 1),
                     "unit": "pairs/s", "ms_per_step": round(ms, 4), "dtype": "bf16", "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
@@ -685,9 +743,13 @@ def run_other(args):
                 layers[1].train_step(h, row_scale=sc, B=B, stream=stream)
         _timed_loop(torch, stream, run16, args.warmup)
         ms = _timed_loop(torch, stream, run16, args.steps) / args.steps
+        prof = run16
         out.update({"metric": "FF train step latency, 784-500-500 fp32, B=64 pairs", "value": round(1e3 * ms / 16, 2),
                     "unit": "us/step", "higher_is_better": False, "ms_per_step": round(ms, 4), "dtype": "f32",
                     "config": {"workload": "ff_train_784-500-500_fp32_B64_16steps"}})
+    if prof is not None:
+        # one more call, each launch timed on its own stream (not the timed calls above)
+        out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, prof, 1), pk)
     print(json.dumps(out), flush=True)
 
 
