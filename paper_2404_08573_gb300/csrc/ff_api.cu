@@ -494,6 +494,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   const size_t oSa = off; off += align256((size_t)R * 4);
   const size_t oSb = off; off += align256((size_t)R * 4);
   const size_t oP = off; off += align256((size_t)ntmax * R * 4);
+  const size_t oP2 = off; off += align256(b16 ? (size_t)ntmax * R * 4 : 0);
   const size_t oG = off; off += align256(goodness ? 0 : (size_t)n * 10 * 4);
   if (off > L0->pws_bytes) {
     FF_TRY(cudaStreamSynchronize(L0->last_stream), "sync before predict scratch growth");
@@ -511,7 +512,9 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   float* cols = reinterpret_cast<float*>(w + oCols);
   void* Hb[2] = {w + oH0, w + oH1};
   float* Sb[2] = {reinterpret_cast<float*>(w + oSa), reinterpret_cast<float*>(w + oSb)};
-  float* gpart = reinterpret_cast<float*>(w + oP);
+  // goodness partials of the forward GEMMs, alternating between layers on the
+  // tensor-core path (a GEMM reads the previous layer's while writing its own)
+  float* gpb[2] = {reinterpret_cast<float*>(w + oP), reinterpret_cast<float*>(w + (b16 ? oP2 : oP))};
   float* G = goodness ? goodness : reinterpret_cast<float*>(w + oG);
   int* err = &L0->ds->err;
 
@@ -543,11 +546,21 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
                             Sb[0], n_layers == 1 ? Gc : nullptr, err, st),
               "layer-1 expansion");
     int cur = 0;
+    int nt_prev = 0;
     for (int k = 1; k < n_layers; ++k) {
       ff_layer* Lk = layers[k];
+      float* gpart = gpb[k & 1];
       EpiArgs ep{Sb[cur], Lk->cfg.has_bias ? Lk->b : nullptr, Hb[cur ^ 1], Lk->ldN, gpart};
       int nt;
       if (b16) {
+        if (k >= 2) {
+          // the row scale and layer k-1's share of G come from layer k-1's
+          // goodness partials inside this GEMM (no separate finalize)
+          ep.row_scale = nullptr;
+          ep.gpart_in = gpb[(k - 1) & 1];
+          ep.ntiles_in = nt_prev;
+          ep.G_acc = Gc;
+        }
         nt = tc_fwd_ntiles(Lk->N);
         FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
                   tc_gemm_fwd(static_cast<const bf16*>(Hb[cur]), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep,
@@ -559,14 +572,17 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
                   simt_gemm_fwd(static_cast<const float*>(Hb[cur]), Lk->ldK, Lk->W, Lk->K, rows, Lk->N, Lk->K, ep, st),
                   "predict forward GEMM (fp32)");
       }
-      FinalizeArgs fa{};
-      fa.gpart = gpart;
-      fa.ntiles = nt;
-      fa.M = rows;
-      fa.s_next = (k + 1 < n_layers) ? Sb[cur ^ 1] : nullptr;
-      fa.G_acc = Gc;
-      fa.err = err;
-      FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 12), st, launch_finalize(fa, st), "predict goodness");
+      nt_prev = nt;
+      if (!b16 || k + 1 == n_layers) {
+        FinalizeArgs fa{};
+        fa.gpart = gpart;
+        fa.ntiles = nt;
+        fa.M = rows;
+        fa.s_next = (k + 1 < n_layers) ? Sb[cur ^ 1] : nullptr;
+        fa.G_acc = Gc;
+        fa.err = err;
+        FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 12), st, launch_finalize(fa, st), "predict goodness");
+      }
       cur ^= 1;
     }
   }

@@ -20,13 +20,6 @@
 namespace ff {
 namespace {
 
-constexpr float kNormEps = 1e-12f;
-
-// 1 / max(sqrt(ss), 1e-12), with NaN propagated (fmaxf alone would drop it).
-__device__ __forceinline__ float inv_norm(float ss) {
-  const float r = sqrtf(ss);
-  return r != r ? r : 1.f / fmaxf(r, kNormEps);
-}
 // ReLU that keeps NaN visible to the non-finite check.
 __device__ __forceinline__ float relu_nan(float z) { return z != z ? z : fmaxf(z, 0.f); }
 
@@ -57,21 +50,6 @@ __device__ __forceinline__ float block_sum_256(float v, float* red /*[8]*/) {
   }
   __syncthreads();
   return t;
-}
-
-// g = sum over t of gpart[t * M + i], t = 0..ntiles-1, in that order; the
-// loads are issued together (8 at a time) rather than one per dependent add.
-__device__ __forceinline__ float sum_partials(const float* __restrict__ gpart, int ntiles, int M, int i) {
-  float g = 0.f;
-  for (int t0 = 0; t0 < ntiles; t0 += 8) {
-    float v[8];
-#pragma unroll
-    for (int u = 0; u < 8; ++u) v[u] = (t0 + u < ntiles) ? __ldg(gpart + (size_t)(t0 + u) * M + i) : 0.f;
-#pragma unroll
-    for (int u = 0; u < 8; ++u)
-      if (t0 + u < ntiles) g += v[u];
-  }
-  return g;
 }
 
 // ------------------------------------------------------------------ overlay

@@ -266,14 +266,30 @@ __global__ void __launch_bounds__(NTHREADS, 1)
     const int ew = warp - 2;          // 0 .. EPI_WARPS-1
     const int half = ew / 4;
     const int cbase = half * CPW;     // this warp's first column within the tile
-    float s0 = 0.f;
+    float srow[MT];
+#pragma unroll
+    for (int mt = 0; mt < MT; ++mt) srow[mt] = 0.f;
     if (MODE == MODE_FWD) {
       // While the mainloop runs: the tile's bias (zero past N or without bias)
-      // into shared memory and this thread's first row scale into a register.
+      // into shared memory and this thread's row scales into registers.
       for (int c = (int)threadIdx.x - 64; c < BN; c += 32 * EPI_WARPS)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
-      const int gi0 = m0 + q * 32 + lane;
-      if (gi0 < M) s0 = __ldg(ep.row_scale + gi0);
+#pragma unroll
+      for (int mt = 0; mt < MT; ++mt) {
+        const int gi = m0 + mt * BM + q * 32 + lane;
+        if (gi >= M) continue;
+        if (ep.gpart_in) {
+          const float gprev = sum_partials(ep.gpart_in, ep.ntiles_in, M, gi);
+          srow[mt] = inv_norm(gprev);
+          if (blockIdx.y == 0 && half == 0) {  // one thread per row
+            if (!isfinite(gprev)) atomicOr(err, DEVERR_NONFINITE);
+            if (ep.G_acc) ep.G_acc[gi] += gprev;
+            if (ep.s_out) ep.s_out[gi] = srow[mt];
+          }
+        } else {
+          srow[mt] = __ldg(ep.row_scale + gi);
+        }
+      }
       ptx::named_bar(1, 32 * EPI_WARPS);
     }
     const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
@@ -294,8 +310,7 @@ __global__ void __launch_bounds__(NTHREADS, 1)
         // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
         uint8_t* stage = smem + (MODE == MODE_FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
         const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS + cbase);
-        float s = s0;
-        if (MODE == MODE_FWD && mt > 0) s = gi < M ? __ldg(ep.row_scale + gi) : 0.f;
+        const float s = srow[mt];
         float g = 0.f;
         // Columns past N and rows past M hold zero products (their operand rows
         // were zero-filled); the TMA store clips them and gpart skips them.

@@ -662,6 +662,7 @@ struct HeadWork {
   float* S[kMaxSegs + 2];   // S[k]: row scale of layer k's input (S[L]: of the last activity)
   void* Hk[kMaxSegs + 1];
   float* gpart;
+  float* gpart2;   // the tensor-core forward alternates between gpart and gpart2
   float* logits;
   float* zpart;
   float* dz;
@@ -692,6 +693,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   size_t oH[kMaxSegs + 1];
   for (int k = 0; k < L; ++k) { oH[k] = off; off += align256((size_t)rows * layers[k]->ldN * es); }
   size_t oG = off; off += align256((size_t)ntmax * rows * 4);
+  size_t oG2 = off; off += align256(b16 ? (size_t)ntmax * rows * 4 : 0);
   size_t oZ = off; off += align256((size_t)rows * kClasses * 4);
   size_t oZP = off; off += align256(chain_zpart_floats(layers, L, rows) * 4);
   size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
@@ -710,6 +712,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   for (int k = 0; k <= L; ++k) w->S[k] = reinterpret_cast<float*>(base + oS[k]);
   for (int k = 0; k < L; ++k) w->Hk[k] = base + oH[k];
   w->gpart = reinterpret_cast<float*>(base + oG);
+  w->gpart2 = reinterpret_cast<float*>(base + (b16 ? oG2 : oG));
   w->logits = reinterpret_cast<float*>(base + oZ);
   w->zpart = reinterpret_cast<float*>(base + oZP);
   w->dz = train ? reinterpret_cast<float*>(base + oD) : nullptr;
@@ -728,11 +731,21 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
   FF_LAUNCH(K_OVERLAY, (double)rows * (L0->K * 4.0 + L0->ldK * es + 4), st,
             launch_overlay(x, nullptr, rows, L0->K, w.X0, L0->ldK, b16, w.S[0], 2, st), "neutral-label overlay");
   const void* in = w.X0;
+  int nt_prev = 0;
   for (int k = 0; k < L; ++k) {
     ff_layer* Lk = layers[k];
-    EpiArgs ep{w.S[k], Lk->cfg.has_bias ? Lk->b : nullptr, w.Hk[k], Lk->ldN, w.gpart};
+    float* gpart = b16 && (k & 1) ? w.gpart2 : w.gpart;
+    EpiArgs ep{w.S[k], Lk->cfg.has_bias ? Lk->b : nullptr, w.Hk[k], Lk->ldN, gpart};
     int nt;
     if (b16) {
+      if (k >= 1) {
+        // layer k-1's activity scale S[k] comes from its goodness partials
+        // inside this GEMM (no separate finalize)
+        ep.row_scale = nullptr;
+        ep.gpart_in = (k - 1) & 1 ? w.gpart2 : w.gpart;
+        ep.ntiles_in = nt_prev;
+        ep.s_out = w.S[k];
+      }
       nt = tc_fwd_ntiles(Lk->N);
       FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
                 tc_gemm_fwd(static_cast<const bf16*>(in), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep, err, st),
@@ -743,13 +756,16 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
                 simt_gemm_fwd(static_cast<const float*>(in), Lk->ldK, Lk->W, Lk->K, rows, Lk->N, Lk->K, ep, st),
                 "head forward GEMM (fp32)");
     }
-    FinalizeArgs fa{};
-    fa.gpart = w.gpart;
-    fa.ntiles = nt;
-    fa.M = rows;
-    fa.s_next = w.S[k + 1];
-    fa.err = err;
-    FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 4), st, launch_finalize(fa, st), "head activity scale");
+    nt_prev = nt;
+    if (!b16 || k + 1 == L) {
+      FinalizeArgs fa{};
+      fa.gpart = gpart;
+      fa.ntiles = nt;
+      fa.M = rows;
+      fa.s_next = w.S[k + 1];
+      fa.err = err;
+      FF_LAUNCH(K_FINALIZE, (double)rows * (nt * 4.0 + 4), st, launch_finalize(fa, st), "head activity scale");
+    }
     in = w.Hk[k];
   }
   return FF_OK;

@@ -32,6 +32,29 @@ __device__ __forceinline__ bool ff_dcheck(bool, int*) { return true; }
 // innermost coordinate times the element size is a multiple of 16.
 __device__ __forceinline__ bool tma_x_aligned(int x, int esize) { return ((long long)x * esize) % 16 == 0; }
 
+// Row scale and goodness helpers shared by the element-wise and GEMM kernels.
+constexpr float kNormEps = 1e-12f;
+
+// 1 / max(sqrt(ss), 1e-12), with NaN propagated (fmaxf alone would drop it).
+__device__ __forceinline__ float inv_norm(float ss) {
+  const float r = sqrtf(ss);
+  return r != r ? r : 1.f / fmaxf(r, kNormEps);
+}
+// g = sum over t of gpart[t * M + i], t = 0..ntiles-1, in that order; the
+// loads are issued together (8 at a time) rather than one per dependent add.
+__device__ __forceinline__ float sum_partials(const float* __restrict__ gpart, int ntiles, int M, int i) {
+  float g = 0.f;
+  for (int t0 = 0; t0 < ntiles; t0 += 8) {
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) v[u] = (t0 + u < ntiles) ? __ldg(gpart + (size_t)(t0 + u) * M + i) : 0.f;
+#pragma unroll
+    for (int u = 0; u < 8; ++u)
+      if (t0 + u < ntiles) g += v[u];
+  }
+  return g;
+}
+
 // Bound on every spin-wait in a kernel: after this many nanoseconds of
 // %globaltimer the wait gives up, latches DEVERR_TIMEOUT and the kernel
 // winds down.
@@ -128,6 +151,15 @@ struct EpiArgs {
   const float* bias;   // null: no bias
   void* out; int ldo;
   float* gpart;        // forward only
+  // Forward GEMMs of the tensor-core path only: with gpart_in set, the row
+  // scale is inv_norm of the previous layer's goodness (its partials
+  // gpart_in[t * M + i], t < ntiles_in, summed as k_finalize does) instead of
+  // row_scale[i]; the first column tile adds that goodness to G_acc[i] and
+  // stores the scale in s_out[i] (each when set) and flags a non-finite one.
+  const float* gpart_in;
+  int ntiles_in;
+  float* G_acc;
+  float* s_out;
 };
 
 // Tensor-core (tcgen05) bf16 GEMMs, fp32 accumulate.
