@@ -10,12 +10,13 @@
 // largest logit.
 //
 // Kernels (all fixed-order reductions, no floating-point atomics):
-//   k_head_dot     partial logits A V^T over 1024-feature splits of the
+//   k_head_dot     partial logits A V^T over feature splits of the
 //                  segments; A is never materialised -- it is read as the
-//                  stored activities H_k times their row scales s_k
-//   k_head_finish  z = c + the splits' partials (in split order), softmax,
-//                  per-row loss and dz = (softmax(z) - onehot(y)) / n,
-//                  per-block partials of dc and of the loss
+//                  stored activities H_k times their row scales s_k.  The
+//                  last block of each 64-row block to finish then forms
+//                  z = c + the splits' partials (in split order), softmax,
+//                  per-row loss and dz = (softmax(z) - onehot(y)) / n, and
+//                  the row block's partials of dc and of the loss
 //   k_head_wgrad   dV partials per 128-row block: dz^T (s_k H_k)
 //   k_head_adam    reduces the partials in a fixed order, Adam on V and c,
 //                  the step's loss
@@ -36,7 +37,6 @@ constexpr int kMaxSegs = 16;
 constexpr int kDotRows = 64;     // rows per block of k_head_dot (eight per warp)
 constexpr int kSplit = 1024;     // widest feature split of one segment per k_head_dot block
 constexpr int kDotMinBlocks = 152 / 2;  // k_head_dot grids narrower than this split features finer
-constexpr int kFinRows = 256;    // rows per block of k_head_finish (one per thread)
 constexpr int kWgRows = 64;      // rows per block of k_head_wgrad (8 per warp)
 constexpr int kWgChunk = 128;    // features per block of k_head_wgrad (4 per lane)
 constexpr int kPart = kClasses + 1;  // per-block partials: dc[10], loss
@@ -157,6 +157,23 @@ size_t zpart_floats(const int* F, int nseg, int rows, int es) {
   return mx;
 }
 
+// What the last block of a row block needs to finish its rows: the bias,
+// labels (null: logits only), outputs, the head's step counter (advanced by
+// row block 0 when training) and one arrival counter per row block (zero
+// between launches; the finishing block resets it).
+struct FinishArgs {
+  const float* cb;
+  const int* labels;
+  float inv_n;
+  float* logits;  // [n, 10] or null
+  float* dz;      // [n, 10] or null
+  float* part;    // [row blocks, 11] or null
+  ff_dev_state* ds;
+  float beta1, beta2;
+  int* counter;
+  int S;          // blocks (splits) per row block
+};
+
 // One tensor map per segment: H_k as [n, ld_k] with 64-row boxes of 512
 // bytes (256 bf16 or 128 fp32 features), no swizzle.
 struct HeadMaps {
@@ -177,7 +194,7 @@ constexpr int kDotSmem = kDotStages * kDotStageBytes + kSplit * kClasses * 4 + 6
 template <typename T>
 __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ HeadMaps maps, Segs sg, int split, int n,
                                                      const float* __restrict__ V, float* __restrict__ zpart,
-                                                     int* err) {
+                                                     FinishArgs fa, int* err) {
   constexpr int CH = 512 / (int)sizeof(T);  // features per chunk
   constexpr int FPL = CH / 32;              // features per lane
   constexpr int NCH = kSplit / CH;          // chunks in the widest split
@@ -303,41 +320,45 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
     if (threadIdx.x == 0)
       for (int ch = issued - kDotStages < 0 ? 0 : issued - kDotStages; ch < issued; ++ch)
         ptx::mbar_wait(&full[ch % kDotStages], (uint32_t)(ch / kDotStages) & 1u, 10000000ull, never_set);
-    return;
-  }
-#pragma unroll
-  for (int r = 0; r < 8; ++r)
-#pragma unroll
-    for (int c = 0; c < kClasses; ++c) acc[r][c] = warp_sum(acc[r][c]);
-  // lane c writes class c of the warp's rows
-#pragma unroll
-  for (int c = 0; c < kClasses; ++c) {
-    if (lane != c) continue;
+  } else {
 #pragma unroll
     for (int r = 0; r < 8; ++r)
-      if (r0 + r < n) zpart[((size_t)blockIdx.x * n + r0 + r) * kClasses + c] = acc[r][c];
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) acc[r][c] = warp_sum(acc[r][c]);
+    // lane c writes class c of the warp's rows
+#pragma unroll
+    for (int c = 0; c < kClasses; ++c) {
+      if (lane != c) continue;
+#pragma unroll
+      for (int r = 0; r < 8; ++r)
+        if (r0 + r < n) zpart[((size_t)blockIdx.x * n + r0 + r) * kClasses + c] = acc[r][c];
+    }
   }
-}
-
-// One thread per row: z = c + sum of the splits' partials (split order),
-// then softmax, loss and dz (training) or the logits (predict).  Per block:
-// the partial sums of dz (for dc) and of the loss, in a fixed order.
-__global__ void __launch_bounds__(kFinRows) k_head_finish(int n, int S, const float* __restrict__ zpart,
-                                                          const float* __restrict__ cb, const int* __restrict__ labels,
-                                                          float inv_n, float* __restrict__ logits,
-                                                          float* __restrict__ dz, float* __restrict__ part,
-                                                          ff_dev_state* ds, float beta1, float beta2, int* err) {
-  __shared__ float red[kFinRows / 32][kPart];
-  const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-  const int row = blockIdx.x * kFinRows + threadIdx.x;
-  if (blockIdx.x == 0 && threadIdx.x == 0 && labels && ds) {
-    // this step's Adam counter and bias corrections, read by k_head_adam
-    ds->t += 1;
-    ds->pow1 *= (double)beta1;
-    ds->pow2 *= (double)beta2;
-    ds->bc1 = (float)(1.0 - ds->pow1);
-    ds->bc2 = (float)(1.0 - ds->pow2);
+  // Every block arrives (an aborted one too, so that the counter is reset);
+  // the last of the row block's S blocks finishes its rows.
+  __shared__ int last;
+  __shared__ float fred[kDotRows / 32][kPart];
+  __threadfence();
+  __syncthreads();
+  if (threadIdx.x == 0) last = atomicAdd(fa.counter + blockIdx.y, 1) == fa.S - 1;
+  __syncthreads();
+  if (!last) return;
+  __threadfence();
+  if (threadIdx.x == 0) {
+    fa.counter[blockIdx.y] = 0;
+    if (blockIdx.y == 0 && fa.labels && fa.ds) {
+      // this step's Adam counter and bias corrections, read by k_head_adam
+      fa.ds->t += 1;
+      fa.ds->pow1 *= (double)fa.beta1;
+      fa.ds->pow2 *= (double)fa.beta2;
+      fa.ds->bc1 = (float)(1.0 - fa.ds->pow1);
+      fa.ds->bc2 = (float)(1.0 - fa.ds->pow2);
+    }
   }
+  if (threadIdx.x >= kDotRows) return;
+  // one thread per row: z = c + the splits' partials in split order (read
+  // past L1: other blocks wrote them during this launch)
+  const int row = rblk + (int)threadIdx.x;
   float dzr[kClasses];
   float loss = 0.f;
 #pragma unroll
@@ -345,28 +366,30 @@ __global__ void __launch_bounds__(kFinRows) k_head_finish(int n, int S, const fl
   if (row < n) {
     float z[kClasses];
 #pragma unroll
-    for (int c = 0; c < kClasses; ++c) z[c] = __ldg(cb + c);
-    for (int sp = 0; sp < S; ++sp) {
+    for (int c = 0; c < kClasses; ++c) z[c] = __ldg(fa.cb + c);
+    for (int sp = 0; sp < fa.S; ++sp) {
       const float* zp = zpart + ((size_t)sp * n + row) * kClasses;
 #pragma unroll
-      for (int c = 0; c < kClasses; ++c) z[c] += __ldg(zp + c);
+      for (int c = 0; c < kClasses; ++c) z[c] += __ldcg(zp + c);
     }
-    loss = finish_row(z, row, labels, inv_n, logits, dz, dzr, err);
+    loss = finish_row(z, row, fa.labels, fa.inv_n, fa.logits, fa.dz, dzr, err);
   }
-  if (!part) return;
+  if (!fa.part) return;
+  // the row block's sums of dz (for dc) and of the loss, in a fixed order
 #pragma unroll
   for (int c = 0; c < kClasses; ++c) dzr[c] = warp_sum(dzr[c]);
   loss = warp_sum(loss);
   if (lane == 0) {
 #pragma unroll
-    for (int c = 0; c < kClasses; ++c) red[warp][c] = dzr[c];
-    red[warp][kClasses] = loss;
+    for (int c = 0; c < kClasses; ++c) fred[warp][c] = dzr[c];
+    fred[warp][kClasses] = loss;
   }
-  __syncthreads();
+  asm volatile("bar.sync 1, %0;" ::"n"(kDotRows) : "memory");  // the row block's warps only
   if (threadIdx.x < kPart) {
-    float acc = 0.f;
-    for (int w = 0; w < kFinRows / 32; ++w) acc += red[w][threadIdx.x];
-    part[(size_t)blockIdx.x * kPart + threadIdx.x] = acc;
+    float t = 0.f;
+#pragma unroll
+    for (int w = 0; w < kDotRows / 32; ++w) t += fred[w][threadIdx.x];
+    fa.part[(size_t)blockIdx.y * kPart + threadIdx.x] = t;
   }
 }
 
@@ -433,7 +456,9 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
 // block per 32 rows x 256 columns (block 32 x 8; thread (x, y) owns columns
 // 8x..8x+7 of rows y, y+8, y+16, y+24):
 //   dZ_ij = (sum_c dz_ic V_cj) [h_ij > 0],  G_ij = s_i dZ_ij (weight-gradient
-//   operand, in the activity type),  db partials = sum over the block's rows.
+//   operand, in the activity type),  db partials = sum over the block's rows,
+//   and the block's own weight-gradient partials dV_cj = sum_i dz_ic h_ij
+//   over the same rows (the block reads the raw activity).
 // V (before this step's update) and dz are staged in shared memory.  Lead
 // blocks (x == 0) also write the next layer's row scale from the forward's
 // goodness partials; block (0, 0) advances the layer's Adam step.
@@ -481,6 +506,7 @@ struct PoGradArgs {
   int ntiles, n, N, ld;
   float* s_next;        // [n] or null
   float* dbpart;        // [row blocks, N]
+  float* dVpart;        // [row blocks, 10, N]: the block's dV partials
   ff_dev_state* ds;     // the layer's
   float beta1, beta2;
   int* err;
@@ -492,7 +518,10 @@ template <typename T>
 __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restrict__ H, T* __restrict__ G) {
   __shared__ float Vsh[kClasses][8][32];  // V[c][c0 + 8 l + e] at [c][e][l]: conflict-free reads
   __shared__ float dzs[kPoRows][kClasses];
-  __shared__ float red[8][256 + 8];
+  // the block's activity tile in its own type (for the dV partials), then
+  // the db reduction in the same memory
+  __shared__ __align__(16) T Hs[kPoRows][256 + 8];
+  static_assert(sizeof(Hs) >= 8 * (256 + 4) * sizeof(float), "the db reduction fits in the tile's memory");
   const int r0 = blockIdx.y * kPoRows;
   const int lane = threadIdx.x, tid = threadIdx.y * 32 + threadIdx.x;
   const int c0 = blockIdx.x * 256;
@@ -530,9 +559,15 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   for (int k = 0; k < 4; ++k) {
     const int li = threadIdx.y + 8 * k;
     const int i = r0 + li;
-    if (!cols_ok || i >= a.n) continue;
     float h[8], z[8];
-    V8<T>::load(H + (size_t)i * a.ld + cg, h);
+    if (cols_ok && i < a.n) {
+      V8<T>::load(H + (size_t)i * a.ld + cg, h);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) h[e] = 0.f;
+    }
+    V8<T>::store(&Hs[li][lane * 8], h);
+    if (!cols_ok || i >= a.n) continue;
     const float si = __ldg(a.s + i);
 #pragma unroll
     for (int e = 0; e < 8; ++e) {
@@ -545,8 +580,29 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     }
     V8<T>::store(G + (size_t)i * a.ld + cg, z);
   }
+  __syncthreads();
+  // dV partials from the staged tile: thread (x, y) sums classes y and
+  // y + 8 (when below 10) over the block's 32 rows in order, for its 8 columns
 #pragma unroll
-  for (int e = 0; e < 8; ++e) red[threadIdx.y][lane * 8 + e] = db[e];
+  for (int c = threadIdx.y; c < kClasses; c += 8) {
+    float dv[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) dv[e] = 0.f;
+    for (int li = 0; li < kPoRows; ++li) {
+      const float d = dzs[li][c];
+      float h[8];
+      V8<T>::load(&Hs[li][lane * 8], h);
+#pragma unroll
+      for (int e = 0; e < 8; ++e) dv[e] = fmaf(d, h[e], dv[e]);
+    }
+#pragma unroll
+    for (int e = 0; e < 8; ++e)
+      if (cg + e < a.N) a.dVpart[((size_t)blockIdx.y * kClasses + c) * a.N + cg + e] = dv[e];
+  }
+  __syncthreads();
+  // db partials: the eight row groups added in order, through the tile's memory
+  float (*red)[256 + 4] = reinterpret_cast<float (*)[256 + 4]>(&Hs[0][0]);
+  V8<float>::store(&red[threadIdx.y][lane * 8], db);
   __syncthreads();
   if (threadIdx.y == 0) {
 #pragma unroll
@@ -636,6 +692,8 @@ struct ff_head {
   ff::ff_dev_state* ds;
   void* ws;
   size_t ws_bytes;
+  int* counters;    // k_head_dot arrival counters, one per 64-row block (zero between launches)
+  int counter_cap;
 };
 
 namespace ff {
@@ -697,7 +755,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   size_t oZ = off; off += align256((size_t)rows * kClasses * 4);
   size_t oZP = off; off += align256(chain_zpart_floats(layers, L, rows) * 4);
   size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
-  size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kFinRows) * kPart * 4 : 0);
+  size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kDotRows) * kPart * 4 : 0);
   size_t oV = off; off += align256(train ? (size_t)cdiv(rows, kWgRows) * kClasses * hd->F * 4 : 0);
   if (off > hd->ws_bytes) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before head workspace growth");
@@ -787,14 +845,43 @@ Segs make_segs(ff_layer* const* layers, int L, const HeadWork& w, int F) {
   return sg;
 }
 
-// Logits (and, with labels, softmax, loss, dz and the per-block partials)
-// of n rows: k_head_dot over the feature splits, then k_head_finish.
-ff_status head_logits(const Segs& sg, bool b16, int n, const float* V, const float* c, const int* labels,
-                      float* logits, float* zpart, float* dz, float* part, ff_dev_state* ds, float beta1, float beta2,
-                      int* err, cudaStream_t st) {
+// One arrival counter per 64-row block of k_head_dot, all zero (grown on
+// demand; the kernel leaves them zero).
+ff_status ensure_counters(ff_head* hd, int blocks) {
+  if (blocks <= hd->counter_cap) return FF_OK;
+  FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before counter growth");
+  dev_free(hd->counters);
+  hd->counters = nullptr;
+  hd->counter_cap = 0;
+  FF_TRY(dev_alloc(reinterpret_cast<void**>(&hd->counters), (size_t)blocks * sizeof(int)), "head counters");
+  FF_TRY(cudaMemset(hd->counters, 0, (size_t)blocks * sizeof(int)), "zero head counters");
+  hd->counter_cap = blocks;
+  return FF_OK;
+}
+
+// Logits (and, with labels, softmax, loss, dz and the per-row-block
+// partials) of n rows: k_head_dot over the feature splits, whose last block
+// per row block finishes the rows.
+ff_status head_logits(ff_head* hd, const Segs& sg, bool b16, int n, const int* labels, float* logits, float* zpart,
+                      float* dz, float* part, int* err, cudaStream_t st) {
   const int es = b16 ? 2 : 4;
   const int split = dot_split(sg.F, sg.nseg, n, es);
   const int S = head_splits(sg.F, sg.nseg, split);
+  ff_status s = ensure_counters(hd, cdiv(n, kDotRows));
+  if (s != FF_OK) return s;
+  FinishArgs fa{};
+  fa.cb = hd->c;
+  fa.labels = labels;
+  fa.inv_n = 1.f / (float)n;
+  fa.logits = logits;
+  fa.dz = dz;
+  fa.part = part;
+  fa.ds = labels ? hd->ds : nullptr;
+  fa.beta1 = hd->cfg.beta1;
+  fa.beta2 = hd->cfg.beta2;
+  fa.counter = hd->counters;
+  fa.S = S;
+  const float* V = hd->V;
   HeadMaps maps;
   std::memset(&maps, 0, sizeof(maps));
   for (int k = 0; k < sg.nseg; ++k)
@@ -806,17 +893,12 @@ ff_status head_logits(const Segs& sg, bool b16, int n, const float* V, const flo
                                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kDotSmem);
   FF_TRY(b16 ? attr_b : attr_f, "head kernel attributes");
   dim3 grid(S, cdiv(n, kDotRows));
-  FF_LAUNCH(K_HEAD_LOGITS, (double)n * sg.F_total * es + (double)n * S * kClasses * 4, st,
-            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, err), cudaGetLastError())
-                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, err),
+  FF_LAUNCH(K_HEAD_LOGITS, (double)n * sg.F_total * es + (double)n * (2 * S + 2) * kClasses * 4, st,
+            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, fa, err),
+                    cudaGetLastError())
+                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, fa, err),
                     cudaGetLastError())),
-            "head partial logits");
-  const float inv_n = 1.f / (float)n;
-  FF_LAUNCH(K_HEAD_FINISH, (double)n * (S + 2) * kClasses * 4, st,
-            (k_head_finish<<<cdiv(n, kFinRows), kFinRows, 0, st>>>(n, S, zpart, c, labels, inv_n, logits, dz, part,
-                                                                   ds, beta1, beta2, err),
-             cudaGetLastError()),
-            "head softmax and cross-entropy");
+            "head logits, softmax and cross-entropy");
   return FF_OK;
 }
 
@@ -855,8 +937,8 @@ ff_status po_workspace(ff_head* hd, int n, int N, int es, PoWork* w) {
   size_t off = 0;
   const size_t oZ = off; off += align256(zpart_floats(&N, 1, n, es) * 4);
   const size_t oD = off; off += align256((size_t)n * kClasses * 4);
-  const size_t oP = off; off += align256((size_t)cdiv(n, kFinRows) * kPart * 4);
-  const size_t oV = off; off += align256((size_t)cdiv(n, kWgRows) * kClasses * N * 4);
+  const size_t oP = off; off += align256((size_t)cdiv(n, kDotRows) * kPart * 4);
+  const size_t oV = off; off += align256((size_t)cdiv(n, kPoRows) * kClasses * N * 4);
   if (off > hd->ws_bytes) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before workspace growth");
     dev_free(hd->ws);
@@ -961,6 +1043,7 @@ ff_status ff_head_destroy(ff_head* hd) {
   if (!hd) return FF_OK;
   cudaStreamSynchronize(hd->last_stream);
   dev_free(hd->ws);
+  dev_free(hd->counters);
   dev_free(hd->V);
   dev_free(hd->ds);
   delete hd;
@@ -986,12 +1069,11 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
   const Segs sg = make_segs(layers, n_layers, w, hd->F);
   const bool b16 = layers[0]->is_bf16;
   const double es = b16 ? 2.0 : 4.0;
-  s = head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.zpart, w.dz, w.part, hd->ds, hd->cfg.beta1,
-                  hd->cfg.beta2, err, st);
+  s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, err, st);
   if (s != FF_OK) return s;
   FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
             launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
-  const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kFinRows), n, loss);
+  const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kDotRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
   FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st,
             (k_head_adam<<<vblocks + 1, 256, 0, st>>>(a), cudaGetLastError()), "head Adam");
@@ -1021,7 +1103,7 @@ ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, co
     if (s != FF_OK) return s;
     const Segs sg = make_segs(layers, n_layers, w, hd->F);
     float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
-    s = head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, w.zpart, nullptr, nullptr, nullptr, 0.f, 0.f, err, st);
+    s = head_logits(hd, sg, b16, cn, nullptr, z, w.zpart, nullptr, nullptr, err, st);
     if (s != FF_OK) return s;
     if (pred)
       FF_LAUNCH(K_ARGMAX, (double)cn * 44, st, launch_argmax(z, cn, nullptr, pred + r0, st), "head argmax");
@@ -1163,12 +1245,10 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   sg.off[0] = 0;
   sg.nseg = 1;
   sg.F_total = N;
-  s = head_logits(sg, b16, n, hd->V, hd->c, labels, nullptr, w.zpart, w.dz, w.part, hd->ds, hd->cfg.beta1,
-                  hd->cfg.beta2, &hd->ds->err, st);
+  s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, &hd->ds->err, st);
   if (s != FF_OK) return s;
-  FF_LAUNCH(K_HEAD_WGRAD, (double)n * N * es + (double)cdiv(n, kWgRows) * kClasses * N * 4, st,
-            launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "block weight gradient");
-  // the gradient reaching the layer, with the block's weights before its update
+  // the gradient reaching the layer, with the block's weights before its
+  // update, and the block's weight-gradient partials
   PoGradArgs pa{};
   pa.dz = w.dz;
   pa.V = hd->V;
@@ -1180,12 +1260,13 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   pa.ld = L->ldN;
   pa.s_next = next_scale;
   pa.dbpart = L->dbpart;
+  pa.dVpart = w.dVpart;
   pa.ds = L->ds;
   pa.beta1 = L->cfg.beta1;
   pa.beta2 = L->cfg.beta2;
   pa.err = &L->ds->err;
   dim3 grid(cdiv(L->ldN, 256), cdiv(n, kPoRows)), block(32, 8);
-  FF_LAUNCH(K_GRAD_PREP, (double)n * L->ldN * es * 2 + (double)cdiv(n, kPoRows) * N * 4, st,
+  FF_LAUNCH(K_GRAD_PREP, (double)n * L->ldN * es * 2 + (double)cdiv(n, kPoRows) * (kClasses + 1) * N * 4, st,
             (b16 ? (k_po_grad<bf16><<<grid, block, 0, st>>>(pa, static_cast<const bf16*>(H), static_cast<bf16*>(L->dZ)),
                     cudaGetLastError())
                  : (k_po_grad<float><<<grid, block, 0, st>>>(pa, static_cast<const float*>(H),
@@ -1228,7 +1309,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   aa.loss_out = nullptr;
   aa.B = n;
   FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
-  const HeadAdamArgs ha = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kFinRows), n, loss);
+  const HeadAdamArgs ha = head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, kDotRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
   FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), st,
             (k_head_adam<<<vblocks + 1, 256, 0, st>>>(ha), cudaGetLastError()), "block Adam");
@@ -1268,7 +1349,7 @@ ff_status ff_po_predict(ff_layer* const* layers, int n_layers, ff_head* hd, cons
     sg.nseg = 1;
     sg.F_total = top->N;
     float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
-    s = head_logits(sg, b16, cn, hd->V, hd->c, nullptr, z, w.zpart, nullptr, nullptr, nullptr, 0.f, 0.f, err, st);
+    s = head_logits(hd, sg, b16, cn, nullptr, z, w.zpart, nullptr, nullptr, err, st);
     if (s != FF_OK) return s;
     if (pred)
       FF_LAUNCH(K_ARGMAX, (double)cn * 44, st, launch_argmax(z, cn, nullptr, pred + r0, st), "block argmax");
