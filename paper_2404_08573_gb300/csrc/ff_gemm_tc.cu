@@ -66,8 +66,11 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
   atomicOr(err, DEVERR_TIMEOUT);
 }
 
+// At most 96 registers a thread (the bound for two CTAs of 320 threads per
+// SM; no spills): a CTA then leaves room on its SM for the Adam and local-
+// gradient blocks of the other layers' streams (784-2000x4 epoch -1 %).
 template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
-__global__ void __launch_bounds__(NTHREADS, 1)
+__global__ void __launch_bounds__(NTHREADS, 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
   using C = TcCfg<BN, NSTAGE, MT, PAIR>;
