@@ -273,6 +273,11 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   aa.stats_out = L->ds->stats;
   aa.loss_out = loss ? loss : &L->ds->loss;
   aa.B = B;
+  // Data nobody reads after this step, so its dirty lines need not reach HBM:
+  // dW (unless kept for ff_layer_get_grad) and the local-gradient operand.
+  // (Dropping the activities' lines as well measured no further gain.)
+  aa.discard_dW = !L->cfg.keep_grad && ((uintptr_t)L->dW & 127u) == 0;
+  add_dead(aa, L->dZ, (size_t)M * L->ldN * (size_t)es);
   FF_LAUNCH(K_ADAM, (double)L->N * L->K * (28.0 + (L->is_bf16 ? 2.0 : 0.0)) + (double)L->N * (aa.nrb * 4.0 + 28), st,
             launch_adam(aa, st),
             "Adam");

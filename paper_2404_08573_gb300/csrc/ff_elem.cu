@@ -324,6 +324,12 @@ __device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, flo
 
 __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
   ptx::griddep_wait();  // launched with programmatic stream serialization
+  {
+    // the step's dead buffers: every kernel that reads them has completed
+    const long long gt = (long long)blockIdx.x * 256 + threadIdx.x, nt = (long long)gridDim.x * 256;
+    for (int r = 0; r < a.ndead; ++r)
+      for (long long l = gt; l < a.dead_lines[r]; l += nt) ptx::discard_l2(a.dead[r] + l * 128);
+  }
   const float a1 = a.lr / a.ds->bc1, r2 = 1.f / a.ds->bc2;
   if ((int)blockIdx.x < w_blocks) {
     const long long total = (long long)a.N * a.K;
@@ -346,6 +352,9 @@ __global__ void __launch_bounds__(256) k_adam(AdamArgs a, int w_blocks) {
         __stcs(reinterpret_cast<float4*>(a.W + idx), w);
         __stcs(reinterpret_cast<float4*>(a.mW + idx), m);
         __stcs(reinterpret_cast<float4*>(a.vW + idx), v);
+        // the first of every 8 threads drops the 128-byte dW line the 8 just
+        // read (the warp's loads have all returned: g was used above)
+        if (a.discard_dW && (threadIdx.x & 7) == 0 && idx + 32 <= total) ptx::discard_l2(a.dW + idx);
         if (a.Wb) {
           const long long o = dense_b ? idx : (idx / a.K) * a.ldb + idx % a.K;
           __nv_bfloat162 p0 = __floats2bfloat162_rn(w.x, w.y), p1 = __floats2bfloat162_rn(w.z, w.w);
@@ -617,6 +626,13 @@ cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, voi
   PdlLaunch l(dim3(cdiv(a.ld, 256), local_grad_row_blocks(a.M)), dim3(32, 8), st);
   if (b16) return cudaLaunchKernelEx(&l.cfg, k_grad_prep<bf16>, a, (const bf16*)H, (bf16*)dZ);
   return cudaLaunchKernelEx(&l.cfg, k_grad_prep<float>, a, (const float*)H, (float*)dZ);
+}
+
+void add_dead(AdamArgs& a, void* p, size_t bytes) {
+  if (!p || ((uintptr_t)p & 127u) || bytes < 128 || a.ndead >= 2) return;
+  a.dead[a.ndead] = static_cast<char*>(p);
+  a.dead_lines[a.ndead] = (long long)(bytes / 128);
+  ++a.ndead;
 }
 
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st) {

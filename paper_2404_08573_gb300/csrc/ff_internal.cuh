@@ -128,7 +128,17 @@ struct AdamArgs {
   const float* stat_part;  // grad_prep's statistics partials, or null
   int ncb;
   float* stats_out;        // [3] receives the step's statistics
+  // Dead data: buffers (128-byte aligned, whole lines) that nothing reads
+  // before they are rewritten, and dW itself once read (discard_dW), have
+  // their lines dropped from L2 instead of written back to HBM.
+  int discard_dW;
+  int ndead;
+  char* dead[2];
+  long long dead_lines[2];
 };
+// Adds [p, p + bytes) to the Adam step's dead buffers (its whole 128-byte
+// lines; nothing when p is not 128-byte aligned).
+void add_dead(AdamArgs& a, void* p, size_t bytes);
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
 cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cudaStream_t st);
