@@ -366,6 +366,35 @@ def test_repeat_runs_are_bitwise_equal(env):
     assert np.array_equal(outs[0][0], outs[1][0]) and np.array_equal(outs[0][1], outs[1][1])
 
 
+def test_dropped_gradient_lines_change_nothing(env):
+    """Without keep_grad the Adam kernel drops dW's L2 lines once read (and
+    the local-gradient operand's); a layer that keeps its gradient does not
+    drop dW.  Both train a hidden and a first layer bit for bit alike over
+    several steps, at a size whose state does not fit in L2."""
+    torch, ff = env
+    B = 1024
+    x2, l2 = pair_inputs(B, seed=78)
+    xg, lg = torch.from_numpy(x2).cuda(), torch.from_numpy(l2).cuda()
+    outs = []
+    for keep in (True, False):
+        l1 = ff.Layer(784, 2000, prec="bf16", init_seed=5, keep_grad=keep)
+        l2_ = ff.Layer(2000, 2000, prec="bf16", init_seed=6, keep_grad=keep)
+        h = l1.new_activation(2 * B)
+        sc = torch.empty(2 * B, device="cuda")
+        loss = torch.empty(4, 2, device="cuda")
+        for t in range(4):
+            l1.train_step(xg, labels=lg, B=B, h_out=h, next_scale=sc, loss=loss[t, 0:1])
+            l2_.train_step(h, row_scale=sc, B=B, loss=loss[t, 1:2])
+        torch.cuda.synchronize()
+        l1.check()
+        l2_.check()
+        outs.append((loss.cpu().numpy(), [l.get_state() for l in (l1, l2_)]))
+    assert np.array_equal(outs[0][0], outs[1][0])
+    for a, b in zip(outs[0][1], outs[1][1]):
+        for k in ("W", "b", "mW", "vW", "mb", "vb"):
+            assert np.array_equal(np.asarray(a[k]), np.asarray(b[k])), k
+
+
 # ---------------------------------------------------------------- edges
 def test_edge_cases(env):
     torch, ff = env
