@@ -494,8 +494,9 @@ constexpr int WGRAD_BN = 256;
 //   pairs, one subtile per CTA (128 CTAs per GEMM), 6 / 4 stages  9.90 / 10.52
 //   pairs, two subtiles per CTA (64 CTAs per GEMM), 4 / 3 stages  9.05 / 8.78
 // With 128 CTAs a GEMM alone is faster (20 vs 29 us for 2048x2000x2000) but
-// two layers' GEMMs no longer fit on the GPU side by side; earlier 128 x 256
-// tiles and 4-CTA multicast clusters measured 9.8 and 11.1 ms.
+// two layers' GEMMs no longer fit on the GPU side by side (re-measured with
+// dependent launch and the later Adam changes: 9.54 against 8.32 ms); earlier
+// 128 x 256 tiles and 4-CTA multicast clusters measured 9.8 and 11.1 ms.
 constexpr bool USE_PAIR = true;
 constexpr int NSTAGES = 3;       // operand ring depth
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
