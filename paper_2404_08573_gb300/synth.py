@@ -125,14 +125,15 @@ def pair_batch(x: np.ndarray, y: np.ndarray, y_neg: np.ndarray):
     return np.ascontiguousarray(x2), l2
 
 
-def learnable_task(n: int, seed: int = 0, features: int = 784, start_row: int = 0):
+def learnable_task(n: int, seed: int = 0, features: int = 784, start_row: int = 0, on_support: float = 0.5):
     """A learnable MNIST-shaped task for end-to-end accuracy checks.
 
     Class c owns a fixed random support of 157 feature positions among
     features 10..783.  Each feature of a sample of class c is nonzero with
     probability 0.2; a nonzero feature lands on the class support with
-    probability 0.5 (else anywhere), so about 20 % of features are nonzero and
-    the class is recoverable from where the mass sits.  Values are U(0, 1).
+    probability ``on_support`` (else anywhere), so about 20 % of features are
+    nonzero and the class is recoverable from where the mass sits (less
+    reliably for a smaller ``on_support``).  Values are U(0, 1).
     Returns (x [n, features] float32, y [n] int32).
     """
     rng_support = uniform(seed, STREAM_PROTOTYPES, N_CLASSES * (features - 10))
@@ -141,12 +142,12 @@ def learnable_task(n: int, seed: int = 0, features: int = 784, start_row: int = 
     y = labels(n, seed, start=start_row)
     u = uniform(seed, STREAM_FEATURES, n * features * 2, start=start_row * features * 2).reshape(n, features, 2)
     x = np.zeros((n, features), dtype=np.float64)
-    on_support = np.zeros((n, features), dtype=bool)
-    on_support[np.arange(n)[:, None], support[y]] = True
+    on = np.zeros((n, features), dtype=bool)
+    on[np.arange(n)[:, None], support[y]] = True
     # nonzero probability: features on the class support carry the class mass.
-    p_on = 0.2 * 0.5 * features / 157.0 + 0.2 * 0.5
-    p_off = 0.2 * 0.5
-    p = np.where(on_support, p_on, p_off)
+    p_on = 0.2 * on_support * features / 157.0 + 0.2 * (1.0 - on_support)
+    p_off = 0.2 * (1.0 - on_support)
+    p = np.where(on, p_on, p_off)
     p[:, :10] = 0.0
     x = np.where(u[..., 0] < p, u[..., 1], 0.0)
     return x.astype(np.float32), y
