@@ -189,7 +189,7 @@ def test_train_step(env, prec, B, K, N, first):
     # the activity handed to the next layer and its scale
     assert_close(h.float().cpu().numpy()[:, :N], ref["H"], 1e-5 if not emul else 2.0 ** -8 + 1e-3, 1e-5, "activity")
     assert_close(sn.cpu().numpy(), 1.0 / np.maximum(np.sqrt(ref["g"]), 1e-12), gtol, 0, "next scale")
-    # against the plain fp64 definition, at the benchmark spec's tolerances
+    # against the plain fp64 definition, at the tolerances of each precision
     plain = fo.layer_train_step(fo.LayerState(W, b), xin, B, theta, fo.AdamHyper(lr=lr))
     if not emul:
         assert_close(g.cpu().numpy(), plain["g"], 1e-4, 1e-4, "goodness vs fp64")
