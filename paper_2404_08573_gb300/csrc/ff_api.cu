@@ -119,6 +119,8 @@ ff_status ensure_capacity(ff_layer* L, int rows) {
 
 static void free_layer(ff_layer* L) {
   if (!L) return;
+  dev_free(L->kpart);
+  dev_free(L->kcnt);
   dev_free(L->W);
   dev_free(L->mW);  // also holds v_W
   dev_free(L->dW);
@@ -143,9 +145,37 @@ struct FwdResult {
   int ntiles;
 };
 
+// Split-K scratch of an fp32 layer's forward and weight-gradient GEMMs on M
+// rows (grown on demand; new counters start at zero).
+static ff_status ensure_split(ff_layer* L, int M) {
+  const size_t fwd = simt_split_floats(M, L->N, L->K), wg = simt_split_floats(L->N, L->K, M);
+  const size_t need = fwd > wg ? fwd : wg;
+  if (need == 0) return FF_OK;
+  const int t1 = simt_split_tiles(M, L->N), t2 = simt_split_tiles(L->N, L->K);
+  const int tiles = t1 > t2 ? t1 : t2;
+  if (need <= L->kpart_cap && tiles <= L->kcnt_cap) return FF_OK;
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync before split scratch growth");
+  dev_free(L->kpart);
+  dev_free(L->kcnt);
+  L->kpart = nullptr;
+  L->kcnt = nullptr;
+  L->kpart_cap = 0;
+  L->kcnt_cap = 0;
+  FF_TRY(dev_alloc(reinterpret_cast<void**>(&L->kpart), need * sizeof(float)), "split scratch");
+  FF_TRY(dev_alloc(reinterpret_cast<void**>(&L->kcnt), (size_t)tiles * sizeof(int)), "split counters");
+  FF_TRY(cudaMemset(L->kcnt, 0, (size_t)tiles * sizeof(int)), "zero split counters");
+  L->kpart_cap = need;
+  L->kcnt_cap = tiles;
+  return FF_OK;
+}
+
 static ff_status forward_core(ff_layer* L, const void* x, const int* labels, const float* row_scale, int M,
                               void* h_out, cudaStream_t st, cudaEvent_t ev_input_read, FwdResult* r) {
   const int K = L->K, N = L->N;
+  if (!L->is_bf16) {
+    const ff_status ss = ensure_split(L, M);
+    if (ss != FF_OK) return ss;
+  }
   const double es = L->is_bf16 ? 2.0 : 4.0;
   const float* s;
   const void* X;
@@ -176,6 +206,10 @@ static ff_status forward_core(ff_layer* L, const void* x, const int* labels, con
               "forward GEMM (tcgen05)");
   } else {
     ntiles = simt_fwd_ntiles(N);
+    ep.kpart = L->kpart;
+    ep.kpart_cap = L->kpart_cap;
+    ep.kcnt = L->kcnt;
+    ep.kcnt_cap = L->kcnt_cap;
     FF_LAUNCH(K_FWD_SIMT, 2.0 * M * N * K, st,
               simt_gemm_fwd(static_cast<const float*>(X), L->ldK, L->W, K, M, N, K, ep, st), "forward GEMM (fp32)");
   }
@@ -241,9 +275,14 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
                             L->N, L->K, L->dW, L->K, &L->ds->err, st),
               "weight-gradient GEMM (tcgen05)");
   } else {
+    EpiArgs split{};
+    split.kpart = L->kpart;
+    split.kpart_cap = L->kpart_cap;
+    split.kcnt = L->kcnt;
+    split.kcnt_cap = L->kcnt_cap;
     FF_LAUNCH(K_WGRAD_SIMT, 2.0 * M * L->N * L->K, st,
               simt_gemm_wgrad(static_cast<const float*>(L->dZ), L->ldN, static_cast<const float*>(fr.X), L->ldK, M,
-                              L->N, L->K, L->dW, L->K, st),
+                              L->N, L->K, L->dW, L->K, st, &split),
               "weight-gradient GEMM (fp32)");
   }
   AdamArgs aa{};

@@ -170,6 +170,13 @@ struct EpiArgs {
   int ntiles_in;
   float* G_acc;
   float* s_out;
+  // fp32 SIMT GEMMs only: split-K scratch (partial tiles, capacity in floats,
+  // and one arrival counter per output tile, zero between launches); null: no
+  // split.
+  float* kpart;
+  size_t kpart_cap;
+  int* kcnt;
+  int kcnt_cap;
 };
 
 // Tensor-core (tcgen05) bf16 GEMMs, fp32 accumulate.
@@ -191,14 +198,19 @@ int tc_gemm_fwd_ctas(int M, int N);
 bool make_plain_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
                     int box_rows);
 
-// SIMT fp32 GEMMs with the same contracts.
+// SIMT fp32 GEMMs with the same contracts.  A GEMM of few output tiles
+// splits its contraction over blockIdx.z when the EpiArgs carry split-K
+// scratch of the size simt_split_floats / simt_split_tiles give (the wgrad
+// form takes the scratch from `split`).
 int simt_fwd_ntiles(int N);
+size_t simt_split_floats(int M, int N, int K);
+int simt_split_tiles(int M, int N);
 cudaError_t simt_gemm_fwd(const float* A, int lda, const float* B, int ldb, int M, int N, int K,
                           const EpiArgs& ep, cudaStream_t st);
 cudaError_t simt_gemm_store(const float* A, int lda, const float* B, int ldb, int M, int N, int K,
                             float* C, int ldc, cudaStream_t st);
 cudaError_t simt_gemm_wgrad(const float* G, int ldg, const float* X, int ldx, int R, int N, int K,
-                            float* C, int ldc, cudaStream_t st);
+                            float* C, int ldc, cudaStream_t st, const EpiArgs* split = nullptr);
 
 }  // namespace ff
 
@@ -230,4 +242,7 @@ struct ff_layer {
   float* stat_part;  // [row blocks * (2 + column blocks)] step statistics partials
   // predict scratch (owned here when this layer is layers[0] of ff_predict)
   void* pws; size_t pws_bytes;
+  // split-K scratch of the fp32 GEMMs (grown on demand; counters kept zero)
+  float* kpart; size_t kpart_cap;
+  int* kcnt; int kcnt_cap;
 };
