@@ -209,12 +209,30 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
       for (int e = 0; e < 8; ++e) h[k][e] = 0.f;
     }
   }
-  // lanes 0..3: row r0 + y + 8 * lane
+  // The warp's 4 rows r0 + y + 8k: lanes 8k .. 8k+7 share row k's goodness,
+  // lane 8k + p loading partials p, p + 8, ... (one round trip for up to 64
+  // column-tile partials) and a fixed xor tree adding the 8 lane sums; lane 8k
+  // then forms the row's loss terms.
   float cc = 0.f, sc = 0.f, lv = 0.f, gp = 0.f, gn = 0.f;
-  if (lane < 4) {
-    const int i = r0 + threadIdx.y + 8 * lane;
+  {
+    const int k = lane >> 3, p = lane & 7;
+    const int i = r0 + threadIdx.y + 8 * k;
+    float g = 0.f;
     if (i < a.M) {
-      const float g = sum_partials(a.gpart, a.ntiles, a.M, i);
+      float v[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int t = p + 8 * u;
+        v[u] = t < a.ntiles ? __ldg(a.gpart + (size_t)t * a.M + i) : 0.f;
+      }
+      for (int t = p + 64; t < a.ntiles; t += 8) v[0] += __ldg(a.gpart + (size_t)t * a.M + i);  // past 64 tiles
+#pragma unroll
+      for (int u = 0; u < 8; ++u) g += v[u];
+    }
+    g += __shfl_xor_sync(0xffffffffu, g, 4);
+    g += __shfl_xor_sync(0xffffffffu, g, 2);
+    g += __shfl_xor_sync(0xffffffffu, g, 1);
+    if (p == 0 && i < a.M) {
       const bool pos = i < a.B;
       const float tt = pos ? a.theta - g : g - a.theta;  // the pair member's margin error
       const float sg = sigmoid_f(tt);
@@ -234,7 +252,7 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
   for (int e = 0; e < 8; ++e) db[e] = 0.f;
 #pragma unroll
   for (int k = 0; k < 4; ++k) {
-    const float ck = __shfl_sync(0xffffffffu, cc, k), sk = __shfl_sync(0xffffffffu, sc, k);
+    const float ck = __shfl_sync(0xffffffffu, cc, 8 * k), sk = __shfl_sync(0xffffffffu, sc, 8 * k);
     const int i = r0 + threadIdx.y + 8 * k;
     float z[8];
 #pragma unroll
@@ -245,7 +263,7 @@ __global__ void __launch_bounds__(256) k_grad_prep(GradPrepArgs a, const T* __re
     if (cols_ok && i < a.M) Vec8<T>::store(dZ + (size_t)i * a.ld + cg, z);
   }
   if (lead) {
-    lv = warp_sum(lv);  // lanes 4..31 contribute 0
+    lv = warp_sum(lv);  // only lanes 0, 8, 16, 24 contribute
     gp = warp_sum(gp);
     gn = warp_sum(gn);
     if (lane == 0) {
