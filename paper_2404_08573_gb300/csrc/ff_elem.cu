@@ -6,8 +6,9 @@
 //   grad_prep    the same goodness, the pair loss softplus(theta - g_pos) +
 //                softplus(g_neg - theta) and its derivative dL/dg, then
 //                dZ = dL/dg * 2h (h = 0 where z <= 0), the weight-gradient
-//                operand s*dZ and per-64-row partial sums for db
-//   adam         Adam (§5.1) on W and b, refreshing the bf16 copy of W
+//                operand s*dZ and per-32-row partial sums for db
+//   adam         Adam (§5.1) on W and b, refreshing the bf16 copy of W, and
+//                dropping the step's dead data (dW, s*dZ) from L2
 //   init         He-uniform W from a counter-based SplitMix64 stream
 //   predict      label columns of W1, per-label expansion of layer 1,
 //                argmax over the 10 labels (§3 "Prediction"), and over
@@ -177,9 +178,10 @@ struct Vec8<float> {
 
 // Train-step epilogue of the forward GEMM, one block per 32 rows x 256
 // columns (block 32 x 8).  Thread (x, y) owns columns 8x..8x+7 of rows
-// y, y+8, y+16, y+24: it issues those activity loads first; meanwhile lanes
-// 0..3 of its warp reduce the per-tile goodness partials of the warp's four
-// rows and form dL/dg, broadcast to the warp by shuffles.  Then
+// y, y+8, y+16, y+24: it issues those activity loads first; meanwhile the
+// warp's lanes, 8 per row, reduce the per-tile goodness partials of its four
+// rows and lanes 0, 8, 16, 24 form dL/dg, broadcast to the warp by shuffles.
+// Then
 //   dZ'_ij = s_i * 2 dL/dg_i * h_ij (h = 0 where z <= 0) in the operand type,
 //   and the block's column sums of dZ for db.
 // Blocks of column 0 also write g, the next layer's scale
