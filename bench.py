@@ -296,11 +296,20 @@ def run_ours(args):
         cstream = torch.cuda.Stream(device=dev)
         loss_h = torch.empty(len(layers), pin_memory=True)
 
-        def epoch_e2e():
-            def fetch(t):
-                start, b = bl[t]
+        nb = len(bl)
+
+        def run_e2e(n_epochs):
+            # the epochs' batches as one stream: batch g of the run is copied
+            # into ring slot g % RING on the copy stream, RING - 1 batches
+            # ahead of the step that reads it (across epoch boundaries too, as
+            # a data loader would); each epoch ends with the net synced and
+            # its loss read back to the host
+            total = n_epochs * nb
+
+            def fetch(g):
+                start, b = bl[g % nb]
                 r0 = 2 * start
-                j = t % RING
+                j = g % RING
                 with torch.cuda.stream(cstream):
                     cstream.wait_event(freed[j])      # the step that last read slot j is past layer 1
                     xbuf[j][:2 * b].copy_(Xp[r0:r0 + 2 * b], non_blocking=True)
@@ -308,29 +317,31 @@ def run_ours(args):
                     copied[j].record(cstream)
             begin = torch.cuda.Event()
             begin.record(stream)
-            cstream.wait_event(begin)             # no copy starts before the step does
-            for t in range(min(RING - 1, len(bl))):
-                fetch(t)
-            for t, (start, b) in enumerate(bl):
-                if t + RING - 1 < len(bl):
-                    fetch(t + RING - 1)
-                j = t % RING
+            cstream.wait_event(begin)             # no copy starts before the run does
+            for g in range(min(RING - 1, total)):
+                fetch(g)
+            for g in range(total):
+                if g + RING - 1 < total:
+                    fetch(g + RING - 1)
+                t = g % nb
+                start, b = bl[t]
+                j = g % RING
                 stream.wait_event(copied[j])
                 net.train_step(xbuf[j][:2 * b], lbuf[j][:2 * b], B=b, loss=loss[t], stream=stream)
                 freed[j].record(stream)  # ff_net_train_step returns with `stream` ordered after layer 1 read x
-            net.sync(stream)
-            loss_h.copy_(loss[-1], non_blocking=True)
+                if t == nb - 1:
+                    net.sync(stream)
+                    loss_h.copy_(loss[-1], non_blocking=True)
 
         for j in range(RING):
             freed[j].record(stream)
         with torch.cuda.stream(stream):
-            epoch_e2e()
+            run_e2e(1)
         barrier()
         e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
         with torch.cuda.stream(stream):
             e0.record(stream)
-            for _ in range(args.steps):
-                epoch_e2e()
+            run_e2e(args.steps)
             e1.record(stream)
         barrier()
         e2e_value, ems = replica_throughput(e0.elapsed_time(e1), PAIRS_PER_EPOCH * args.steps, world, dist)
