@@ -54,11 +54,6 @@ struct Segs {
   int F_total;
 };
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-  return v;
-}
 
 // h[0..W) = H[row, f .. f+W) as float, zero past the segment or the rows.
 template <typename T, int W>
@@ -462,42 +457,6 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
 // V (before this step's update) and dz are staged in shared memory.  Lead
 // blocks (x == 0) also write the next layer's row scale from the forward's
 // goodness partials; block (0, 0) advances the layer's Adam step.
-template <typename T>
-struct V8;
-template <>
-struct V8<bf16> {
-  static __device__ __forceinline__ void load(const bf16* p, float (&v)[8]) {
-    const uint4 u = *reinterpret_cast<const uint4*>(p);
-    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-    for (int e = 0; e < 4; ++e) {
-      const float2 f = __bfloat1622float2(h[e]);
-      v[2 * e] = f.x;
-      v[2 * e + 1] = f.y;
-    }
-  }
-  static __device__ __forceinline__ void store(bf16* p, const float (&v)[8]) {
-    uint4 u;
-    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
-#pragma unroll
-    for (int e = 0; e < 4; ++e) h[e] = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
-    *reinterpret_cast<uint4*>(p) = u;
-  }
-};
-template <>
-struct V8<float> {
-  static __device__ __forceinline__ void load(const float* p, float (&v)[8]) {
-    const float4 a = *reinterpret_cast<const float4*>(p);
-    const float4 b = *reinterpret_cast<const float4*>(p + 4);
-    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
-    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
-  }
-  static __device__ __forceinline__ void store(float* p, const float (&v)[8]) {
-    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
-    *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
-  }
-};
-
 struct PoGradArgs {
   const float* dz;      // [n, 10]
   const float* V;       // [10, N] (before this step's update)
@@ -561,12 +520,12 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     const int i = r0 + li;
     float h[8], z[8];
     if (cols_ok && i < a.n) {
-      V8<T>::load(H + (size_t)i * a.ld + cg, h);
+      Vec8<T>::load(H + (size_t)i * a.ld + cg, h);
     } else {
 #pragma unroll
       for (int e = 0; e < 8; ++e) h[e] = 0.f;
     }
-    V8<T>::store(&Hs[li][lane * 8], h);
+    Vec8<T>::store(&Hs[li][lane * 8], h);
     if (!cols_ok || i >= a.n) continue;
     const float si = __ldg(a.s + i);
 #pragma unroll
@@ -578,7 +537,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
       db[e] += d;
       z[e] = si * d;
     }
-    V8<T>::store(G + (size_t)i * a.ld + cg, z);
+    Vec8<T>::store(G + (size_t)i * a.ld + cg, z);
   }
   __syncthreads();
   // dV partials from the staged tile: thread (x, y) sums classes y and
@@ -591,7 +550,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     for (int li = 0; li < kPoRows; ++li) {
       const float d = dzs[li][c];
       float h[8];
-      V8<T>::load(&Hs[li][lane * 8], h);
+      Vec8<T>::load(&Hs[li][lane * 8], h);
 #pragma unroll
       for (int e = 0; e < 8; ++e) dv[e] = fmaf(d, h[e], dv[e]);
     }
@@ -602,7 +561,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   __syncthreads();
   // db partials: the eight row groups added in order, through the tile's memory
   float (*red)[256 + 4] = reinterpret_cast<float (*)[256 + 4]>(&Hs[0][0]);
-  V8<float>::store(&red[threadIdx.y][lane * 8], db);
+  Vec8<float>::store(&red[threadIdx.y][lane * 8], db);
   __syncthreads();
   if (threadIdx.y == 0) {
 #pragma unroll
@@ -630,12 +589,6 @@ struct HeadAdamArgs {
   float* dc_out;        // [10] or null
 };
 
-__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float a1, float b1, float b2, float eps,
-                                      float r2) {
-  m = b1 * m + (1.f - b1) * g;
-  v = b2 * v + (1.f - b2) * g * g;
-  w -= a1 * m / (sqrtf(v * r2) + eps);
-}
 
 // Threads 0 .. 10F-1 of the grid own one V element each; the last block owns
 // the 10 biases (warp w: columns w and w + 8 of the partials, column 10 being

@@ -55,6 +55,63 @@ __device__ __forceinline__ float sum_partials(const float* __restrict__ gpart, i
   return g;
 }
 
+// Device helpers shared by the kernel files.
+__device__ __forceinline__ float warp_sum(float v) {
+#pragma unroll
+  for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+  return v;
+}
+
+// Eight consecutive values of an activity row (16 bytes of bf16 or 32 of
+// fp32) as floats, and back (bf16: round to nearest even).
+template <typename T>
+struct Vec8;
+template <>
+struct Vec8<bf16> {
+  static __device__ __forceinline__ void load(const bf16* p, float (&v)[8]) {
+    const uint4 u = *reinterpret_cast<const uint4*>(p);
+    const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) {
+      const float2 f = __bfloat1622float2(h[e]);
+      v[2 * e] = f.x;
+      v[2 * e + 1] = f.y;
+    }
+  }
+  static __device__ __forceinline__ void store(bf16* p, const float (&v)[8]) {
+    uint4 u;
+    __nv_bfloat162* h = reinterpret_cast<__nv_bfloat162*>(&u);
+#pragma unroll
+    for (int e = 0; e < 4; ++e) h[e] = __floats2bfloat162_rn(v[2 * e], v[2 * e + 1]);
+    *reinterpret_cast<uint4*>(p) = u;
+  }
+};
+template <>
+struct Vec8<float> {
+  static __device__ __forceinline__ void load(const float* p, float (&v)[8]) {
+    const float4 a = *reinterpret_cast<const float4*>(p);
+    const float4 b = *reinterpret_cast<const float4*>(p + 4);
+    v[0] = a.x; v[1] = a.y; v[2] = a.z; v[3] = a.w;
+    v[4] = b.x; v[5] = b.y; v[6] = b.z; v[7] = b.w;
+  }
+  static __device__ __forceinline__ void store(float* p, const float (&v)[8]) {
+    *reinterpret_cast<float4*>(p) = make_float4(v[0], v[1], v[2], v[3]);
+    *reinterpret_cast<float4*>(p + 4) = make_float4(v[4], v[5], v[6], v[7]);
+  }
+};
+
+// One Adam step of one parameter.  a1 = lr / (1 - beta1^t) and
+// r2 = 1 / (1 - beta2^t) are formed once per thread, so the update
+// lr * (m / bc1) / (sqrt(v / bc2) + eps) costs one division per parameter
+// instead of three (the kernel is otherwise limited by those divisions, not
+// by HBM).
+__device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float a1, float b1, float b2, float eps,
+                                      float r2) {
+  m = b1 * m + (1.f - b1) * g;
+  v = b2 * v + (1.f - b2) * g * g;
+  w -= a1 * m / (sqrtf(v * r2) + eps);
+}
+
 // Bound on every spin-wait in a kernel: after this many nanoseconds of
 // %globaltimer the wait gives up, latches DEVERR_TIMEOUT and the kernel
 // winds down.
