@@ -33,21 +33,6 @@ __device__ __forceinline__ bf16 from_f<bf16>(float v) { return __float2bfloat16_
 __device__ __forceinline__ float to_f(float v) { return v; }
 __device__ __forceinline__ float to_f(bf16 v) { return __bfloat162float(v); }
 
-
-// Fixed-order block sum for blockDim.x == 256; result valid in thread 0.
-__device__ __forceinline__ float block_sum_256(float v, float* red /*[8]*/) {
-  v = warp_sum(v);
-  if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = v;
-  __syncthreads();
-  float t = 0.f;
-  if (threadIdx.x == 0) {
-#pragma unroll
-    for (int w = 0; w < 8; ++w) t += red[w];
-  }
-  __syncthreads();
-  return t;
-}
-
 // ------------------------------------------------------------------ overlay
 template <typename T>
 __device__ __forceinline__ void store4(T* p, float a, float b, float c, float d);
