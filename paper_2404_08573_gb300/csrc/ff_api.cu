@@ -57,7 +57,7 @@ static size_t align256(size_t b) { return (b + 255) & ~(size_t)255; }
 
 // goodness partials per row: the most either forward GEMM writes
 static int gpart_tiles_max(int N) {
-  const int a = tc_fwd_ntiles(N), b = simt_fwd_ntiles(N);
+  const int a = tc_fwd_ntiles_max(N), b = simt_fwd_ntiles(N);
   return a > b ? a : b;
 }
 
@@ -200,7 +200,7 @@ static ff_status forward_core(ff_layer* L, const void* x, const int* labels, con
   EpiArgs ep{s, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
   int ntiles;
   if (L->is_bf16) {
-    ntiles = tc_fwd_ntiles(N);
+    ntiles = tc_fwd_ntiles(M, N, false);
     FF_LAUNCH(K_FWD_TC, 2.0 * M * N * K, st,
               tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, M, N, K, ep, &L->ds->err, st),
               "forward GEMM (tcgen05)");
@@ -494,7 +494,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   int ldmax = 0, ntmax = 0;
   for (int k = 0; k < n_layers; ++k) {
     if (layers[k]->ldN > ldmax) ldmax = layers[k]->ldN;
-    const int nt = b16 ? tc_fwd_ntiles(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
+    const int nt = b16 ? tc_fwd_ntiles_max(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
     if (nt > ntmax) ntmax = nt;
   }
   // Samples per chunk: about 40 MB of activations per buffer, so that one
@@ -515,7 +515,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
       double best = -1.0;
       int bestC = C;
       for (int c = C; c >= C / 2 && c >= 64; --c) {
-        const int ctas = tc_gemm_fwd_ctas(10 * c, Nw);
+        const int ctas = tc_gemm_fwd_ctas(10 * c, Nw, true);
         const double eff = (double)ctas / ((double)cdiv(ctas, sms) * sms);
         if (eff > best + 1e-9) {
           best = eff;
@@ -595,6 +595,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
       ff_layer* Lk = layers[k];
       float* gpart = gpb[k & 1];
       EpiArgs ep{Sb[cur], Lk->cfg.has_bias ? Lk->b : nullptr, Hb[cur ^ 1], Lk->ldN, gpart};
+      ep.narrow = true;
       int nt;
       if (b16) {
         if (k >= 2) {
@@ -605,7 +606,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
           ep.ntiles_in = nt_prev;
           ep.G_acc = Gc;
         }
-        nt = tc_fwd_ntiles(Lk->N);
+        nt = tc_fwd_ntiles(rows, Lk->N, true);
         FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
                   tc_gemm_fwd(static_cast<const bf16*>(Hb[cur]), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep,
                               err, st),

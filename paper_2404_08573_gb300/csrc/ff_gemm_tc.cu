@@ -500,16 +500,23 @@ constexpr int WGRAD_BN = 256;
 constexpr bool USE_PAIR = true;
 constexpr int NSTAGES = 3;       // operand ring depth
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
-constexpr int B_BOX_ROWS = USE_PAIR ? FWD_BN / 2 : FWD_BN;
+constexpr int CLUSTER_M = USE_PAIR ? 2 : 1;
 // A GEMM that would get fewer than kSmallGridCtas CTAs with two subtiles per
-// CTA (at most a third of the GPU, e.g. 1024 batch rows of a 2000-wide
+// CTA (at most a third of the GPU, e.g. 1216 batch rows of a 2000-wide
 // layer) runs with one subtile per CTA instead: twice the CTAs, each with a
-// 6-stage ring of 32 KB stages.
+// 6-stage ring of 32 KB stages.  One whose one-subtile grid still fills at
+// most half the SMs (1024 rows of a 2000-wide layer: 64 CTAs) also halves
+// the tile width to 128 columns (128 CTAs, 8-stage ring of 24 KB stages).
 constexpr int kSmallGridCtas = 64;
 constexpr int NSTAGES_SMALL = 6;
-bool small_grid(int M, int N, int bn) {
-  constexpr int CM = USE_PAIR ? 2 : 1;
-  return (long long)cdiv(cdiv(M, BM * ROW_SUBTILES), CM) * CM * cdiv(N, bn) < kSmallGridCtas;
+constexpr int TINY_BN = 128;
+constexpr int kTinyGridCtas = 152 / 2;
+constexpr int NSTAGES_TINY = 8;
+enum Shape { SHAPE_FULL, SHAPE_SMALL, SHAPE_TINY };
+int grid_ctas(int M, int N, int mt, int bn) { return cdiv(cdiv(M, BM * mt), CLUSTER_M) * CLUSTER_M * cdiv(N, bn); }
+Shape shape_of(int M, int N, int bn) {
+  if (grid_ctas(M, N, ROW_SUBTILES, bn) >= kSmallGridCtas) return SHAPE_FULL;
+  return grid_ctas(M, N, 1, bn) > kTinyGridCtas ? SHAPE_SMALL : SHAPE_TINY;
 }
 
 }  // namespace
@@ -526,21 +533,35 @@ bool tc_supported() {
   return major == 10 && encode_fn() != nullptr;
 }
 
-int tc_fwd_ntiles(int N) { return cdiv(N, FWD_BN) * (EPI_WARPS / 4); }  // goodness partials per row
-
-int tc_gemm_fwd_ctas(int M, int N) {
-  constexpr int CM = USE_PAIR ? 2 : 1;
-  const int mt = small_grid(M, N, FWD_BN) ? 1 : ROW_SUBTILES;
-  return cdiv(cdiv(M, BM * mt), CM) * CM * cdiv(N, FWD_BN);
+// goodness partials per row: one per epilogue warp's column half of each column tile
+int tc_fwd_ntiles(int M, int N, bool narrow) {
+  return cdiv(N, narrow && shape_of(M, N, FWD_BN) == SHAPE_TINY ? TINY_BN : FWD_BN) * (EPI_WARPS / 4);
 }
+int tc_fwd_ntiles_max(int N) { return cdiv(N, TINY_BN) * (EPI_WARPS / 4); }
+
+int tc_gemm_fwd_ctas(int M, int N, bool narrow) {
+  switch (shape_of(M, N, FWD_BN)) {
+    case SHAPE_FULL: return grid_ctas(M, N, ROW_SUBTILES, FWD_BN);
+    case SHAPE_SMALL: return grid_ctas(M, N, 1, FWD_BN);
+    default: return grid_ctas(M, N, 1, narrow ? TINY_BN : FWD_BN);
+  }
+}
+
+// B (the weights, [N, K]) is loaded per CTA in boxes of the CTA's share of a tile's columns.
+static constexpr int b_box_rows(int bn) { return USE_PAIR ? bn / 2 : bn; }
 
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
                         int* err, cudaStream_t st) {
+  Shape sh = shape_of(M, N, FWD_BN);
+  if (sh == SHAPE_TINY && !ep.narrow) sh = SHAPE_SMALL;
+  const int bn = sh == SHAPE_TINY ? TINY_BN : FWD_BN;
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, B_BOX_ROWS) ||
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(bn)) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
-  if (small_grid(M, N, FWD_BN))
+  if (sh == SHAPE_TINY)
+    return launch_tc<TINY_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_TINY, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
+  if (sh == SHAPE_SMALL)
     return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
   return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
 }
@@ -554,12 +575,12 @@ static bool store_map(CUtensorMap* tc, float* C, int ldc, int rows, int cols) {
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, float* Cm,
                           int ldc, int* err, cudaStream_t st) {
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, B_BOX_ROWS))
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(FWD_BN)))
     return cudaErrorInvalidValue;
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  if (small_grid(M, N, FWD_BN))
+  if (shape_of(M, N, FWD_BN) != SHAPE_FULL)
     return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, M, N, K, ep, err,
                                                                                    st);
   return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
@@ -575,7 +596,7 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  if (small_grid(N, K, WGRAD_BN))
+  if (shape_of(N, K, WGRAD_BN) != SHAPE_FULL)
     return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, N, K, R, ep, err,
                                                                                    st);
   return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);

@@ -694,7 +694,7 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   const size_t es = b16 ? 2 : 4;
   int ntmax = 0;
   for (int k = 0; k < L; ++k) {
-    const int nt = b16 ? tc_fwd_ntiles(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
+    const int nt = b16 ? tc_fwd_ntiles_max(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
     if (nt > ntmax) ntmax = nt;
   }
   size_t off = 0;
@@ -747,6 +747,7 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
     ff_layer* Lk = layers[k];
     float* gpart = b16 && (k & 1) ? w.gpart2 : w.gpart;
     EpiArgs ep{w.S[k], Lk->cfg.has_bias ? Lk->b : nullptr, w.Hk[k], Lk->ldN, gpart};
+    ep.narrow = true;
     int nt;
     if (b16) {
       if (k >= 1) {
@@ -757,7 +758,7 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
         ep.ntiles_in = nt_prev;
         ep.s_out = w.S[k];
       }
-      nt = tc_fwd_ntiles(Lk->N);
+      nt = tc_fwd_ntiles(rows, Lk->N, true);
       FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
                 tc_gemm_fwd(static_cast<const bf16*>(in), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep, err, st),
                 "head forward GEMM (tcgen05)");
@@ -1180,7 +1181,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   EpiArgs ep{sc, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
   int ntiles;
   if (b16) {
-    ntiles = tc_fwd_ntiles(N);
+    ntiles = tc_fwd_ntiles(n, N, false);
     FF_LAUNCH(K_FWD_TC, 2.0 * n * N * K, st,
               tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, n, N, K, ep, &L->ds->err, st),
               "forward GEMM (tcgen05)");

@@ -234,12 +234,21 @@ struct EpiArgs {
   size_t kpart_cap;
   int* kcnt;
   int kcnt_cap;
+  // Tensor-core forward GEMMs: a grid that would fill at most half the SMs
+  // may use 128-column tiles (twice the CTAs).  Set where the GEMM has the
+  // GPU to itself (the layer chains of predict and of the softmax head); the
+  // net's concurrent per-layer GEMMs run faster on the wider tiles.
+  bool narrow;
 };
 
 // Tensor-core (tcgen05) bf16 GEMMs, fp32 accumulate.
 //   fwd/store: C[M,N] = A[M,K] B[N,K]^T  (A, B row-major, K contiguous)
 //   wgrad:     C[N,K] = G[R,N]^T X[R,K]  (contraction over R rows)
-int tc_fwd_ntiles(int N);
+// Goodness partials per row the forward GEMM writes for an M x N output (its
+// tile shape depends on both and on EpiArgs::narrow), and the most it writes
+// for any M.
+int tc_fwd_ntiles(int M, int N, bool narrow);
+int tc_fwd_ntiles_max(int N);
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
                         const EpiArgs& ep, int* err, cudaStream_t st);
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
@@ -248,7 +257,7 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
                           float* C, int ldc, int* err, cudaStream_t st);
 bool tc_supported();
 // CTAs of the forward GEMM for an M x N output (its tile configuration).
-int tc_gemm_fwd_ctas(int M, int N);
+int tc_gemm_fwd_ctas(int M, int N, bool narrow);
 // Tensor map of a row-major [rows, cols] bf16 (esize 2) or fp32 (esize 4)
 // matrix with row stride ld, boxes of box_rows x box_cols, no swizzle; false
 // if the pointer or the stride is not 16-byte aligned.

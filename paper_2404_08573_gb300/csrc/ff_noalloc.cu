@@ -55,7 +55,7 @@ extern "C" FF_API ff_status ff_forward_noalloc(const void* x, const float* row_s
   if (rows < 0 || in_features < 1 || out_features < 1) return FF_ERR_INVALID_ARG;
   if (rows == 0) return FF_OK;
   if (!x || !row_scale || !W_bf16 || !h_out) return FF_ERR_INVALID_ARG;
-  const size_t partials = (size_t)tc_fwd_ntiles(out_features) * (size_t)rows;
+  const size_t partials = (size_t)tc_fwd_ntiles(rows, out_features, false) * (size_t)rows;
   if (partials > kNoAllocScratchFloats - kNoAllocPartialOffset) return FF_ERR_INVALID_ARG;
   if (!tc_supported()) return FF_ERR_UNSUPPORTED;
   float* scratch = nullptr;
@@ -75,7 +75,7 @@ extern "C" FF_API ff_status ff_forward_noalloc(const void* x, const float* row_s
   if (e != cudaSuccess) return FF_ERR_CUDA;
   FinalizeArgs fa{};
   fa.gpart = gpart;
-  fa.ntiles = tc_fwd_ntiles(out_features);
+  fa.ntiles = tc_fwd_ntiles(rows, out_features, false);
   fa.M = rows;
   fa.g_out = goodness;
   fa.s_next = next_scale;

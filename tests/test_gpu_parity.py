@@ -75,6 +75,9 @@ def test_overlay_kernel(env, prec):
 FWD_CASES = [
     ("fp32", 300, 784, 600), ("bf16", 300, 784, 600), ("bf16", 1, 11, 5), ("fp32", 1, 11, 5),
     ("bf16", 130, 2003, 777), ("fp32", 130, 2003, 777), ("bf16", 257, 64, 256), ("bf16", 2048, 2000, 2000),
+    # the bf16 GEMM's three tile shapes: 128-column tiles (at most 76 CTAs of
+    # one 128-row subtile each), 256-column tiles of one subtile, of two
+    ("bf16", 1024, 300, 2000), ("bf16", 1216, 300, 2000),
 ]
 
 
