@@ -109,6 +109,7 @@ __device__ __forceinline__ float sigmoid_f(float t) {
 }
 
 __global__ void __launch_bounds__(256) k_finalize(FinalizeArgs a) {
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   const int i = blockIdx.x * 256 + threadIdx.x;
   if (i >= a.M) return;
   const float g = sum_partials(a.gpart, a.ntiles, a.M, i);
@@ -553,28 +554,11 @@ int finalize_grid(int M) { return cdiv(M, 256); }
 
 cudaError_t launch_finalize(const FinalizeArgs& a, cudaStream_t st) {
   if (a.M <= 0) return cudaSuccess;
-  k_finalize<<<finalize_grid(a.M), 256, 0, st>>>(a);
-  return cudaGetLastError();
+  PdlLaunch l(dim3(finalize_grid(a.M)), dim3(256), st);
+  return cudaLaunchKernelEx(&l.cfg, k_finalize, a);
 }
 
 int local_grad_row_blocks(int M) { return cdiv(M, kGradRows); }
-
-// Launch configuration with programmatic stream serialization: the kernel
-// may start while the previous kernel of the stream finishes and waits for it
-// with griddep_wait() before touching memory.
-struct PdlLaunch {
-  cudaLaunchConfig_t cfg = {};
-  cudaLaunchAttribute attr[1];
-  PdlLaunch(dim3 grid, dim3 block, cudaStream_t st) {
-    cfg.gridDim = grid;
-    cfg.blockDim = block;
-    cfg.stream = st;
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[0].val.programmaticStreamSerializationAllowed = 1;
-    cfg.attrs = attr;
-    cfg.numAttrs = 1;
-  }
-};
 
 cudaError_t launch_grad_prep(const GradPrepArgs& a, bool b16, const void* H, void* dZ, cudaStream_t st) {
   PdlLaunch l(dim3(cdiv(a.ld, 256), local_grad_row_blocks(a.M)), dim3(32, 8), st);

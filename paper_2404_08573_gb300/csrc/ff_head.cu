@@ -224,6 +224,7 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
     ptx::prefetch_tmap(map);
   }
   __syncthreads();
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   if (threadIdx.x == 0) {
     for (; issued < kDotStages && issued < nch; ++issued) {
       if (!ff_dcheck(tma_x_aligned(fs + issued * CH, (int)sizeof(T)), err)) {
@@ -362,10 +363,21 @@ __global__ void __launch_bounds__(256, 1) k_head_dot(const __grid_constant__ Hea
     float z[kClasses];
 #pragma unroll
     for (int c = 0; c < kClasses; ++c) z[c] = __ldg(fa.cb + c);
-    for (int sp = 0; sp < fa.S; ++sp) {
-      const float* zp = zpart + ((size_t)sp * n + row) * kClasses;
+    // four splits' loads in flight at a time, added in split order
+    for (int sp0 = 0; sp0 < fa.S; sp0 += 4) {
+      float t[4][kClasses];
 #pragma unroll
-      for (int c = 0; c < kClasses; ++c) z[c] += __ldcg(zp + c);
+      for (int u = 0; u < 4; ++u) {
+        const float* zp = zpart + ((size_t)(sp0 + u) * n + row) * kClasses;
+#pragma unroll
+        for (int c = 0; c < kClasses; ++c) t[u][c] = sp0 + u < fa.S ? __ldcg(zp + c) : 0.f;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u)
+        if (sp0 + u < fa.S) {
+#pragma unroll
+          for (int c = 0; c < kClasses; ++c) z[c] += t[u][c];
+        }
     }
     loss = finish_row(z, row, fa.labels, fa.inv_n, fa.logits, fa.dz, dzr, err);
   }
@@ -397,6 +409,7 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
                                                     float* __restrict__ dVpart) {
   __shared__ float dzs[kWgRows][kClasses];
   __shared__ float red[8][kClasses][kWgChunk];
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   // segment and chunk of this block
   int k = 0, chunk = blockIdx.x;
@@ -485,6 +498,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   const int lane = threadIdx.x, tid = threadIdx.y * 32 + threadIdx.x;
   const int c0 = blockIdx.x * 256;
   const int cg = c0 + lane * 8;
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   for (int idx = tid; idx < kClasses * 256; idx += 256) {
     const int c = idx / 256, j = idx % 256;
     Vsh[c][j % 8][j / 8] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
@@ -494,8 +508,7 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     dzs[i][c] = (r0 + i < a.n) ? __ldg(a.dz + (size_t)(r0 + i) * kClasses + c) : 0.f;
   }
   if (blockIdx.x == 0 && tid < kPoRows && r0 + tid < a.n) {
-    float g = 0.f;
-    for (int t = 0; t < a.ntiles; ++t) g += __ldg(a.gpart + (size_t)t * a.n + r0 + tid);
+    const float g = sum_partials(a.gpart, a.ntiles, a.n, r0 + tid);
     if (!isfinite(g)) atomicOr(a.err, DEVERR_NONFINITE);
     if (a.s_next) {
       const float r = sqrtf(g);
@@ -594,14 +607,15 @@ struct HeadAdamArgs {
 // the 10 biases (warp w: columns w and w + 8 of the partials, column 10 being
 // the loss).
 __global__ void __launch_bounds__(256) k_head_adam(HeadAdamArgs a) {
+  ptx::griddep_wait();  // launched with programmatic stream serialization
   const float a1 = a.lr / a.ds->bc1, r2 = 1.f / a.ds->bc2;
   const int total = kClasses * a.F;
   const int vblocks = (total + 255) / 256;
   if ((int)blockIdx.x < vblocks) {
     const int idx = blockIdx.x * 256 + threadIdx.x;
     if (idx >= total) return;
-    float g = 0.f;
-    for (int rb = 0; rb < a.nrb; ++rb) g += __ldg(a.dVpart + (size_t)rb * total + idx);
+    // the row blocks' partials in order, eight loads in flight
+    const float g = sum_partials(a.dVpart, a.nrb, total, idx);
     if (a.dV_out) a.dV_out[idx] = g;
     float w = a.V[idx], m = a.mV[idx], v = a.vV[idx];
     adam1(w, m, v, g, a1, a.beta1, a.beta2, a.eps, r2);
@@ -847,11 +861,10 @@ ff_status head_logits(ff_head* hd, const Segs& sg, bool b16, int n, const int* l
                                                          cudaFuncAttributeMaxDynamicSharedMemorySize, kDotSmem);
   FF_TRY(b16 ? attr_b : attr_f, "head kernel attributes");
   dim3 grid(S, cdiv(n, kDotRows));
+  PdlLaunch l(grid, dim3(256), st, kDotSmem);
   FF_LAUNCH(K_HEAD_LOGITS, (double)n * sg.F_total * es + (double)n * (2 * S + 2) * kClasses * 4, st,
-            (b16 ? (k_head_dot<bf16><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, fa, err),
-                    cudaGetLastError())
-                 : (k_head_dot<float><<<grid, 256, kDotSmem, st>>>(maps, sg, split, n, V, zpart, fa, err),
-                    cudaGetLastError())),
+            (b16 ? cudaLaunchKernelEx(&l.cfg, k_head_dot<bf16>, maps, sg, split, n, V, zpart, fa, err)
+                 : cudaLaunchKernelEx(&l.cfg, k_head_dot<float>, maps, sg, split, n, V, zpart, fa, err)),
             "head logits, softmax and cross-entropy");
   return FF_OK;
 }
@@ -859,12 +872,9 @@ ff_status head_logits(ff_head* hd, const Segs& sg, bool b16, int n, const int* l
 cudaError_t launch_head_wgrad(const Segs& sg, bool b16, int n, const float* dz, float* dVpart, cudaStream_t st) {
   int chunks = 0;
   for (int k = 0; k < sg.nseg; ++k) chunks += cdiv(sg.F[k], kWgChunk);
-  dim3 grid(chunks, cdiv(n, kWgRows));
-  if (b16)
-    k_head_wgrad<bf16><<<grid, 256, 0, st>>>(sg, n, dz, dVpart);
-  else
-    k_head_wgrad<float><<<grid, 256, 0, st>>>(sg, n, dz, dVpart);
-  return cudaGetLastError();
+  PdlLaunch l(dim3(chunks, cdiv(n, kWgRows)), dim3(256), st);
+  return b16 ? cudaLaunchKernelEx(&l.cfg, k_head_wgrad<bf16>, sg, n, dz, dVpart)
+             : cudaLaunchKernelEx(&l.cfg, k_head_wgrad<float>, sg, n, dz, dVpart);
 }
 
 }  // namespace
@@ -1029,8 +1039,9 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
             launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
   const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kDotRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
-  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st,
-            (k_head_adam<<<vblocks + 1, 256, 0, st>>>(a), cudaGetLastError()), "head Adam");
+  PdlLaunch l(dim3(vblocks + 1), dim3(256), st);
+  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st, cudaLaunchKernelEx(&l.cfg, k_head_adam, a),
+            "head Adam");
   return FF_OK;
 }
 
@@ -1219,13 +1230,12 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   pa.beta1 = L->cfg.beta1;
   pa.beta2 = L->cfg.beta2;
   pa.err = &L->ds->err;
-  dim3 grid(cdiv(L->ldN, 256), cdiv(n, kPoRows)), block(32, 8);
+  PdlLaunch pl(dim3(cdiv(L->ldN, 256), cdiv(n, kPoRows)), dim3(32, 8), st);
   FF_LAUNCH(K_GRAD_PREP, (double)n * L->ldN * es * 2 + (double)cdiv(n, kPoRows) * (kClasses + 1) * N * 4, st,
-            (b16 ? (k_po_grad<bf16><<<grid, block, 0, st>>>(pa, static_cast<const bf16*>(H), static_cast<bf16*>(L->dZ)),
-                    cudaGetLastError())
-                 : (k_po_grad<float><<<grid, block, 0, st>>>(pa, static_cast<const float*>(H),
-                                                            static_cast<float*>(L->dZ)),
-                    cudaGetLastError())),
+            (b16 ? cudaLaunchKernelEx(&pl.cfg, k_po_grad<bf16>, pa, static_cast<const bf16*>(H),
+                                      static_cast<bf16*>(L->dZ))
+                 : cudaLaunchKernelEx(&pl.cfg, k_po_grad<float>, pa, static_cast<const float*>(H),
+                                      static_cast<float*>(L->dZ))),
             "block gradient into the layer");
   if (b16) {
     FF_LAUNCH(K_WGRAD_TC, 2.0 * n * N * K, st,
@@ -1268,8 +1278,9 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
   const HeadAdamArgs ha = head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, kDotRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
+  PdlLaunch hl(dim3(vblocks + 1), dim3(256), st);
   FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), st,
-            (k_head_adam<<<vblocks + 1, 256, 0, st>>>(ha), cudaGetLastError()), "block Adam");
+            cudaLaunchKernelEx(&hl.cfg, k_head_adam, ha), "block Adam");
   return FF_OK;
 }
 

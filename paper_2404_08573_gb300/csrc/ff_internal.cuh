@@ -196,6 +196,25 @@ struct AdamArgs {
 // Adds [p, p + bytes) to the Adam step's dead buffers (its whole 128-byte
 // lines; nothing when p is not 128-byte aligned).
 void add_dead(AdamArgs& a, void* p, size_t bytes);
+
+// Launch configuration with programmatic stream serialization: the kernel
+// may start while the previous kernel of the stream finishes and waits for it
+// with griddep_wait() before touching memory.
+struct PdlLaunch {
+  cudaLaunchConfig_t cfg = {};
+  cudaLaunchAttribute attr[1];
+  PdlLaunch(dim3 grid, dim3 block, cudaStream_t st, size_t smem = 0) {
+    cfg.gridDim = grid;
+    cfg.blockDim = block;
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = st;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+  }
+};
+
 cudaError_t launch_adam(const AdamArgs& a, cudaStream_t st);
 cudaError_t launch_init_weights(float* W, int N, int K, unsigned long long seed, cudaStream_t st);
 cudaError_t launch_to_bf16(const float* W, int N, int K, bf16* Wb, int ldb, cudaStream_t st);
