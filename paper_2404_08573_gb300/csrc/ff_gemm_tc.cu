@@ -40,6 +40,9 @@ constexpr int EPI_WARPS = 8;                 // two per TMEM lane quarter, each 
 constexpr int NTHREADS = 64 + 32 * EPI_WARPS;  // producer warp, MMA warp, epilogue warps
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
+constexpr int MODE_FWD_LOGITS = 2;  // forward, plus partial logits of a 10-class block (EpiArgs::logit_V)
+constexpr int kLogitClasses = 10;
+constexpr int kLogitStride = 12;    // floats per column of the staged block weights (three float4)
 
 template <int BN, int NSTAGE, int MT, bool PAIR>
 struct TcCfg {
@@ -74,6 +77,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
   using C = TcCfg<BN, NSTAGE, MT, PAIR>;
+  constexpr bool FWD = MODE != MODE_STORE;
+  constexpr bool LOGITS = MODE == MODE_FWD_LOGITS;
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -87,6 +92,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tslot + 1);
   volatile int* never_set = reinterpret_cast<volatile int*>(tslot + 2);  // drain waits ignore the abort
   float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [BN] bias of this tile
+  float* sVt = sbias + BN;  // LOGITS: [BN][kLogitStride] block weights of this tile's columns
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -119,7 +125,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
-    if (MODE == MODE_FWD || tma_store) ptx::prefetch_tmap(&tmC);
+    if (FWD || tma_store) ptx::prefetch_tmap(&tmC);
   }
   if (warp == 1) {
     if constexpr (PAIR) {
@@ -272,11 +278,17 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     float srow[MT];
 #pragma unroll
     for (int mt = 0; mt < MT; ++mt) srow[mt] = 0.f;
-    if (MODE == MODE_FWD) {
+    if (FWD) {
       // While the mainloop runs: the tile's bias (zero past N or without bias)
       // into shared memory and this thread's row scales into registers.
       for (int c = (int)threadIdx.x - 64; c < BN; c += 32 * EPI_WARPS)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
+      if constexpr (LOGITS) {
+        for (int idx = (int)threadIdx.x - 64; idx < kLogitClasses * BN; idx += 32 * EPI_WARPS) {
+          const int c = idx / BN, j = idx % BN;
+          sVt[j * kLogitStride + c] = n0 + j < N ? __ldg(ep.logit_V + (size_t)c * ep.logit_ldV + n0 + j) : 0.f;
+        }
+      }
 #pragma unroll
       for (int mt = 0; mt < MT; ++mt) {
         const int gi = m0 + mt * BM + q * 32 + lane;
@@ -301,26 +313,29 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     ptx::tc_fence_after();
     // tcgen05.ld is warp-collective: decide for the whole warp at once
     if (__all_sync(0xffffffffu, ok && !*abort_flag)) {
-      constexpr int ES = MODE == MODE_FWD ? 2 : 4;      // staged element size
+      constexpr int ES = FWD ? 2 : 4;      // staged element size
       constexpr int CW = 128 / ES;                       // columns per 128-byte swizzle row
       const uint32_t sw = (uint32_t)(lane & 7);
-      const bool staged = MODE == MODE_FWD || tma_store;
+      const bool staged = FWD || tma_store;
       int fchunk = 0;  // fp32 chunks streamed so far (slot parity)
 #pragma unroll 1
       for (int mt = 0; mt < MT; ++mt) {
         const int rbase = m0 + mt * BM + q * 32;  // this warp's first row in subtile mt
         const int gi = rbase + lane;
         // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
-        uint8_t* stage = smem + (MODE == MODE_FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
+        uint8_t* stage = smem + (FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
         const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS + cbase);
         const float s = srow[mt];
         float g = 0.f;
+        float zl[kLogitClasses];  // LOGITS: this row's partial logits over the warp's columns
+#pragma unroll
+        for (int c = 0; c < kLogitClasses; ++c) zl[c] = 0.f;
         // Columns past N and rows past M hold zero products (their operand rows
         // were zero-filled); the TMA store clips them and gpart skips them.
         // c0 counts columns within this warp's half.
         auto process = [&](const uint32_t (&r)[32], int c0) {
           const int col0 = n0 + cbase + c0;
-          if (MODE == MODE_FWD) {
+          if (FWD) {
             uint32_t packed[16];
             const float4* b4 = reinterpret_cast<const float4*>(sbias + cbase + c0);
 #pragma unroll
@@ -338,6 +353,19 @@ __global__ void __launch_bounds__(NTHREADS, 2)
               __nv_bfloat162 p1 = __floats2bfloat162_rn(h[2], h[3]);
               packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
               packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
+              if constexpr (LOGITS) {
+                // the block reads the stored (bf16-rounded) activity
+                const float2 lo = __bfloat1622float2(p0), hi = __bfloat1622float2(p1);
+                const float hr[4] = {lo.x, lo.y, hi.x, hi.y};
+#pragma unroll
+                for (int e = 0; e < 4; ++e) {
+                  const float4* vt = reinterpret_cast<const float4*>(sVt + (cbase + c0 + 4 * v + e) * kLogitStride);
+                  const float4 v0 = vt[0], v1 = vt[1], v2 = vt[2];
+                  const float vv[kLogitClasses] = {v0.x, v0.y, v0.z, v0.w, v1.x, v1.y, v1.z, v1.w, v2.x, v2.y};
+#pragma unroll
+                  for (int c = 0; c < kLogitClasses; ++c) zl[c] = fmaf(hr[e], vv[c], zl[c]);
+                }
+              }
             }
             uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
 #pragma unroll
@@ -384,8 +412,13 @@ __global__ void __launch_bounds__(NTHREADS, 2)
           process(rb, c0 + 32);
           ptx::tmem_ld_wait();
         }
-        if (MODE == MODE_FWD && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
-        if (MODE == MODE_FWD) {
+        if (FWD && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
+        if (LOGITS && gi < M) {
+          float2* zp = reinterpret_cast<float2*>(ep.zpart + ((size_t)(blockIdx.y * HALVES + half) * M + gi) * kLogitClasses);
+#pragma unroll
+          for (int c = 0; c < kLogitClasses; c += 2) zp[c / 2] = make_float2(zl[c], zl[c + 1]);
+        }
+        if (FWD) {
           ptx::fence_async_smem();
           __syncwarp();
           if (lane == 0 && rbase < M) {
@@ -460,8 +493,10 @@ template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st) {
   using C = TcCfg<BN, NSTAGE, MT, PAIR>;
+  constexpr int SMEM = C::SMEM + (MODE == MODE_FWD_LOGITS ? BN * kLogitStride * 4 : 0);
+  static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
   auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT>;
-  static cudaError_t attr = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, C::SMEM);
+  static cudaError_t attr = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
   if (attr != cudaSuccess) return attr;
   cudaLaunchConfig_t cfg = {};
   // tile rows padded to whole pairs; a padding CTA loads zeros, supplies its
@@ -469,7 +504,7 @@ cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtens
   constexpr int CM = PAIR ? 2 : 1;
   cfg.gridDim = dim3(cdiv(cdiv(M, BM * MT), CM) * CM, cdiv(N, BN), 1);
   cfg.blockDim = dim3(NTHREADS, 1, 1);
-  cfg.dynamicSmemBytes = C::SMEM;
+  cfg.dynamicSmemBytes = SMEM;
   cfg.stream = st;
   cudaLaunchAttribute at[2];
   at[0].id = cudaLaunchAttributeClusterDimension;
@@ -559,6 +594,15 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
   if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(bn)) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
+  if (ep.logit_V) {
+    // the Performance-Optimized step's forward (never narrowed)
+    if (!ep.zpart || ep.logit_ldV < N || ep.narrow) return cudaErrorInvalidValue;
+    if (sh == SHAPE_FULL)
+      return launch_tc<FWD_BN, false, false, MODE_FWD_LOGITS, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K,
+                                                                                               ep, err, st);
+    return launch_tc<FWD_BN, false, false, MODE_FWD_LOGITS, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, 1, M, N, K, ep, err,
+                                                                                        st);
+  }
   if (sh == SHAPE_TINY)
     return launch_tc<TINY_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_TINY, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
   if (sh == SHAPE_SMALL)

@@ -20,6 +20,7 @@
 //   k_head_wgrad   dV partials per 128-row block: dz^T (s_k H_k)
 //   k_head_adam    reduces the partials in a fixed order, Adam on V and c,
 //                  the step's loss
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <new>
@@ -470,8 +471,21 @@ __global__ void __launch_bounds__(256) k_head_wgrad(Segs sg, int n, const float*
 // V (before this step's update) and dz are staged in shared memory.  Lead
 // blocks (x == 0) also write the next layer's row scale from the forward's
 // goodness partials; block (0, 0) advances the layer's Adam step.
+// With zpart set (bf16 layers), dz is not given: the forward GEMM wrote the
+// block's partial logits, and every block finishes its own rows from them
+// (bias + partials in tile order, softmax, cross-entropy; the blocks of a row
+// block compute identical values); lead blocks then write the row block's dz
+// and loss sums, and block (0, 0) also advances the block's Adam step.
 struct PoGradArgs {
-  const float* dz;      // [n, 10]
+  const float* dz;      // [n, 10], or null with zpart
+  const float* zpart;   // [zt, n, 10] partial logits, or null
+  int zt;
+  const float* cb;      // [10] block bias
+  const int* labels;    // [n]
+  float inv_n;
+  float* part;          // [row blocks, 11]: sums of dz and of the loss (with zpart)
+  ff_dev_state* hds;    // the block's Adam state (with zpart)
+  float hbeta1, hbeta2;
   const float* V;       // [10, N] (before this step's update)
   const float* s;       // [n] row scale of the layer input
   const float* gpart;   // forward goodness partials [ntiles, n]
@@ -503,9 +517,54 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     const int c = idx / 256, j = idx % 256;
     Vsh[c][j % 8][j / 8] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
   }
-  for (int idx = tid; idx < kPoRows * kClasses; idx += 256) {
-    const int i = idx / kClasses, c = idx % kClasses;
-    dzs[i][c] = (r0 + i < a.n) ? __ldg(a.dz + (size_t)(r0 + i) * kClasses + c) : 0.f;
+  if (a.zpart) {
+    // logits of the block's rows: thread per (row, class), partials in tile order
+    for (int idx = tid; idx < kPoRows * kClasses; idx += 256) {
+      const int i = idx / kClasses, c = idx % kClasses;
+      dzs[i][c] = r0 + i < a.n ? __ldg(a.cb + c) + sum_partials(a.zpart, a.zt, a.n * kClasses, (r0 + i) * kClasses + c)
+                               : 0.f;
+    }
+    __syncthreads();
+    if (threadIdx.y == 0) {
+      // warp 0: softmax, loss and dz of row r0 + lane, in place
+      float z[kClasses], dzr[kClasses];
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) z[c] = dzs[lane][c];
+      float loss = 0.f;
+      if (r0 + lane < a.n) {
+        loss = finish_row(z, r0 + lane, a.labels, a.inv_n, nullptr, nullptr, dzr, &a.hds->err);
+      } else {
+#pragma unroll
+        for (int c = 0; c < kClasses; ++c) dzr[c] = 0.f;
+      }
+#pragma unroll
+      for (int c = 0; c < kClasses; ++c) dzs[lane][c] = dzr[c];
+      if (blockIdx.x == 0) {
+        // the row block's sums of dz (for dc) and of the loss, in a fixed order
+#pragma unroll
+        for (int c = 0; c < kClasses; ++c) dzr[c] = warp_sum(dzr[c]);
+        loss = warp_sum(loss);
+        if (lane < kPart) {
+          float t = loss;
+#pragma unroll
+          for (int c = 0; c < kClasses; ++c)
+            if (lane == c) t = dzr[c];
+          a.part[(size_t)blockIdx.y * kPart + lane] = t;
+        }
+        if (blockIdx.y == 0 && lane == 0) {
+          a.hds->t += 1;
+          a.hds->pow1 *= (double)a.hbeta1;
+          a.hds->pow2 *= (double)a.hbeta2;
+          a.hds->bc1 = (float)(1.0 - a.hds->pow1);
+          a.hds->bc2 = (float)(1.0 - a.hds->pow2);
+        }
+      }
+    }
+  } else {
+    for (int idx = tid; idx < kPoRows * kClasses; idx += 256) {
+      const int i = idx / kClasses, c = idx % kClasses;
+      dzs[i][c] = (r0 + i < a.n) ? __ldg(a.dz + (size_t)(r0 + i) * kClasses + c) : 0.f;
+    }
   }
   if (blockIdx.x == 0 && tid < kPoRows && r0 + tid < a.n) {
     const float g = sum_partials(a.gpart, a.ntiles, a.n, r0 + tid);
@@ -899,9 +958,12 @@ struct PoWork {
 
 ff_status po_workspace(ff_head* hd, int n, int N, int es, PoWork* w) {
   size_t off = 0;
-  const size_t oZ = off; off += align256(zpart_floats(&N, 1, n, es) * 4);
+  // partial logits: k_head_dot's (fp32 layers) or the forward GEMM's (bf16)
+  size_t zf = zpart_floats(&N, 1, n, es);
+  if (es == 2) zf = std::max(zf, (size_t)tc_fwd_ntiles_max(N) * n * kClasses);
+  const size_t oZ = off; off += align256(zf * 4);
   const size_t oD = off; off += align256((size_t)n * kClasses * 4);
-  const size_t oP = off; off += align256((size_t)cdiv(n, kDotRows) * kPart * 4);
+  const size_t oP = off; off += align256((size_t)cdiv(n, std::min(kDotRows, kPoRows)) * kPart * 4);
   const size_t oV = off; off += align256((size_t)cdiv(n, kPoRows) * kClasses * N * 4);
   if (off > hd->ws_bytes) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before workspace growth");
@@ -1192,6 +1254,10 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   EpiArgs ep{sc, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
   int ntiles;
   if (b16) {
+    // the block's partial logits come out of the forward GEMM's epilogue
+    ep.logit_V = hd->V;
+    ep.logit_ldV = N;
+    ep.zpart = w.zpart;
     ntiles = tc_fwd_ntiles(n, N, false);
     FF_LAUNCH(K_FWD_TC, 2.0 * n * N * K, st,
               tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, n, N, K, ep, &L->ds->err, st),
@@ -1201,21 +1267,36 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
     FF_LAUNCH(K_FWD_SIMT, 2.0 * n * N * K, st,
               simt_gemm_fwd(static_cast<const float*>(X), L->ldK, L->W, K, n, N, K, ep, st), "forward GEMM (fp32)");
   }
-  // the block on the raw activity: logits, cross-entropy, dz, dV partials
-  Segs sg{};
-  sg.H[0] = H;
-  sg.s[0] = nullptr;
-  sg.ld[0] = L->ldN;
-  sg.F[0] = N;
-  sg.off[0] = 0;
-  sg.nseg = 1;
-  sg.F_total = N;
-  s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, &hd->ds->err, st);
-  if (s != FF_OK) return s;
+  if (!b16) {
+    // the block on the raw activity: logits, cross-entropy, dz
+    Segs sg{};
+    sg.H[0] = H;
+    sg.s[0] = nullptr;
+    sg.ld[0] = L->ldN;
+    sg.F[0] = N;
+    sg.off[0] = 0;
+    sg.nseg = 1;
+    sg.F_total = N;
+    s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, &hd->ds->err, st);
+    if (s != FF_OK) return s;
+  }
   // the gradient reaching the layer, with the block's weights before its
-  // update, and the block's weight-gradient partials
+  // update, and the block's weight-gradient partials (bf16: after finishing
+  // the block's rows from the GEMM's partial logits)
   PoGradArgs pa{};
-  pa.dz = w.dz;
+  if (b16) {
+    pa.zpart = w.zpart;
+    pa.zt = ntiles;
+    pa.cb = hd->c;
+    pa.labels = labels;
+    pa.inv_n = 1.f / (float)n;
+    pa.part = w.part;
+    pa.hds = hd->ds;
+    pa.hbeta1 = hd->cfg.beta1;
+    pa.hbeta2 = hd->cfg.beta2;
+  } else {
+    pa.dz = w.dz;
+  }
   pa.V = hd->V;
   pa.s = sc;
   pa.gpart = L->gpart;
@@ -1276,7 +1357,8 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   aa.discard_dW = !L->cfg.keep_grad && ((uintptr_t)L->dW & 127u) == 0;
   add_dead(aa, L->dZ, (size_t)n * L->ldN * (size_t)es);
   FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
-  const HeadAdamArgs ha = head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, kDotRows), n, loss);
+  const HeadAdamArgs ha =
+      head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, b16 ? kPoRows : kDotRows), n, loss);
   const int vblocks = cdiv((long long)kClasses * hd->F, 256);
   PdlLaunch hl(dim3(vblocks + 1), dim3(256), st);
   FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), st,

@@ -258,6 +258,14 @@ struct EpiArgs {
   // GPU to itself (the layer chains of predict and of the softmax head); the
   // net's concurrent per-layer GEMMs run faster on the wider tiles.
   bool narrow;
+  // Tensor-core forward GEMMs: with logit_V set ([10, logit_ldV] fp32, the
+  // weights of a 10-class softmax block on this layer's activity), each
+  // epilogue warp also writes its rows' partial logits over its columns,
+  // zpart[(t * M + i) * 10 + c] = sum over the columns j of tile-half t of
+  // bf16(H_ij) V_cj, with t indexing like the goodness partials.
+  const float* logit_V;
+  int logit_ldV;
+  float* zpart;
 };
 
 // Tensor-core (tcgen05) bf16 GEMMs, fp32 accumulate.
