@@ -5,6 +5,9 @@
 //            (the linear+ReLU of §3 on the concatenated batch of §4, and the
 //            sum of squared activities of Eq. 1 taken from the fp32
 //            accumulator);
+//            -- optionally also per-tile partial logits of a 10-class
+//            softmax block on the stored activity (the Performance-
+//            Optimized layer of §4);
 //   store    C = X W^T in fp32 (the label-free part of layer 1 in predict);
 //   wgrad    dW = G^T X with G = diag(s) dZ, contracting over the batch rows
 //            (both operands are read MN-major straight from their row-major

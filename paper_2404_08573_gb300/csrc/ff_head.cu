@@ -17,9 +17,14 @@
 //                  z = c + the splits' partials (in split order), softmax,
 //                  per-row loss and dz = (softmax(z) - onehot(y)) / n, and
 //                  the row block's partials of dc and of the loss
-//   k_head_wgrad   dV partials per 128-row block: dz^T (s_k H_k)
+//   k_head_wgrad   dV partials per 64-row block: dz^T (s_k H_k)
 //   k_head_adam    reduces the partials in a fixed order, Adam on V and c,
 //                  the step's loss
+//   k_po_grad      the Performance-Optimized step (§4): the gradient through
+//                  a layer's own block into the layer and the block's dV
+//                  partials; with bf16 layers it first finishes its rows'
+//                  softmax from the partial logits that the forward GEMM's
+//                  epilogue wrote (no k_head_dot pass)
 #include <algorithm>
 #include <cmath>
 #include <cstring>
