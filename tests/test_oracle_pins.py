@@ -659,3 +659,60 @@ def test_po_layer_special_cases():
     o = fo.po_layer_train_step(fo.LayerState(Wd, np.zeros(N)), fo.HeadState(V, np.zeros(10)), x, y,
                                fo.AdamHyper(), fo.AdamHyper())
     assert not o["dW"][2].any() and o["db"][2] == 0.0
+
+
+def _brute_po_predict(Ws, bs, V, c, x):
+    """The last block's argmax with explicit loops: neutral label (0.1 in the
+    10 label features), each layer's input scaled to unit length (1e-12
+    floor), ReLU layers, logits V h + c on the last raw activity, lowest
+    class on ties."""
+    preds = []
+    for row in x:
+        a = [0.1] * 10 + [float(v) for v in row[10:]]
+        for W, b in zip(Ws, bs):
+            nrm = math.sqrt(sum(v * v for v in a))
+            s = 1.0 / max(nrm, 1e-12)
+            h = []
+            for j in range(len(W)):
+                z = b[j] + sum(W[j][k] * a[k] * s for k in range(len(a)))
+                h.append(z if z > 0 else 0.0)
+            a = h
+        z = [c[k] + sum(V[k][j] * a[j] for j in range(len(a))) for k in range(10)]
+        best = 0
+        for k in range(1, 10):
+            if z[k] > z[best]:
+                best = k
+        preds.append(best)
+    return np.array(preds)
+
+
+@pytest.mark.parametrize("dims", [(14, 6, 5), (14, 7)])
+def test_po_predict_matches_brute_force(dims):
+    rng = np.random.default_rng(31)
+    Ws = [rng.standard_normal((dims[i + 1], dims[i])) for i in range(len(dims) - 1)]
+    bs = [rng.standard_normal(dims[i + 1]) * 0.2 for i in range(len(dims) - 1)]
+    V = rng.standard_normal((10, dims[-1]))
+    c = rng.standard_normal(10) * 0.1
+    x = rng.random((40, dims[0]))
+    states = [fo.LayerState(W, b) for W, b in zip(Ws, bs)]
+    heads = [fo.HeadState(rng.standard_normal((10, d)), np.zeros(10)) for d in dims[1:-1]] + [fo.HeadState(V, c)]
+    pred, z = fo.po_predict(states, heads, x)
+    bp = _brute_po_predict([W.tolist() for W in Ws], [b.tolist() for b in bs], V.tolist(), c.tolist(), x)
+    assert np.array_equal(pred, bp)
+    # only the last layer's block decides: the earlier blocks are ignored
+    heads2 = [fo.HeadState(np.zeros((10, d)), np.ones(10)) for d in dims[1:-1]] + [fo.HeadState(V, c)]
+    assert np.array_equal(fo.po_predict(states, heads2, x)[0], pred)
+
+
+def test_po_predict_hand_built_block_selects_the_class():
+    # one layer copying features 10..19 through the ReLU; the block maps unit j to class j
+    K = 24
+    W = np.zeros((10, K)); W[np.arange(10), 10 + np.arange(10)] = 1.0
+    V = np.eye(10)
+    x = np.zeros((10, K))
+    for k in range(10):
+        x[k, 10 + k] = 1.0          # the only nonzero image feature of sample k
+    pred, z = fo.po_predict([fo.LayerState(W, np.zeros(10))], [fo.HeadState(V, np.zeros(10))], x)
+    assert np.array_equal(pred, np.arange(10))
+    # the neutral label area (10 x 0.1) only enters through the input norm: z_k = 1 / sqrt(1.1)
+    np.testing.assert_allclose(z[np.arange(10), np.arange(10)], 1.0 / math.sqrt(1.1), rtol=1e-14)
