@@ -59,7 +59,10 @@ def _bounds(out, x_in, V, emul):
 
 
 @pytest.mark.parametrize("prec,raw,K,N,n", [("fp32", True, 784, 256, 300), ("bf16", True, 784, 256, 300),
-                                            ("bf16", False, 256, 136, 257), ("fp32", False, 200, 96, 64)])
+                                            ("bf16", False, 256, 136, 257), ("fp32", False, 200, 96, 64),
+                                            # a full-size hidden layer: the forward GEMM's logits
+                                            # epilogue on two 128-row subtiles per CTA
+                                            ("bf16", False, 2000, 2000, 2048)])
 def test_po_step_matches_oracle(env, prec, raw, K, N, n):
     torch, ff = env
     layer, W, b = _layer(ff, K, N, prec, seed=K + N)
@@ -108,10 +111,21 @@ def test_po_step_matches_oracle(env, prec, raw, K, N, n):
     ls, bs = layer.get_state(), block.get_state()
     assert ls["t"] == 1 and bs["t"] == 1
     z = np.zeros_like(W, dtype=np.float64)
-    assert_adam_state(ls["W"], ls["mW"], ls["vW"], W, z, z, 1, out["dW"], bW, hpl, "W")
-    assert_adam_state(ls["b"], ls["mb"], ls["vb"], b, np.zeros(N), np.zeros(N), 1, out["db"], bb, hpl, "b")
+    # the Adam kernels applied to the GPU's own gradients, with the float32 hyper-parameters: tight
+    f32 = lambda hp: fo.AdamHyper(*[float(np.float32(v)) for v in (hp.lr, hp.beta1, hp.beta2, hp.eps)])
+    assert_adam_state(ls["W"], ls["mW"], ls["vW"], W, z, z, 1, dW.astype(np.float64), 0 * z, f32(hpl), "W (own grad)",
+                      rtol=1e-5, w_floor=0.05, max_band_frac=0.0)
+    # against the oracle's gradients: 1e-4 plus Adam's spread over each element's bound.  With
+    # bf16 operands the stored s*dZ rounds to a neighbouring bf16 value wherever the GPU's
+    # fp32 dz (from fp32 logits) and the oracle's fp64 dz straddle a rounding boundary; over
+    # a 2048-row contraction of mixed-sign terms that moves up to ~8 % of the dW elements by
+    # more than 1e-4 relative (each inside its bound, checked above and by the band here).
+    band = 0.15 if emul and n >= 1024 else 0.05
+    assert_adam_state(ls["W"], ls["mW"], ls["vW"], W, z, z, 1, out["dW"], bW, hpl, "W", max_band_frac=band)
+    assert_adam_state(ls["b"], ls["mb"], ls["vb"], b, np.zeros(N), np.zeros(N), 1, out["db"], bb, hpl, "b",
+                      max_band_frac=band)
     zv = np.zeros_like(V, dtype=np.float64)
-    assert_adam_state(bs["V"], bs["mV"], bs["vV"], V, zv, zv, 1, out["dV"], bV, hpb, "V")
+    assert_adam_state(bs["V"], bs["mV"], bs["vV"], V, zv, zv, 1, out["dV"], bV, hpb, "V", max_band_frac=band)
 
 
 def test_po_net_learns_and_predicts(env):
