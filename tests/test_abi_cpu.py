@@ -85,3 +85,11 @@ def test_invalid_arguments_are_rejected_on_the_host(libff):
     assert libff.ff_net_train_step(None, None, None, 1, None, None) == 1
     assert libff.ff_layer_get_state(None, None, None, None, None, None, None, None) == 1
     assert libff.ff_layer_check(None) == 1
+    # the allocation-free forward: sizes and pointers checked, and the scratch limit
+    # (rows * 2 * ceil(out / 256) partials) applied, before any CUDA call
+    fake = ctypes.c_void_p(256)
+    assert libff.ff_forward_noalloc(None, None, None, None, -1, 16, 8, None, None, None, None, None) == 1
+    assert libff.ff_forward_noalloc(None, None, None, None, 0, 16, 8, None, None, None, None, None) == 0
+    assert libff.ff_forward_noalloc(None, None, None, None, 4, 16, 8, None, None, None, None, None) == 1
+    assert libff.ff_forward_noalloc(fake, fake, fake, None, 4, 0, 8, fake, None, None, None, None) == 1
+    assert libff.ff_forward_noalloc(fake, fake, fake, None, 1 << 21, 16, 8, fake, None, None, None, None) == 1
