@@ -293,13 +293,16 @@ def run_ours(args):
     value, ms = replica_throughput(ms, PAIRS_PER_EPOCH * args.steps, world, dist)
 
     # end to end through the public API: pinned host batches copied in per
-    # batch on a copy stream, RING batches ahead of the layer that reads them
+    # batch on a copy stream, RING batches ahead of the layer that reads them;
+    # each image travels once per pair (ff_net_train_step_images), with the
+    # true and the wrong labels
     e2e = None
     if not args.no_e2e:
-        Xp = torch.from_numpy(X_h).pin_memory()
+        X_img = np.concatenate([X_h[2 * start:2 * start + b] for start, b in bl])   # positive halves
+        Xp = torch.from_numpy(X_img).pin_memory()
         Lp = torch.from_numpy(L_h).pin_memory()
         RING = 3
-        xbuf = [torch.empty(2 * BATCH, NET[0], device=dev) for _ in range(RING)]
+        xbuf = [torch.empty(BATCH, NET[0], device=dev) for _ in range(RING)]
         lbuf = [torch.empty(2 * BATCH, dtype=torch.int32, device=dev) for _ in range(RING)]
         copied = [torch.cuda.Event() for _ in range(RING)]
         freed = [torch.cuda.Event() for _ in range(RING)]
@@ -322,7 +325,7 @@ def run_ours(args):
                 j = g % RING
                 with torch.cuda.stream(cstream):
                     cstream.wait_event(freed[j])      # the step that last read slot j is past layer 1
-                    xbuf[j][:2 * b].copy_(Xp[r0:r0 + 2 * b], non_blocking=True)
+                    xbuf[j][:b].copy_(Xp[start:start + b], non_blocking=True)
                     lbuf[j][:2 * b].copy_(Lp[r0:r0 + 2 * b], non_blocking=True)
                     copied[j].record(cstream)
             begin = torch.cuda.Event()
@@ -337,8 +340,8 @@ def run_ours(args):
                 start, b = bl[t]
                 j = g % RING
                 stream.wait_event(copied[j])
-                net.train_step(xbuf[j][:2 * b], lbuf[j][:2 * b], B=b, loss=loss[t], stream=stream)
-                freed[j].record(stream)  # ff_net_train_step returns with `stream` ordered after layer 1 read x
+                net.train_step_images(xbuf[j][:b], lbuf[j][:2 * b], loss=loss[t], stream=stream)
+                freed[j].record(stream)  # the step returns with `stream` ordered after layer 1 read x
                 if t == nb - 1:
                     net.sync(stream)
                     loss_h.copy_(loss[-1], non_blocking=True)
@@ -356,8 +359,8 @@ def run_ours(args):
         barrier()
         e2e_value, ems = replica_throughput(e0.elapsed_time(e1), PAIRS_PER_EPOCH * args.steps, world, dist)
         e2e = {"value": e2e_value, "unit": "pairs/s",
-               "h2d_bytes_per_step": int(X_h.nbytes + L_h.nbytes), "d2h_bytes_per_step": int(loss_h.numel() * 4),
-               "ms_per_step": ems / args.steps}
+               "h2d_bytes_per_step": int(X_img.nbytes + L_h.nbytes), "d2h_bytes_per_step": int(loss_h.numel() * 4),
+               "ms_per_step": ems / args.steps, "input": "one image per pair (ff_net_train_step_images)"}
 
     # Per-kernel device time: the same epochs with the layers run one after
     # another on one stream (each kernel alone on the GPU), every launch

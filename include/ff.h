@@ -297,7 +297,8 @@ FF_API ff_status ff_po_train_step(ff_layer* layer, ff_head* block, const void* x
  * batch t while layer k-1 trains batch t+1; bitwise the same as calling
  * ff_po_train_step layer after layer.  max_rows: the largest batch (rows);
  * depth: activation (and label) ring slots.  ff_net_sync, ff_net_wait and
- * ff_net_destroy apply; ff_net_train_step does not (FF_ERR_INVALID_ARG). */
+ * ff_net_destroy apply; ff_net_train_step and ff_net_train_step_images do
+ * not (FF_ERR_INVALID_ARG). */
 FF_API ff_status ff_net_create_po(ff_layer* const* layers, ff_head* const* blocks, int n_layers,
                                   int max_rows, int depth, ff_net** out);
 /* One batch: x [rows, in] raw float32 (neutral label on layer 1), labels
@@ -363,6 +364,15 @@ FF_API ff_status ff_net_destroy(ff_net* net);
  * each layer's loss asynchronously; call ff_net_sync before reading it. */
 FF_API ff_status ff_net_train_step(ff_net* net, const float* x, const int* labels, int B,
                             float* loss, void* stream);
+
+/* As ff_net_train_step, with each image sent once per pair: x raw float32
+ * [B, in] (the positive and the negative row of pair i share image i, as in
+ * §3 "Negative Data"), labels [2B] (true labels then wrong labels).  Layer 1
+ * overlays image i with labels[i] for row i and with labels[B + i] for row
+ * B + i; the result is bitwise that of ff_net_train_step on x stacked twice.
+ * Halves the input bytes a caller copies per step. */
+FF_API ff_status ff_net_train_step_images(ff_net* net, const float* x, const int* labels, int B,
+                                          float* loss, void* stream);
 
 /* Makes `stream` wait for all work the net has enqueued so far.  The steps
  * enqueued between two ff_net_sync calls on one stream depend on nothing

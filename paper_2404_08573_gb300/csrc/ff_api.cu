@@ -169,8 +169,11 @@ static ff_status ensure_split(ff_layer* L, int M) {
   return FF_OK;
 }
 
+// x_rows: rows of the raw input x when labels are given (0: M; M / 2: one
+// image per pair, read for the positive and the negative row).
 static ff_status forward_core(ff_layer* L, const void* x, const int* labels, const float* row_scale, int M,
-                              void* h_out, cudaStream_t st, cudaEvent_t ev_input_read, FwdResult* r) {
+                              void* h_out, cudaStream_t st, cudaEvent_t ev_input_read, FwdResult* r,
+                              int x_rows = 0) {
   const int K = L->K, N = L->N;
   if (!L->is_bf16) {
     const ff_status ss = ensure_split(L, M);
@@ -181,7 +184,8 @@ static ff_status forward_core(ff_layer* L, const void* x, const int* labels, con
   const void* X;
   if (labels) {
     FF_LAUNCH(K_OVERLAY, (double)M * (K * 4.0 + L->ldK * es + 8), st,
-              launch_overlay(static_cast<const float*>(x), labels, M, K, L->X, L->ldK, L->is_bf16, L->s_in, 0, st),
+              launch_overlay(static_cast<const float*>(x), labels, M, K, L->X, L->ldK, L->is_bf16, L->s_in, 0, st,
+                             x_rows),
               "overlay");
     if (ev_input_read) FF_TRY(cudaEventRecord(ev_input_read, st), "event record");
     X = L->X;
@@ -230,7 +234,7 @@ static ff_status check_call(ff_layer* L, const void* x, const int* labels, int r
 
 ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B, void* h_out,
                           float* next_scale, float* goodness, float* loss, cudaStream_t st,
-                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done) {
+                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done, bool images_once) {
   ff_status cs = check_call(L, x, labels, B);
   if (cs != FF_OK) return cs;
   if (h_out && !aligned16(h_out)) return FF_ERR_INVALID_ARG;
@@ -242,7 +246,8 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   L->last_stream = st;
   const double es = L->is_bf16 ? 2.0 : 4.0;
   FwdResult fr;
-  ff_status fs = forward_core(L, x, labels, row_scale, M, h_out, st, ev_input_read, &fr);
+  ff_status fs = forward_core(L, x, labels, row_scale, M, h_out, st, ev_input_read, &fr,
+                              images_once && labels ? B : 0);
   if (fs != FF_OK) return fs;
 
   GradPrepArgs ga{};

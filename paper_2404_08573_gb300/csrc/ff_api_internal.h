@@ -28,9 +28,11 @@ ff_status ensure_capacity(ff_layer* L, int rows);
 // not null, is recorded once the raw input x has been consumed (after the
 // overlay; only meaningful when labels are given); ev_forward_done, if not
 // null, once the activity, goodness and next-layer scale are written.
+// images_once (with labels): x holds B images, one per pair, read for both
+// the positive row i and the negative row B + i.
 ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const float* row_scale, int B,
                           void* h_out, float* next_scale, float* goodness, float* loss, cudaStream_t st,
-                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done);
+                          cudaEvent_t ev_input_read, cudaEvent_t ev_forward_done, bool images_once = false);
 
 }  // namespace ff
 

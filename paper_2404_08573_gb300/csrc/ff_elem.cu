@@ -50,11 +50,11 @@ __device__ __forceinline__ void store4<bf16>(bf16* p, float a, float b, float c,
 // when x is) move as float4; others element by element.
 template <typename T>
 __global__ void k_overlay(const float* __restrict__ x, const int* __restrict__ labels, int rows, int F,
-                          T* __restrict__ out, int ldo, float* __restrict__ s_out, int mode) {
+                          T* __restrict__ out, int ldo, float* __restrict__ s_out, int mode, int src_rows) {
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   const int row = blockIdx.x * 8 + warp;
   if (row >= rows) return;
-  const float* xr = x + (size_t)row * F;
+  const float* xr = x + (size_t)(row % src_rows) * F;
   T* orow = out + (size_t)row * ldo;
   const int lab = (mode == 0 && labels) ? labels[row] : -1;
   float ss = 0.f;
@@ -530,13 +530,14 @@ int grid_for(long long work, int per_block, int cap) {
 }  // namespace
 
 cudaError_t launch_overlay(const float* x, const int* labels, int rows, int F, void* out, int ldo, bool out_bf16,
-                           float* s_out, int mode, cudaStream_t st) {
+                           float* s_out, int mode, cudaStream_t st, int src_rows) {
   if (rows <= 0) return cudaSuccess;
+  if (src_rows <= 0 || src_rows > rows) src_rows = rows;
   const int grid = cdiv(rows, 8);
   if (out_bf16)
-    k_overlay<bf16><<<grid, 256, 0, st>>>(x, labels, rows, F, (bf16*)out, ldo, s_out, mode);
+    k_overlay<bf16><<<grid, 256, 0, st>>>(x, labels, rows, F, (bf16*)out, ldo, s_out, mode, src_rows);
   else
-    k_overlay<float><<<grid, 256, 0, st>>>(x, labels, rows, F, (float*)out, ldo, s_out, mode);
+    k_overlay<float><<<grid, 256, 0, st>>>(x, labels, rows, F, (float*)out, ldo, s_out, mode, src_rows);
   return cudaGetLastError();
 }
 

@@ -138,8 +138,11 @@ inline int cdiv(long long a, long long b) { return (int)((a + b - 1) / b); }
 //   mode 0: out[:,0..9] = one-hot(labels[r]); mode 1: out[:,0..9] = 0 and the
 //   norm counts one extra 1.0 (the one-hot every predict overlay adds);
 //   mode 2: out[:,0..9] = 0.1, the neutral label of the softmax head (§3).
+// Output row r reads input row r % src_rows (src_rows 0: rows): with
+// src_rows = B the B images of a pair batch are read once each for both
+// their positive and their negative row.
 cudaError_t launch_overlay(const float* x, const int* labels, int rows, int F, void* out,
-                           int ldo, bool out_bf16, float* s_out, int mode, cudaStream_t st);
+                           int ldo, bool out_bf16, float* s_out, int mode, cudaStream_t st, int src_rows = 0);
 // s_r = 1 / max(||x_r||, 1e-12) of an activation buffer.
 cudaError_t launch_row_scale(const void* x, int ldx, bool x_bf16, int rows, int F,
                              float* s_out, cudaStream_t st);

@@ -201,8 +201,9 @@ ff_status ff_net_destroy(ff_net* n) {
   return FF_OK;
 }
 
-ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
-  ff::NvtxRange nvtx_("ff_net_train_step");
+// One batch through every layer; images_once: x holds one image per pair.
+static ff_status net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream,
+                                bool images_once) {
   if (!n || !x || !labels || B < 0 || B > n->max_B || n->po) return FF_ERR_INVALID_ARG;
   if (B == 0) return FF_OK;
   cudaStream_t cs = static_cast<cudaStream_t>(stream);
@@ -228,7 +229,7 @@ ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B,
     float* sn = k + 1 < n->L ? n->sbuf[k][slot] : nullptr;
     s = ff::train_step_impl(n->layers[k], xin, k == 0 ? labels : nullptr, scale, B, hout, sn, nullptr,
                             loss ? loss + k : nullptr, st, k == 0 ? n->ev_x_done : nullptr,
-                            k + 1 < n->L ? n->ready[k][slot] : nullptr);
+                            k + 1 < n->L ? n->ready[k][slot] : nullptr, images_once && k == 0);
     if (s != FF_OK) return s;
     if (k > 0) {
       s = ff::cuda_status(cudaEventRecord(n->consumed[k - 1][slot], st), "record consumed event");
@@ -281,6 +282,16 @@ ff_status ff_net_po_train_step(ff_net* n, const float* x, const int* labels, int
   ++n->step;
   ++n->since_sync;
   return FF_OK;
+}
+
+ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_net_train_step");
+  return net_train_step(n, x, labels, B, loss, stream, false);
+}
+
+ff_status ff_net_train_step_images(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_net_train_step_images");
+  return net_train_step(n, x, labels, B, loss, stream, true);
 }
 
 ff_status ff_net_sync(ff_net* n, void* stream) {

@@ -91,6 +91,7 @@ def lib():
             "ff_net_create": [c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_destroy": [c_void_p],
             "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
+            "ff_net_train_step_images": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_sync": [c_void_p, c_void_p],
             "ff_net_create_po": [c_void_p, c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_po_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
@@ -327,6 +328,17 @@ class Net:
         _check(lib().ff_net_train_step(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
                                        int(B), _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
                "ff_net_train_step")
+
+    def train_step_images(self, x, labels, loss=None, stream=None):
+        """ff_net_train_step_images: x [B, in] holds one image per pair, labels
+        [2B] the true labels then the wrong ones."""
+        B = x.shape[0]
+        if labels.shape[0] != 2 * B:
+            raise ValueError("labels must hold 2 * x.shape[0] entries (true labels, then wrong labels)")
+        _check(lib().ff_net_train_step_images(self._h, _ptr(x, torch.float32, "x"),
+                                              _ptr(labels, torch.int32, "labels"), int(B),
+                                              _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
+               "ff_net_train_step_images")
 
     def sync(self, stream=None):
         _check(lib().ff_net_sync(self._h, c_void_p(_stream(stream))), "ff_net_sync")

@@ -83,6 +83,7 @@ def test_invalid_arguments_are_rejected_on_the_host(libff):
     assert libff.ff_pff_run(None, None, None, 0, 1, None, None) == 1
     assert libff.ff_net_create(None, 2, 8, 2, ctypes.byref(out)) == 1
     assert libff.ff_net_train_step(None, None, None, 1, None, None) == 1
+    assert libff.ff_net_train_step_images(None, None, None, 1, None, None) == 1
     assert libff.ff_layer_get_state(None, None, None, None, None, None, None, None) == 1
     assert libff.ff_layer_check(None) == 1
     # the allocation-free forward: sizes and pointers checked, and the scratch limit
@@ -93,3 +94,18 @@ def test_invalid_arguments_are_rejected_on_the_host(libff):
     assert libff.ff_forward_noalloc(None, None, None, None, 4, 16, 8, None, None, None, None, None) == 1
     assert libff.ff_forward_noalloc(fake, fake, fake, None, 4, 0, 8, fake, None, None, None, None) == 1
     assert libff.ff_forward_noalloc(fake, fake, fake, None, 1 << 21, 16, 8, fake, None, None, None, None) == 1
+
+
+def test_every_function_the_binding_calls_has_a_declared_signature(libff):
+    """ctypes passes an undeclared argument list as C ints: a device pointer
+    would lose its upper 32 bits.  Every ff_* function the binding calls must
+    therefore have its argument types set, and exist in include/ff.h."""
+    from paper_2404_08573_gb300 import ff
+    src = open(os.path.join(ROOT, "paper_2404_08573_gb300", "ff.py")).read()
+    called = sorted(set(re.findall(r"lib\(\)\.(ff_\w+)\(", src)))
+    assert called, "no calls found"
+    L = ff.lib()
+    declared = set(_declared())
+    for name in called:
+        assert name in declared, f"{name} is called by the binding but not declared in ff.h"
+        assert getattr(L, name).argtypes is not None, f"{name} has no argtypes in the binding"

@@ -324,6 +324,35 @@ def test_adaptive_negatives_label_outside_range_is_plain_prediction(env):
     ff.adaptive_negatives(layers, empty, torch.empty(0, dtype=torch.int32, device="cuda"))
 
 
+# ------------------------------------------------- one image per pair == stacked pairs
+@pytest.mark.parametrize("prec", ["bf16", "fp32"])
+def test_net_step_with_one_image_per_pair_equals_stacked_pairs(env, prec):
+    torch, ff = env
+    dims, Bmax = (784, 192, 160), 96
+    mk = lambda: [ff.Layer(dims[i], dims[i + 1], prec=prec, init_seed=70 + i) for i in range(2)]
+    a, b = mk(), mk()
+    net_a, net_b = ff.Net(a, max_B=Bmax, depth=2), ff.Net(b, max_B=Bmax, depth=2)
+    Bs = [96, 37, 96, 1]                                  # full and ragged batches
+    la = torch.empty(len(Bs), 2, device="cuda")
+    lb = torch.empty(len(Bs), 2, device="cuda")
+    for t, B in enumerate(Bs):
+        x2, l2 = pair_inputs(B, seed=300 + t)
+        assert np.array_equal(x2[:B], x2[B:])             # the pair rows share their image
+        lg = torch.from_numpy(l2).cuda()
+        net_a.train_step(torch.from_numpy(x2).cuda(), lg, B=B, loss=la[t])
+        net_b.train_step_images(torch.from_numpy(np.ascontiguousarray(x2[:B])).cuda(), lg, loss=lb[t])
+    net_a.sync()
+    net_b.sync()
+    torch.cuda.synchronize()
+    assert torch.equal(la, lb)
+    for p, q in zip(a, b):
+        sp, sq = p.get_state(), q.get_state()
+        for k in ("W", "b", "mW", "vW"):
+            assert np.array_equal(sp[k], sq[k]), k
+    with pytest.raises(ValueError):
+        net_b.train_step_images(torch.zeros(4, 784, device="cuda"), torch.zeros(4, dtype=torch.int32, device="cuda"))
+
+
 # ----------------------------------------------- multi-stream net == sequential
 def test_net_on_streams_is_bitwise_sequential(env):
     torch, ff = env
