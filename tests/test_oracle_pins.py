@@ -181,6 +181,31 @@ def test_adam_first_step_closed_form_and_zero_gradient():
         w_t = w_n
 
 
+def test_adam_two_steps_with_different_gradients_pin_both_decay_rates():
+    """Two steps with g1 != g2 (a constant gradient hides beta1 and beta2,
+    since then m_hat = g and v_hat = g^2 for any rates).  The expected values
+    are worked out by hand with beta1 = 0.9, beta2 = 0.999, lr = 0.03,
+    eps = 1e-8 and written as decimals:
+      element 0: w0 = 0.5, g1 = 2, g2 = -1
+        m1 = 0.2, v1 = 0.004, w1 = 0.5 - 0.06/(2 + 1e-8)
+        m2 = 0.08, v2 = 0.004996, m_hat2 = 8/19, v_hat2 = 4996/1999
+      element 1: w0 = 0, g1 = 1, g2 = 3
+        m1 = 0.1, v1 = 0.001, w1 = -0.03/(1 + 1e-8)
+        m2 = 0.39, v2 = 0.009999, m_hat2 = 39/19, v_hat2 = 9999/1999
+    (w2 to 40 digits by decimal arithmetic)."""
+    hp = fo.AdamHyper(lr=0.03, beta1=0.9, beta2=0.999, eps=1e-8)
+    w0 = np.array([0.5, 0.0])
+    z = np.zeros(2)
+    w1, m1, v1 = fo.adam_update(w0, np.array([2.0, 1.0]), z, z, 1, hp)
+    assert np.allclose(m1, [0.2, 0.1], rtol=1e-15, atol=0)
+    assert np.allclose(v1, [0.004, 0.001], rtol=1e-14, atol=0)
+    assert np.allclose(w1, [0.47000000014999999925, -0.02999999970000000300], rtol=1e-15, atol=1e-16)
+    w2, m2, v2 = fo.adam_update(w1, np.array([-1.0, 3.0]), m1, v1, 2, hp)
+    assert np.allclose(m2, [0.08, 0.39], rtol=1e-14, atol=0)
+    assert np.allclose(v2, [0.004996, 0.009999], rtol=1e-14, atol=0)
+    assert np.allclose(w2, [0.46200988901072940735, -0.05753343314630051164], rtol=1e-14, atol=1e-16)
+
+
 # ---------------------------------------------------------------- predict
 def _brute_predict(Ws, bs, x, n_classes=10):
     """Pure-Python loops, no NumPy algebra: overlay, normalise, ReLU layers,

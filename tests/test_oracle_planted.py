@@ -169,6 +169,41 @@ def test_adam_with_eps_inside_the_root_is_caught(monkeypatch):
     _caught(pins.test_adam_first_step_closed_form_and_zero_gradient)
 
 
+def _adam_with_rates(b1, b2):
+    """Adam whose moment decay rates are b1 (first) and b2 (second)
+    regardless of the hyper-parameters passed in."""
+    def bad(w, grad, m, v, t, hp):
+        grad = np.asarray(grad, dtype=np.float64)
+        m = b1 * np.asarray(m, dtype=np.float64) + (1.0 - b1) * grad
+        v = b2 * np.asarray(v, dtype=np.float64) + (1.0 - b2) * grad * grad
+        m_hat, v_hat = m / (1.0 - b1 ** t), v / (1.0 - b2 ** t)
+        return np.asarray(w, dtype=np.float64) - hp.lr * m_hat / (np.sqrt(v_hat) + hp.eps), m, v
+    return bad
+
+
+def test_adam_with_the_decay_rates_swapped_is_caught(monkeypatch):
+    # swapped consistently in the moments and their bias corrections: the
+    # one-step and constant-gradient pins cannot see it
+    monkeypatch.setattr(fo, "adam_update", _adam_with_rates(0.999, 0.9))
+    pins.test_adam_first_step_closed_form_and_zero_gradient()
+    _caught(pins.test_adam_two_steps_with_different_gradients_pin_both_decay_rates)
+
+
+def test_adam_with_a_wrong_second_moment_rate_is_caught(monkeypatch):
+    monkeypatch.setattr(fo, "adam_update", _adam_with_rates(0.9, 0.99))
+    _caught(pins.test_adam_two_steps_with_different_gradients_pin_both_decay_rates)
+
+
+def test_adam_with_a_wrong_first_moment_rate_is_caught(monkeypatch):
+    monkeypatch.setattr(fo, "adam_update", _adam_with_rates(0.8, 0.999))
+    _caught(pins.test_adam_two_steps_with_different_gradients_pin_both_decay_rates)
+
+
+def test_the_planted_adam_copy_with_the_right_rates_passes(monkeypatch):
+    monkeypatch.setattr(fo, "adam_update", _adam_with_rates(0.9, 0.999))
+    pins.test_adam_two_steps_with_different_gradients_pin_both_decay_rates()
+
+
 # ---------------------------------------------------------------- predict
 def test_predict_counting_layer_one_is_caught(monkeypatch):
     def bad(states, x_raw, emulate_bf16=False, n_classes=fo.N_CLASSES):
