@@ -405,9 +405,11 @@ FF_API ff_status ff_net_wait(ff_net* net, unsigned int timeout_ms);
  *   - Limit: rows * 2 * ceil(out_features / 256) <= 1048512 (two goodness
  *     partials per 256-column tile and row); larger requests return
  *     FF_ERR_INVALID_ARG before anything is enqueued.
- *   - The first call on a device looks up that array's device address (once
- *     per device, with that device current); make that first call before any
+ *   - Every call looks up that array's device address on the caller's
+ *     current device (the lookup enqueues nothing).  The first call on a
+ *     device also loads the library's device code there: make it before any
  *     stream capture.
+ *   - rows == 0 computes nothing and still sets device_status to 0.
  *   - Every call shares the array and it keeps the last call's contents:
  *     calls whose work overlaps on the GPU (other streams, other threads)
  *     race; order them on one stream.

@@ -8,8 +8,6 @@
 // kernel live in the file-scope array below instead of a layer workspace.
 // That array is a fixed part of every device that loads this library, held
 // until the process exits.
-#include <mutex>
-
 #include "ff_internal.cuh"
 
 namespace ff {
@@ -21,25 +19,17 @@ constexpr size_t kNoAllocScratchFloats = size_t(1) << 20;  // 4 MiB
 constexpr size_t kNoAllocPartialOffset = 64;
 static __device__ __align__(256) float g_noalloc_scratch[kNoAllocScratchFloats];
 
-constexpr int kMaxDevices = 64;
-std::mutex g_mu;
-float* g_scratch_addr[kMaxDevices] = {nullptr};
-
-// Device address of the scratch array on the current device, looked up once
-// per device.  In host code the array's name is only a host-side stand-in.
+// Device address of the scratch array on the current device.  In host code
+// the array's name is only a host-side stand-in, so the address is looked up
+// with the caller's device current -- on every call rather than cached, so
+// that a context recreated after cudaDeviceReset never sees a stale address
+// (the lookup enqueues nothing; the first one on a device also loads the
+// library's device code there).
 cudaError_t scratch_address(float** out) {
-  int dev = 0;
-  cudaError_t e = cudaGetDevice(&dev);
+  void* p = nullptr;
+  const cudaError_t e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
   if (e != cudaSuccess) return e;
-  if (dev < 0 || dev >= kMaxDevices) return cudaErrorInvalidDevice;
-  std::lock_guard<std::mutex> lock(g_mu);
-  if (!g_scratch_addr[dev]) {
-    void* p = nullptr;
-    e = cudaGetSymbolAddress(&p, g_noalloc_scratch);
-    if (e != cudaSuccess) return e;
-    g_scratch_addr[dev] = static_cast<float*>(p);
-  }
-  *out = g_scratch_addr[dev];
+  *out = static_cast<float*>(p);
   return cudaSuccess;
 }
 
@@ -53,7 +43,12 @@ extern "C" FF_API ff_status ff_forward_noalloc(const void* x, const float* row_s
                                                void* h_out, float* goodness, float* next_scale, int* device_status,
                                                void* stream) {
   if (rows < 0 || in_features < 1 || out_features < 1) return FF_ERR_INVALID_ARG;
-  if (rows == 0) return FF_OK;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  if (rows == 0) {
+    // nothing to compute; the status word still reads 0 afterwards
+    if (device_status && cudaMemsetAsync(device_status, 0, sizeof(int), st) != cudaSuccess) return FF_ERR_CUDA;
+    return FF_OK;
+  }
   if (!x || !row_scale || !W_bf16 || !h_out) return FF_ERR_INVALID_ARG;
   const size_t partials = (size_t)tc_fwd_ntiles(rows, out_features, false) * (size_t)rows;
   if (partials > kNoAllocScratchFloats - kNoAllocPartialOffset) return FF_ERR_INVALID_ARG;
@@ -61,7 +56,6 @@ extern "C" FF_API ff_status ff_forward_noalloc(const void* x, const float* row_s
   float* scratch = nullptr;
   cudaError_t e = scratch_address(&scratch);
   if (e != cudaSuccess) return FF_ERR_CUDA;
-  cudaStream_t st = static_cast<cudaStream_t>(stream);
   int* err = device_status ? device_status : reinterpret_cast<int*>(scratch);
   // the error word must start at zero; the partials are written before they are read
   e = cudaMemsetAsync(err, 0, sizeof(int), st);
