@@ -374,6 +374,33 @@ FF_API ff_status ff_net_train_step(ff_net* net, const float* x, const int* label
 FF_API ff_status ff_net_train_step_images(ff_net* net, const float* x, const int* labels, int B,
                                           float* loss, void* stream);
 
+/* A whole run of batches through the net (§4: layer i trains on the output
+ * of layer i-1 computed with that layer's weights before the same step's
+ * update; §3 Eq. 1 and §5.1 per layer), in one persistent kernel: the
+ * tensor-core tiles of every layer's forward and weight-gradient GEMMs, and
+ * the label overlay, local gradient and Adam of every layer, run as tasks
+ * on all SMs at once, the layers as a wavefront (layer k on batch t - k: the
+ * single-GPU analogue of Single-Layer PFF, Algorithm 1).  Bitwise the same
+ * result as ff_net_train_step (or _images) called once per batch.
+ *   x: images_per_pair_row = 2: [2 * n_pairs, in] float32 pair batches laid
+ *      out as ff_net_train_step takes them, batch t (B pairs, the last one
+ *      n_pairs % B) in rows 2tB .. 2tB + 2b (b positive rows, then the same
+ *      images again for the negative rows); images_per_pair_row = 1:
+ *      [n_pairs, in], one image per pair, as ff_net_train_step_images.
+ *   labels: [2 * n_pairs] int32, per batch b true labels then b wrong ones.
+ *   loss: [ceil(n_pairs / B), n_layers] (device) or NULL: each batch's loss
+ *      per layer.
+ * Runs in the persistent kernel when every layer is FF_BF16 with in and out
+ * features multiples of 8 (at most 16384 out), at most 8 layers, and 2B a
+ * multiple of 256 (at most 16384); the last partial batch, and any net
+ * outside these limits, goes through ff_net_train_step.  The first call for
+ * a given (B, batch count, layout) builds and keeps a plan (task tables,
+ * tensor maps, activation rings; it allocates).  Returns with `stream`
+ * ordered after all of it (as ff_net_sync).  Not on a Performance-Optimized
+ * net (FF_ERR_INVALID_ARG). */
+FF_API ff_status ff_net_train_epoch(ff_net* net, const float* x, const int* labels, int n_pairs, int B,
+                                    int images_per_pair_row, float* loss, void* stream);
+
 /* Makes `stream` wait for all work the net has enqueued so far.  The steps
  * enqueued between two ff_net_sync calls on one stream depend on nothing
  * outside them but that stream, so such a sequence can be captured into a

@@ -27,7 +27,7 @@ CHECKED_BUILD_DIR = os.path.join(HERE, "_build_checked")
 CHECKED_LIB_PATH = os.path.join(HERE, "libff_checked.so")
 
 SOURCES = ["ff_api.cu", "ff_net.cu", "ff_elem.cu", "ff_gemm_tc.cu", "ff_gemm_simt.cu", "ff_prof.cu", "ff_noalloc.cu",
-           "ff_head.cu", "ff_pff.cu"]
+           "ff_head.cu", "ff_pff.cu", "ff_epoch.cu"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 NVCC_FLAGS = ARCH + [
     "-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-O2", "-Xcompiler", "-fvisibility=hidden",

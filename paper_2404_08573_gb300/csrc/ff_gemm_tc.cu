@@ -564,6 +564,11 @@ bool make_plain_map(CUtensorMap* m, const void* ptr, int esize, int cols, int ro
   return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_NONE);
 }
 
+bool make_sw128_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
+                    int box_rows) {
+  return make_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows);
+}
+
 bool tc_supported() {
   int dev = 0, major = 0;
   if (cudaGetDevice(&dev) != cudaSuccess) return false;

@@ -105,11 +105,14 @@ struct Vec8<float> {
 // lr * (m / bc1) / (sqrt(v / bc2) + eps) costs one division per parameter
 // instead of three (the kernel is otherwise limited by those divisions, not
 // by HBM).
+// Every operation is spelled out (which product is fused, every rounding),
+// so all kernels that call it produce the same bits whatever the compiler's
+// contraction choices at each call site.
 __device__ __forceinline__ void adam1(float& w, float& m, float& v, float g, float a1, float b1, float b2, float eps,
                                       float r2) {
-  m = b1 * m + (1.f - b1) * g;
-  v = b2 * v + (1.f - b2) * g * g;
-  w -= a1 * m / (sqrtf(v * r2) + eps);
+  m = fmaf(b1, m, __fmul_rn(1.f - b1, g));
+  v = fmaf(b2, v, __fmul_rn(__fmul_rn(1.f - b2, g), g));
+  w = __fsub_rn(w, __fdiv_rn(__fmul_rn(a1, m), __fadd_rn(__fsqrt_rn(__fmul_rn(v, r2)), eps)));
 }
 
 // Bound on every spin-wait in a kernel: after this many nanoseconds of
@@ -292,6 +295,10 @@ int tc_gemm_fwd_ctas(int M, int N, bool narrow);
 // matrix with row stride ld, boxes of box_rows x box_cols, no swizzle; false
 // if the pointer or the stride is not 16-byte aligned.
 bool make_plain_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
+                    int box_rows);
+// The same with 128-byte swizzle (the layout the tensor-core GEMMs' shared
+// memory descriptors expect); out-of-range elements of a box read as zero.
+bool make_sw128_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols,
                     int box_rows);
 
 // SIMT fp32 GEMMs with the same contracts.  A GEMM of few output tiles

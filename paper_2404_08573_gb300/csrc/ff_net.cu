@@ -19,27 +19,9 @@
 #include <vector>
 
 #include "ff_api_internal.h"
+#include "ff_net_internal.h"
 #include "ff_prof.h"
 
-struct ff_net {
-  std::vector<ff_layer*> layers;
-  int L = 0, max_B = 0, depth = 0;
-  std::vector<cudaStream_t> streams;
-  std::vector<std::vector<void*>> hbuf;
-  std::vector<std::vector<float*>> sbuf;
-  std::vector<std::vector<cudaEvent_t>> ready, consumed;
-  std::vector<cudaEvent_t> tail;
-  cudaEvent_t ev_x_in = nullptr, ev_x_done = nullptr;
-  long long step = 0;
-  long long since_sync = 0;  // steps enqueued since the last ff_net_sync
-  void* mem = nullptr;
-  // Performance-Optimized nets: one softmax block per layer, label ring
-  bool po = false;
-  int max_rows = 0;
-  std::vector<ff_head*> blocks;
-  std::vector<int*> lab;
-  std::vector<cudaEvent_t> lab_done;
-};
 
 namespace {
 
@@ -68,6 +50,7 @@ void release(ff_net* n) {
   if (n->ev_x_done) cudaEventDestroy(n->ev_x_done);
   for (auto st : n->streams)
     if (st) cudaStreamDestroy(st);
+  ff::epoch_plan_free(n->epoch);
   ff::dev_free(n->mem);
   delete n;
 }
@@ -172,37 +155,10 @@ ff_status create_net(ff_layer* const* layers, ff_head* const* blocks, int n_laye
 
 }  // namespace
 
-extern "C" {
-
-ff_status ff_net_create(ff_layer* const* layers, int n_layers, int max_B, int depth, ff_net** out) {
-  if (max_B < 1 || max_B > (1 << 29)) {
-    if (out) *out = nullptr;
-    return FF_ERR_INVALID_ARG;
-  }
-  return create_net(layers, nullptr, n_layers, 2 * max_B, depth, out);
-}
-
-ff_status ff_net_create_po(ff_layer* const* layers, ff_head* const* blocks, int n_layers, int max_rows, int depth,
-                           ff_net** out) {
-  if (!blocks || !layers || n_layers < 1) {
-    if (out) *out = nullptr;
-    return FF_ERR_INVALID_ARG;
-  }
-  for (int k = 0; k < n_layers; ++k)
-    if (!blocks[k] || !layers[k] || ff::head_features(blocks[k]) != layers[k]->N) {
-      if (out) *out = nullptr;
-      return FF_ERR_INVALID_ARG;
-    }
-  return create_net(layers, blocks, n_layers, max_rows, depth, out);
-}
-
-ff_status ff_net_destroy(ff_net* n) {
-  release(n);
-  return FF_OK;
-}
+namespace ff {
 
 // One batch through every layer; images_once: x holds one image per pair.
-static ff_status net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream,
+ff_status net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream,
                                 bool images_once) {
   if (!n || !x || !labels || B < 0 || B > n->max_B || n->po) return FF_ERR_INVALID_ARG;
   if (B == 0) return FF_OK;
@@ -240,6 +196,37 @@ static ff_status net_train_step(ff_net* n, const float* x, const int* labels, in
   if (s != FF_OK) return s;
   ++n->step;
   ++n->since_sync;
+  return FF_OK;
+}
+
+}  // namespace ff
+
+extern "C" {
+
+ff_status ff_net_create(ff_layer* const* layers, int n_layers, int max_B, int depth, ff_net** out) {
+  if (max_B < 1 || max_B > (1 << 29)) {
+    if (out) *out = nullptr;
+    return FF_ERR_INVALID_ARG;
+  }
+  return create_net(layers, nullptr, n_layers, 2 * max_B, depth, out);
+}
+
+ff_status ff_net_create_po(ff_layer* const* layers, ff_head* const* blocks, int n_layers, int max_rows, int depth,
+                           ff_net** out) {
+  if (!blocks || !layers || n_layers < 1) {
+    if (out) *out = nullptr;
+    return FF_ERR_INVALID_ARG;
+  }
+  for (int k = 0; k < n_layers; ++k)
+    if (!blocks[k] || !layers[k] || ff::head_features(blocks[k]) != layers[k]->N) {
+      if (out) *out = nullptr;
+      return FF_ERR_INVALID_ARG;
+    }
+  return create_net(layers, blocks, n_layers, max_rows, depth, out);
+}
+
+ff_status ff_net_destroy(ff_net* n) {
+  release(n);
   return FF_OK;
 }
 
@@ -286,12 +273,12 @@ ff_status ff_net_po_train_step(ff_net* n, const float* x, const int* labels, int
 
 ff_status ff_net_train_step(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
   ff::NvtxRange nvtx_("ff_net_train_step");
-  return net_train_step(n, x, labels, B, loss, stream, false);
+  return ff::net_train_step(n, x, labels, B, loss, stream, false);
 }
 
 ff_status ff_net_train_step_images(ff_net* n, const float* x, const int* labels, int B, float* loss, void* stream) {
   ff::NvtxRange nvtx_("ff_net_train_step_images");
-  return net_train_step(n, x, labels, B, loss, stream, true);
+  return ff::net_train_step(n, x, labels, B, loss, stream, true);
 }
 
 ff_status ff_net_sync(ff_net* n, void* stream) {

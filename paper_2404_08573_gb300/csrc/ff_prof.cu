@@ -23,7 +23,8 @@ const char* const kNames[K_NUM] = {"overlay",     "row_scale",    "fwd_gemm_tc",
                                    "finalize",    "grad_prep",   "wgrad_gemm_tc", "wgrad_gemm_simt",
                                    "adam",        "init_weights", "to_bf16",       "label_columns",
                                    "store_gemm_tc", "store_gemm_simt", "expand",   "argmax",
-                                   "head_logits", "head_wgrad",   "head_adam"};
+                                   "head_logits", "head_wgrad",   "head_adam",
+                                   "epoch_gemm_tc"};
 
 struct Rec {
   int kind;

@@ -8,7 +8,7 @@ namespace ff {
 enum KernelKind {
   K_OVERLAY, K_ROW_SCALE, K_FWD_TC, K_FWD_SIMT, K_FINALIZE, K_GRAD_PREP, K_WGRAD_TC, K_WGRAD_SIMT,
   K_ADAM, K_INIT, K_TO_BF16, K_LABEL_COLS, K_STORE_TC, K_STORE_SIMT, K_EXPAND, K_ARGMAX,
-  K_HEAD_LOGITS, K_HEAD_WGRAD, K_HEAD_ADAM, K_NUM
+  K_HEAD_LOGITS, K_HEAD_WGRAD, K_HEAD_ADAM, K_EPOCH, K_NUM
 };
 
 // Counts one launch; when timing is enabled records an event on `st` now and

@@ -93,6 +93,7 @@ def lib():
             "ff_net_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_train_step_images": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_sync": [c_void_p, c_void_p],
+            "ff_net_train_epoch": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p],
             "ff_net_create_po": [c_void_p, c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_po_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
@@ -339,6 +340,19 @@ class Net:
                                               _ptr(labels, torch.int32, "labels"), int(B),
                                               _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
                "ff_net_train_step_images")
+
+    def train_epoch(self, x, labels, n_pairs: int, B: int, images_per_pair_row: int = 2, loss=None, stream=None):
+        """ff_net_train_epoch: n_pairs pairs in batches of B pairs through the
+        net in one persistent kernel (the tail batch stepwise); x holds
+        images_per_pair_row rows per pair (2: stacked pair batches, 1: one
+        image per pair), labels [2 * n_pairs] (per batch the true labels, then
+        the wrong ones)."""
+        if x.shape[0] != images_per_pair_row * n_pairs or labels.shape[0] != 2 * n_pairs:
+            raise ValueError("x must have images_per_pair_row * n_pairs rows and labels 2 * n_pairs entries")
+        _check(lib().ff_net_train_epoch(self._h, _ptr(x, torch.float32, "x"), _ptr(labels, torch.int32, "labels"),
+                                        int(n_pairs), int(B), int(images_per_pair_row),
+                                        _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
+               "ff_net_train_epoch")
 
     def sync(self, stream=None):
         _check(lib().ff_net_sync(self._h, c_void_p(_stream(stream))), "ff_net_sync")
