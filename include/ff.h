@@ -401,6 +401,18 @@ FF_API ff_status ff_net_train_step_images(ff_net* net, const float* x, const int
 FF_API ff_status ff_net_train_epoch(ff_net* net, const float* x, const int* labels, int n_pairs, int B,
                                     int images_per_pair_row, float* loss, void* stream);
 
+/* Instrumentation of ff_net_train_epoch (not part of the method).
+ * enable = 1 / 0 switches per-task tracing of later epoch calls on or off
+ * (-1 leaves it); with `out` (host) it waits for the device and copies the
+ * last traced epoch: out[0] = GEMM tasks G, out[1] = stream tasks S, then per
+ * task (the G GEMM tasks in their queue order, then the S stream tasks) six
+ * words of %globaltimer ns: GEMM tasks -- dequeued, dependencies met, MMAs
+ * started, last MMA issued, epilogue started, done; stream tasks --
+ * dequeued, dependencies met, the SM that ran it (not a time), unused,
+ * unused, done.  Returns the words written, 0 if there is no trace, -1 on an
+ * error. */
+FF_API long long ff_net_epoch_trace(ff_net* net, int enable, unsigned long long* out, long long capacity);
+
 /* Makes `stream` wait for all work the net has enqueued so far.  The steps
  * enqueued between two ff_net_sync calls on one stream depend on nothing
  * outside them but that stream, so such a sequence can be captured into a

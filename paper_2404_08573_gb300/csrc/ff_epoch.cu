@@ -23,10 +23,10 @@
 //   warp 0        TMA producer (the even CTA's lane 0 also dequeues GEMM tasks
 //                 and hands them to both CTAs through a shared-memory ring)
 //   warp 1        tcgen05.mma issuer (even CTA), TMEM owner
-//   warps 2..9    GEMM epilogue (TMEM -> registers -> TMA stores), with two
+//   warps 2..5    GEMM epilogue (TMEM -> registers -> TMA stores), with two
 //                 256-column accumulators so a tile's epilogue overlaps the
 //                 next tile's mainloop
-//   warps 10..15  streamers: OV, LG and ADAM tasks (HBM-bound), dequeued one
+//   warps 6..31   streamers: OV, LG and ADAM tasks (HBM-bound), dequeued one
 //                 at a time by the CTA
 // So Adam's HBM stream and the local gradient run on every SM beside the
 // tensor-core tiles.  Tasks are dequeued in a fixed global order in which
@@ -61,16 +61,17 @@ constexpr int STAGES = 4;
 constexpr int A_BYTES = BM * BK * 2;
 constexpr int B_BYTES = HB * BK * 2;
 constexpr int STAGE = A_BYTES + B_BYTES;
-constexpr int EPI_WARPS = 8;
-constexpr int STR_WARPS = 6;   // 16 warps in all: up to 128 registers a thread
+constexpr int EPI_WARPS = 4;    // one per TMEM lane quarter, both column halves
+constexpr int STR_WARPS = 26;   // 32 warps in all (64 registers a thread): many loads in flight per SM
 constexpr int EPI0 = 2;
 constexpr int STR0 = EPI0 + EPI_WARPS;
 constexpr int NTHREADS = 32 * (STR0 + STR_WARPS);
 constexpr int NSTR = 32 * STR_WARPS;  // streamer threads
 constexpr int TQ = 4;             // task ring slots between the GEMM roles
 constexpr uint32_t TMEM_COLS = 512;  // two 256-column accumulators
-constexpr int EPI_BYTES = 8192;   // staging per epilogue warp
-constexpr int LG_ROWS = 32;
+constexpr int EPI_BYTES = 16384;  // staging per epilogue warp: its 32 rows x 256 bf16 columns
+constexpr int LG_ROWS = 32;      // rows of a bias-gradient partial (as k_grad_prep)
+constexpr int LG_TASK_ROWS = 64; // rows of a local-gradient task
 constexpr int OV_ROWS = 64;
 constexpr int ADAM_ROWS = 16;
 constexpr int BAR_EPI = 1, BAR_STR = 2;
@@ -78,12 +79,12 @@ constexpr int BAR_EPI = 1, BAR_STR = 2;
 constexpr int OFF_EPI = STAGES * STAGE;
 constexpr int OFF_BIAS = OFF_EPI + EPI_WARPS * EPI_BYTES;
 constexpr int OFF_RED = OFF_BIAS + BN * 4;
-constexpr int RED_FLOATS = 8 * (256 + 8) + 4 * 8;
+constexpr int RED_FLOATS = 4 * LG_TASK_ROWS + 6 * 8 + 2 * 64;  // rows' terms, row-group sums, active counts
 constexpr int OFF_BARS = OFF_RED + RED_FLOATS * 4;
 // full[STAGES], empty[STAGES], accf[2], acce[2], tqf[TQ], tqe[TQ], drain
 constexpr int NBARS = 2 * STAGES + 4 + 2 * TQ + 1;
 constexpr int OFF_TQ = OFF_BARS + NBARS * 8;
-constexpr int OFF_MISC = OFF_TQ + TQ * 8;
+constexpr int OFF_MISC = OFF_TQ + TQ * 12;
 constexpr int SMEM_BYTES = OFF_MISC + 64 + 1024;  // + 1024-byte alignment slack
 static_assert(24 + 4 * EPI_WARPS <= 64, "misc slots");
 static_assert(SMEM_BYTES <= 227 * 1024, "shared memory per CTA");
@@ -151,6 +152,9 @@ struct EpochP {
   int* cnt;
   int* err;
   float* loss;              // [nb, L] or null
+  // optional trace: per task (GEMM tasks first, then stream tasks) its
+  // dequeue, dependencies-met and done times (%globaltimer, ns) and SM id
+  unsigned long long* trace;
   LayerP lay[kMaxLayers];
 };
 
@@ -168,6 +172,15 @@ __device__ __forceinline__ void fence_proxy_async_global() {
   asm volatile("fence.proxy.async.global;" ::: "memory");
 }
 __device__ __forceinline__ void bulk_wait_all() { asm volatile("cp.async.bulk.wait_group 0;" ::: "memory"); }
+// Starts bringing [p, p + bytes) into L2 (16-byte aligned, in pieces of at
+// most 32 KB); nothing waits for it.
+__device__ __forceinline__ void prefetch_l2(const void* p, size_t bytes) {
+  const char* c = static_cast<const char*>(p);
+  for (size_t off = 0; off < bytes; off += 32768) {
+    const uint32_t n = (uint32_t)(bytes - off < 32768 ? bytes - off : 32768) & ~15u;
+    if (n) asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(c + off), "r"(n) : "memory");
+  }
+}
 
 __device__ __forceinline__ uint4 ldcg16(const void* p) { return __ldcg(reinterpret_cast<const uint4*>(p)); }
 
@@ -187,6 +200,10 @@ __device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t pa
       : "memory");
   return ok != 0;
 }
+__device__ __forceinline__ void st_remote_u1(int* local_slot, uint32_t rank, int v) {
+  const uint32_t a = ptx::mapa_shared(ptx::smem_u32(local_slot), rank);
+  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
+}
 __device__ __forceinline__ void st_remote_u2(uint2* local_slot, uint32_t rank, uint2 v) {
   const uint32_t a = ptx::mapa_shared(ptx::smem_u32(local_slot), rank);
   asm volatile("st.shared::cluster.v2.u32 [%0], {%1, %2};" ::"r"(a), "r"(v.x), "r"(v.y) : "memory");
@@ -201,16 +218,20 @@ __device__ __forceinline__ bool aborted(const EpochP& P) {
 }
 
 // Bounded wait on an mbarrier phase (cluster-scope acquire); false on abort
-// or timeout (the latter latched).
+// or timeout (the latter latched).  The abort flag lives in global memory, so
+// it is read only every 64th poll: a read in every poll would put an L2
+// round trip between a phase completing and the waiter seeing it.
 __device__ bool bar_wait(const EpochP& P, uint64_t* bar, uint32_t parity) {
   if (mbar_try_wait_cluster(bar, parity)) return true;
   const uint64_t t0 = ptx::globaltimer();
-  while (true) {
+  for (uint32_t n = 1;; ++n) {
     if (mbar_try_wait_cluster(bar, parity)) return true;
-    if (aborted(P)) return false;
-    if (ptx::globaltimer() - t0 > kWaitTimeoutNs) {
-      latch_abort(P);
-      return false;
+    if ((n & 63u) == 0) {
+      if (aborted(P)) return false;
+      if (ptx::globaltimer() - t0 > kWaitTimeoutNs) {
+        latch_abort(P);
+        return false;
+      }
     }
   }
 }
@@ -220,20 +241,40 @@ __device__ void bar_drain(uint64_t* bar, uint32_t parity, unsigned long long tim
   while (!mbar_try_wait_cluster(bar, parity))
     if (ptx::globaltimer() - t0 > timeout_ns) return;
 }
-// Bounded wait until counter >= target.
+// Bounded wait until counter >= target (the abort flag read every 16th poll).
 __device__ bool wait_count(const EpochP& P, int idx, int target) {
   const int* p = P.cnt + idx;
   if (ld_acquire(p) >= target) return true;
   const uint64_t t0 = ptx::globaltimer();
-  while (true) {
+  for (uint32_t n = 1;; ++n) {
     if (ld_acquire(p) >= target) return true;
-    if (aborted(P)) return false;
-    if (ptx::globaltimer() - t0 > kWaitTimeoutNs) {
-      latch_abort(P);
-      return false;
+    if ((n & 15u) == 0) {
+      if (aborted(P)) return false;
+      if (ptx::globaltimer() - t0 > kWaitTimeoutNs) {
+        latch_abort(P);
+        return false;
+      }
     }
-    __nanosleep(100);
   }
+}
+
+__device__ __forceinline__ uint32_t smid() {
+  uint32_t r;
+  asm volatile("mov.u32 %0, %%smid;" : "=r"(r));
+  return r;
+}
+// Trace words per task: GEMM tasks -- 0 dequeued, 1 dependencies met
+// (producer), 2 MMAs started, 3 last MMA issued, 4 epilogue started, 5 done;
+// stream tasks -- 0 dequeued, 1 dependencies met, 5 done; word 2 of a
+// stream task is its SM.
+}  // namespace
+constexpr int kTraceWords = 6;
+namespace {
+__device__ __forceinline__ void trace_at(const EpochP& P, int idx, int field) {
+  if (P.trace) P.trace[(size_t)idx * kTraceWords + field] = ptx::globaltimer();
+}
+__device__ __forceinline__ void trace_sm(const EpochP& P, int idx) {
+  if (P.trace) P.trace[(size_t)idx * kTraceWords + 2] = smid();
 }
 
 __device__ __forceinline__ uint32_t t_type(uint2 t) { return t.x & 7u; }
@@ -260,7 +301,7 @@ __device__ bool wait_deps(const EpochP& P, uint2 t) {
       // the input rows of this row tile, and their row scale
       if (k == 0) {
         if (!wait_count(P, c_ov(b % P.D, a), (BN / OV_ROWS) * (b / P.D + 1))) return false;
-      } else if (!wait_count(P, c_lgrt(k - 1, a), (BN / LG_ROWS) * (b + 1))) {
+      } else if (!wait_count(P, c_lgrt(k - 1, a), (BN / LG_TASK_ROWS) * (b + 1))) {
         return false;
       }
       // this column tile's rows of W and b after the previous batch's update
@@ -273,7 +314,7 @@ __device__ bool wait_deps(const EpochP& P, uint2 t) {
       return true;
     }
     case T_WG:
-      return wait_count(P, c_lgall(k), (b + 1) * (P.M / LG_ROWS));
+      return wait_count(P, c_lgall(k), (b + 1) * (P.M / LG_TASK_ROWS));
     case T_OV:
       if (b >= P.D) {
         const LayerP& l0 = P.lay[0];
@@ -281,7 +322,7 @@ __device__ bool wait_deps(const EpochP& P, uint2 t) {
       }
       return true;
     case T_LG:
-      return wait_count(P, c_fwd(k, a / (BN / LG_ROWS)), (b + 1) * 2 * P.lay[k].n_ct);
+      return wait_count(P, c_fwd(k, a / (BN / LG_TASK_ROWS)), (b + 1) * 2 * P.lay[k].n_ct);
     case T_ADAM:
       return wait_count(P, c_wgnt(k, a * ADAM_ROWS / BN), (b + 1) * 2 * P.lay[k].n_kt);
   }
@@ -298,7 +339,7 @@ __device__ void signal_done(const EpochP& P, uint2 t) {
       break;
     case T_OV: red_release_add(P.cnt + c_ov(t_batch(t) % P.D, a / (BN / OV_ROWS)), 1); break;
     case T_LG:
-      red_release_add(P.cnt + c_lgrt(k, a / (BN / LG_ROWS)), 1);
+      red_release_add(P.cnt + c_lgrt(k, a / (BN / LG_TASK_ROWS)), 1);
       red_release_add(P.cnt + c_lgall(k), 1);
       break;
     case T_ADAM: red_release_add(P.cnt + c_adam(k, a * ADAM_ROWS / BN), 1); break;
@@ -327,11 +368,14 @@ __device__ __forceinline__ void load_h8(const bf16* p, float (&v)[8]) {
 // s: streamer thread 0..NSTR-1 (s >> 5 its warp, lane its lane).
 
 // OV(b, r64): the label overlay of §3 for 64 rows of batch b, as k_overlay
-// (mode 0): features 0..9 <- one-hot(label), bf16 cast, row scale.
-__device__ void task_overlay(const EpochP& P, int b, int r64, int s) {
+// (mode 0): features 0..9 <- one-hot(label), bf16 cast, row scale.  A warp
+// takes a row; all of a lane's loads of the row are issued before its first
+// store (the row scale sums each lane's values in k_overlay's order).
+constexpr int OV_VEC_MAX = 8;  // float4 loads per lane and row: rows up to 4096 features
+__device__ __noinline__ void task_overlay(const EpochP& P, int b, int r64, int s) {
   const int y = s >> 5, lane = s & 31;
   const int F = P.K0, ldo = P.ldK0, slot = b % P.D;
-  const bool vec = (F & 3) == 0 && (reinterpret_cast<uintptr_t>(P.x) & 15u) == 0;
+  const bool vec = (F & 3) == 0 && (reinterpret_cast<uintptr_t>(P.x) & 15u) == 0 && ldo <= 128 * OV_VEC_MAX;
   for (int rr = y; rr < OV_ROWS; rr += STR_WARPS) {
     const int row = r64 * OV_ROWS + rr;
     const float* xr = P.xrp == 2 ? P.x + ((size_t)b * P.M + row) * F : P.x + ((size_t)b * P.B + row % P.B) * F;
@@ -339,12 +383,17 @@ __device__ void task_overlay(const EpochP& P, int b, int r64, int s) {
     const int lab = __ldg(P.labels + (size_t)b * P.M + row);
     float ss = 0.f;
     if (vec) {
-      for (int f = 4 * lane; f < ldo; f += 128) {
-        float v[4] = {0.f, 0.f, 0.f, 0.f};
-        if (f < F) {
-          const float4 q = __ldg(reinterpret_cast<const float4*>(xr + f));
-          v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
-        }
+      float4 q[OV_VEC_MAX];
+#pragma unroll
+      for (int it = 0; it < OV_VEC_MAX; ++it) {
+        const int f = 4 * lane + 128 * it;
+        q[it] = f < F ? __ldg(reinterpret_cast<const float4*>(xr + f)) : make_float4(0.f, 0.f, 0.f, 0.f);
+      }
+#pragma unroll
+      for (int it = 0; it < OV_VEC_MAX; ++it) {
+        const int f = 4 * lane + 128 * it;
+        if (f >= ldo) break;
+        float v[4] = {q[it].x, q[it].y, q[it].z, q[it].w};
 #pragma unroll
         for (int u = 0; u < 4; ++u) {
           if (f + u < 10) v[u] = (f + u == lab) ? 1.f : 0.f;
@@ -367,155 +416,156 @@ __device__ void task_overlay(const EpochP& P, int b, int r64, int s) {
   }
 }
 
-// LG(k, b, rb): the local gradient of 32 rows, for every 256-column block the
-// computation of one k_grad_prep block (same thread mapping and orders).
-__device__ void task_local_grad(const EpochP& P, int k, int b, int rb, int s, float* smem_red) {
+// LG(k, b, t): the local gradient of rows [64t, 64t + 64) -- two 32-row
+// blocks, each what the 256-column blocks of k_grad_prep compute for it, with
+// the same reduction orders:
+//   1. warps 0..15 (per block, k_grad_prep's 8 row groups ty with 8 lanes per
+//      row) sum each row's goodness partials and form dL/dg, the next layer's
+//      scale and the row's loss and goodness terms (summed per row group,
+//      then over the groups in order);
+//   2. every streamer thread takes (block, 8-column chunk) items: dZ' =
+//      (s 2 dL/dg) h for the block's 32 rows, and the bias-gradient partial of
+//      each column as k_grad_prep sums it (per row group its 4 rows in
+//      order, then the 8 groups in order).
+__device__ __noinline__ void task_local_grad(const EpochP& P, int k, int b, int t, int s, float* smem_red) {
   const LayerP& lp = P.lay[k];
   const int slot = b % P.D;
   const int M = P.M, N = lp.N, ld = lp.ldN;
   const int ntiles = 2 * lp.n_ct;
   const int nrb = M / LG_ROWS, ncb = (ld + 255) / 256;
+  constexpr int NBLK = LG_TASK_ROWS / LG_ROWS;
   const bf16* H = lp.h_ring + (size_t)slot * M * ld;
   const float* gpart = lp.g_ring + (size_t)slot * ntiles * M;
   const float* sin = lp.s_in_ring + (size_t)slot * M;
   float* s_next = lp.sn_ring ? lp.sn_ring + (size_t)slot * M : nullptr;
-  float (*red)[256 + 8] = reinterpret_cast<float (*)[256 + 8]>(smem_red);
-  float* lred = smem_red + 8 * (256 + 8);
-  float* gpred = lred + 8;
-  float* gnred = gpred + 8;
-  float* ared = gnred + 8;
-  // The 8 row groups (ty) of a k_grad_prep block run on the STR_WARPS warps
-  // in turn; each group's sums are formed alone and combined in the same
-  // fixed order afterwards.
-  const int wy = s >> 5, lane = s & 31;
-  const int r0 = rb * LG_ROWS;
-  for (int cb = 0; cb < ncb; ++cb) {
-    const bool lead = cb == 0;
-    const int cg = cb * 256 + lane * 8;
-    const bool cols_ok = cg < ld;
-    for (int ty = wy; ty < 8; ty += STR_WARPS) {
-      float h[4][8];
+  float* sc_row = smem_red;                    // [64] s_i * 2 dL/dg_i
+  float* c_row = sc_row + LG_TASK_ROWS;        // [64] 2 dL/dg_i
+  float* lred = c_row + LG_TASK_ROWS;          // [2][8] per block and row group: loss
+  float* gpred = lred + NBLK * 8;              // positive rows' goodness
+  float* gnred = gpred + NBLK * 8;             // negative rows' goodness
+  int* actc = reinterpret_cast<int*>(gnred + NBLK * 8);  // [2][64] active ReLUs per block and 256-column block
+  const int w = s >> 5, lane = s & 31;
+  const int r0 = t * LG_TASK_ROWS;
+  for (int i = s; i < NBLK * 64; i += NSTR) actc[i] = 0;
+  if (w < NBLK * 8) {
+    const int blk = w >> 3, ty = w & 7, q = lane >> 3, p = lane & 7;
+    const int lr = blk * LG_ROWS + ty + 8 * q;  // row within the task
+    const int i = r0 + lr;
+    float g = 0.f;
+    float v[8];
+#pragma unroll
+    for (int u = 0; u < 8; ++u) {
+      const int tt = p + 8 * u;
+      v[u] = tt < ntiles ? __ldcg(gpart + (size_t)tt * M + i) : 0.f;
+    }
+    for (int tt = p + 64; tt < ntiles; tt += 8) v[0] += __ldcg(gpart + (size_t)tt * M + i);
+#pragma unroll
+    for (int u = 0; u < 8; ++u) g += v[u];
+    g += __shfl_xor_sync(0xffffffffu, g, 4);
+    g += __shfl_xor_sync(0xffffffffu, g, 2);
+    g += __shfl_xor_sync(0xffffffffu, g, 1);
+    float lv = 0.f, gp = 0.f, gn = 0.f;
+    if (p == 0) {
+      const bool pos = i < P.B;
+      const float tt = pos ? lp.theta - g : g - lp.theta;
+      const float sg = sigmoid_f(tt);
+      const float cc = 2.f * (pos ? -sg : sg) / (float)P.B;
+      c_row[lr] = cc;
+      sc_row[lr] = __ldcg(sin + i) * cc;
+      if (!isfinite(g)) atomicOr(&lp.ds->err, DEVERR_NONFINITE);
+      if (s_next) s_next[i] = inv_norm(g);
+      lv = softplus_f(tt);
+      (pos ? gp : gn) = g;
+    }
+    lv = warp_sum(lv);
+    gp = warp_sum(gp);
+    gn = warp_sum(gn);
+    if (lane == 0) {
+      lred[w] = lv;
+      gpred[w] = gp;
+      gnred[w] = gn;
+    }
+  }
+  ptx::named_bar(BAR_STR, NSTR);
+  if (s < NBLK) {
+    const int rb = t * NBLK + s;
+    float tl = 0.f, tp = 0.f, tn = 0.f;
+#pragma unroll
+    for (int yy = 0; yy < 8; ++yy) {
+      tl += lred[s * 8 + yy];
+      tp += gpred[s * 8 + yy];
+      tn += gnred[s * 8 + yy];
+    }
+    lp.loss_part[rb] = tl;
+    lp.stat_part[rb] = tp;
+    lp.stat_part[nrb + rb] = tn;
+    if (rb == 0) {
+      // the Adam update that follows is step t; beta^t kept as running
+      // products (read around L1: other SMs wrote them earlier in this launch)
+      ff_dev_state* ds = lp.ds;
+      const double p1 = __ldcg(&ds->pow1) * lp.beta1d, p2 = __ldcg(&ds->pow2) * lp.beta2d;
+      ds->t = __ldcg(&ds->t) + 1;
+      ds->pow1 = p1;
+      ds->pow2 = p2;
+      ds->bc1 = (float)(1.0 - p1);
+      ds->bc2 = (float)(1.0 - p2);
+    }
+  }
+  const int nch = ld / 8;  // 8-column chunks (ld is a multiple of 8)
+  for (int item = s; item < NBLK * nch; item += NSTR) {
+    const int blk = item / nch, ch = item - blk * nch;
+    const int cg = 8 * ch, rb0 = r0 + blk * LG_ROWS, lb = blk * LG_ROWS;
+    // row group y holds rows y, y + 8, y + 16, y + 24 of the block (kept
+    // packed: 8 bf16 in 4 registers; the many streamer threads keep enough
+    // of these loads in flight)
+    auto load_group = [&](int y, uint4 (&hv)[4]) {
+#pragma unroll
+      for (int q = 0; q < 4; ++q) hv[q] = ldcg16(H + (size_t)(rb0 + y + 8 * q) * ld + cg);
+    };
+    float tsum[8];
+#pragma unroll
+    for (int e = 0; e < 8; ++e) tsum[e] = 0.f;
+    int act = 0;
+    auto use_group = [&](int y, const uint4 (&hp)[4]) {
+      float acc[8];
+#pragma unroll
+      for (int e = 0; e < 8; ++e) acc[e] = 0.f;
 #pragma unroll
       for (int q = 0; q < 4; ++q) {
-        const int i = r0 + ty + 8 * q;
-        if (cols_ok) {
-          load_h8(H + (size_t)i * ld + cg, h[q]);
-        } else {
+        const float ck = c_row[lb + y + 8 * q], sk = sc_row[lb + y + 8 * q];
+        const __nv_bfloat162* h2 = reinterpret_cast<const __nv_bfloat162*>(&hp[q]);
+        uint4 outp;
+        __nv_bfloat162* o2 = reinterpret_cast<__nv_bfloat162*>(&outp);
 #pragma unroll
-          for (int e = 0; e < 8; ++e) h[q][e] = 0.f;
+        for (int e = 0; e < 4; ++e) {
+          const float2 f = __bfloat1622float2(h2[e]);
+          acc[2 * e] = fmaf(ck, f.x, acc[2 * e]);
+          acc[2 * e + 1] = fmaf(ck, f.y, acc[2 * e + 1]);
+          act += (f.x > 0.f ? 1 : 0) + (f.y > 0.f ? 1 : 0);
+          o2[e] = __floats2bfloat162_rn(sk * f.x, sk * f.y);
         }
-      }
-      float cc = 0.f, sc = 0.f, lv = 0.f, gp = 0.f, gn = 0.f;
-      {
-        const int q = lane >> 3, p = lane & 7;
-        const int i = r0 + ty + 8 * q;
-        float g = 0.f;
-        float v[8];
-#pragma unroll
-        for (int u = 0; u < 8; ++u) {
-          const int t = p + 8 * u;
-          v[u] = t < ntiles ? __ldcg(gpart + (size_t)t * M + i) : 0.f;
-        }
-        for (int t = p + 64; t < ntiles; t += 8) v[0] += __ldcg(gpart + (size_t)t * M + i);
-#pragma unroll
-        for (int u = 0; u < 8; ++u) g += v[u];
-        g += __shfl_xor_sync(0xffffffffu, g, 4);
-        g += __shfl_xor_sync(0xffffffffu, g, 2);
-        g += __shfl_xor_sync(0xffffffffu, g, 1);
-        if (p == 0) {
-          const bool pos = i < P.B;
-          const float tt = pos ? lp.theta - g : g - lp.theta;
-          const float sg = sigmoid_f(tt);
-          cc = 2.f * (pos ? -sg : sg) / (float)P.B;
-          sc = __ldcg(sin + i) * cc;
-          if (lead) {
-            if (!isfinite(g)) atomicOr(&lp.ds->err, DEVERR_NONFINITE);
-            if (s_next) s_next[i] = inv_norm(g);
-            lv = softplus_f(tt);
-            (pos ? gp : gn) = g;
-          }
-        }
-      }
-      float db[8];
-#pragma unroll
-      for (int e = 0; e < 8; ++e) db[e] = 0.f;
-#pragma unroll
-      for (int q = 0; q < 4; ++q) {
-        const float ck = __shfl_sync(0xffffffffu, cc, 8 * q), sk = __shfl_sync(0xffffffffu, sc, 8 * q);
-        const int i = r0 + ty + 8 * q;
-        float z[8];
-#pragma unroll
-        for (int e = 0; e < 8; ++e) {
-          z[e] = sk * h[q][e];
-          db[e] = fmaf(ck, h[q][e], db[e]);
-        }
-        if (cols_ok) Vec8<bf16>::store(lp.dZ + (size_t)i * ld + cg, z);
-      }
-      if (lead) {
-        lv = warp_sum(lv);
-        gp = warp_sum(gp);
-        gn = warp_sum(gn);
-        if (lane == 0) {
-          lred[ty] = lv;
-          gpred[ty] = gp;
-          gnred[ty] = gn;
-        }
-      }
-      {
-        float act = 0.f;
-#pragma unroll
-        for (int q = 0; q < 4; ++q)
-#pragma unroll
-          for (int e = 0; e < 8; ++e) act += h[q][e] > 0.f ? 1.f : 0.f;
-        act = warp_sum(act);
-        if (lane == 0) ared[ty] = act;
+        *reinterpret_cast<uint4*>(lp.dZ + (size_t)(rb0 + y + 8 * q) * ld + cg) = outp;
       }
 #pragma unroll
-      for (int e = 0; e < 8; ++e) red[ty][lane * 8 + e] = db[e];
+      for (int e = 0; e < 8; ++e) tsum[e] += acc[e];
+    };
+#pragma unroll 1
+    for (int y = 0; y < 8; ++y) {
+      uint4 hv[4];
+      load_group(y, hv);
+      use_group(y, hv);
     }
-    ptx::named_bar(BAR_STR, NSTR);
-    if (wy == 0) {
+    const int rb = t * NBLK + blk;
 #pragma unroll
-      for (int e = 0; e < 8; ++e) {
-        const int j = cg + e;
-        float t = 0.f;
-#pragma unroll
-        for (int yy = 0; yy < 8; ++yy) t += red[yy][lane * 8 + e];
-        if (j < N) lp.dbpart[(size_t)rb * N + j] = t;
-      }
-      if (lane == 0) {
-        float t = 0.f;
-#pragma unroll
-        for (int yy = 0; yy < 8; ++yy) t += ared[yy];
-        lp.stat_part[2 * nrb + (size_t)rb * ncb + cb] = t;
-      }
-      if (lead && lane == 0) {
-        float t = 0.f;
-#pragma unroll
-        for (int yy = 0; yy < 8; ++yy) t += lred[yy];
-        lp.loss_part[rb] = t;
-        float tp = 0.f, tn = 0.f;
-#pragma unroll
-        for (int yy = 0; yy < 8; ++yy) {
-          tp += gpred[yy];
-          tn += gnred[yy];
-        }
-        lp.stat_part[rb] = tp;
-        lp.stat_part[nrb + rb] = tn;
-      }
-      if (lead && rb == 0 && lane == 0) {
-        // the Adam update that follows is step t; beta^t kept as running
-        // products (read around L1: other SMs wrote them earlier in this launch)
-        ff_dev_state* ds = lp.ds;
-        const double p1 = __ldcg(&ds->pow1) * lp.beta1d, p2 = __ldcg(&ds->pow2) * lp.beta2d;
-        ds->t = __ldcg(&ds->t) + 1;
-        ds->pow1 = p1;
-        ds->pow2 = p2;
-        ds->bc1 = (float)(1.0 - p1);
-        ds->bc2 = (float)(1.0 - p2);
-      }
-    }
-    ptx::named_bar(BAR_STR, NSTR);  // red / lred reused by the next column block
+    for (int e = 0; e < 8; ++e)
+      if (cg + e < N) lp.dbpart[(size_t)rb * N + cg + e] = tsum[e];
+    // active ReLUs per 256-column block: whole counts, exact in any order
+    if (act) atomicAdd(&actc[blk * 64 + ch / 32], act);
+  }
+  ptx::named_bar(BAR_STR, NSTR);
+  for (int i = s; i < NBLK * ncb; i += NSTR) {
+    const int blk = i / ncb, cb = i - blk * ncb;
+    lp.stat_part[2 * nrb + (size_t)(t * NBLK + blk) * ncb + cb] = (float)actc[blk * 64 + cb];
   }
 }
 
@@ -538,7 +588,7 @@ __device__ __forceinline__ void st_stream8(float* p, const float (&v)[8]) {
 // ADAM(k, b, c): Adam (§5.1) on rows [16c, 16c + 16) of W and of b, as k_adam
 // does it element by element (same bias-gradient reduction order); chunk 0
 // also forms the step's loss and statistics.
-__device__ void task_adam(const EpochP& P, int k, int b, int c, int s) {
+__device__ __noinline__ void task_adam(const EpochP& P, int k, int b, int c, int s) {
   const LayerP& lp = P.lay[k];
   const int K = lp.K, N = lp.N;
   const int n0 = c * ADAM_ROWS, n1 = n0 + ADAM_ROWS < N ? n0 + ADAM_ROWS : N;
@@ -547,8 +597,8 @@ __device__ void task_adam(const EpochP& P, int k, int b, int c, int s) {
   const long long base = (long long)n0 * K, end = (long long)n1 * K;
   const long long total = (long long)N * K;
   // 8 parameters per thread and array per step (K % 8 == 0: every chunk
-  // starts and ends on 8), two steps in flight
-  constexpr int U = 2;
+  // starts and ends on 8)
+  constexpr int U = 1;
   for (long long q0 = base / 8 + s; q0 * 8 < end; q0 += NSTR * U) {
     float w[U][8], m[U][8], v[U][8], g[U][8];
 #pragma unroll
@@ -650,6 +700,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
   uint64_t* tqe = tqf + TQ;
   uint64_t* drain = tqe + TQ;
   uint2* tq = reinterpret_cast<uint2*>(smem + OFF_TQ);
+  int* tqi = reinterpret_cast<int*>(smem + OFF_TQ + TQ * 8);  // [TQ] the tasks' indices (trace)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(smem + OFF_MISC);
   uint2* stask_slot = reinterpret_cast<uint2*>(smem + OFF_MISC + 8);
   volatile int* evote = reinterpret_cast<volatile int*>(smem + OFF_MISC + 24);  // [EPI_WARPS]
@@ -700,6 +751,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
           if (!bar_wait(P, &tqe[j], ph ^ 1u)) break;
           const int idx = atomicAdd(P.cnt + C_QG, 1);
           task = idx < P.n_gtask ? __ldg(P.gtask + idx) : make_uint2(T_END, 0u);
+          if (idx < P.n_gtask) {
+            trace_at(P, idx, 0);
+            tqi[j] = idx;
+            st_remote_u1(&tqi[j], 1u, idx);
+          }
           tq[j] = task;
           st_remote_u2(&tq[j], 1u, task);
           ptx::mbar_arrive(&tqf[j]);
@@ -711,6 +767,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
         }
         if (t_type(task) == T_END) break;
         if (!wait_deps(P, task)) break;
+        if (even) trace_at(P, tqi[j], 1);
         fence_proxy_async_global();
         const int k = t_layer(task), b = t_batch(task), a = t_a(task), c = t_c(task);
         const LayerP& lp = P.lay[k];
@@ -779,11 +836,13 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
         const int j = i % TQ;
         if (!bar_wait(P, &tqf[j], (uint32_t)(i / TQ) & 1u)) break;
         const uint2 task = tq[j];
+        const int tidx = tqi[j];
         ptx::mbar_arrive(&tqe[j]);
         if (t_type(task) == T_END) break;
         const int buf = i & 1;
         if (!bar_wait(P, &acce[buf], ((uint32_t)(i >> 1) & 1u) ^ 1u)) break;
         ptx::tc_fence_after();
+        trace_at(P, tidx, 2);
         const bool fwd = t_type(task) == T_FWD;
         const LayerP& lp = P.lay[t_layer(task)];
         const int nkb = fwd ? (lp.K + BK - 1) / BK : P.M / BK;
@@ -815,6 +874,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
         }
         if (!ok) break;
         ptx::umma_commit_pair(&accf[buf], pmask);
+        trace_at(P, tidx, 3);
       }
       // every MMA issued so far has completed before TMEM can be released
       if (issued_any) {
@@ -824,14 +884,15 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
     }
   } else if (warp < STR0) {
     // ------------------------------------------------------ epilogue
+    // Warp w reads TMEM lane quarter q = w % 4 (rows 32q.. of this CTA's 128)
+    // over both 128-column halves in turn, each half with its own goodness
+    // partial (the per-128-column partials of the per-step forward GEMM).
     const int q = warp & 3;
     const int ew = warp - EPI0;
-    const int half = ew / 4;
-    const int cbase = half * (BN / 2);
     uint8_t* stage = smem + OFF_EPI + ew * EPI_BYTES;
     const uint32_t sw = (uint32_t)(lane & 7);
-    // Named barriers among the 8 epilogue warps must be reached by all of
-    // them or by none: every go/stop decision after a bounded wait is a vote.
+    // Named barriers among the epilogue warps must be reached by all of them
+    // or by none: every go/stop decision after a bounded wait is a vote.
     auto vote = [&](bool ok) {
       ok = __all_sync(0xffffffffu, ok);
       if (lane == 0) evote[ew] = ok ? 1 : 0;
@@ -846,6 +907,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
       const int j = i % TQ;
       const bool got = bar_wait(P, &tqf[j], (uint32_t)(i / TQ) & 1u);
       const uint2 task = got ? tq[j] : make_uint2(T_END, 0u);
+      const int tidx = got ? tqi[j] : 0;  // read before the slot is released
       __syncwarp();
       if (got && lane == 0) {
         if (even)
@@ -874,17 +936,25 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
       }
       const bool ready = bar_wait(P, &accf[buf], (uint32_t)(i >> 1) & 1u);
       ptx::tc_fence_after();
-      if (vote(ready)) {
+      if (!vote(ready)) break;
+      if (even && warp == EPI0 && lane == 0) trace_at(P, tidx, 4);
+      const CUtensorMap* mC = lp.tm + (fwd ? TM_FWD_C : TM_WG_C);
+      int fchunk = 0;
+#pragma unroll 1
+      for (int hh = 0; hh < 2; ++hh) {
+        const int cbase = hh * (BN / 2);
         const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(buf * BN + cbase);
         float g = 0.f;
-        int fchunk = 0;
-        const CUtensorMap* mC = lp.tm + (fwd ? TM_FWD_C : TM_WG_C);
-        auto process = [&](const uint32_t (&r)[32], int c0) {
-          if (fwd) {
-            uint32_t packed[16];
+        if (fwd) {
+          // 16 columns at a time (a 16-column TMEM load), the next load in
+          // flight while these are used: H = ReLU(s acc + b) to bf16 in the
+          // 128-byte-swizzled staging, goodness from the fp32 values in
+          // column order
+          auto process = [&](const uint32_t (&r)[16], int c0) {
+            uint32_t packed[8];
             const float4* b4 = reinterpret_cast<const float4*>(sbias + cbase + c0);
 #pragma unroll
-            for (int v = 0; v < 8; ++v) {
+            for (int v = 0; v < 4; ++v) {
               const float4 bb = b4[v];
               const float bv[4] = {bb.x, bb.y, bb.z, bb.w};
               float h[4];
@@ -899,24 +969,57 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
               packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
               packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
             }
-            uint8_t* base = stage + (c0 / 64) * (32 * 128) + lane * 128;
+            uint8_t* base = stage + hh * 8192 + (c0 / 64) * (32 * 128) + lane * 128;
 #pragma unroll
-            for (int v = 0; v < 4; ++v) {
+            for (int v = 0; v < 2; ++v) {
               const uint32_t jj = (uint32_t)((c0 % 64) / 8 + v);
               *reinterpret_cast<uint4*>(base + ((jj ^ sw) << 4)) =
                   make_uint4(packed[4 * v], packed[4 * v + 1], packed[4 * v + 2], packed[4 * v + 3]);
             }
-          } else {
-            // fp32 dW: chunk n through slot n & 1, refilled once the store
-            // issued from it two chunks ago has read it
+          };
+          uint32_t ra[16], rb[16];
+          ptx::tmem_ld16(trow, ra);
+          ptx::tmem_ld_wait();
+#pragma unroll 1
+          for (int c0 = 0; c0 < BN / 2; c0 += 32) {
+            ptx::tmem_ld16(trow + (uint32_t)(c0 + 16), rb);
+            process(ra, c0);
+            ptx::tmem_ld_wait();
+            if (c0 + 32 < BN / 2) ptx::tmem_ld16(trow + (uint32_t)(c0 + 32), ra);
+            process(rb, c0 + 16);
+            ptx::tmem_ld_wait();
+            if (c0 % 64 == 32) {
+              // a full 64-column box: out to the activity ring
+              ptx::fence_async_smem();
+              __syncwarp();
+              const int col = n0 + cbase + c0 - 32;
+              if (lane == 0) {
+                if (col < lp.ldN) ptx::tma_store_2d(mC, stage + hh * 8192 + (c0 / 64) * (32 * 128), col, slot * P.M + rloc);
+                ptx::bulk_commit();
+              }
+            }
+          }
+        } else {
+          // fp32 dW, 32 columns (one 4 KB box) at a time through slot n & 1,
+          // refilled once the store issued from it two boxes ago has read it
+#pragma unroll 1
+          for (int c0 = 0; c0 < BN / 2; c0 += 32) {
+            uint32_t ra[16], rb[16];
+            ptx::tmem_ld16(trow + (uint32_t)c0, ra);
+            ptx::tmem_ld16(trow + (uint32_t)(c0 + 16), rb);
             uint8_t* sbuf = stage + (fchunk & 1) * 4096;
             if (lane == 0 && fchunk >= 2) ptx::bulk_wait_read1();
             __syncwarp();
+            ptx::tmem_ld_wait();
             uint8_t* base = sbuf + lane * 128;
 #pragma unroll
-            for (int v = 0; v < 8; ++v)
+            for (int v = 0; v < 4; ++v)
               *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
-                  make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+                  make_uint4(ra[4 * v], ra[4 * v + 1], ra[4 * v + 2], ra[4 * v + 3]);
+#pragma unroll
+            for (int v = 0; v < 4; ++v)
+              *reinterpret_cast<uint4*>(base + (((uint32_t)(v + 4) ^ sw) << 4)) =
+                  make_uint4(rb[4 * v], rb[4 * v + 1], rb[4 * v + 2], rb[4 * v + 3]);
             ptx::fence_async_smem();
             __syncwarp();
             const int col0 = n0 + cbase + c0;
@@ -924,64 +1027,57 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
             if (lane == 0) ptx::bulk_commit();
             ++fchunk;
           }
-        };
-        uint32_t ra[32], rb[32];
-        ptx::tmem_ld32(trow, ra);
-        ptx::tmem_ld_wait();
-#pragma unroll 1
-        for (int c0 = 0; c0 < BN / 2; c0 += 64) {
-          ptx::tmem_ld32(trow + (uint32_t)(c0 + 32), rb);
-          process(ra, c0);
-          ptx::tmem_ld_wait();
-          if (c0 + 64 < BN / 2) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
-          process(rb, c0 + 32);
-          ptx::tmem_ld_wait();
         }
-        // TMEM of this buffer is read: the MMA may refill it
-        ptx::tc_fence_before();
-        __syncwarp();
-        if (lane == 0) {
-          if (even)
-            ptx::mbar_arrive(&acce[buf]);
-          else
-            mbar_arrive_remote(&acce[buf], 0u);
-        }
-        if (fwd) {
-          lp.g_ring[((size_t)slot * 2 * lp.n_ct + (size_t)(c * 2 + half)) * P.M + rloc + lane] = g;
-          ptx::fence_async_smem();
-          __syncwarp();
-          if (lane == 0) {
-#pragma unroll 1
-            for (int ch = 0; ch < (BN / 2) / 64; ++ch) {
-              const int col = n0 + cbase + ch * 64;
-              if (col < lp.ldN) ptx::tma_store_2d(mC, stage + ch * (32 * 128), col, slot * P.M + rloc);
-            }
-            ptx::bulk_commit();
-          }
-        }
-        // the task's outputs are written (TMA stores complete) before it is
-        // counted done
-        if (lane == 0) {
-          bulk_wait_all();
-          fence_proxy_async_global();
-        }
-        __threadfence();
-        ptx::named_bar(BAR_EPI, 32 * EPI_WARPS);
-        if (warp == EPI0 && lane == 0) signal_done(P, task);
-      } else {
-        break;
+        if (fwd) lp.g_ring[((size_t)slot * 2 * lp.n_ct + (size_t)(c * 2 + hh)) * P.M + rloc + lane] = g;
+      }
+      // TMEM of this buffer is read: the MMA may refill it
+      ptx::tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (even)
+          ptx::mbar_arrive(&acce[buf]);
+        else
+          mbar_arrive_remote(&acce[buf], 0u);
+      }
+      // the task's outputs are written (TMA stores complete) before it is
+      // counted done
+      if (lane == 0) {
+        bulk_wait_all();
+        fence_proxy_async_global();
+      }
+      __threadfence();
+      ptx::named_bar(BAR_EPI, 32 * EPI_WARPS);
+      if (warp == EPI0 && lane == 0) {
+        signal_done(P, task);
+        if (even) trace_at(P, tidx, 5);
       }
     }
     if (lane == 0) bulk_wait_all();
   } else {
     // ----------------------------------------------------- streamers
     const int s = (int)threadIdx.x - 32 * STR0;
+    int sidx = 0;
     for (int i = 0;; ++i) {
       uint2* slotp = stask_slot + (i & 1);
       if (s == 0) {
         const int idx = atomicAdd(P.cnt + C_QS, 1);
         uint2 t = idx < P.n_stask ? __ldg(P.stask + idx) : make_uint2(T_END, 0u);
+        sidx = P.n_gtask + idx;
+        if (t_type(t) != T_END) trace_at(P, sidx, 0);
+        // the operands that do not wait on this batch start their way into
+        // L2 now: an Adam chunk's W and moments, an overlay block's images
+        if (t_type(t) == T_ADAM) {
+          const LayerP& lp = P.lay[t_layer(t)];
+          const int n0 = t_a(t) * ADAM_ROWS, n1 = n0 + ADAM_ROWS < lp.N ? n0 + ADAM_ROWS : lp.N;
+          const size_t off = (size_t)n0 * lp.K, bytes = (size_t)(n1 - n0) * lp.K * 4;
+          prefetch_l2(lp.W + off, bytes);
+          prefetch_l2(lp.mW + off, bytes);
+          prefetch_l2(lp.vW + off, bytes);
+        } else if (t_type(t) == T_OV && P.xrp == 2 && (P.K0 & 3) == 0) {
+          prefetch_l2(P.x + ((size_t)t_batch(t) * P.M + (size_t)t_a(t) * OV_ROWS) * P.K0, (size_t)OV_ROWS * P.K0 * 4);
+        }
         if (t_type(t) != T_END && !wait_deps(P, t)) t = make_uint2(T_END, 0u);
+        if (t_type(t) != T_END) trace_at(P, sidx, 1);
         *slotp = t;
       }
       ptx::named_bar(BAR_STR, NSTR);
@@ -994,7 +1090,11 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
       }
       __threadfence();
       ptx::named_bar(BAR_STR, NSTR);
-      if (s == 0) signal_done(P, t);
+      if (s == 0) {
+        signal_done(P, t);
+        trace_at(P, sidx, 5);
+        trace_sm(P, sidx);
+      }
     }
   }
 
@@ -1010,6 +1110,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
 // ------------------------------------------------------------------- host
 struct EpochPlan {
   int B = 0, nb = 0, xrp = 0;
+  unsigned long long* trace = nullptr;  // [4 * (GEMM + stream tasks)] when tracing
   std::vector<void*> ws;   // each layer's workspace when the plan was built
   void* mem = nullptr;
   EpochP P{};
@@ -1019,6 +1120,7 @@ struct EpochPlan {
 
 void epoch_plan_free(EpochPlan* p) {
   if (!p) return;
+  dev_free(p->trace);
   dev_free(p->mem);
   delete p;
 }
@@ -1052,7 +1154,7 @@ ff_status build_plan(ff_net* n, int B, int nb, int xrp, cudaStream_t st, EpochPl
     for (int k = 0; k < L; ++k) {
       const int b = tau - k;
       if (b < 0 || b >= nb) continue;
-      for (int rb = 0; rb < M / LG_ROWS; ++rb) stt.push_back(mk_task(T_LG, k, b, rb, 0));
+      for (int rb = 0; rb < M / LG_TASK_ROWS; ++rb) stt.push_back(mk_task(T_LG, k, b, rb, 0));
     }
     for (int k = 0; k < L; ++k) {
       const int b = tau - k;
@@ -1247,6 +1349,12 @@ ff_status net_train_epoch(ff_net* n, const float* x, const int* labels, int n_pa
       p = n->epoch;
     }
     EpochP P = p->P;
+    if (n->epoch_trace && !p->trace) {
+      const size_t bytes = (size_t)kTraceWords * (p->P.n_gtask + p->P.n_stask) * sizeof(unsigned long long);
+      FF_TRY(dev_alloc(reinterpret_cast<void**>(&p->trace), bytes), "epoch trace");
+      FF_TRY(cudaMemsetAsync(p->trace, 0, bytes, st), "epoch trace");
+    }
+    P.trace = n->epoch_trace ? p->trace : nullptr;
     P.x = x;
     P.labels = labels;
     P.loss = loss;
@@ -1309,4 +1417,21 @@ extern "C" FF_API ff_status ff_net_train_epoch(ff_net* n, const float* x, const 
     return ff_net_sync(n, stream);
   }
   return ff::net_train_epoch(n, x, labels, n_pairs, B, images_per_pair_row, loss, st);
+}
+
+extern "C" FF_API long long ff_net_epoch_trace(ff_net* n, int enable, unsigned long long* out, long long capacity) {
+  if (!n) return -1;
+  if (enable >= 0) n->epoch_trace = enable != 0;
+  if (!out) return 0;
+  ff::EpochPlan* p = n->epoch;
+  if (!p || !p->trace || capacity < 2) return 0;
+  const long long recs = (long long)p->P.n_gtask + p->P.n_stask;
+  long long words = ff::kTraceWords * recs;
+  if (words > capacity - 2) words = (capacity - 2) / ff::kTraceWords * ff::kTraceWords;
+  if (cudaDeviceSynchronize() != cudaSuccess) return -1;
+  out[0] = (unsigned long long)p->P.n_gtask;
+  out[1] = (unsigned long long)p->P.n_stask;
+  if (cudaMemcpy(out + 2, p->trace, (size_t)words * sizeof(unsigned long long), cudaMemcpyDeviceToHost) != cudaSuccess)
+    return -1;
+  return words + 2;
 }

@@ -35,5 +35,6 @@ struct ff_net {
   std::vector<cudaEvent_t> lab_done;
   // the persistent train-epoch plan (ff_net_train_epoch), built on first use
   ff::EpochPlan* epoch = nullptr;
+  bool epoch_trace = false;  // record per-task times in the epoch kernel (ff_net_epoch_trace)
 };
 

@@ -94,6 +94,7 @@ def lib():
             "ff_net_train_step_images": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_net_sync": [c_void_p, c_void_p],
             "ff_net_train_epoch": [c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p],
+            "ff_net_epoch_trace": [c_void_p, c_int, c_void_p, c_longlong],
             "ff_net_create_po": [c_void_p, c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
             "ff_net_po_train_step": [c_void_p, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
             "ff_forward_noalloc": [c_void_p, c_void_p, c_void_p, c_void_p, c_int, c_int, c_int, c_void_p, c_void_p,
@@ -353,6 +354,24 @@ class Net:
                                         int(n_pairs), int(B), int(images_per_pair_row),
                                         _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
                "ff_net_train_epoch")
+
+    def epoch_trace(self, enable=None):
+        """ff_net_epoch_trace: with enable=True/False switches per-task tracing
+        of later train_epoch calls; returns the last traced epoch as
+        (gemm [G, 6], stream [S, 6]) uint64 arrays (see include/ff.h), or None."""
+        L = lib()
+        L.ff_net_epoch_trace.restype = c_longlong
+        if enable is not None:
+            L.ff_net_epoch_trace(self._h, 1 if enable else 0, None, 0)
+            return None
+        cap = 2 + 6 * (1 << 22)
+        buf = np.zeros(cap, np.uint64)
+        n = L.ff_net_epoch_trace(self._h, -1, buf.ctypes.data, cap)
+        if n < 2:
+            return None
+        g, st = int(buf[0]), int(buf[1])
+        rec = buf[2:n].reshape(-1, 6)
+        return rec[:g], rec[g:g + st]
 
     def sync(self, stream=None):
         _check(lib().ff_net_sync(self._h, c_void_p(_stream(stream))), "ff_net_sync")
