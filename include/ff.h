@@ -74,7 +74,7 @@ typedef struct {
                         fp32 accumulate, fp32 master weights and moments */
   unsigned long long init_seed; /* W ~ U(+-sqrt(6/K)) from this seed; b = 0 */
   int max_rows;      /* workspace capacity in rows (2B); grows on demand if exceeded */
-  int keep_grad;     /* 1: keep dW, db of the last train step for ff_layer_get_grad */
+  int keep_grad;     /* 1: keep dW, db and the operand G of the last train step (ff_layer_get_grad, _operand) */
 } ff_layer_config;
 
 typedef struct ff_layer ff_layer; /* opaque */
@@ -339,6 +339,17 @@ FF_API ff_status ff_layer_get_stats(const ff_layer* layer, float* stats);
  * or device pointers; NULL skips).  Needs cfg.keep_grad = 1, else
  * FF_ERR_UNSUPPORTED.  Synchronous. */
 FF_API ff_status ff_layer_get_grad(const ff_layer* layer, float* dW, float* db);
+
+/* The weight-gradient operand of the last train step (of ff_layer_train_step
+ * or ff_po_train_step): G = diag(s) dZ, the local gradient scaled by each
+ * row's input scale, rows [rows, ff_row_stride(out_features)] in the layer's
+ * operand type (bf16 in FF_BF16 mode, rounded to nearest even as the
+ * weight-gradient GEMM reads it; fp32 otherwise), so that dW = G^T x.
+ * rows: the step's rows (2B for a train step, n for a Performance-Optimized
+ * step).  Host or device pointer.  Needs cfg.keep_grad = 1 (the operand is
+ * otherwise dropped from the cache once read), else FF_ERR_UNSUPPORTED.
+ * Synchronous. */
+FF_API ff_status ff_layer_get_grad_operand(const ff_layer* layer, void* out, int rows);
 
 /* Waits for the layer's last stream and returns the first latched kernel
  * error (FF_ERR_TIMEOUT, FF_ERR_NONFINITE) or FF_ERR_CUDA, then clears it. */

@@ -321,7 +321,7 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   // dW (unless kept for ff_layer_get_grad) and the local-gradient operand.
   // (Dropping the activities' lines as well measured no further gain.)
   aa.discard_dW = !L->cfg.keep_grad && ((uintptr_t)L->dW & 127u) == 0;
-  add_dead(aa, L->dZ, (size_t)M * L->ldN * (size_t)es);
+  if (!L->cfg.keep_grad) add_dead(aa, L->dZ, (size_t)M * L->ldN * (size_t)es);
   FF_LAUNCH(K_ADAM, (double)L->N * L->K * (28.0 + (L->is_bf16 ? 2.0 : 0.0)) + (double)L->N * (aa.nrb * 4.0 + 28), st,
             launch_adam(aa, st),
             "Adam");
@@ -700,6 +700,16 @@ ff_status ff_layer_get_grad(const ff_layer* Lc, float* dW, float* db) {
   FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
   if (dW) FF_TRY(cudaMemcpy(dW, L->dW, (size_t)L->N * L->K * 4, kind_default()), "copy dW");
   if (db) FF_TRY(cudaMemcpy(db, L->db, (size_t)L->N * 4, kind_default()), "copy db");
+  return FF_OK;
+}
+
+ff_status ff_layer_get_grad_operand(const ff_layer* Lc, void* out, int rows) {
+  if (!Lc || !out || rows < 0) return FF_ERR_INVALID_ARG;
+  if (!Lc->cfg.keep_grad) return FF_ERR_UNSUPPORTED;
+  if (rows > Lc->cap) return FF_ERR_INVALID_ARG;
+  ff_layer* L = const_cast<ff_layer*>(Lc);
+  FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
+  if (rows) FF_TRY(cudaMemcpy(out, L->dZ, (size_t)rows * L->ldN * (L->is_bf16 ? 2 : 4), kind_default()), "copy G");
   return FF_OK;
 }
 

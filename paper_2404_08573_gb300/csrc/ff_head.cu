@@ -1360,7 +1360,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   aa.B = n;
   // data nobody reads after this step (see the FF train step)
   aa.discard_dW = !L->cfg.keep_grad && ((uintptr_t)L->dW & 127u) == 0;
-  add_dead(aa, L->dZ, (size_t)n * L->ldN * (size_t)es);
+  if (!L->cfg.keep_grad) add_dead(aa, L->dZ, (size_t)n * L->ldN * (size_t)es);
   FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
   const HeadAdamArgs ha =
       head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, b16 ? kPoRows : kDotRows), n, loss);

@@ -85,6 +85,7 @@ def lib():
             "ff_layer_get_state": [c_void_p] + [c_void_p] * 6 + [POINTER(c_longlong)],
             "ff_layer_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
             "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
+            "ff_layer_get_grad_operand": [c_void_p, c_void_p, c_int],
             "ff_layer_check": [c_void_p],
             "ff_layer_get_stats": [c_void_p, c_void_p],
             "ff_layer_selftest_wait": [c_void_p, ctypes.c_uint, c_void_p],
@@ -258,6 +259,19 @@ class Layer:
         dW = np.empty((N, K), np.float32); db = np.empty(N, np.float32)
         _check(lib().ff_layer_get_grad(self._h, dW.ctypes.data, db.ctypes.data), "ff_layer_get_grad")
         return dW, db
+
+    def get_grad_operand(self, rows: int):
+        """ff_layer_get_grad_operand: the last step's weight-gradient operand
+        G = diag(s) dZ [rows, ff_row_stride(out_features)] as float64 (from
+        bf16 or fp32; exact)."""
+        ld = row_stride(self.out_features)
+        if self.prec == "bf16":
+            raw = np.empty((rows, ld), np.uint16)
+            _check(lib().ff_layer_get_grad_operand(self._h, raw.ctypes.data, int(rows)), "ff_layer_get_grad_operand")
+            return (raw.astype(np.uint32) << 16).view(np.float32).astype(np.float64)
+        out = np.empty((rows, ld), np.float32)
+        _check(lib().ff_layer_get_grad_operand(self._h, out.ctypes.data, int(rows)), "ff_layer_get_grad_operand")
+        return out.astype(np.float64)
 
     def stats(self):
         """ff_layer_get_stats: (mean positive goodness, mean negative goodness,
