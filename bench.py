@@ -548,7 +548,16 @@ def run_ours(args):
 FP32_ALU_TFLOPS = 152 * 128 * 2 * 2.07e9 / 1e12
 
 
-def _kernel_profile(lib, torch, fn, pk):
+def _traffic(workload, kernel):
+    """DRAM bytes per launch of `kernel` in `workload` from profiles/traffic.json, or None."""
+    try:
+        with open(os.path.join(ROOT, "profiles", "traffic.json")) as f:
+            return json.load(f).get(workload, {}).get(kernel)
+    except Exception:
+        return None
+
+
+def _kernel_profile(lib, torch, fn, pk, workload=None):
     """Per-kernel device time of one more call of `fn`, every launch bracketed
     by CUDA events on its own stream by libff's profiler: the kernel table and
     the roofline of the kernel with the most device time (tensor-core GEMMs
@@ -586,8 +595,8 @@ def _kernel_profile(lib, torch, fn, pk):
         else:
             bound, peak, src = "hbm", pk["hbm"], pk["src"] + " HBM copy"
         roof = {"kernel": top["kernel"], "bound": bound, "achieved": top["achieved"], "peak": round(peak, 1),
-                "unit": top["unit"], "frac": round(top["achieved"] / peak, 4), "peak_source": src, "traffic": None,
-                "share": top["share"]}
+                "unit": top["unit"], "frac": round(top["achieved"] / peak, 4), "peak_source": src,
+                "traffic": _traffic(workload, top["kernel"]) if workload else None, "share": top["share"]}
     return kernels, roof
 
 
@@ -849,6 +858,33 @@ def run_other(args):
                     "config": {"workload": "ff_train_3072-8192x4_bf16_B4096_theta8",
                                "timing": f"{args.steps} consecutive steps, one sync at the end"}})
         net.close()
+    elif w == "epoch_kernel":
+        # the 784-2000x4 epoch in one persistent kernel (ff_net_train_epoch), lr 1e-3 (a live
+        # net, as the default workload's headline), every timed call from the same state;
+        # --epoch-pairs shortens the epoch (whole batches of 1024 pairs)
+        pairs = min(args.epoch_pairs or PAIRS_PER_EPOCH, PAIRS_PER_EPOCH)
+        X_h, L_h = epoch_inputs()
+        X = torch.from_numpy(X_h[:2 * pairs]).to(dev)
+        Lb = torch.from_numpy(L_h[:2 * pairs]).to(dev)
+        tr = _Trainer(ff, torch, dev, LIVE_LR, BATCH)
+        nbat = -(-pairs // BATCH)
+        loss = torch.zeros(nbat, len(NET) - 1, device=dev)
+        fn = lambda: tr.net.train_epoch(X, Lb, pairs, BATCH, loss=loss, stream=stream)
+        tr.restore()
+        _timed_loop(torch, stream, fn, args.warmup)
+        total = 0.0
+        for _ in range(args.steps):
+            tr.restore()
+            total += _timed_loop(torch, stream, fn, 1)
+        ms = total / args.steps
+        flops = pairs * train_flops_per_pair()
+        tf = flops / (ms / 1e3) / 1e12
+        prof = fn
+        out.update({"metric": "FF train pairs/s on 4x2000 net, one persistent kernel per epoch (ff_net_train_epoch)",
+                    "value": round(pairs / (ms / 1e3), 1), "unit": "pairs/s", "ms_per_step": round(ms, 4),
+                    "dtype": "bf16", "tflops": round(tf, 2), "frac_of_bf16_peak": round(tf / pk["bf16"], 4),
+                    "config": {"workload": f"ff_train_784-2000x4_bf16_epoch{pairs}_B{BATCH}_persistent",
+                               "lr": LIVE_LR, "state": "every timed call from the same initial state"}})
     elif w == "tiny_fp32":
         # 784-500-500 fp32, 16 steps of 64 pairs (latency-bound)
         B = 64
@@ -874,7 +910,8 @@ def run_other(args):
                     "config": {"workload": "ff_train_784-500-500_fp32_B64_16steps"}})
     if prof is not None:
         # one more call, each launch timed on its own stream (not the timed calls above)
-        out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, prof, 1), pk)
+        out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, prof, 1), pk,
+                                                          out.get("config", {}).get("workload"))
     print(json.dumps(out), flush=True)
 
 
@@ -911,7 +948,9 @@ def main():
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
     ap.add_argument("--workload", default="train_4x2000",
                     choices=["train_4x2000", "predict_bf16", "predict_fp32", "adaptive_neg", "softmax_predict",
-                             "softmax_train", "po_train", "pff_4x2000", "pipeline_5x2000", "wide_4x8192", "tiny_fp32"])
+                             "softmax_train", "po_train", "pff_4x2000", "pipeline_5x2000", "wide_4x8192", "tiny_fp32",
+                             "epoch_kernel"])
+    ap.add_argument("--epoch-pairs", type=int, default=0, help="epoch_kernel: pairs per epoch (default 60000)")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-graph", action="store_true")
     ap.add_argument("--no-profile", action="store_true")
