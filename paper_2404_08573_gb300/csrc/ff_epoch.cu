@@ -6,7 +6,7 @@
 //   OV(b, 64 rows)        label overlay, cast to bf16, row scale (layer 1 input)
 //   FWD(k, b, rt, ct)     256 x 256 tile of H = ReLU(s X W^T + b) with its
 //                         per-128-column goodness partials (tcgen05, pair of CTAs)
-//   LG(k, b, 32 rows)     goodness, loss, dL/dg, next-layer scale, dZ' = s 2 dL/dg H,
+//   LG(k, b, 64 rows)     goodness, loss, dL/dg, next-layer scale, dZ' = s 2 dL/dg H,
 //                         bias-gradient partials
 //   WG(k, b, nt, kt)      256 x 256 tile of dW = dZ'^T X (tcgen05, pair of CTAs)
 //   ADAM(k, b, 16 rows)   Adam on 16 rows of W and their bias elements; refreshes
