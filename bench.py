@@ -209,10 +209,16 @@ class _Trainer:
     Adam state kept on the device so that every timed epoch starts from the
     same state (restored outside the timed region)."""
 
+    # True (--fused-local-grad): the local step in the forward GEMM's epilogue
+    # instead of its own kernel after each forward (same results; slower here)
+    fused_local_grad = False
+
     def __init__(self, ff, torch, dev, lr, max_B):
         self.ff, self.torch, self.dev = ff, torch, dev
         self.layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", theta=THETA, lr=lr, init_seed=1000 + k,
                                 max_rows=2 * max_B) for k in range(len(NET) - 1)]
+        for l in self.layers:
+            l.set_fused_local_grad(self.fused_local_grad)
         self.net = ff.Net(self.layers, max_B=max_B, depth=2)
         self.W0 = [torch.from_numpy(l.get_state()["W"]).to(dev) for l in self.layers]
         self.zeros = torch.zeros(max(NET[k] * NET[k + 1] for k in range(len(NET) - 1)), device=dev)
@@ -519,7 +525,9 @@ def run_ours(args):
                        "state": "every timed epoch starts from the same initial weights and Adam state "
                                 "(restored outside the timed region)",
                        "parallelism": f"{world} replica(s); per GPU 4 layers on 4 CUDA streams",
-                       "l2": "inputs larger than L2 (376 MB of pair batches per step)"},
+                       "l2": "inputs larger than L2 (376 MB of pair batches per step)",
+                       "local_grad": "in the forward GEMM's epilogue" if _Trainer.fused_local_grad
+                       else "separate kernel after the forward GEMM"},
             "launch": mode,
             "ms_per_step_eager": round(ms_eager / args.steps, 4),
             "ms_per_step_graph": round(ms_graph / args.steps, 4) if ms_graph is not None else None,
@@ -957,9 +965,12 @@ def main():
     ap.add_argument("--no-cfg-lr", action="store_true", help="skip the epoch timed at the workload's lr 0.03")
     ap.add_argument("--no-epoch-kernel", action="store_true", help="skip the persistent epoch kernel mode")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--fused-local-grad", action="store_true",
+                    help="form the local step in the forward GEMM's epilogue (same results; for comparison)")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--cpu-worker", type=float, default=None, help=argparse.SUPPRESS)
     args = ap.parse_args()
+    _Trainer.fused_local_grad = args.fused_local_grad
     if args.cpu_worker is not None:
         v, done, el, _ = oracle_sample(args.cpu_worker)
         print(json.dumps({"pairs_per_s": v, "steps": done, "elapsed": el}))

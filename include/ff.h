@@ -355,6 +355,18 @@ FF_API ff_status ff_layer_get_grad_operand(const ff_layer* layer, void* out, int
  * error (FF_ERR_TIMEOUT, FF_ERR_NONFINITE) or FF_ERR_CUDA, then clears it. */
 FF_API ff_status ff_layer_check(ff_layer* layer);
 
+/* Where a bf16 train step forms the rest of the local step of §3 (Eq. 1)
+ * after the forward: enable = 1 in the forward GEMM's epilogue -- the CTAs
+ * of a row block exchange their goodness partials in a thread-block cluster
+ * and write dZ', the bias-gradient and loss partials themselves -- wherever
+ * out_features <= 2048; enable = 0 (the default) in a separate kernel after
+ * the forward.  Both give bitwise the same results.  The fused form is
+ * faster for a layer stepped alone on a stream and slower where several
+ * layers' kernels share the GPU (a net on layer streams), since its clusters
+ * of up to 8 CTAs need that many free SMs at once.  No effect on fp32
+ * layers.  Returns FF_ERR_INVALID_ARG for a NULL layer. */
+FF_API ff_status ff_layer_set_fused_local_grad(ff_layer* layer, int enable);
+
 /* A net of layers trained concurrently, one CUDA stream per layer: the
  * single-GPU analogue of Single-Layer PFF (§4.1, Algorithm 1), where node i
  * trains L_i on the output of L_{i-1}.  Here the hand-off is per batch: layer

@@ -143,6 +143,7 @@ struct FwdResult {
   void* H;
   const void* X;
   int ntiles;
+  bool local_grad_done;  // the forward's epilogue also formed the local step (tc_gemm_fwd_lg)
 };
 
 // Split-K scratch of an fp32 layer's forward and weight-gradient GEMMs on M
@@ -171,9 +172,12 @@ static ff_status ensure_split(ff_layer* L, int M) {
 
 // x_rows: rows of the raw input x when labels are given (0: M; M / 2: one
 // image per pair, read for the positive and the negative row).
+// lg (train steps): the local step's arguments; for a bf16 layer whose shape
+// allows it, the forward GEMM forms that step in its epilogue as well
+// (r->local_grad_done), with lg->s set to the row scale used here.
 static ff_status forward_core(ff_layer* L, const void* x, const int* labels, const float* row_scale, int M,
                               void* h_out, cudaStream_t st, cudaEvent_t ev_input_read, FwdResult* r,
-                              int x_rows = 0) {
+                              int x_rows = 0, GradPrepArgs* lg = nullptr) {
   const int K = L->K, N = L->N;
   if (!L->is_bf16) {
     const ff_status ss = ensure_split(L, M);
@@ -203,7 +207,17 @@ static ff_status forward_core(ff_layer* L, const void* x, const int* labels, con
   void* H = h_out ? h_out : L->H;
   EpiArgs ep{s, L->cfg.has_bias ? L->b : nullptr, H, L->ldN, L->gpart};
   int ntiles;
-  if (L->is_bf16) {
+  r->local_grad_done = false;
+  if (L->is_bf16 && lg && L->fuse_local_grad && tc_fwd_lg_supported(M, N)) {
+    ntiles = tc_fwd_ntiles(M, N, false);
+    lg->s = s;
+    ep.gpart = nullptr;
+    FF_LAUNCH(K_FWD_TC, 2.0 * M * N * K, st,
+              tc_gemm_fwd_lg(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, M, N, K, ep, *lg,
+                             static_cast<bf16*>(L->dZ), &L->ds->err, st),
+              "forward GEMM with the local gradient (tcgen05)");
+    r->local_grad_done = true;
+  } else if (L->is_bf16) {
     ntiles = tc_fwd_ntiles(M, N, false);
     FF_LAUNCH(K_FWD_TC, 2.0 * M * N * K, st,
               tc_gemm_fwd(static_cast<const bf16*>(X), L->ldK, L->Wb, L->ldK, M, N, K, ep, &L->ds->err, st),
@@ -245,20 +259,13 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   if (cap_st != FF_OK) return cap_st;
   L->last_stream = st;
   const double es = L->is_bf16 ? 2.0 : 4.0;
-  FwdResult fr;
-  ff_status fs = forward_core(L, x, labels, row_scale, M, h_out, st, ev_input_read, &fr,
-                              images_once && labels ? B : 0);
-  if (fs != FF_OK) return fs;
-
   GradPrepArgs ga{};
   ga.gpart = L->gpart;
-  ga.ntiles = fr.ntiles;
   ga.M = M;
   ga.N = L->N;
   ga.ld = L->ldN;
   ga.B = B;
   ga.theta = L->cfg.theta;
-  ga.s = fr.s;
   ga.g_out = goodness;
   ga.s_next = next_scale;
   ga.dbpart = L->dbpart;
@@ -269,9 +276,17 @@ ff_status train_step_impl(ff_layer* L, const void* x, const int* labels, const f
   ga.beta1 = L->cfg.beta1;
   ga.beta2 = L->cfg.beta2;
   ga.err = &L->ds->err;
-  FF_LAUNCH(K_GRAD_PREP,
-            (double)M * (fr.ntiles * 4.0 + 12) + (double)M * L->ldN * es * 2 + (double)local_grad_row_blocks(M) * L->N * 4,
-            st, launch_grad_prep(ga, L->is_bf16, fr.H, L->dZ, st), "goodness/loss/local gradient");
+  FwdResult fr;
+  ff_status fs = forward_core(L, x, labels, row_scale, M, h_out, st, ev_input_read, &fr,
+                              images_once && labels ? B : 0, &ga);
+  if (fs != FF_OK) return fs;
+  if (!fr.local_grad_done) {
+    ga.ntiles = fr.ntiles;
+    ga.s = fr.s;
+    FF_LAUNCH(K_GRAD_PREP,
+              (double)M * (fr.ntiles * 4.0 + 12) + (double)M * L->ldN * es * 2 + (double)local_grad_row_blocks(M) * L->N * 4,
+              st, launch_grad_prep(ga, L->is_bf16, fr.H, L->dZ, st), "goodness/loss/local gradient");
+  }
   if (ev_forward_done) FF_TRY(cudaEventRecord(ev_forward_done, st), "event record");
 
   if (L->is_bf16) {
@@ -362,9 +377,8 @@ ff_status ff_layer_create(const ff_layer_config* cfg, void* stream, ff_layer** o
   int dev = 0;
   FF_TRY(cudaGetDevice(&dev), "cudaGetDevice");
   if (cfg->prec == FF_BF16 && !tc_supported()) return FF_ERR_UNSUPPORTED;
-  ff_layer* L = new (std::nothrow) ff_layer();
+  ff_layer* L = new (std::nothrow) ff_layer();  // value-initialised: null pointers, zero sizes, defaults
   if (!L) return FF_ERR_OOM;
-  std::memset(L, 0, sizeof(*L));
   L->cfg = *cfg;
   L->K = cfg->in_features;
   L->N = cfg->out_features;
@@ -726,6 +740,12 @@ ff_status ff_layer_get_stats(const ff_layer* Lc, float* stats) {
   ff_layer* L = const_cast<ff_layer*>(Lc);
   FF_TRY(cudaStreamSynchronize(L->last_stream), "sync");
   FF_TRY(cudaMemcpy(stats, L->ds->stats, 3 * sizeof(float), cudaMemcpyDefault), "read statistics");
+  return FF_OK;
+}
+
+ff_status ff_layer_set_fused_local_grad(ff_layer* layer, int enable) {
+  if (!layer) return FF_ERR_INVALID_ARG;
+  layer->fuse_local_grad = enable != 0;
   return FF_OK;
 }
 

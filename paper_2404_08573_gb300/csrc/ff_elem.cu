@@ -101,12 +101,6 @@ __global__ void k_row_scale(const T* __restrict__ x, int ldx, int rows, int F, f
 }
 
 // ----------------------------------------------------------------- finalize
-__device__ __forceinline__ float softplus_f(float t) { return fmaxf(t, 0.f) + log1pf(expf(-fabsf(t))); }
-__device__ __forceinline__ float sigmoid_f(float t) {
-  if (t >= 0.f) return 1.f / (1.f + expf(-t));
-  const float e = expf(t);
-  return e / (1.f + e);
-}
 
 __global__ void __launch_bounds__(256) k_finalize(FinalizeArgs a) {
   ptx::griddep_wait();  // launched with programmatic stream serialization

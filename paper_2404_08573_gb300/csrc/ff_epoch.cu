@@ -184,30 +184,10 @@ __device__ __forceinline__ void prefetch_l2(const void* p, size_t bytes) {
 
 __device__ __forceinline__ uint4 ldcg16(const void* p) { return __ldcg(reinterpret_cast<const uint4*>(p)); }
 
-// Cross-CTA (cluster) forms used by the pair's task ring.
-__device__ __forceinline__ void mbar_arrive_remote(uint64_t* local_bar, uint32_t rank) {
-  const uint32_t a = ptx::mapa_shared(ptx::smem_u32(local_bar), rank);
-  asm volatile("mbarrier.arrive.release.cluster.shared::cluster.b64 _, [%0];" ::"r"(a) : "memory");
-}
-__device__ __forceinline__ bool mbar_try_wait_cluster(uint64_t* bar, uint32_t parity) {
-  uint32_t ok;
-  asm volatile(
-      "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.acquire.cluster.shared::cta.b64 p, [%1], %2;\n\t"
-      "selp.u32 %0, 1, 0, p;\n\t}"
-      : "=r"(ok)
-      : "r"(ptx::smem_u32(bar)), "r"(parity)
-      : "memory");
-  return ok != 0;
-}
-__device__ __forceinline__ void st_remote_u1(int* local_slot, uint32_t rank, int v) {
-  const uint32_t a = ptx::mapa_shared(ptx::smem_u32(local_slot), rank);
-  asm volatile("st.shared::cluster.u32 [%0], %1;" ::"r"(a), "r"(v) : "memory");
-}
-__device__ __forceinline__ void st_remote_u2(uint2* local_slot, uint32_t rank, uint2 v) {
-  const uint32_t a = ptx::mapa_shared(ptx::smem_u32(local_slot), rank);
-  asm volatile("st.shared::cluster.v2.u32 [%0], {%1, %2};" ::"r"(a), "r"(v.x), "r"(v.y) : "memory");
-}
+using ptx::mbar_arrive_remote;
+using ptx::mbar_try_wait_cluster;
+using ptx::st_remote_u1;
+using ptx::st_remote_u2;
 
 __device__ __forceinline__ void latch_abort(const EpochP& P) {
   atomicOr(P.err, DEVERR_TIMEOUT);
@@ -346,12 +326,6 @@ __device__ void signal_done(const EpochP& P, uint2 t) {
   }
 }
 
-__device__ __forceinline__ float softplus_f(float t) { return fmaxf(t, 0.f) + log1pf(expf(-fabsf(t))); }
-__device__ __forceinline__ float sigmoid_f(float t) {
-  if (t >= 0.f) return 1.f / (1.f + expf(-t));
-  const float e = expf(t);
-  return e / (1.f + e);
-}
 
 __device__ __forceinline__ void load_h8(const bf16* p, float (&v)[8]) {
   const uint4 u = ldcg16(p);

@@ -11,13 +11,22 @@
 //   store    C = X W^T in fp32 (the label-free part of layer 1 in predict);
 //   wgrad    dW = G^T X with G = diag(s) dZ, contracting over the batch rows
 //            (both operands are read MN-major straight from their row-major
-//            buffers: no transposed copies).
+//            buffers: no transposed copies);
+//   forward with the local gradient (train step): the forward above, and in
+//            the same epilogue the rest of the layer's local step of §3
+//            (Eq. 1): each row's goodness summed over all column tiles, the
+//            loss, dL/dg, the next layer's row scale, the weight-gradient
+//            operand dZ' = s * 2 dL/dg * h and the bias-gradient partials.
+//            The CTAs holding a row block's column tiles form one cluster and
+//            exchange their goodness partials through distributed shared
+//            memory (plain remote stores and remote mbarrier arrivals).
 //
-// One CTA computes one (ROW_SUBTILES*BM) x BN output tile with three warp roles:
+// One CTA computes one (MT*BM) x (NT*BN) output tile with three warp roles:
 //   warp 0      TMA producer: 128-byte-swizzled tiles into a STAGES-deep ring
 //   warp 1      allocates TMEM, one elected lane issues tcgen05.mma (M=128,
-//               N=BN, K=16; one per row subtile, sharing the B stage) and
-//               commits each stage back to the producer
+//               N=BN, K=16; one per row subtile and column subtile, each
+//               into its own accumulator) and commits each stage back to the
+//               producer
 // In pair mode two CTAs (a cluster of 2 along x) run as one cta_group::2
 // unit: each loads its own A rows and half of B, the even CTA's MMA warp
 // issues M=256 MMAs over both, and each CTA's epilogue reads its own TMEM.
@@ -29,6 +38,8 @@
 // MMAs already in flight and frees TMEM before the CTA exits.
 #include <cudaTypedefs.h>
 
+#include <cstdio>
+#include <cstdlib>
 #include <mutex>
 
 #include "ff_internal.cuh"
@@ -44,27 +55,34 @@ constexpr int NTHREADS = 64 + 32 * EPI_WARPS;  // producer warp, MMA warp, epilo
 constexpr int MODE_FWD = 0;
 constexpr int MODE_STORE = 1;
 constexpr int MODE_FWD_LOGITS = 2;  // forward, plus partial logits of a 10-class block (EpiArgs::logit_V)
+constexpr int MODE_FWD_LG = 3;      // forward, plus the local gradient (GradPrepArgs), cluster-wide goodness
+constexpr int kLgParts = 16;        // goodness partials of a row (128 columns each) a cluster can hold
 constexpr int kLogitClasses = 10;
 constexpr int kLogitStride = 12;    // floats per column of the staged block weights (three float4)
 
-template <int BN, int NSTAGE, int MT, bool PAIR>
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT = 1>
 struct TcCfg {
+  static constexpr int TN = NT * BN;                // columns of the tile (NT column subtiles of BN)
   static constexpr int A_BYTES = MT * BM * BK * 2;  // MT row subtiles of BM rows
-  static constexpr int BH = PAIR ? BN / 2 : BN;     // B columns this CTA loads
-  static constexpr int B_BYTES = BH * BK * 2;
+  static constexpr int BH = PAIR ? BN / 2 : BN;     // B columns of a column subtile this CTA loads
+  static constexpr int B_BYTES = NT * BH * BK * 2;
   static constexpr int STAGE = A_BYTES + B_BYTES;
   static constexpr int STAGES = NSTAGE;
-  static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + BN * 4 /*bias*/;
+  static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + TN * 4 /*bias*/;
+  // the local-gradient epilogue: every partial of the cluster's row block,
+  // and per epilogue warp its rows' 2 dL/dg and s 2 dL/dg
+  static constexpr int LG_SMEM = kLgParts * MT * BM * 4 + EPI_WARPS * 32 * 2 * 4;
   static constexpr uint32_t ACC_COLS = BN <= 32 ? 32 : BN <= 64 ? 64 : BN <= 128 ? 128 : 256;
-  static constexpr uint32_t TMEM_COLS = MT * ACC_COLS;  // one accumulator per row subtile
+  static constexpr uint32_t TMEM_COLS = MT * NT * ACC_COLS;  // one accumulator per (row, column) subtile
   static_assert(BN % 64 == 0 && BN <= 256, "BN must be a multiple of 64, at most 256");
-  static_assert(MT >= 1 && MT * ACC_COLS <= 512, "accumulators must fit in TMEM");
+  static_assert(MT >= 1 && NT >= 1 && MT * NT * ACC_COLS <= 512, "accumulators must fit in TMEM");
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-  static_assert(MT * 4 * 32 * BN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
+  static_assert(MT * 4 * 32 * TN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
   static_assert(EPI_WARPS * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
-  static_assert(BN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
+  static_assert(TN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
+  static_assert(NT == 1 || TN / (EPI_WARPS / 4) == BN, "with column subtiles each epilogue warp reads one accumulator");
   static_assert(!PAIR || BH % 64 == 0, "each CTA of a pair loads whole 64-column B groups");
-  static_assert(2 * STAGES * 8 + 8 + 12 <= 256, "barriers, TMEM slot and flags must fit below the bias tile");
+  static_assert(2 * STAGES * 8 + 8 + 16 + 8 <= 256, "barriers, TMEM slot, flags and the LG barrier fit below the bias tile");
 };
 
 __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
@@ -75,13 +93,19 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
 // At most 96 registers a thread (the bound for two CTAs of 320 threads per
 // SM; no spills): a CTA then leaves room on its SM for the Adam and local-
 // gradient blocks of the other layers' streams (784-2000x4 epoch -1 %).
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
+// MODE_FWD_LG: tmD maps dZ' (as tmC maps H) and lg holds the local step's
+// arguments; the grid's column tiles all lie in one cluster (2 x gridDim.y).
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT>
 __global__ void __launch_bounds__(NTHREADS, 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
-              const __grid_constant__ CUtensorMap tmC, int tma_store, int M, int N, int K, EpiArgs ep, int* err) {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR>;
+              const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmD, int tma_store, int M,
+              int N, int K, EpiArgs ep, GradPrepArgs lg, int* err) {
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT>;
   constexpr bool FWD = MODE != MODE_STORE;
   constexpr bool LOGITS = MODE == MODE_FWD_LOGITS;
+  constexpr bool LG = MODE == MODE_FWD_LG;
+  static_assert(!LG || (PAIR && MT == 1 && NT == 2 && BN == 256 && EPI_WARPS == 8),
+                "the local-gradient epilogue: 128 rows x 512 columns per CTA, a warp per 32 rows x 256 columns");
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -94,15 +118,20 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(tfull + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tslot + 1);
   volatile int* never_set = reinterpret_cast<volatile int*>(tslot + 2);  // drain waits ignore the abort
-  float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [BN] bias of this tile
-  float* sVt = sbias + BN;  // LOGITS: [BN][kLogitStride] block weights of this tile's columns
+  uint64_t* lgbar = reinterpret_cast<uint64_t*>(tslot + 4);  // LG: every partial of the row block has arrived
+  float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [TN] bias of this tile
+  float* sVt = sbias + C::TN;  // LOGITS: [BN][kLogitStride] block weights of this tile's columns
+  // LG: [kLgParts][MT * BM] goodness partials of this CTA's rows (partial t
+  // covers columns 128t ..), then per epilogue warp [2][32] row terms
+  float* sgp = sbias + C::TN;
+  float* scc = sgp + kLgParts * MT * BM;
 
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   // blockIdx.x: row tile (the two CTAs of a pair are consecutive in x, as
   // cta_group::2 requires); blockIdx.y: column tile
   const int m0 = blockIdx.x * (BM * MT);
-  const int n0 = blockIdx.y * BN;
+  const int n0 = blockIdx.y * C::TN;
   const int num_kb = (K + BK - 1) / BK;
 
   // PAIR: the two CTAs of a cluster (consecutive tile rows, same columns)
@@ -113,22 +142,27 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   // even CTA issues the MMAs once both halves of a stage have landed (the odd
   // CTA's copies complete on the even CTA's `full` barrier) and its commits
   // arrive on both CTAs' `empty` and `tfull` barriers.
+  // A cluster may hold several pairs (LG: a pair per column tile); the pair
+  // is the two CTAs whose cluster ranks differ in bit 0.
   uint32_t crank = 0;
   if constexpr (PAIR) crank = ptx::cluster_ctarank();
-  const bool issuer = !PAIR || crank == 0;
-  constexpr uint16_t pmask = 3;
+  const uint32_t pair_lead = crank & ~1u;
+  const bool issuer = !PAIR || (crank & 1u) == 0;
+  const uint16_t pmask = (uint16_t)(3u << pair_lead);
   if (threadIdx.x == 0) {
     for (int s = 0; s < C::STAGES; ++s) {
       ptx::mbar_init(&full[s], 1);
       ptx::mbar_init(&empty[s], 1);
     }
     ptx::mbar_init(tfull, 1);
+    if constexpr (LG) ptx::mbar_init(lgbar, 32 * EPI_WARPS * gridDim.y);  // every epilogue lane of the row block
     *abort_flag = 0;
     *never_set = 0;
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
     if (FWD || tma_store) ptx::prefetch_tmap(&tmC);
+    if constexpr (LG) ptx::prefetch_tmap(&tmD);
   }
   if (warp == 1) {
     if constexpr (PAIR) {
@@ -153,7 +187,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     if (lane == 0) {
       // the stage barriers the copies complete on: the issuing CTA's
       uint32_t full0 = ptx::smem_u32(&full[0]);
-      if constexpr (PAIR) full0 = ptx::mapa_shared(full0, 0u);
+      if constexpr (PAIR) full0 = ptx::mapa_shared(full0, pair_lead);
       auto load = [&](void* dst, const CUtensorMap* map, int s, int c0, int c1) {
         if (!ff_dcheck(tma_x_aligned(c0, 2), err)) {
           *abort_flag = 1;
@@ -164,7 +198,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         else
           ptx::tma_load_2d(dst, map, &full[s], c0, c1);
       };
-      const int nb = n0 + (int)crank * C::BH;  // first B column this CTA loads
+      const int nb = n0 + (int)(crank & 1u) * C::BH;  // first B column this CTA loads (of column subtile 0)
       int issued = 0;
       for (int kb = 0; kb < num_kb; ++kb) {
         const int s = kb % C::STAGES;
@@ -185,7 +219,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
           for (int j = 0; j < MT * BM / 64; ++j) load(a + j * 64 * BK * 2, &tmA, s, m0 + 64 * j, k0);
         }
         if (!B_MN) {
-          load(b, &tmB, s, k0, nb);
+#pragma unroll
+          for (int nt = 0; nt < NT; ++nt) load(b + nt * C::BH * BK * 2, &tmB, s, k0, nb + nt * BN);
         } else {
 #pragma unroll
           for (int j = 0; j < C::BH / 64; ++j) load(b + j * 64 * BK * 2, &tmB, s, nb + 64 * j, k0);
@@ -235,22 +270,28 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const uint32_t b_base = ptx::smem_u32(sB + s * C::B_BYTES);
 #pragma unroll
         for (int k = 0; k < BK / 16; ++k) {
-          // K-major: the 16-element K slice sits 32 bytes further along each
-          // swizzled 128-byte row (SBO = 1024 between 8-row groups).
-          // MN-major: 16 K rows further = 2 x 1024 bytes; LBO = 8192 between
-          // the 64-element MN chunks, SBO = 1024 between 8-row K groups.
-          const uint64_t bd = B_MN ? ptx::sdesc_sw128(b_base + k * 2048, 64 * BK * 2, 1024)
-                                   : ptx::sdesc_sw128(b_base + k * 32, 16, 1024);
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt) {
-            // row subtile mt: BM rows further in the A stage, its own accumulator
-            const uint32_t as = a_base + mt * BM * BK * 2;
-            const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
-                                     : ptx::sdesc_sw128(as + k * 32, 16, 1024);
-            if constexpr (PAIR)
-              ptx::umma_f16_pair(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
-            else
-              ptx::umma_f16(tmem + (uint32_t)(mt * C::ACC_COLS), ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+          for (int nt = 0; nt < NT; ++nt) {
+            // K-major: the 16-element K slice sits 32 bytes further along each
+            // swizzled 128-byte row (SBO = 1024 between 8-row groups).
+            // MN-major: 16 K rows further = 2 x 1024 bytes; LBO = 8192 between
+            // the 64-element MN chunks, SBO = 1024 between 8-row K groups.
+            // Column subtile nt: its own B box, BH rows further.
+            const uint32_t bs = b_base + nt * C::BH * BK * 2;
+            const uint64_t bd = B_MN ? ptx::sdesc_sw128(bs + k * 2048, 64 * BK * 2, 1024)
+                                     : ptx::sdesc_sw128(bs + k * 32, 16, 1024);
+#pragma unroll
+            for (int mt = 0; mt < MT; ++mt) {
+              // row subtile mt: BM rows further in the A stage, its own accumulator
+              const uint32_t as = a_base + mt * BM * BK * 2;
+              const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
+                                       : ptx::sdesc_sw128(as + k * 32, 16, 1024);
+              const uint32_t acc = tmem + (uint32_t)((mt * NT + nt) * C::ACC_COLS);
+              if constexpr (PAIR)
+                ptx::umma_f16_pair(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+              else
+                ptx::umma_f16(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+            }
           }
         }
         if constexpr (PAIR)
@@ -273,7 +314,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     // 128-byte-swizzled layout (conflict-free for row-per-thread 16-byte
     // writes) and one lane writes it out with TMA.
     constexpr int HALVES = EPI_WARPS / 4;
-    constexpr int CPW = BN / HALVES;  // columns per epilogue warp
+    constexpr int CPW = C::TN / HALVES;  // columns per epilogue warp (within one accumulator)
     const int q = warp & 3;
     const int ew = warp - 2;          // 0 .. EPI_WARPS-1
     const int half = ew / 4;
@@ -284,7 +325,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     if (FWD) {
       // While the mainloop runs: the tile's bias (zero past N or without bias)
       // into shared memory and this thread's row scales into registers.
-      for (int c = (int)threadIdx.x - 64; c < BN; c += 32 * EPI_WARPS)
+      for (int c = (int)threadIdx.x - 64; c < C::TN; c += 32 * EPI_WARPS)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
       if constexpr (LOGITS) {
         for (int idx = (int)threadIdx.x - 64; idx < kLogitClasses * BN; idx += 32 * EPI_WARPS) {
@@ -327,9 +368,11 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const int gi = rbase + lane;
         // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
         uint8_t* stage = smem + (FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
-        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) + (uint32_t)(mt * C::ACC_COLS + cbase);
+        const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) +
+                              (uint32_t)((mt * NT + cbase / BN) * C::ACC_COLS + cbase % BN);
         const float s = srow[mt];
         float g = 0.f;
+        float g_lo = 0.f;  // LG: the goodness partial of the warp's first 128 columns
         float zl[kLogitClasses];  // LOGITS: this row's partial logits over the warp's columns
 #pragma unroll
         for (int c = 0; c < kLogitClasses; ++c) zl[c] = 0.f;
@@ -414,8 +457,15 @@ __global__ void __launch_bounds__(NTHREADS, 2)
           if (c0 + 64 < CPW) ptx::tmem_ld32(trow + (uint32_t)(c0 + 64), ra);
           process(rb, c0 + 32);
           ptx::tmem_ld_wait();
+          if constexpr (LG) {
+            // partials per 128 columns, as the tile shapes of the other forms give
+            if (c0 + 64 == 128) {
+              g_lo = g;
+              g = 0.f;
+            }
+          }
         }
-        if (FWD && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
+        if (FWD && !LG && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
         if (LOGITS && gi < M) {
           float2* zp = reinterpret_cast<float2*>(ep.zpart + ((size_t)(blockIdx.y * HALVES + half) * M + gi) * kLogitClasses);
 #pragma unroll
@@ -432,6 +482,147 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
             }
             ptx::bulk_commit();
+          }
+        }
+        if constexpr (LG) {
+          // ---- the rest of the layer's local step (§3, Eq. 1) for the warp's
+          // 32 rows x 256 columns, with every sum in the order of the separate
+          // local-gradient kernel (k_grad_prep), so both give the same bits.
+          const int r = q * 32 + lane;  // row within the CTA
+          // (1) this warp's two partials into every CTA of the row block (this
+          //     one included), then one arrival on each CTA's barrier
+          {
+            const int t0 = (n0 + cbase) / 128;
+            const uint32_t xr = crank & 1u;
+            for (uint32_t y = 0; y < gridDim.y; ++y) {
+              const uint32_t rank = xr + 2u * y;
+              ptx::st_remote_f32(&sgp[t0 * BM + r], rank, g_lo);
+              ptx::st_remote_f32(&sgp[(t0 + 1) * BM + r], rank, g);
+              ptx::mbar_arrive_remote(lgbar, rank);
+            }
+          }
+          // (2) every partial of these rows has arrived (bounded)
+          const bool have = ptx::mbar_wait_cluster(lgbar, 0, kWaitTimeoutNs, abort_flag);
+          if (!have) latch(err, abort_flag);
+          if (__all_sync(0xffffffffu, have && !*abort_flag)) {
+            // (3) the row's goodness: 8 lane-strided sums over the partials
+            //     (the ones past N are +0), then a fixed tree
+            const int nparts = 4 * (int)gridDim.y;
+            float gs[8];
+#pragma unroll
+            for (int p8 = 0; p8 < 8; ++p8) {
+              float a = 0.f;
+              for (int t = p8; t < nparts; t += 8) a += sgp[t * BM + r];
+              gs[p8] = a;
+            }
+            const float gsum = ((gs[0] + gs[4]) + (gs[2] + gs[6])) + ((gs[1] + gs[5]) + (gs[3] + gs[7]));
+            const bool row_ok = gi < M;
+            const bool pos = gi < lg.B;
+            const float tt = pos ? lg.theta - gsum : gsum - lg.theta;  // the pair member's margin error
+            float cc = 0.f, sc = 0.f;  // 2 dL/dg, and times the row scale
+            if (row_ok) {
+              const float sg = sigmoid_f(tt);
+              cc = 2.f * (pos ? -sg : sg) / (float)lg.B;
+              sc = s * cc;
+            }
+            const bool lead = blockIdx.y == 0 && half == 0;  // one thread per row
+            float lv = 0.f, gpv = 0.f, gnv = 0.f;
+            if (lead && row_ok) {
+              if (!isfinite(gsum)) atomicOr(err, DEVERR_NONFINITE);
+              if (lg.g_out) lg.g_out[gi] = gsum;
+              if (lg.s_next) lg.s_next[gi] = inv_norm(gsum);
+              lv = softplus_f(tt);
+              (pos ? gpv : gnv) = gsum;
+            }
+            float* ccw = scc + ew * 64;  // [32] 2 dL/dg, then [32] s 2 dL/dg of the warp's rows
+            ccw[lane] = cc;
+            ccw[32 + lane] = sc;
+            const int rb = rbase / 32;  // the 32-row block
+            const int nrb = (M + 31) / 32;
+            if (lead) {
+              // the block's loss and goodness sums: rows y, y+8, y+16, y+24 as
+              // (y + (y+16)) + ((y+8) + (y+24)), then y = 0..7 in turn
+              auto block_sum = [&](float v) {
+                v += __shfl_down_sync(0xffffffffu, v, 16);
+                v += __shfl_down_sync(0xffffffffu, v, 8);
+                float t = 0.f;
+#pragma unroll
+                for (int y = 0; y < 8; ++y) t += __shfl_sync(0xffffffffu, v, y);
+                return t;
+              };
+              const float tl = block_sum(lv), tp = block_sum(gpv), tn = block_sum(gnv);
+              if (lane == 0 && rbase < M) {
+                lg.loss_part[rb] = tl;
+                if (lg.stat_part) {
+                  lg.stat_part[rb] = tp;
+                  lg.stat_part[nrb + rb] = tn;
+                }
+              }
+              if (blockIdx.x == 0 && q == 0 && lane == 0 && lg.ds) {
+                // the Adam update that follows is step t; beta^t as running products
+                lg.ds->t += 1;
+                lg.ds->pow1 *= lg.beta1;
+                lg.ds->pow2 *= lg.beta2;
+                lg.ds->bc1 = (float)(1.0 - lg.ds->pow1);
+                lg.ds->bc2 = (float)(1.0 - lg.ds->pow2);
+              }
+            }
+            // (4) once the activity's stores have read the staging, turn it in
+            //     place into dZ' = bf16(s 2 dL/dg h) (h as stored; zero on rows
+            //     past M), two columns per lane and pass: lane j takes columns
+            //     64 p + 2j, +1, row by row -- conflict-free in the swizzled
+            //     layout -- and forms their bias-gradient partials over the 32
+            //     rows, db_y = chain of fmas over the rows y + 8k, then y = 0..7
+            if (lane == 0) ptx::bulk_wait_read0();
+            __syncwarp();
+            float act = 0.f;
+            const int nvalid = M - rbase;  // rows of the block below M
+#pragma unroll 1
+            for (int pass = 0; pass < CPW / 64; ++pass) {
+              uint8_t* chunk = stage + pass * (32 * 128) + (lane & 3) * 4;
+              float tA = 0.f, tB = 0.f;
+#pragma unroll 2
+              for (int y = 0; y < 8; ++y) {
+                float dA = 0.f, dB = 0.f;
+#pragma unroll
+                for (int k = 0; k < 4; ++k) {
+                  const int rr_ = y + 8 * k;
+                  uint32_t* wp = reinterpret_cast<uint32_t*>(chunk + rr_ * 128 + ((((uint32_t)lane >> 2) ^ (uint32_t)(rr_ & 7)) << 4));
+                  uint32_t w = *wp;
+                  if (rr_ >= nvalid) w = 0u;
+                  const float2 hf = __bfloat1622float2(*reinterpret_cast<__nv_bfloat162*>(&w));
+                  const float cr = ccw[rr_], sr = ccw[32 + rr_];
+                  dA = fmaf(cr, hf.x, dA);
+                  dB = fmaf(cr, hf.y, dB);
+                  act += (hf.x > 0.f ? 1.f : 0.f) + (hf.y > 0.f ? 1.f : 0.f);
+                  __nv_bfloat162 zb = __floats2bfloat162_rn(sr * hf.x, sr * hf.y);
+                  *wp = *reinterpret_cast<uint32_t*>(&zb);
+                }
+                tA += dA;
+                tB += dB;
+              }
+              const int col = n0 + cbase + pass * 64 + 2 * lane;
+              if (rbase < M) {
+                if (col < N) lg.dbpart[(size_t)rb * N + col] = tA;
+                if (col + 1 < N) lg.dbpart[(size_t)rb * N + col + 1] = tB;
+              }
+            }
+            // (6) dZ' out with TMA, and the block's active-ReLU count
+            ptx::fence_async_smem();
+            __syncwarp();
+            if (lane == 0 && rbase < M) {
+#pragma unroll 1
+              for (int ch = 0; ch < CPW / CW; ++ch) {
+                const int col = n0 + cbase + ch * CW;
+                if (col < ep.ldo && ff_dcheck(col >= 0 && rbase >= 0 && tma_x_aligned(col, 2), err))
+                  ptx::tma_store_2d(&tmD, stage + ch * (32 * 128), col, rbase);
+              }
+              ptx::bulk_commit();
+            }
+            act = warp_sum(act);
+            const int cb = (n0 + cbase) / 256;
+            if (lane == 0 && lg.stat_part && cb < lg.ncb && rbase < M)
+              lg.stat_part[2 * nrb + (size_t)rb * lg.ncb + cb] = act;
           }
         }
       }
@@ -492,34 +683,56 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
   return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT>
-cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
-                      int K, const EpiArgs& ep, int* err, cudaStream_t st) {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR>;
-  constexpr int SMEM = C::SMEM + (MODE == MODE_FWD_LOGITS ? BN * kLogitStride * 4 : 0);
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT, int MODE>
+constexpr int tc_smem() {
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT>;
+  return C::SMEM + (MODE == MODE_FWD_LOGITS ? BN * kLogitStride * 4 : 0) + (MODE == MODE_FWD_LG ? C::LG_SMEM : 0);
+}
+
+// Launch configuration of one instance: the grid (tile rows padded to whole
+// pairs; a padding CTA loads zeros, supplies its half of B and writes
+// nothing), clusters of the pair (LG: of the pair and every column tile),
+// and programmatic stream serialization.
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT>
+struct TcLaunch {
+  static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE>();
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-  auto kern = k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT>;
-  static cudaError_t attr = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
-  if (attr != cudaSuccess) return attr;
+  static constexpr int CM = PAIR ? 2 : 1;
   cudaLaunchConfig_t cfg = {};
-  // tile rows padded to whole pairs; a padding CTA loads zeros, supplies its
-  // half of B and writes nothing
-  constexpr int CM = PAIR ? 2 : 1;
-  cfg.gridDim = dim3(cdiv(cdiv(M, BM * MT), CM) * CM, cdiv(N, BN), 1);
-  cfg.blockDim = dim3(NTHREADS, 1, 1);
-  cfg.dynamicSmemBytes = SMEM;
-  cfg.stream = st;
   cudaLaunchAttribute at[2];
-  at[0].id = cudaLaunchAttributeClusterDimension;
-  at[0].val.clusterDim.x = CM;
-  at[0].val.clusterDim.y = 1;
-  at[0].val.clusterDim.z = 1;
-  cfg.attrs = at;
-  // the next kernel's launch and set-up overlap this one's tail (griddep_*)
-  at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-  at[1].val.programmaticStreamSerializationAllowed = 1;
-  cfg.numAttrs = 2;
-  return cudaLaunchKernelEx(&cfg, kern, ta, tb, tc, tma_store, M, N, K, ep, err);
+  TcLaunch(int M, int N, cudaStream_t st) {
+    cfg.gridDim = dim3(cdiv(cdiv(M, BM * MT), CM) * CM, cdiv(N, NT * BN), 1);
+    cfg.blockDim = dim3(NTHREADS, 1, 1);
+    cfg.dynamicSmemBytes = SMEM;
+    cfg.stream = st;
+    at[0].id = cudaLaunchAttributeClusterDimension;
+    at[0].val.clusterDim.x = CM;
+    at[0].val.clusterDim.y = MODE == MODE_FWD_LG ? cfg.gridDim.y : 1;
+    at[0].val.clusterDim.z = 1;
+    // the next kernel's launch and set-up overlap this one's tail (griddep_*)
+    at[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    at[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = at;
+    cfg.numAttrs = 2;
+  }
+  static auto kernel() { return k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT>; }
+  static cudaError_t set_attrs() {
+    static cudaError_t e = cudaFuncSetAttribute(kernel(), cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
+    return e;
+  }
+};
+
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT = 1>
+cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
+                      int K, const EpiArgs& ep, int* err, cudaStream_t st, const CUtensorMap* td = nullptr,
+                      const GradPrepArgs* lg = nullptr) {
+  using Lc = TcLaunch<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT>;
+  const cudaError_t attr = Lc::set_attrs();
+  if (attr != cudaSuccess) return attr;
+  Lc l(M, N, st);
+  const GradPrepArgs none{};
+  return cudaLaunchKernelEx(&l.cfg, Lc::kernel(), ta, tb, tc, td ? *td : tc, tma_store, M, N, K, ep, lg ? *lg : none,
+                            err);
 }
 
 constexpr int FWD_BN = 256;
@@ -592,6 +805,49 @@ int tc_gemm_fwd_ctas(int M, int N, bool narrow) {
 
 // B (the weights, [N, K]) is loaded per CTA in boxes of the CTA's share of a tile's columns.
 static constexpr int b_box_rows(int bn) { return USE_PAIR ? bn / 2 : bn; }
+
+// The train step's forward with the local gradient: CTA pairs of 256 rows x
+// 512 columns (two 256-column accumulators per CTA; per 64-deep K step a CTA
+// loads 48 KB of operands for 8.4 MFLOP, as the 512 x 256 pairs above) and
+// every column tile of a row block in one cluster, so at most 4 column tiles
+// (N <= 2048) in the portable cluster size of 8.
+using FwdLg = TcLaunch<FWD_BN, false, false, MODE_FWD_LG, true, NSTAGES, 1, 2>;
+constexpr int kLgMaxColTiles = 4;
+
+bool tc_fwd_lg_supported(int M, int N) {
+  if (M <= 0 || N <= 0 || cdiv(N, 2 * FWD_BN) > kLgMaxColTiles) return false;
+  // clusters of 2 x (column tiles) CTAs must fit the GPU (checked once per column-tile count)
+  static int ok[kLgMaxColTiles + 1] = {0, 0, 0, 0, 0};  // 0 unknown, 1 yes, -1 no
+  const int ct = cdiv(N, 2 * FWD_BN);
+  if (ok[ct] == 0) {
+    int clusters = 0;
+    cudaError_t e = FwdLg::set_attrs();
+    if (e == cudaSuccess) {
+      // the occupancy query takes the cluster shape alone (no other launch attributes)
+      FwdLg l(2 * BM, ct * 2 * FWD_BN, nullptr);
+      l.cfg.numAttrs = 1;
+      e = cudaOccupancyMaxActiveClusters(&clusters, FwdLg::kernel(), &l.cfg);
+    }
+    if (e != cudaSuccess) cudaGetLastError();  // leave no sticky launch-configuration error behind
+    if (std::getenv("FF_DEBUG"))
+      std::fprintf(stderr, "[ff] forward with local gradient, %d column tiles: %d clusters of %d CTAs (%s)\n", ct,
+                   clusters, 2 * ct, cudaGetErrorString(e));
+    ok[ct] = e == cudaSuccess && clusters > 0 ? 1 : -1;
+  }
+  return ok[ct] > 0;
+}
+
+cudaError_t tc_gemm_fwd_lg(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
+                           const GradPrepArgs& lg, bf16* dZ, int* err, cudaStream_t st) {
+  if (!tc_fwd_lg_supported(M, N) || ep.gpart_in || ep.logit_V || !lg.loss_part || !lg.dbpart)
+    return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, tc, td;
+  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(FWD_BN)) ||
+      !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32) || !make_map(&td, dZ, 2, ep.ldo, M, ep.ldo, 64, 32))
+    return cudaErrorInvalidValue;
+  return launch_tc<FWD_BN, false, false, MODE_FWD_LG, true, NSTAGES, 1, 2>(ta, tb, tc, 1, M, N, K, ep, err, st, &td,
+                                                                            &lg);
+}
 
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
                         int* err, cudaStream_t st) {

@@ -55,6 +55,15 @@ __device__ __forceinline__ float sum_partials(const float* __restrict__ gpart, i
   return g;
 }
 
+// The FF loss terms of Eq. 1 (reading: the negative log-likelihood of the
+// logistic p(real) = sigmoid(g - theta)), shared by every kernel that forms them.
+__device__ __forceinline__ float softplus_f(float t) { return fmaxf(t, 0.f) + log1pf(expf(-fabsf(t))); }
+__device__ __forceinline__ float sigmoid_f(float t) {
+  if (t >= 0.f) return 1.f / (1.f + expf(-t));
+  const float e = expf(t);
+  return e / (1.f + e);
+}
+
 // Device helpers shared by the kernel files.
 __device__ __forceinline__ float warp_sum(float v) {
 #pragma unroll
@@ -284,6 +293,16 @@ int tc_fwd_ntiles(int M, int N, bool narrow);
 int tc_fwd_ntiles_max(int N);
 cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
                         const EpiArgs& ep, int* err, cudaStream_t st);
+// The train step's forward with the local step fused into its epilogue: the
+// forward above (H into ep.out) and everything the local-gradient kernel
+// (launch_grad_prep) computes from it -- dZ' into dZ ([M, ep.ldo] bf16), the
+// bias-gradient, loss and statistics partials, g_out, s_next and the Adam
+// step counter of lg -- bitwise the same.  lg.gpart and lg.ntiles are not
+// used; ep.row_scale must be lg.s.  For N <= 2048 where the GPU can hold the
+// clusters (tc_fwd_lg_supported); cudaErrorInvalidValue otherwise.
+bool tc_fwd_lg_supported(int M, int N);
+cudaError_t tc_gemm_fwd_lg(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, const EpiArgs& ep,
+                           const GradPrepArgs& lg, bf16* dZ, int* err, cudaStream_t st);
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
                           float* C, int ldc, int* err, cudaStream_t st);
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K,
@@ -348,4 +367,12 @@ struct ff_layer {
   // split-K scratch of the fp32 GEMMs (grown on demand; counters kept zero)
   float* kpart; size_t kpart_cap;
   int* kcnt; int kcnt_cap;
+  // bf16 train steps: the local gradient in the forward GEMM's epilogue
+  // (tc_gemm_fwd_lg) where the shape allows, else the separate kernel.  Off
+  // by default: on the 784-2000x4 epoch with 4 layer streams the fused
+  // forward made the epoch slower (9.0 against 8.1 ms): its 8-CTA clusters
+  // wait for 8 free SMs of one GPC while the other layers' kernels run, and
+  // its longer epilogue holds them, where the separate kernel fills gaps on
+  // every SM; alone on one stream it is 2 % faster than forward + kernel.
+  bool fuse_local_grad = false;
 };

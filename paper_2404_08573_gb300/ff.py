@@ -72,6 +72,8 @@ def lib():
         L.ff_status_string.argtypes = [c_int]
         L.ff_row_stride.restype = c_int
         L.ff_row_stride.argtypes = [c_int]
+        L.ff_kernel_launches.restype = ctypes.c_ulonglong
+        L.ff_kernel_launches.argtypes = []
         sig = {
             "ff_layer_create": [POINTER(LayerConfig), c_void_p, POINTER(c_void_p)],
             "ff_layer_destroy": [c_void_p],
@@ -87,6 +89,7 @@ def lib():
             "ff_layer_get_grad": [c_void_p, c_void_p, c_void_p],
             "ff_layer_get_grad_operand": [c_void_p, c_void_p, c_int],
             "ff_layer_check": [c_void_p],
+            "ff_layer_set_fused_local_grad": [c_void_p, c_int],
             "ff_layer_get_stats": [c_void_p, c_void_p],
             "ff_layer_selftest_wait": [c_void_p, ctypes.c_uint, c_void_p],
             "ff_net_create": [c_void_p, c_int, c_int, c_int, POINTER(c_void_p)],
@@ -132,6 +135,11 @@ def _check(status: int, what: str):
 
 def row_stride(features: int) -> int:
     return lib().ff_row_stride(int(features))
+
+
+def kernel_launches() -> int:
+    """ff_kernel_launches: libff's kernel launches in this process so far."""
+    return int(lib().ff_kernel_launches())
 
 
 def _stream(stream) -> int:
@@ -282,6 +290,12 @@ class Layer:
 
     def check(self):
         _check(lib().ff_layer_check(self._h), "ff_layer_check")
+
+    def set_fused_local_grad(self, enable: bool):
+        """ff_layer_set_fused_local_grad: bf16 train steps form the local step in
+        the forward GEMM's epilogue (True) or in a separate kernel (False, the
+        default); bitwise the same results."""
+        _check(lib().ff_layer_set_fused_local_grad(self._h, 1 if enable else 0), "ff_layer_set_fused_local_grad")
 
     def selftest_wait(self, timeout_us: int, stream=None):
         """ff_layer_selftest_wait: a bounded wait that is made to run out."""
