@@ -420,7 +420,12 @@ FF_API ff_status ff_net_train_step_images(ff_net* net, const float* x, const int
  * a given (B, batch count, layout) builds and keeps a plan (task tables,
  * tensor maps, activation rings; it allocates).  Returns with `stream`
  * ordered after all of it (as ff_net_sync).  Not on a Performance-Optimized
- * net (FF_ERR_INVALID_ARG). */
+ * net (FF_ERR_INVALID_ARG).
+ * Roles: by default every SM runs GEMM tiles and streamed tasks side by side.
+ * With the environment variable FF_EPOCH_GEMM_CLUSTERS=n (read when a plan
+ * is built; 1 <= n < the number of resident CTA pairs) n pairs run only GEMM
+ * tiles and the other CTAs only the streamed tasks -- the same bits, and on
+ * the 784-2000x4 epoch slower for every n. */
 FF_API ff_status ff_net_train_epoch(ff_net* net, const float* x, const int* labels, int n_pairs, int B,
                                     int images_per_pair_row, float* loss, void* stream);
 

@@ -155,6 +155,10 @@ struct EpochP {
   // optional trace: per task (GEMM tasks first, then stream tasks) its
   // dequeue, dependencies-met and done times (%globaltimer, ns) and SM id
   unsigned long long* trace;
+  // Roles by cluster: clusters 0 .. gemm_clusters-1 take GEMM tasks; with
+  // split set they take no stream tasks and the other clusters take only
+  // stream tasks (every CTA takes both otherwise).
+  int gemm_clusters, split;
   LayerP lay[kMaxLayers];
 };
 
@@ -685,6 +689,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
   const uint32_t crank = ptx::cluster_ctarank();
   const bool even = crank == 0;
   constexpr uint16_t pmask = 3;
+  const bool gemm_cta = (int)(blockIdx.x / 2) < P.gemm_clusters;
+  const bool stream_cta = !P.split || !gemm_cta;
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < STAGES; ++s) {
@@ -723,7 +729,8 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
         uint2 task;
         if (even) {
           if (!bar_wait(P, &tqe[j], ph ^ 1u)) break;
-          const int idx = atomicAdd(P.cnt + C_QG, 1);
+          // a cluster without the GEMM role hands its roles the end at once
+          const int idx = gemm_cta ? atomicAdd(P.cnt + C_QG, 1) : P.n_gtask;
           task = idx < P.n_gtask ? __ldg(P.gtask + idx) : make_uint2(T_END, 0u);
           if (idx < P.n_gtask) {
             trace_at(P, idx, 0);
@@ -1027,7 +1034,7 @@ __global__ void __launch_bounds__(NTHREADS, 1) k_epoch(const __grid_constant__ E
       }
     }
     if (lane == 0) bulk_wait_all();
-  } else {
+  } else if (stream_cta) {
     // ----------------------------------------------------- streamers
     const int s = (int)threadIdx.x - 32 * STR0;
     int sidx = 0;
@@ -1285,6 +1292,16 @@ ff_status build_plan(ff_net* n, int B, int nb, int xrp, cudaStream_t st, EpochPl
     return s != FF_OK ? s : FF_ERR_UNSUPPORTED;
   }
   p->grid = 2 * clusters;
+  p->P.gemm_clusters = clusters;
+  p->P.split = 0;
+  if (const char* g = std::getenv("FF_EPOCH_GEMM_CLUSTERS")) {
+    // split the roles: this many clusters run GEMM tiles only, the rest stream
+    const int gc = std::atoi(g);
+    if (gc >= 1 && gc < clusters) {
+      p->P.gemm_clusters = gc;
+      p->P.split = 1;
+    }
+  }
   for (int k = 0; k < L; ++k) p->ws.push_back(Ls[k]->X);
   p->B = B;
   p->nb = nb;

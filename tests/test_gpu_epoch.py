@@ -127,3 +127,27 @@ def test_epoch_kernel_784_2000x4_batch1024(env):
         assert abs(got[k] - o["loss"]) <= 1e-3 * o["loss"], (k, got[k], o["loss"])
     na.close()
     nb_.close()
+
+
+def test_epoch_kernel_with_split_roles_is_bitwise_the_per_step_path(env, monkeypatch):
+    """Roles split by cluster (FF_EPOCH_GEMM_CLUSTERS: that many clusters run
+    only GEMM tiles, the others only the streamed tasks): the same bits."""
+    torch, ff = env
+    monkeypatch.setenv("FF_EPOCH_GEMM_CLUSTERS", "8")
+    dims, B, n_pairs = (784, 512, 264), 256, 4 * 256 + 72
+    la, na, lb, nb_ = _nets(ff, dims, B, 0.003, 90)
+    x2, _, lab = _pairs(n_pairs, B, dims[0], seed=91)
+    xg, lg = torch.from_numpy(x2).cuda(), torch.from_numpy(lab).cuda()
+    nbat = -(-n_pairs // B)
+    loss_a = torch.zeros(nbat, 2, device="cuda")
+    loss_b = torch.zeros(nbat, 2, device="cuda")
+    na.train_epoch(xg, lg, n_pairs, B, loss=loss_a)
+    for t, start in enumerate(range(0, n_pairs, B)):
+        b = min(B, n_pairs - start)
+        nb_.train_step(xg[2 * start:2 * start + 2 * b], lg[2 * start:2 * start + 2 * b], B=b, loss=loss_b[t])
+    nb_.sync()
+    torch.cuda.synchronize()
+    assert torch.equal(loss_a, loss_b), ("per-batch loss differences", (loss_a - loss_b).abs().cpu().numpy())
+    _assert_same_state(la, lb, "split roles")
+    na.close()
+    nb_.close()
