@@ -911,10 +911,24 @@ def run_other(args):
                 layers[0].train_step(xb, labels=lb, B=B, h_out=h, next_scale=sc, stream=stream)
                 layers[1].train_step(h, row_scale=sc, B=B, stream=stream)
         _timed_loop(torch, stream, run16, args.warmup)
-        ms = _timed_loop(torch, stream, run16, args.steps) / args.steps
+        ms_eager = _timed_loop(torch, stream, run16, args.steps) / args.steps
+        ms, launch = ms_eager, "eager"
+        ms_graph = None
+        if not args.no_graph:
+            # the 16 steps captured once as a CUDA graph (the launches are the
+            # cost at this size), replayed per timed call
+            graph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(graph, stream=stream):
+                run16()
+            _timed_loop(torch, stream, graph.replay, args.warmup)
+            ms_graph = _timed_loop(torch, stream, graph.replay, args.steps) / args.steps
+            if ms_graph < ms:
+                ms, launch = ms_graph, "one CUDA graph per 16 steps"
         prof = run16
         out.update({"metric": "FF train step latency, 784-500-500 fp32, B=64 pairs", "value": round(1e3 * ms / 16, 2),
                     "unit": "us/step", "higher_is_better": False, "ms_per_step": round(ms, 4), "dtype": "f32",
+                    "launch": launch, "us_per_step_eager": round(1e3 * ms_eager / 16, 2),
+                    "us_per_step_graph": round(1e3 * ms_graph / 16, 2) if ms_graph is not None else None,
                     "config": {"workload": "ff_train_784-500-500_fp32_B64_16steps"}})
     if prof is not None:
         # one more call, each launch timed on its own stream (not the timed calls above)
