@@ -565,12 +565,18 @@ def _traffic(workload, kernel):
         return None
 
 
-def _kernel_profile(lib, torch, fn, pk, workload=None):
+# TF32 against bf16 dense tensor throughput, nominal (1.1 / 2.25 PFLOP/s)
+TF32_PER_BF16 = 1.1 / 2.25
+
+
+def _kernel_profile(lib, torch, fn, pk, workload=None, tf32x3=False):
     """Per-kernel device time of one more call of `fn`, every launch bracketed
     by CUDA events on its own stream by libff's profiler: the kernel table and
     the roofline of the kernel with the most device time (tensor-core GEMMs
-    against the measured bf16 peak, fp32 SIMT GEMMs against the fp32 FMA peak,
-    the rest against the measured HBM copy bandwidth)."""
+    against the measured bf16 peak -- fp32 ones, tf32x3, against the TF32
+    peak it implies over the three products each fp32 term takes -- fp32 SIMT
+    GEMMs against the fp32 FMA peak, the rest against the measured HBM copy
+    bandwidth)."""
     import ctypes
     torch.cuda.synchronize()
     lib.ff_profile_enable(1)
@@ -598,6 +604,9 @@ def _kernel_profile(lib, torch, fn, pk, workload=None):
         top = max(kernels, key=lambda k: k["ms"])
         if "simt" in top["kernel"]:
             bound, peak, src = "alu", FP32_ALU_TFLOPS, "fp32 FMA peak from unit counts and clock (152 x 128 x 2 x 2.07 GHz)"
+        elif top["unit"] == "TFLOP/s" and tf32x3:
+            bound, peak = "tensor", pk["bf16"] * TF32_PER_BF16 / 3
+            src = pk["src"] + " bf16 burst x nominal TF32/bf16 ratio (1.1/2.25) / 3 TF32 products per fp32 term"
         elif top["unit"] == "TFLOP/s":
             bound, peak, src = "tensor", pk["bf16"], pk["src"] + " bf16 burst"
         else:
@@ -636,6 +645,7 @@ def run_other(args):
            "scaling": "weak", "vs_baseline": None, "higher_is_better": True}
     w = args.workload
     prof = None  # the workload's call, profiled once more after the timed calls
+    tf32x3 = False  # its tensor-core GEMMs take fp32 operands (three TF32 products per term)
     if w.startswith("predict"):
         # 10 000 samples x 10 label overlays through 784-2000x4, goodness of layers 2..4
         prec = "fp32" if w.endswith("fp32") else "bf16"
@@ -654,6 +664,7 @@ def run_other(args):
                     "unit": "samples/s", "ms_per_step": round(ms, 4), "dtype": prec, "tflops": round(tf, 2),
                     "frac_of_bf16_peak": round(tf / pk["bf16"], 4) if prec == "bf16" else None,
                     "config": {"workload": f"ff_predict_784-2000x4_{prec}_n10000", "algorithmic_tflop": flops / 1e12}})
+        tf32x3 = prec == "fp32"
     elif w == "adaptive_neg":
         # AdaptiveNEG refresh of one chapter: the strongest wrong label of all
         # 60 000 training samples under goodness prediction through 784-2000x4
@@ -933,7 +944,7 @@ def run_other(args):
     if prof is not None:
         # one more call, each launch timed on its own stream (not the timed calls above)
         out["kernels"], out["roofline"] = _kernel_profile(lib, torch, lambda: _timed_loop(torch, stream, prof, 1), pk,
-                                                          out.get("config", {}).get("workload"))
+                                                          out.get("config", {}).get("workload"), tf32x3)
     print(json.dumps(out), flush=True)
 
 

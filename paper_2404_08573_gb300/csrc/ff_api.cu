@@ -510,21 +510,26 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
   if (L0->K < 10) return FF_ERR_INVALID_ARG;
   const bool b16 = L0->is_bf16;
   const size_t es = b16 ? 2 : 4;
+  // fp32 layers: the GEMMs on the tensor cores (three TF32 products) where
+  // every layer's rows allow TMA, else on the CUDA cores
+  bool f32tc = !b16;
+  for (int k = 0; k < n_layers && f32tc; ++k) f32tc = tc_f32_supported(layers[k]->K, layers[k]->ldK, layers[k]->K);
   int ldmax = 0, ntmax = 0;
   for (int k = 0; k < n_layers; ++k) {
     if (layers[k]->ldN > ldmax) ldmax = layers[k]->ldN;
-    const int nt = b16 ? tc_fwd_ntiles_max(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
+    const int nt = b16 || f32tc ? tc_fwd_ntiles_max(layers[k]->N) : simt_fwd_ntiles(layers[k]->N);
     if (nt > ntmax) ntmax = nt;
   }
   // Samples per chunk: about 40 MB of activations per buffer, so that one
   // chunk's two activation buffers stay resident in L2 between layers.
   long long per = (40ll << 20) / ((long long)10 * ldmax * es);
   int C = (int)(per < 64 ? 64 : per > 8192 ? 8192 : per);
-  if (b16 && n > C) {
+  if ((b16 || f32tc) && n > C) {
     // Each forward GEMM CTA holds a whole SM, so a chunk whose GEMMs end in a
     // nearly empty last wave wastes most of that wave: among chunk sizes
     // down to half the L2 budget, take the one whose widest hidden GEMM fills
-    // its waves best (the largest on ties).
+    // its waves best (the largest on ties).  (fp32 forward GEMMs never narrow
+    // their tiles.)
     int dev = 0, sms = 0;
     if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) ==
                                                    cudaSuccess && sms > 0 && n_layers > 1) {
@@ -534,7 +539,7 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
       double best = -1.0;
       int bestC = C;
       for (int c = C; c >= C / 2 && c >= 64; --c) {
-        const int ctas = tc_gemm_fwd_ctas(10 * c, Nw, true);
+        const int ctas = tc_gemm_fwd_ctas(10 * c, Nw, b16);
         const double eff = (double)ctas / ((double)cdiv(ctas, sms) * sms);
         if (eff > best + 1e-9) {
           best = eff;
@@ -597,6 +602,11 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
                 tc_gemm_store(static_cast<const bf16*>(X0), L0->ldK, L0->Wb, L0->ldK, cn, N1, L0->K, base, L0->ldN,
                               err, st),
                 "layer-1 base GEMM (tcgen05)");
+    } else if (f32tc) {
+      FF_LAUNCH(K_STORE_TC, 2.0 * cn * N1 * L0->K, st,
+                tc_gemm_store_f32(static_cast<const float*>(X0), L0->ldK, L0->W, L0->K, cn, N1, L0->K, base,
+                                  L0->ldN, err, st),
+                "layer-1 base GEMM (fp32, tcgen05 TF32 x 3)");
     } else {
       FF_LAUNCH(K_STORE_SIMT, 2.0 * cn * N1 * L0->K, st,
                 simt_gemm_store(static_cast<const float*>(X0), L0->ldK, L0->W, L0->K, cn, N1, L0->K, base, L0->ldN,
@@ -630,6 +640,13 @@ static ff_status predict_impl(ff_layer* const* layers, int n_layers, const float
                   tc_gemm_fwd(static_cast<const bf16*>(Hb[cur]), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep,
                               err, st),
                   "predict forward GEMM (tcgen05)");
+      } else if (f32tc) {
+        ep.narrow = false;
+        nt = tc_fwd_ntiles(rows, Lk->N, false);
+        FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
+                  tc_gemm_fwd_f32(static_cast<const float*>(Hb[cur]), Lk->ldK, Lk->W, Lk->K, rows, Lk->N, Lk->K, ep,
+                                  err, st),
+                  "predict forward GEMM (fp32, tcgen05 TF32 x 3)");
       } else {
         nt = simt_fwd_ntiles(Lk->N);
         FF_LAUNCH(K_FWD_SIMT, 2.0 * rows * Lk->N * Lk->K, st,

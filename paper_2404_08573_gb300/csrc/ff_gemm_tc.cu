@@ -33,6 +33,13 @@
 //   warps 2..9  epilogue: tcgen05.ld of TMEM lanes 32*(warp%4).., one half of
 //               the columns each -> registers, fused scale/bias/ReLU/goodness
 //               (partials per 128-column half) or plain store
+// fp32 operands (OPB = 4, the exact-precision mode's forward and store
+// GEMMs): the tensor cores' TF32 products in three terms, A B ~ Ah Bh + Ah Bl +
+// Al Bh, where xh is x with the 13 low mantissa bits cleared (exactly a TF32
+// value) and xl = x - xh (exact in fp32); the dropped Al Bl and the TF32
+// truncation of xl leave a relative error near 2^-21 per product.  The
+// epilogue warps, idle during the mainloop, split each landed stage in
+// shared memory (hi in place, lo beside it) before the MMAs read it.
 // Every mbarrier wait is bounded (kWaitTimeoutNs); a timeout latches
 // DEVERR_TIMEOUT in *err, tells the other roles to stop, waits for copies and
 // MMAs already in flight and frees TMEM before the CTA exits.
@@ -60,13 +67,18 @@ constexpr int kLgParts = 16;        // goodness partials of a row (128 columns e
 constexpr int kLogitClasses = 10;
 constexpr int kLogitStride = 12;    // floats per column of the staged block weights (three float4)
 
-template <int BN, int NSTAGE, int MT, bool PAIR, int NT = 1>
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT = 1, int OPB = 2>
 struct TcCfg {
+  // OPB: bytes per operand element (2: bf16; 4: fp32 through three TF32
+  // products).  A k-block is one 128-byte swizzle row either way: BKE
+  // elements, so tile byte sizes do not depend on the type.
+  static constexpr int BKE = 128 / OPB;
   static constexpr int TN = NT * BN;                // columns of the tile (NT column subtiles of BN)
-  static constexpr int A_BYTES = MT * BM * BK * 2;  // MT row subtiles of BM rows
+  static constexpr int A_BYTES = MT * BM * 128;     // MT row subtiles of BM rows
   static constexpr int BH = PAIR ? BN / 2 : BN;     // B columns of a column subtile this CTA loads
-  static constexpr int B_BYTES = NT * BH * BK * 2;
-  static constexpr int STAGE = A_BYTES + B_BYTES;
+  static constexpr int B_BYTES = NT * BH * 128;
+  static constexpr int IN_BYTES = A_BYTES + B_BYTES;  // what TMA brings per stage
+  static constexpr int STAGE = (OPB == 4 ? 2 : 1) * IN_BYTES;  // fp32: the lo parts beside
   static constexpr int STAGES = NSTAGE;
   static constexpr int SMEM = STAGES * STAGE + 1024 /*alignment slack*/ + 256 /*barriers*/ + TN * 4 /*bias*/;
   // the local-gradient epilogue: every partial of the cluster's row block,
@@ -77,12 +89,13 @@ struct TcCfg {
   static_assert(BN % 64 == 0 && BN <= 256, "BN must be a multiple of 64, at most 256");
   static_assert(MT >= 1 && NT >= 1 && MT * NT * ACC_COLS <= 512, "accumulators must fit in TMEM");
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
-  static_assert(MT * 4 * 32 * TN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
+  static_assert(OPB == 4 || MT * 4 * 32 * TN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
+  static_assert(OPB == 2 || OPB == 4, "bf16 or fp32 operands");
   static_assert(EPI_WARPS * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
   static_assert(TN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
   static_assert(NT == 1 || TN / (EPI_WARPS / 4) == BN, "with column subtiles each epilogue warp reads one accumulator");
   static_assert(!PAIR || BH % 64 == 0, "each CTA of a pair loads whole 64-column B groups");
-  static_assert(2 * STAGES * 8 + 8 + 16 + 8 <= 256, "barriers, TMEM slot, flags and the LG barrier fit below the bias tile");
+  static_assert(3 * STAGES * 8 + 8 + 16 + 8 <= 256, "barriers, TMEM slot, flags and the LG barrier fit below the bias tile");
 };
 
 __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
@@ -95,15 +108,18 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
 // gradient blocks of the other layers' streams (784-2000x4 epoch -1 %).
 // MODE_FWD_LG: tmD maps dZ' (as tmC maps H) and lg holds the local step's
 // arguments; the grid's column tiles all lie in one cluster (2 x gridDim.y).
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB>
 __global__ void __launch_bounds__(NTHREADS, 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmD, int tma_store, int M,
               int N, int K, EpiArgs ep, GradPrepArgs lg, int* err) {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT>;
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB>;
   constexpr bool FWD = MODE != MODE_STORE;
   constexpr bool LOGITS = MODE == MODE_FWD_LOGITS;
   constexpr bool LG = MODE == MODE_FWD_LG;
+  constexpr bool TF32 = OPB == 4;
+  static_assert(!TF32 || (!A_MN && !B_MN && (MODE == MODE_FWD || MODE == MODE_STORE)),
+                "fp32 operands: K-major forward and store GEMMs");
   static_assert(!LG || (PAIR && MT == 1 && NT == 2 && BN == 256 && EPI_WARPS == 8),
                 "the local-gradient epilogue: 128 rows x 512 columns per CTA, a warp per 32 rows x 256 columns");
   extern __shared__ uint8_t smem_raw[];
@@ -112,13 +128,16 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   uint8_t* smem = smem_raw + ((1024u - (raw_s & 1023u)) & 1023u);
   uint8_t* sA = smem;
   uint8_t* sB = smem + C::STAGES * C::A_BYTES;
-  uint64_t* full = reinterpret_cast<uint64_t*>(sB + C::STAGES * C::B_BYTES);
+  // fp32: the lo parts of A and B, at the same offsets one ring further on
+  constexpr int LO = C::STAGES * C::IN_BYTES;
+  uint64_t* full = reinterpret_cast<uint64_t*>(smem + C::STAGES * C::STAGE);
   uint64_t* empty = full + C::STAGES;
   uint64_t* tfull = empty + C::STAGES;
   uint32_t* tslot = reinterpret_cast<uint32_t*>(tfull + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tslot + 1);
   volatile int* never_set = reinterpret_cast<volatile int*>(tslot + 2);  // drain waits ignore the abort
   uint64_t* lgbar = reinterpret_cast<uint64_t*>(tslot + 4);  // LG: every partial of the row block has arrived
+  uint64_t* conv = lgbar + 1;  // fp32: [STAGES] both CTAs' splits of a stage are done
   float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [TN] bias of this tile
   float* sVt = sbias + C::TN;  // LOGITS: [BN][kLogitStride] block weights of this tile's columns
   // LG: [kLgParts][MT * BM] goodness partials of this CTA's rows (partial t
@@ -132,7 +151,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   // cta_group::2 requires); blockIdx.y: column tile
   const int m0 = blockIdx.x * (BM * MT);
   const int n0 = blockIdx.y * C::TN;
-  const int num_kb = (K + BK - 1) / BK;
+  const int num_kb = (K + C::BKE - 1) / C::BKE;
 
   // PAIR: the two CTAs of a cluster (consecutive tile rows, same columns)
   // compute their 2 x MT x BM rows with cta_group::2 MMAs (M = 256).  Each
@@ -156,6 +175,8 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     }
     ptx::mbar_init(tfull, 1);
     if constexpr (LG) ptx::mbar_init(lgbar, 32 * EPI_WARPS * gridDim.y);  // every epilogue lane of the row block
+    if constexpr (TF32)
+      for (int s = 0; s < C::STAGES; ++s) ptx::mbar_init(&conv[s], (PAIR ? 2 : 1) * EPI_WARPS);
     *abort_flag = 0;
     *never_set = 0;
     ptx::fence_mbar_init();
@@ -189,11 +210,13 @@ __global__ void __launch_bounds__(NTHREADS, 2)
       uint32_t full0 = ptx::smem_u32(&full[0]);
       if constexpr (PAIR) full0 = ptx::mapa_shared(full0, pair_lead);
       auto load = [&](void* dst, const CUtensorMap* map, int s, int c0, int c1) {
-        if (!ff_dcheck(tma_x_aligned(c0, 2), err)) {
+        if (!ff_dcheck(tma_x_aligned(c0, OPB), err)) {
           *abort_flag = 1;
           return;
         }
-        if constexpr (PAIR)
+        // fp32: each CTA's copies complete on its own barrier (its epilogue
+        // warps split them before the pair's MMAs read them)
+        if constexpr (PAIR && !TF32)
           ptx::tma_load_2d_pair(dst, map, full0 + 8u * (uint32_t)s, c0, c1);
         else
           ptx::tma_load_2d(dst, map, &full[s], c0, c1);
@@ -207,10 +230,13 @@ __global__ void __launch_bounds__(NTHREADS, 2)
           latch(err, abort_flag);
           break;
         }
-        if (issuer) ptx::mbar_arrive_expect_tx(&full[s], PAIR ? 2 * C::STAGE : C::STAGE);
+        if constexpr (TF32)
+          ptx::mbar_arrive_expect_tx(&full[s], C::IN_BYTES);
+        else if (issuer)
+          ptx::mbar_arrive_expect_tx(&full[s], PAIR ? 2 * C::STAGE : C::STAGE);
         uint8_t* a = sA + s * C::A_BYTES;
         uint8_t* b = sB + s * C::B_BYTES;
-        const int k0 = kb * BK;
+        const int k0 = kb * C::BKE;
         if (!A_MN) {
 #pragma unroll
           for (int mt = 0; mt < MT; ++mt) load(a + mt * BM * BK * 2, &tmA, s, k0, m0 + BM * mt);
@@ -239,7 +265,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         }
       }
       if (*abort_flag) {
-        if (issuer) {
+        if (issuer || TF32) {
           // let copies already issued land before the CTA's shared memory goes away
           int lo = issued - C::STAGES;
           if (lo < 0) lo = 0;
@@ -257,11 +283,15 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   } else if (warp == 1) {
     // ----------------------------------------------------------------- MMA
     if (lane == 0 && issuer) {
-      constexpr uint32_t idesc = ptx::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
+      constexpr uint32_t idesc = TF32 ? ptx::idesc_tf32_f32(PAIR ? 2 * BM : BM, BN)
+                                      : ptx::idesc_bf16_f32(PAIR ? 2 * BM : BM, BN, A_MN ? 1 : 0, B_MN ? 1 : 0);
       for (int kb = 0; kb < num_kb; ++kb) {
         const int s = kb % C::STAGES;
         const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
-        if (!ptx::mbar_wait(&full[s], ph, kWaitTimeoutNs, abort_flag)) {
+        // fp32: the stage is split in both CTAs (remote arrivals: cluster-scope acquire)
+        const bool ready = TF32 ? ptx::mbar_wait_cluster(&conv[s], ph, kWaitTimeoutNs, abort_flag)
+                                : ptx::mbar_wait(&full[s], ph, kWaitTimeoutNs, abort_flag);
+        if (!ready) {
           latch(err, abort_flag);
           break;
         }
@@ -287,10 +317,24 @@ __global__ void __launch_bounds__(NTHREADS, 2)
               const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
                                        : ptx::sdesc_sw128(as + k * 32, 16, 1024);
               const uint32_t acc = tmem + (uint32_t)((mt * NT + nt) * C::ACC_COLS);
-              if constexpr (PAIR)
+              if constexpr (TF32) {
+                // Ah Bh + Ah Bl + Al Bh (the lo parts LO bytes further on)
+                const uint64_t adl = ptx::sdesc_sw128(as + LO + k * 32, 16, 1024);
+                const uint64_t bdl = ptx::sdesc_sw128(bs + LO + k * 32, 16, 1024);
+                if constexpr (PAIR) {
+                  ptx::umma_tf32_pair(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+                  ptx::umma_tf32_pair(acc, ad, bdl, idesc, 1u);
+                  ptx::umma_tf32_pair(acc, adl, bd, idesc, 1u);
+                } else {
+                  ptx::umma_tf32(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+                  ptx::umma_tf32(acc, ad, bdl, idesc, 1u);
+                  ptx::umma_tf32(acc, adl, bd, idesc, 1u);
+                }
+              } else if constexpr (PAIR) {
                 ptx::umma_f16_pair(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
-              else
+              } else {
                 ptx::umma_f16(acc, ad, bd, idesc, (kb | k) != 0 ? 1u : 0u);
+              }
             }
           }
         }
@@ -351,13 +395,49 @@ __global__ void __launch_bounds__(NTHREADS, 2)
       }
       ptx::named_bar(1, 32 * EPI_WARPS);
     }
+    if constexpr (TF32) {
+      // Split every stage this CTA receives: x -> xh = x with the 13 low
+      // mantissa bits cleared (in place), xl = x - xh (LO bytes further on);
+      // then one arrival per warp on the pair's (even CTA's) barrier.
+      constexpr int V4 = C::IN_BYTES / 16;  // 16-byte words per stage
+      const int t = (int)threadIdx.x - 64;
+      for (int kb = 0; kb < num_kb; ++kb) {
+        const int s = kb % C::STAGES;
+        const uint32_t ph = (uint32_t)(kb / C::STAGES) & 1u;
+        const bool got = ptx::mbar_wait(&full[s], ph, kWaitTimeoutNs, abort_flag);
+        if (!got) latch(err, abort_flag);
+        if (!__all_sync(0xffffffffu, got && !*abort_flag)) break;
+        // the stage's A and B boxes: A_BYTES at sA + s A_BYTES, B_BYTES at sB + s B_BYTES
+        for (int i = t; i < V4; i += 32 * EPI_WARPS) {
+          const int byte = i * 16;
+          uint8_t* p = byte < C::A_BYTES ? sA + s * C::A_BYTES + byte : sB + s * C::B_BYTES + (byte - C::A_BYTES);
+          uint4 x = *reinterpret_cast<uint4*>(p);
+          uint4 h, l;
+          h.x = x.x & 0xFFFFE000u; h.y = x.y & 0xFFFFE000u; h.z = x.z & 0xFFFFE000u; h.w = x.w & 0xFFFFE000u;
+          l.x = __float_as_uint(__fsub_rn(__uint_as_float(x.x), __uint_as_float(h.x)));
+          l.y = __float_as_uint(__fsub_rn(__uint_as_float(x.y), __uint_as_float(h.y)));
+          l.z = __float_as_uint(__fsub_rn(__uint_as_float(x.z), __uint_as_float(h.z)));
+          l.w = __float_as_uint(__fsub_rn(__uint_as_float(x.w), __uint_as_float(h.w)));
+          *reinterpret_cast<uint4*>(p) = h;
+          *reinterpret_cast<uint4*>(p + LO) = l;
+        }
+        ptx::fence_async_smem();  // the MMAs (async proxy) read what these generic writes left
+        __syncwarp();
+        if (lane == 0) {
+          if (issuer)
+            ptx::mbar_arrive(&conv[s]);
+          else
+            ptx::mbar_arrive_remote(&conv[s], pair_lead);
+        }
+      }
+    }
     const bool ok = ptx::mbar_wait(tfull, 0, kWaitTimeoutNs, abort_flag);
     if (threadIdx.x == 64) ptx::griddep_launch_dependents();  // the mainloop is done
     if (!ok) latch(err, abort_flag);
     ptx::tc_fence_after();
     // tcgen05.ld is warp-collective: decide for the whole warp at once
     if (__all_sync(0xffffffffu, ok && !*abort_flag)) {
-      constexpr int ES = FWD ? 2 : 4;      // staged element size
+      constexpr int ES = FWD && !TF32 ? 2 : 4;  // staged element size (the output's)
       constexpr int CW = 128 / ES;                       // columns per 128-byte swizzle row
       const uint32_t sw = (uint32_t)(lane & 7);
       const bool staged = FWD || tma_store;
@@ -367,7 +447,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const int rbase = m0 + mt * BM + q * 32;  // this warp's first row in subtile mt
         const int gi = rbase + lane;
         // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
-        uint8_t* stage = smem + (FWD ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
+        uint8_t* stage = smem + (FWD && !TF32 ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
         const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)((mt * NT + cbase / BN) * C::ACC_COLS + cbase % BN);
         const float s = srow[mt];
@@ -381,7 +461,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         // c0 counts columns within this warp's half.
         auto process = [&](const uint32_t (&r)[32], int c0) {
           const int col0 = n0 + cbase + c0;
-          if (FWD) {
+          if (FWD && !TF32) {
             uint32_t packed[16];
             const float4* b4 = reinterpret_cast<const float4*>(sbias + cbase + c0);
 #pragma unroll
@@ -428,9 +508,22 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             __syncwarp();
             uint8_t* base = sbuf + lane * 128;
 #pragma unroll
-            for (int v = 0; v < 8; ++v)
-              *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) =
-                  make_uint4(r[4 * v], r[4 * v + 1], r[4 * v + 2], r[4 * v + 3]);
+            for (int v = 0; v < 8; ++v) {
+              uint32_t o[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                if constexpr (FWD) {
+                  // fp32 forward: the activity itself, and its goodness
+                  const float z = fmaf(s, __uint_as_float(r[4 * v + e]), sbias[cbase + c0 + 4 * v + e]);
+                  const float h = z != z ? z : fmaxf(z, 0.f);
+                  g = fmaf(h, h, g);
+                  o[e] = __float_as_uint(h);
+                } else {
+                  o[e] = r[4 * v + e];
+                }
+              }
+              *reinterpret_cast<uint4*>(base + (((uint32_t)v ^ sw) << 4)) = make_uint4(o[0], o[1], o[2], o[3]);
+            }
             ptx::fence_async_smem();
             __syncwarp();
             if (lane == 0 && rbase < M && col0 < ep.ldo &&
@@ -471,7 +564,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
 #pragma unroll
           for (int c = 0; c < kLogitClasses; c += 2) zp[c / 2] = make_float2(zl[c], zl[c + 1]);
         }
-        if (FWD) {
+        if (FWD && !TF32) {
           ptx::fence_async_smem();
           __syncwarp();
           if (lane == 0 && rbase < M) {
@@ -683,9 +776,9 @@ bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, in
   return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
 
-template <int BN, int NSTAGE, int MT, bool PAIR, int NT, int MODE>
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT, int MODE, int OPB>
 constexpr int tc_smem() {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT>;
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB>;
   return C::SMEM + (MODE == MODE_FWD_LOGITS ? BN * kLogitStride * 4 : 0) + (MODE == MODE_FWD_LG ? C::LG_SMEM : 0);
 }
 
@@ -693,9 +786,9 @@ constexpr int tc_smem() {
 // pairs; a padding CTA loads zeros, supplies its half of B and writes
 // nothing), clusters of the pair (LG: of the pair and every column tile),
 // and programmatic stream serialization.
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB = 2>
 struct TcLaunch {
-  static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE>();
+  static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE, OPB>();
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
   static constexpr int CM = PAIR ? 2 : 1;
   cudaLaunchConfig_t cfg = {};
@@ -715,18 +808,18 @@ struct TcLaunch {
     cfg.attrs = at;
     cfg.numAttrs = 2;
   }
-  static auto kernel() { return k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT>; }
+  static auto kernel() { return k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB>; }
   static cudaError_t set_attrs() {
     static cudaError_t e = cudaFuncSetAttribute(kernel(), cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     return e;
   }
 };
 
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT = 1>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT = 1, int OPB = 2>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st, const CUtensorMap* td = nullptr,
                       const GradPrepArgs* lg = nullptr) {
-  using Lc = TcLaunch<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT>;
+  using Lc = TcLaunch<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB>;
   const cudaError_t attr = Lc::set_attrs();
   if (attr != cudaSuccess) return attr;
   Lc l(M, N, st);
@@ -908,6 +1001,47 @@ cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R,
     return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, N, K, R, ep, err,
                                                                                    st);
   return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
+}
+
+// ------------------------------------------------ fp32 operands (3 x TF32)
+// Stages of fp32 tiles with their lo parts: 96 KB with two 128-row subtiles
+// per CTA (2 fit), 64 KB with one (3 fit).
+constexpr int NSTAGES_F32 = 2;
+constexpr int NSTAGES_F32_SMALL = 3;
+
+bool tc_f32_supported(int K, int lda, int ldb) {
+  // TMA rows of 16-byte multiples: fp32 row strides and K in multiples of 4
+  return tc_supported() && (K & 3) == 0 && (lda & 3) == 0 && (ldb & 3) == 0;
+}
+
+cudaError_t tc_gemm_fwd_f32(const float* A, int lda, const float* B, int ldb, int M, int N, int K, const EpiArgs& ep,
+                            int* err, cudaStream_t st) {
+  if (!tc_f32_supported(K, lda, ldb) || ep.logit_V || ep.gpart_in || (ep.ldo & 3)) return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, tc;
+  if (!make_map(&ta, A, 4, K, M, lda, 32, BM) || !make_map(&tb, B, 4, K, N, ldb, 32, b_box_rows(FWD_BN)) ||
+      !make_map(&tc, ep.out, 4, ep.ldo, M, ep.ldo, 32, 32))
+    return cudaErrorInvalidValue;
+  if (shape_of(M, N, FWD_BN) != SHAPE_FULL)
+    return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_F32_SMALL, 1, 1, 4>(ta, tb, tc, 1, M, N, K, ep,
+                                                                                          err, st);
+  return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_F32, ROW_SUBTILES, 1, 4>(ta, tb, tc, 1, M, N, K,
+                                                                                              ep, err, st);
+}
+
+cudaError_t tc_gemm_store_f32(const float* A, int lda, const float* B, int ldb, int M, int N, int K, float* Cm,
+                              int ldc, int* err, cudaStream_t st) {
+  if (!tc_f32_supported(K, lda, ldb)) return cudaErrorInvalidValue;
+  CUtensorMap ta, tb, tc;
+  if (!make_map(&ta, A, 4, K, M, lda, 32, BM) || !make_map(&tb, B, 4, K, N, ldb, 32, b_box_rows(FWD_BN)))
+    return cudaErrorInvalidValue;
+  const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
+  if (!tma) tc = ta;  // unused
+  EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
+  if (shape_of(M, N, FWD_BN) != SHAPE_FULL)
+    return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_F32_SMALL, 1, 1, 4>(ta, tb, tc, tma, M, N, K,
+                                                                                            ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_F32, ROW_SUBTILES, 1, 4>(ta, tb, tc, tma, M, N,
+                                                                                                K, ep, err, st);
 }
 
 }  // namespace ff

@@ -305,6 +305,15 @@ cudaError_t tc_gemm_fwd_lg(const bf16* A, int lda, const bf16* B, int ldb, int M
                            const GradPrepArgs& lg, bf16* dZ, int* err, cudaStream_t st);
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K,
                           float* C, int ldc, int* err, cudaStream_t st);
+// The same forward (without gpart_in or block logits) and store GEMMs on fp32
+// operands, as three TF32 tensor-core products per term (Ah Bh + Ah Bl +
+// Al Bh; relative error near 2^-21 per product); H is written in fp32.  For K
+// and both row strides multiples of 4 (tc_f32_supported).
+bool tc_f32_supported(int K, int lda, int ldb);
+cudaError_t tc_gemm_fwd_f32(const float* A, int lda, const float* B, int ldb, int M, int N, int K, const EpiArgs& ep,
+                            int* err, cudaStream_t st);
+cudaError_t tc_gemm_store_f32(const float* A, int lda, const float* B, int ldb, int M, int N, int K, float* C, int ldc,
+                              int* err, cudaStream_t st);
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K,
                           float* C, int ldc, int* err, cudaStream_t st);
 bool tc_supported();

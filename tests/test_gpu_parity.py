@@ -248,7 +248,10 @@ def test_config0_sixteen_steps_fp32(env):
 
 # ---------------------------------------------------------------- predict
 @pytest.mark.parametrize("prec,dims,n", [("fp32", (784, 256, 256, 128), 300), ("bf16", (784, 256, 256, 128), 300),
-                                         ("bf16", (784, 96), 40), ("bf16", (784, 200, 128), 9000)])
+                                         ("bf16", (784, 96), 40), ("bf16", (784, 200, 128), 9000),
+                                         # fp32 on the tensor cores (three TF32 products) at several tile
+                                         # shapes, and widths that are not multiples of 4 (CUDA-core GEMMs)
+                                         ("fp32", (784, 200, 128), 3000), ("fp32", (786, 130, 66), 250)])
 def test_predict(env, prec, dims, n):
     torch, ff = env
     layers, states = [], []
@@ -258,7 +261,7 @@ def test_predict(env, prec, dims, n):
         l.set_state(W=W, b=b)
         layers.append(l)
         states.append(fo.LayerState(W, b))
-    x = synth.mnist_like(n, seed=31)
+    x = synth.mnist_like(n, seed=31, features=dims[0])
     G = torch.empty(n, 10, device="cuda")
     pred, _ = ff.predict(layers, torch.from_numpy(x).cuda(), goodness=G)
     torch.cuda.synchronize()
