@@ -706,9 +706,14 @@ def run_other(args):
             y = torch.from_numpy(synth.labels(n, seed=7)).to(dev)
             steps = [(r, min(BATCH, n - r)) for r in range(0, n, BATCH)]
 
-            def fn():
+            def per_step():
                 for r, b in steps:
                     head.train_step(layers, x[r:r + b], y[r:r + b], stream=stream)
+
+            # the same steps, the features of 16 steps formed by one forward pass
+            fn = lambda: head.train_epoch(layers, x, y, BATCH, stream=stream)
+            _timed_loop(torch, stream, per_step, args.warmup)
+            out["ms_per_step_one_call_per_step"] = round(_timed_loop(torch, stream, per_step, args.steps) / args.steps, 4)
             flops = n * (fwd_flops + 4.0 * 10 * F)
             label = f"ff_softmax_train_784-2000x4_bf16_epoch{n}_B{BATCH}"
             metric = "FF softmax-head train samples/s (neutral pass, CE backprop through the head, Adam) on 4x2000 net"

@@ -196,6 +196,18 @@ FF_API ff_status ff_head_train_step(ff_head* head, ff_layer* const* layers, int 
                                     const float* x, const int* labels, int n, float* loss,
                                     void* stream);
 
+/* ceil(n / B) consecutive train steps of the head, as ff_head_train_step on
+ * rows [tB, tB + B) of x and labels for t = 0, 1, ... (the last step takes the
+ * rest), bitwise the same.  The layers do not change during head training,
+ * so the neutral forward runs once over many steps' rows (up to 16384 per
+ * pass, whole steps) and each step's logits, gradient and Adam update read
+ * their rows of the stored activities.  B <= max_rows; the workspace grows to
+ * the rows of one forward pass.  loss [ceil(n / B)] (device) or NULL receives
+ * each step's mean cross-entropy. */
+FF_API ff_status ff_head_train_epoch(ff_head* head, ff_layer* const* layers, int n_layers,
+                                     const float* x, const int* labels, int n, int B, float* loss,
+                                     void* stream);
+
 /* Softmax prediction of n raw input rows (any n; processed in chunks of
  * max_rows): pred [n] int32 = the class with the largest logit (the lowest
  * on ties) and/or logits [n, 10] float32; either may be NULL, not both. */

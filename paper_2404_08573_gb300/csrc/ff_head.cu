@@ -811,9 +811,13 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
 }
 
 // Neutral-labelled forward of `rows` raw input rows through every layer:
-// H_k and the row scale of every activity.
+// H_k and the row scale of every activity.  narrow: the forward GEMMs may take
+// 128-column tiles when their grid is small (predict); training keeps
+// 256-column tiles at every row count, so that a row's goodness partials --
+// and with them every activity scale -- do not depend on how many rows share
+// the GEMM (ff_head_train_epoch runs many steps' rows at once).
 ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows, const HeadWork& w, int* err,
-                       cudaStream_t st) {
+                       cudaStream_t st, bool narrow) {
   ff_layer* L0 = layers[0];
   const bool b16 = L0->is_bf16;
   const double es = b16 ? 2.0 : 4.0;
@@ -825,7 +829,7 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
     ff_layer* Lk = layers[k];
     float* gpart = b16 && (k & 1) ? w.gpart2 : w.gpart;
     EpiArgs ep{w.S[k], Lk->cfg.has_bias ? Lk->b : nullptr, w.Hk[k], Lk->ldN, gpart};
-    ep.narrow = true;
+    ep.narrow = narrow;
     int nt;
     if (b16) {
       if (k >= 1) {
@@ -836,7 +840,7 @@ ff_status head_forward(ff_layer* const* layers, int L, const float* x, int rows,
         ep.ntiles_in = nt_prev;
         ep.s_out = w.S[k];
       }
-      nt = tc_fwd_ntiles(rows, Lk->N, true);
+      nt = tc_fwd_ntiles(rows, Lk->N, narrow);
       FF_LAUNCH(K_FWD_TC, 2.0 * rows * Lk->N * Lk->K, st,
                 tc_gemm_fwd(static_cast<const bf16*>(in), Lk->ldK, Lk->Wb, Lk->ldK, rows, Lk->N, Lk->K, ep, err, st),
                 "head forward GEMM (tcgen05)");
@@ -1081,6 +1085,34 @@ ff_status ff_head_destroy(ff_head* hd) {
   return FF_OK;
 }
 
+// Rows of stored features ff_head_train_epoch forms per forward pass.
+constexpr int kEpochFeatureRows = 16384;
+
+// The head's part of one train step on n rows of the features in w, starting
+// at row r0 of the stored activities: logits, softmax, loss and dz
+// (k_head_dot), dV partials (k_head_wgrad), Adam on V and c (k_head_adam).
+static ff_status head_step_on_features(ff_head* hd, ff_layer* const* layers, int n_layers, const HeadWork& w, int r0,
+                                       const int* labels, int n, float* loss, cudaStream_t st) {
+  Segs sg = make_segs(layers, n_layers, w, hd->F);
+  const bool b16 = layers[0]->is_bf16;
+  const double es = b16 ? 2.0 : 4.0;
+  for (int j = 0; j < sg.nseg; ++j) {
+    sg.H[j] = static_cast<const char*>(sg.H[j]) + (size_t)r0 * sg.ld[j] * (size_t)es;
+    sg.s[j] += r0;
+  }
+  int* err = &hd->ds->err;
+  ff_status s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, err, st);
+  if (s != FF_OK) return s;
+  FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
+            launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
+  const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kDotRows), n, loss);
+  const int vblocks = cdiv((long long)kClasses * hd->F, 256);
+  PdlLaunch l(dim3(vblocks + 1), dim3(256), st);
+  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st, cudaLaunchKernelEx(&l.cfg, k_head_adam, a),
+            "head Adam");
+  return FF_OK;
+}
+
 ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, const int* labels,
                              int n, float* loss, void* stream) {
   ff::NvtxRange nvtx_("ff_head_train_step");
@@ -1095,20 +1127,40 @@ ff_status ff_head_train_step(ff_head* hd, ff_layer* const* layers, int n_layers,
   if (s != FF_OK) return s;
   hd->last_stream = st;
   int* err = &hd->ds->err;
-  s = head_forward(layers, n_layers, x, n, w, err, st);
+  s = head_forward(layers, n_layers, x, n, w, err, st, false);
   if (s != FF_OK) return s;
-  const Segs sg = make_segs(layers, n_layers, w, hd->F);
-  const bool b16 = layers[0]->is_bf16;
-  const double es = b16 ? 2.0 : 4.0;
-  s = head_logits(hd, sg, b16, n, labels, nullptr, w.zpart, w.dz, w.part, err, st);
+  return head_step_on_features(hd, layers, n_layers, w, 0, labels, n, loss, st);
+}
+
+ff_status ff_head_train_epoch(ff_head* hd, ff_layer* const* layers, int n_layers, const float* x, const int* labels,
+                              int n, int B, float* loss, void* stream) {
+  ff::NvtxRange nvtx_("ff_head_train_epoch");
+  if (!hd || n < 0 || B < 1) return FF_ERR_INVALID_ARG;
+  ff_status s = head_layers(hd, layers, n_layers);
   if (s != FF_OK) return s;
-  FF_LAUNCH(K_HEAD_WGRAD, (double)n * hd->F * es + (double)cdiv(n, kWgRows) * kClasses * hd->F * 4, st,
-            launch_head_wgrad(sg, b16, n, w.dz, w.dVpart, st), "head weight gradient");
-  const HeadAdamArgs a = head_adam_args(hd, w.dVpart, cdiv(n, kWgRows), w.part, cdiv(n, kDotRows), n, loss);
-  const int vblocks = cdiv((long long)kClasses * hd->F, 256);
-  PdlLaunch l(dim3(vblocks + 1), dim3(256), st);
-  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (a.nrb * 4.0 + 28), st, cudaLaunchKernelEx(&l.cfg, k_head_adam, a),
-            "head Adam");
+  if (n == 0) return FF_OK;
+  if (!x || !labels || B > hd->cfg.max_rows) return FF_ERR_INVALID_ARG;
+  cudaStream_t st = static_cast<cudaStream_t>(stream);
+  // Rows whose features one forward pass forms: whole steps, up to
+  // kEpochFeatureRows (at least one step).
+  const int steps_per_chunk = kEpochFeatureRows / B > 0 ? kEpochFeatureRows / B : 1;
+  const int R = (int)((long long)steps_per_chunk * B < n ? (long long)steps_per_chunk * B : n);
+  HeadWork w;
+  s = head_workspace(hd, layers, n_layers, R, true, &w);
+  if (s != FF_OK) return s;
+  hd->last_stream = st;
+  int* err = &hd->ds->err;
+  const int K0 = layers[0]->K;
+  for (int r0 = 0, t = 0; r0 < n; r0 += R) {
+    const int rows = n - r0 < R ? n - r0 : R;
+    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, rows, w, err, st, false);
+    if (s != FF_OK) return s;
+    for (int q = 0; q < rows; q += B, ++t) {
+      const int b = rows - q < B ? rows - q : B;
+      s = head_step_on_features(hd, layers, n_layers, w, q, labels + r0 + q, b, loss ? loss + t : nullptr, st);
+      if (s != FF_OK) return s;
+    }
+  }
   return FF_OK;
 }
 
@@ -1131,7 +1183,7 @@ ff_status ff_head_predict(ff_head* hd, ff_layer* const* layers, int n_layers, co
   const int K0 = layers[0]->K;
   for (int r0 = 0; r0 < n; r0 += C) {
     const int cn = (n - r0) < C ? (n - r0) : C;
-    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, cn, w, err, st);
+    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, cn, w, err, st, true);
     if (s != FF_OK) return s;
     const Segs sg = make_segs(layers, n_layers, w, hd->F);
     float* z = logits ? logits + (size_t)r0 * kClasses : w.logits;
@@ -1394,7 +1446,7 @@ ff_status ff_po_predict(ff_layer* const* layers, int n_layers, ff_head* hd, cons
   ff_layer* top = layers[n_layers - 1];
   for (int r0 = 0; r0 < n; r0 += C) {
     const int cn = (n - r0) < C ? (n - r0) : C;
-    s = head_forward(layers, n_layers, x + (size_t)r0 * layers[0]->K, cn, w, err, st);
+    s = head_forward(layers, n_layers, x + (size_t)r0 * layers[0]->K, cn, w, err, st, true);
     if (s != FF_OK) return s;
     Segs sg{};
     sg.H[0] = w.Hk[n_layers - 1];

@@ -106,6 +106,7 @@ def lib():
             "ff_head_create": [POINTER(HeadConfig), POINTER(c_void_p)],
             "ff_head_destroy": [c_void_p],
             "ff_head_train_step": [c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_void_p, c_void_p],
+            "ff_head_train_epoch": [c_void_p, c_void_p, c_int, c_void_p, c_void_p, c_int, c_int, c_void_p, c_void_p],
             "ff_head_predict": [c_void_p, c_void_p, c_int, c_void_p, c_int, c_void_p, c_void_p, c_void_p],
             "ff_head_get_state": [c_void_p] + [c_void_p] * 6 + [POINTER(c_longlong)],
             "ff_head_set_state": [c_void_p] + [c_void_p] * 6 + [c_longlong],
@@ -473,6 +474,17 @@ class Head:
         _check(lib().ff_head_train_step(self._h, _layer_array(layers), len(layers), _ptr(x, torch.float32, "x"),
                                         _ptr(labels, torch.int32, "labels"), n, _ptr(loss, torch.float32, "loss"),
                                         c_void_p(_stream(stream))), "ff_head_train_step")
+
+    def train_epoch(self, layers, x, labels, B, loss=None, stream=None):
+        """ff_head_train_epoch: ceil(n / B) train steps on consecutive rows, the
+        features of many steps formed by one forward pass."""
+        n = x.shape[0]
+        if labels.shape[0] != n:
+            raise ValueError("labels must have one entry per row of x")
+        _check(lib().ff_head_train_epoch(self._h, _layer_array(layers), len(layers), _ptr(x, torch.float32, "x"),
+                                         _ptr(labels, torch.int32, "labels"), n, int(B),
+                                         _ptr(loss, torch.float32, "loss"), c_void_p(_stream(stream))),
+               "ff_head_train_epoch")
 
     def predict(self, layers, x, pred=None, logits=None, stream=None):
         """Returns (pred, logits)."""

@@ -150,6 +150,38 @@ def test_head_predict_matches_oracle(env, prec, dims, n, max_rows):
     assert np.array_equal(p, np.argmax(logits.cpu().numpy(), axis=1))
 
 
+@pytest.mark.parametrize("prec,dims,n,B", [
+    ("bf16", (784, 256, 256, 128), 5 * 512 + 100, 512),      # one forward pass, a ragged last step
+    ("bf16", (784, 512, 256), 17 * 1024 + 300, 1024),        # two forward passes (16384 rows, then the rest)
+    ("fp32", (784, 200, 136), 3 * 256 + 17, 256),
+])
+def test_head_train_epoch_is_bitwise_the_per_step_calls(env, prec, dims, n, B):
+    """ff_head_train_epoch forms many steps' features in one forward pass; its
+    steps must give exactly the per-step path's losses and head state."""
+    torch, ff = env
+    layers, _ = _net(ff, dims, prec, 40)
+    F = ff.Head.features_of(layers)
+    x = torch.from_numpy(synth.mnist_like(n, seed=41)).cuda()
+    y = torch.from_numpy(synth.labels(n, seed=41)).cuda()
+    nsteps = -(-n // B)
+    ha, hb = ff.Head(F, lr=1e-3, max_rows=B), ff.Head(F, lr=1e-3, max_rows=B)
+    la = torch.zeros(nsteps, device="cuda")
+    lb = torch.zeros(nsteps, device="cuda")
+    ha.train_epoch(layers, x, y, B, loss=la)
+    for t in range(nsteps):
+        r = t * B
+        hb.train_step(layers, x[r:r + B], y[r:r + B], loss=lb[t:t + 1])
+    torch.cuda.synchronize()
+    ha.check()
+    hb.check()
+    assert torch.equal(la, lb), ("per-step losses differ", (la - lb).abs().max().item())
+    sa, sb = ha.get_state(), hb.get_state()
+    for key in sa:
+        assert np.array_equal(np.asarray(sa[key]), np.asarray(sb[key])), key
+    ha.close()
+    hb.close()
+
+
 def test_head_features_are_unit_norm_segments(env):
     """With V = a selector of one feature per class, the logits are those
     features of A: checks the neutral label, the layer order and the
