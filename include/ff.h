@@ -201,8 +201,10 @@ FF_API ff_status ff_head_train_step(ff_head* head, ff_layer* const* layers, int 
  * rest), bitwise the same.  The layers do not change during head training,
  * so the neutral forward runs once over many steps' rows (up to 16384 per
  * pass, whole steps) and each step's logits, gradient and Adam update read
- * their rows of the stored activities.  B <= max_rows; the workspace grows to
- * the rows of one forward pass.  loss [ceil(n / B)] (device) or NULL receives
+ * their rows of the stored activities.  With several passes the next pass's
+ * forward runs on a side stream of the head's, into a second workspace,
+ * while `stream` runs the current pass's steps.  B <= max_rows; the
+ * workspaces grow to the rows of one forward pass.  loss [ceil(n / B)] (device) or NULL receives
  * each step's mean cross-entropy. */
 FF_API ff_status ff_head_train_epoch(ff_head* head, ff_layer* const* layers, int n_layers,
                                      const float* x, const int* labels, int n, int B, float* loss,

@@ -725,6 +725,13 @@ struct ff_head {
   size_t ws_bytes;
   int* counters;    // k_head_dot arrival counters, one per 64-row block (zero between launches)
   int counter_cap;
+  // ff_head_train_epoch: a second feature workspace and a side stream, so
+  // that the next pass's neutral forward runs while the head steps read the
+  // current one (created on first use)
+  void* ws2;
+  size_t ws2_bytes;
+  cudaStream_t side;
+  cudaEvent_t ev_start, ev_fwd[2], ev_use[2];
 };
 
 namespace ff {
@@ -766,8 +773,12 @@ size_t chain_zpart_floats(ff_layer* const* layers, int L, int rows) {
   return zpart_floats(F, nseg, rows, layers[0]->is_bf16 ? 2 : 4);
 }
 
-// Carves the head's workspace for `rows` rows (grown on demand).
-ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, bool train, HeadWork* w) {
+// Carves the head's workspace for `rows` rows (grown on demand); buf 1: the
+// second workspace of ff_head_train_epoch.
+ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, bool train, HeadWork* w,
+                         int buf = 0) {
+  void*& wsp = buf ? hd->ws2 : hd->ws;
+  size_t& wsb = buf ? hd->ws2_bytes : hd->ws_bytes;
   const bool b16 = layers[0]->is_bf16;
   const size_t es = b16 ? 2 : 4;
   int ntmax = 0;
@@ -788,15 +799,16 @@ ff_status head_workspace(ff_head* hd, ff_layer* const* layers, int L, int rows, 
   size_t oD = off; off += align256(train ? (size_t)rows * kClasses * 4 : 0);
   size_t oP = off; off += align256(train ? (size_t)cdiv(rows, kDotRows) * kPart * 4 : 0);
   size_t oV = off; off += align256(train ? (size_t)cdiv(rows, kWgRows) * kClasses * hd->F * 4 : 0);
-  if (off > hd->ws_bytes) {
+  if (off > wsb) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before head workspace growth");
-    dev_free(hd->ws);
-    hd->ws = nullptr;
-    hd->ws_bytes = 0;
-    FF_TRY(dev_alloc(&hd->ws, off), "head workspace");
-    hd->ws_bytes = off;
+    if (hd->side) FF_TRY(cudaStreamSynchronize(hd->side), "sync before head workspace growth");
+    dev_free(wsp);
+    wsp = nullptr;
+    wsb = 0;
+    FF_TRY(dev_alloc(&wsp, off), "head workspace");
+    wsb = off;
   }
-  char* base = static_cast<char*>(hd->ws);
+  char* base = static_cast<char*>(wsp);
   w->X0 = base + oX;
   for (int k = 0; k <= L; ++k) w->S[k] = reinterpret_cast<float*>(base + oS[k]);
   for (int k = 0; k < L; ++k) w->Hk[k] = base + oH[k];
@@ -1077,6 +1089,16 @@ ff_status ff_head_create(const ff_head_config* cfg, ff_head** out) {
 ff_status ff_head_destroy(ff_head* hd) {
   if (!hd) return FF_OK;
   cudaStreamSynchronize(hd->last_stream);
+  if (hd->side) {
+    cudaStreamSynchronize(hd->side);
+    cudaStreamDestroy(hd->side);
+    cudaEventDestroy(hd->ev_start);
+    for (int i = 0; i < 2; ++i) {
+      cudaEventDestroy(hd->ev_fwd[i]);
+      cudaEventDestroy(hd->ev_use[i]);
+    }
+  }
+  dev_free(hd->ws2);
   dev_free(hd->ws);
   dev_free(hd->counters);
   dev_free(hd->V);
@@ -1145,21 +1167,48 @@ ff_status ff_head_train_epoch(ff_head* hd, ff_layer* const* layers, int n_layers
   // kEpochFeatureRows (at least one step).
   const int steps_per_chunk = kEpochFeatureRows / B > 0 ? kEpochFeatureRows / B : 1;
   const int R = (int)((long long)steps_per_chunk * B < n ? (long long)steps_per_chunk * B : n);
-  HeadWork w;
-  s = head_workspace(hd, layers, n_layers, R, true, &w);
-  if (s != FF_OK) return s;
+  const int npass = cdiv(n, R);
+  if (npass > 1 && !hd->side) {
+    FF_TRY(cudaStreamCreateWithFlags(&hd->side, cudaStreamNonBlocking), "head side stream");
+    FF_TRY(cudaEventCreateWithFlags(&hd->ev_start, cudaEventDisableTiming), "head event");
+    for (int i = 0; i < 2; ++i) {
+      FF_TRY(cudaEventCreateWithFlags(&hd->ev_fwd[i], cudaEventDisableTiming), "head event");
+      FF_TRY(cudaEventCreateWithFlags(&hd->ev_use[i], cudaEventDisableTiming), "head event");
+    }
+  }
+  HeadWork w[2];
+  for (int i = 0; i < (npass > 1 ? 2 : 1); ++i) {
+    s = head_workspace(hd, layers, n_layers, R, true, &w[i], i);
+    if (s != FF_OK) return s;
+  }
   hd->last_stream = st;
   int* err = &hd->ds->err;
   const int K0 = layers[0]->K;
-  for (int r0 = 0, t = 0; r0 < n; r0 += R) {
+  // Pass p's forward fills workspace p % 2 on the side stream (after the
+  // head steps of pass p - 2 have read it); its head steps run on `stream`
+  // after that forward, while the side stream forms pass p + 1.  One pass:
+  // everything on `stream`.
+  cudaStream_t fs = npass > 1 ? hd->side : st;
+  if (npass > 1) {
+    FF_TRY(cudaEventRecord(hd->ev_start, st), "event record");
+    FF_TRY(cudaStreamWaitEvent(fs, hd->ev_start, 0), "stream wait");
+  }
+  for (int p = 0, r0 = 0, t = 0; p < npass; ++p, r0 += R) {
     const int rows = n - r0 < R ? n - r0 : R;
-    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, rows, w, err, st, false);
+    const int buf = p & 1;
+    if (npass > 1 && p >= 2) FF_TRY(cudaStreamWaitEvent(fs, hd->ev_use[buf], 0), "stream wait");
+    s = head_forward(layers, n_layers, x + (size_t)r0 * K0, rows, w[buf], err, fs, false);
     if (s != FF_OK) return s;
+    if (npass > 1) {
+      FF_TRY(cudaEventRecord(hd->ev_fwd[buf], fs), "event record");
+      FF_TRY(cudaStreamWaitEvent(st, hd->ev_fwd[buf], 0), "stream wait");
+    }
     for (int q = 0; q < rows; q += B, ++t) {
       const int b = rows - q < B ? rows - q : B;
-      s = head_step_on_features(hd, layers, n_layers, w, q, labels + r0 + q, b, loss ? loss + t : nullptr, st);
+      s = head_step_on_features(hd, layers, n_layers, w[buf], q, labels + r0 + q, b, loss ? loss + t : nullptr, st);
       if (s != FF_OK) return s;
     }
+    if (npass > 1) FF_TRY(cudaEventRecord(hd->ev_use[buf], st), "event record");
   }
   return FF_OK;
 }
