@@ -941,10 +941,35 @@ def run_other(args):
             if ms_graph < ms:
                 ms, launch = ms_graph, "one CUDA graph per 16 steps"
         prof = run16
+        # the same 16 steps through a net of the two layers (one CUDA stream
+        # each: layer 2's forward overlaps layer 1's weight gradient and Adam;
+        # bitwise the sequential result), eager and as one CUDA graph
+        nl = [ff.Layer(784, 500, prec="fp32", init_seed=0), ff.Layer(500, 500, prec="fp32", init_seed=1)]
+        net = ff.Net(nl, max_B=B, depth=2)
+
+        def run16_net():
+            for xb, lb in batches16:
+                net.train_step(xb, lb, B=B, stream=stream)
+            net.sync(stream)
+        _timed_loop(torch, stream, run16_net, args.warmup)
+        ms_net = _timed_loop(torch, stream, run16_net, args.steps) / args.steps
+        if ms_net < ms:
+            ms, launch = ms_net, "2 layer streams (ff_net), eager"
+        ms_net_graph = None
+        if not args.no_graph:
+            gnet = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(gnet, stream=stream):
+                run16_net()
+            _timed_loop(torch, stream, gnet.replay, args.warmup)
+            ms_net_graph = _timed_loop(torch, stream, gnet.replay, args.steps) / args.steps
+            if ms_net_graph < ms:
+                ms, launch = ms_net_graph, "2 layer streams (ff_net) as one CUDA graph per 16 steps"
         out.update({"metric": "FF train step latency, 784-500-500 fp32, B=64 pairs", "value": round(1e3 * ms / 16, 2),
                     "unit": "us/step", "higher_is_better": False, "ms_per_step": round(ms, 4), "dtype": "f32",
                     "launch": launch, "us_per_step_eager": round(1e3 * ms_eager / 16, 2),
                     "us_per_step_graph": round(1e3 * ms_graph / 16, 2) if ms_graph is not None else None,
+                    "us_per_step_net": round(1e3 * ms_net / 16, 2),
+                    "us_per_step_net_graph": round(1e3 * ms_net_graph / 16, 2) if ms_net_graph is not None else None,
                     "config": {"workload": "ff_train_784-500-500_fp32_B64_16steps"}})
     if prof is not None:
         # one more call, each launch timed on its own stream (not the timed calls above)
