@@ -212,6 +212,8 @@ class _Trainer:
     # True (--fused-local-grad): the local step in the forward GEMM's epilogue
     # instead of its own kernel after each forward (same results; slower here)
     fused_local_grad = False
+    # batches of activations each layer may run ahead of the next (--net-depth)
+    depth = 2
 
     def __init__(self, ff, torch, dev, lr, max_B):
         self.ff, self.torch, self.dev = ff, torch, dev
@@ -219,7 +221,7 @@ class _Trainer:
                                 max_rows=2 * max_B) for k in range(len(NET) - 1)]
         for l in self.layers:
             l.set_fused_local_grad(self.fused_local_grad)
-        self.net = ff.Net(self.layers, max_B=max_B, depth=2)
+        self.net = ff.Net(self.layers, max_B=max_B, depth=self.depth)
         self.W0 = [torch.from_numpy(l.get_state()["W"]).to(dev) for l in self.layers]
         self.zeros = torch.zeros(max(NET[k] * NET[k + 1] for k in range(len(NET) - 1)), device=dev)
 
@@ -1022,10 +1024,13 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused-local-grad", action="store_true",
                     help="form the local step in the forward GEMM's epilogue (same results; for comparison)")
+    ap.add_argument("--net-depth", type=int, default=2,
+                    help="activation ring depth of the layer-stream net: batches a layer may run ahead of the next")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
     ap.add_argument("--cpu-worker", type=float, default=None, help=argparse.SUPPRESS)
     args = ap.parse_args()
     _Trainer.fused_local_grad = args.fused_local_grad
+    _Trainer.depth = args.net_depth
     if args.cpu_worker is not None:
         v, done, el, _ = oracle_sample(args.cpu_worker)
         print(json.dumps({"pairs_per_s": v, "steps": done, "elapsed": el}))
