@@ -86,6 +86,12 @@ def test_invalid_arguments_are_rejected_on_the_host(libff):
     assert libff.ff_net_train_step_images(None, None, None, 1, None, None) == 1
     assert libff.ff_layer_get_state(None, None, None, None, None, None, None, None) == 1
     assert libff.ff_layer_check(None) == 1
+    assert libff.ff_layer_set_fused_local_grad(None, 1) == 1
+    assert libff.ff_layer_get_grad_operand(None, None, 4) == 1
+    assert libff.ff_net_train_epoch(None, None, None, 4, 2, 2, None, None) == 1
+    libff.ff_net_epoch_trace.restype = ctypes.c_longlong
+    assert libff.ff_net_epoch_trace(None, 1, None, ctypes.c_longlong(0)) == -1
+    assert libff.ff_head_train_epoch(None, None, 1, None, None, 4, 2, None, None) == 1
     # the allocation-free forward: sizes and pointers checked, and the scratch limit
     # (rows * 2 * ceil(out / 256) partials) applied, before any CUDA call
     fake = ctypes.c_void_p(256)
