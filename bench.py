@@ -442,10 +442,26 @@ def run_ours(args):
             run_e2e()
         barrier()
         ems, _, _ = timed_epochs(live, run_e2e, args.steps)
+        e2e_launch = "eager"
+        if not args.no_graph:
+            # the same epoch -- its host-to-device copies, steps and loss read
+            # back -- captured once as a CUDA graph and replayed per epoch
+            live.restore()
+            egraph = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(egraph, stream=stream):
+                run_e2e()
+            with torch.cuda.stream(stream):
+                egraph.replay()
+            barrier()
+            gms, _, _ = timed_epochs(live, egraph.replay, args.steps)
+            if gms < ems:
+                ems, e2e_launch = gms, "one CUDA graph per epoch (copies, steps and the loss read back)"
+            del egraph
         e2e_value, ems = replica_throughput(ems, PAIRS_PER_EPOCH * args.steps, world, dist)
         e2e = {"value": round(e2e_value, 1), "unit": "pairs/s",
                "h2d_bytes_per_step": int(X_img.nbytes + L_h.nbytes), "d2h_bytes_per_step": int(loss_h.numel() * 4),
-               "ms_per_step": round(ems / args.steps, 4), "input": "one image per pair (ff_net_train_step_images)"}
+               "ms_per_step": round(ems / args.steps, 4), "input": "one image per pair (ff_net_train_step_images)",
+               "launch": e2e_launch}
 
     # Per-kernel device time: the same epochs with the layers run one after
     # another on one stream (each kernel alone on the GPU), every launch
