@@ -214,13 +214,16 @@ class _Trainer:
     fused_local_grad = False
     # batches of activations each layer may run ahead of the next (--net-depth)
     depth = 2
+    # --fused-layers: the layers (0-based) that take the fused form; None: all or none
+    fused_layers = None
 
     def __init__(self, ff, torch, dev, lr, max_B):
         self.ff, self.torch, self.dev = ff, torch, dev
         self.layers = [ff.Layer(NET[k], NET[k + 1], prec="bf16", theta=THETA, lr=lr, init_seed=1000 + k,
                                 max_rows=2 * max_B) for k in range(len(NET) - 1)]
-        for l in self.layers:
-            l.set_fused_local_grad(self.fused_local_grad)
+        for k, l in enumerate(self.layers):
+            fused = self.fused_local_grad if self.fused_layers is None else k in self.fused_layers
+            l.set_fused_local_grad(fused)
         self.net = ff.Net(self.layers, max_B=max_B, depth=self.depth)
         self.W0 = [torch.from_numpy(l.get_state()["W"]).to(dev) for l in self.layers]
         self.zeros = torch.zeros(max(NET[k] * NET[k + 1] for k in range(len(NET) - 1)), device=dev)
@@ -544,8 +547,10 @@ def run_ours(args):
                                 "(restored outside the timed region)",
                        "parallelism": f"{world} replica(s); per GPU 4 layers on 4 CUDA streams",
                        "l2": "inputs larger than L2 (376 MB of pair batches per step)",
-                       "local_grad": "in the forward GEMM's epilogue" if _Trainer.fused_local_grad
-                       else "separate kernel after the forward GEMM"},
+                       "local_grad": ("in the forward GEMM's epilogue on layers " + ",".join(
+                           str(k) for k in sorted(_Trainer.fused_layers)) if _Trainer.fused_layers is not None
+                                      else "in the forward GEMM's epilogue" if _Trainer.fused_local_grad
+                                      else "separate kernel after the forward GEMM")},
             "launch": mode,
             "ms_per_step_eager": round(ms_eager / args.steps, 4),
             "ms_per_step_graph": round(ms_graph / args.steps, 4) if ms_graph is not None else None,
@@ -1040,6 +1045,8 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--fused-local-grad", action="store_true",
                     help="form the local step in the forward GEMM's epilogue (same results; for comparison)")
+    ap.add_argument("--fused-layers", default="",
+                    help="comma-separated layers (0-based) whose local step runs in the forward epilogue")
     ap.add_argument("--net-depth", type=int, default=2,
                     help="activation ring depth of the layer-stream net: batches a layer may run ahead of the next")
     ap.add_argument("--cpu-seconds", type=float, default=12.0)
@@ -1047,6 +1054,8 @@ def main():
     args = ap.parse_args()
     _Trainer.fused_local_grad = args.fused_local_grad
     _Trainer.depth = args.net_depth
+    if args.fused_layers:
+        _Trainer.fused_layers = {int(v) for v in args.fused_layers.split(",")}
     if args.cpu_worker is not None:
         v, done, el, _ = oracle_sample(args.cpu_worker)
         print(json.dumps({"pairs_per_s": v, "steps": done, "elapsed": el}))
