@@ -95,7 +95,7 @@ struct TcCfg {
   static_assert(TN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
   static_assert(NT == 1 || TN / (EPI_WARPS / 4) == BN, "with column subtiles each epilogue warp reads one accumulator");
   static_assert(!PAIR || BH % 64 == 0, "each CTA of a pair loads whole 64-column B groups");
-  static_assert(3 * STAGES * 8 + 8 + 16 + 8 <= 256, "barriers, TMEM slot, flags and the LG barrier fit below the bias tile");
+  static_assert(3 * STAGES * 8 + 8 + 16 + 8 + 32 <= 256, "barriers, TMEM slot, flags, LG and logits barriers fit below the bias");
 };
 
 __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
@@ -122,6 +122,14 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 "fp32 operands: K-major forward and store GEMMs");
   static_assert(!LG || (PAIR && MT == 1 && NT == 2 && BN == 256 && EPI_WARPS == 8),
                 "the local-gradient epilogue: 128 rows x 512 columns per CTA, a warp per 32 rows x 256 columns");
+  // Block logits on the tensor cores (one 128-row subtile per CTA leaves TMEM
+  // room for them): per column half, a pair MMA of the staged bf16 activity
+  // (M = 256 across the pair, K = 128) with the block's weights (N = 16
+  // classes, 8 per CTA, as a hi and a lo bf16 part) into 16 spare TMEM
+  // columns.  With two subtiles the CUDA cores form them (10 fmas an element).
+  constexpr bool LMMA = LOGITS && PAIR && MT == 1 && NT == 1 && BN == 256 && EPI_WARPS == 8;
+  constexpr uint32_t TCOLS = LMMA ? 512 : C::TMEM_COLS;  // + the logits' 2 x 16 columns (a power of 2)
+  constexpr uint32_t LCOL = MT * NT * C::ACC_COLS;       // first logits column
   extern __shared__ uint8_t smem_raw[];
   // 128-byte swizzled tiles need 1024-byte aligned shared addresses.
   const uint32_t raw_s = ptx::smem_u32(smem_raw);
@@ -136,10 +144,16 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   uint32_t* tslot = reinterpret_cast<uint32_t*>(tfull + 1);
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tslot + 1);
   volatile int* never_set = reinterpret_cast<volatile int*>(tslot + 2);  // drain waits ignore the abort
+  volatile int* lgiss = reinterpret_cast<volatile int*>(tslot + 3);     // LMMA: bit h, half h's MMAs issued
   uint64_t* lgbar = reinterpret_cast<uint64_t*>(tslot + 4);  // LG: every partial of the row block has arrived
   uint64_t* conv = lgbar + 1;  // fp32: [STAGES] both CTAs' splits of a stage are done
+  uint64_t* hst = conv + C::STAGES;  // LMMA: [2] both CTAs' activity of a column half is staged
+  uint64_t* lgd = hst + 2;           // LMMA: [2] that half's logits MMAs are done
   float* sbias = reinterpret_cast<float*>(reinterpret_cast<uint8_t*>(full) + 256);  // [TN] bias of this tile
   float* sVt = sbias + C::TN;  // LOGITS: [BN][kLogitStride] block weights of this tile's columns
+  // LMMA: the weights as MMA operands, 1024-byte aligned after the bias:
+  // [half][hi, lo][64-column atom] tiles of 8 classes x 128 bytes
+  uint8_t* sVb = reinterpret_cast<uint8_t*>(full) + 2048;
   // LG: [kLgParts][MT * BM] goodness partials of this CTA's rows (partial t
   // covers columns 128t ..), then per epilogue warp [2][32] row terms
   float* sgp = sbias + C::TN;
@@ -177,8 +191,14 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     if constexpr (LG) ptx::mbar_init(lgbar, 32 * EPI_WARPS * gridDim.y);  // every epilogue lane of the row block
     if constexpr (TF32)
       for (int s = 0; s < C::STAGES; ++s) ptx::mbar_init(&conv[s], (PAIR ? 2 : 1) * EPI_WARPS);
+    if constexpr (LMMA)
+      for (int h = 0; h < 2; ++h) {
+        ptx::mbar_init(&hst[h], 2 * (EPI_WARPS / 2));  // the 4 warps of the half in each CTA
+        ptx::mbar_init(&lgd[h], 1);
+      }
     *abort_flag = 0;
     *never_set = 0;
+    *lgiss = 0;
     ptx::fence_mbar_init();
     ptx::prefetch_tmap(&tmA);
     ptx::prefetch_tmap(&tmB);
@@ -187,10 +207,10 @@ __global__ void __launch_bounds__(NTHREADS, 2)
   }
   if (warp == 1) {
     if constexpr (PAIR) {
-      ptx::tmem_alloc_pair(tslot, C::TMEM_COLS);
+      ptx::tmem_alloc_pair(tslot, TCOLS);
       ptx::tmem_relinquish_pair();
     } else {
-      ptx::tmem_alloc(tslot, C::TMEM_COLS);
+      ptx::tmem_alloc(tslot, TCOLS);
       ptx::tmem_relinquish();
     }
   }
@@ -371,7 +391,23 @@ __global__ void __launch_bounds__(NTHREADS, 2)
       // into shared memory and this thread's row scales into registers.
       for (int c = (int)threadIdx.x - 64; c < C::TN; c += 32 * EPI_WARPS)
         sbias[c] = (ep.bias != nullptr && n0 + c < N) ? __ldg(ep.bias + n0 + c) : 0.f;
-      if constexpr (LOGITS) {
+      if constexpr (LMMA) {
+        // this CTA's 8 classes (the pair splits the 16 padded classes of the
+        // MMA's N) of the tile's 256 columns, as bf16 hi = rn(v) and
+        // lo = rn(v - hi), in 128-byte-swizzled K-major tiles
+        const int cl0 = 8 * (int)(crank & 1u);
+        for (int idx = (int)threadIdx.x - 64; idx < 2 * 2 * 8 * 64; idx += 32 * EPI_WARPS) {
+          const int j = idx & 63, i = (idx >> 6) & 7, a = (idx >> 9) & 1, h = idx >> 10;
+          const int cl = cl0 + i, col = n0 + h * 128 + a * 64 + j;
+          const float v = cl < kLogitClasses && col < N ? __ldg(ep.logit_V + (size_t)cl * ep.logit_ldV + col) : 0.f;
+          const bf16 hi = __float2bfloat16_rn(v);
+          const bf16 lo = __float2bfloat16_rn(v - __bfloat162float(hi));
+          const int off = i * 128 + (((j >> 3) ^ (i & 7)) << 4) + (j & 7) * 2;
+          *reinterpret_cast<bf16*>(sVb + ((h * 2 + 0) * 2 + a) * 1024 + off) = hi;
+          *reinterpret_cast<bf16*>(sVb + ((h * 2 + 1) * 2 + a) * 1024 + off) = lo;
+        }
+        ptx::fence_async_smem();  // read by the logits MMAs (async proxy)
+      } else if constexpr (LOGITS) {
         for (int idx = (int)threadIdx.x - 64; idx < kLogitClasses * BN; idx += 32 * EPI_WARPS) {
           const int c = idx / BN, j = idx % BN;
           sVt[j * kLogitStride + c] = n0 + j < N ? __ldg(ep.logit_V + (size_t)c * ep.logit_ldV + n0 + j) : 0.f;
@@ -448,6 +484,12 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const int gi = rbase + lane;
         // bf16: the warp's 32 x CPW block per subtile; fp32: two 32 x 32 slots, streamed
         uint8_t* stage = smem + (FWD && !TF32 ? (ew * MT + mt) * (32 * CPW * 2) : ew * 8192);
+        // the warp's 32 rows of its 64-column chunk ch of the activity; LMMA:
+        // inside the half's 128-row swizzle atoms (the logits MMA's A operand)
+        auto chunk = [&](int ch) -> uint8_t* {
+          if constexpr (LMMA) return smem + (half * 2 + ch) * 16384 + q * 32 * 128;
+          return stage + ch * (32 * 128);
+        };
         const uint32_t trow = tmem + ((uint32_t)(q * 32) << 16) +
                               (uint32_t)((mt * NT + cbase / BN) * C::ACC_COLS + cbase % BN);
         const float s = srow[mt];
@@ -479,7 +521,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
               __nv_bfloat162 p1 = __floats2bfloat162_rn(h[2], h[3]);
               packed[2 * v] = *reinterpret_cast<uint32_t*>(&p0);
               packed[2 * v + 1] = *reinterpret_cast<uint32_t*>(&p1);
-              if constexpr (LOGITS) {
+              if constexpr (LOGITS && !LMMA) {
                 // the block reads the stored (bf16-rounded) activity
                 const float2 lo = __bfloat1622float2(p0), hi = __bfloat1622float2(p1);
                 const float hr[4] = {lo.x, lo.y, hi.x, hi.y};
@@ -493,7 +535,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
                 }
               }
             }
-            uint8_t* base = stage + (c0 / CW) * (32 * 128) + lane * 128;
+            uint8_t* base = chunk(c0 / CW) + lane * 128;
 #pragma unroll
             for (int v = 0; v < 4; ++v) {
               const uint32_t j = (uint32_t)((c0 % CW) / 8 + v);
@@ -559,7 +601,7 @@ __global__ void __launch_bounds__(NTHREADS, 2)
           }
         }
         if (FWD && !LG && gi < M) ep.gpart[(size_t)(blockIdx.y * HALVES + half) * M + gi] = g;
-        if (LOGITS && gi < M) {
+        if (LOGITS && !LMMA && gi < M) {
           float2* zp = reinterpret_cast<float2*>(ep.zpart + ((size_t)(blockIdx.y * HALVES + half) * M + gi) * kLogitClasses);
 #pragma unroll
           for (int c = 0; c < kLogitClasses; c += 2) zp[c / 2] = make_float2(zl[c], zl[c + 1]);
@@ -572,9 +614,55 @@ __global__ void __launch_bounds__(NTHREADS, 2)
             for (int ch = 0; ch < CPW / CW; ++ch) {
               const int col = n0 + cbase + ch * CW;
               if (col < ep.ldo && ff_dcheck(col >= 0 && rbase >= 0 && tma_x_aligned(col, 2), err))
-                ptx::tma_store_2d(&tmC, stage + ch * (32 * 128), col, rbase);
+                ptx::tma_store_2d(&tmC, chunk(ch), col, rbase);
             }
             ptx::bulk_commit();
+          }
+        }
+        if constexpr (LMMA) {
+          // The block's partial logits of this half: once the 4 warps of the
+          // half have staged their rows in both CTAs, one thread of the even
+          // CTA issues the pair MMAs (K = 128 as 8 steps of 16, the weights'
+          // hi and lo parts), committed to both CTAs' barrier.
+          if (lane == 0) {
+            if (issuer)
+              ptx::mbar_arrive(&hst[half]);
+            else
+              ptx::mbar_arrive_remote(&hst[half], pair_lead);
+          }
+          if (issuer && q == 0 && lane == 0) {
+            if (ptx::mbar_wait_cluster(&hst[half], 0, kWaitTimeoutNs, abort_flag)) {
+              ptx::tc_fence_after();
+              constexpr uint32_t idesc_l = ptx::idesc_bf16_f32(2 * BM, 16, 0, 0);
+#pragma unroll
+              for (int sp = 0; sp < 2; ++sp)
+#pragma unroll
+                for (int kk = 0; kk < 8; ++kk) {
+                  const uint32_t a_addr = ptx::smem_u32(smem + (half * 2 + (kk >> 2)) * 16384) + (kk & 3) * 32;
+                  const uint32_t b_addr = ptx::smem_u32(sVb + ((half * 2 + sp) * 2 + (kk >> 2)) * 1024) + (kk & 3) * 32;
+                  ptx::umma_f16_pair(tmem + LCOL + 16 * half, ptx::sdesc_sw128(a_addr, 16, 1024),
+                                     ptx::sdesc_sw128(b_addr, 16, 1024), idesc_l, (sp | kk) != 0 ? 1u : 0u);
+                }
+              ptx::umma_commit_pair(&lgd[half], pmask);
+              atomicOr(const_cast<int*>(lgiss), 1 << half);
+            } else {
+              latch(err, abort_flag);
+            }
+          }
+          const bool done = ptx::mbar_wait(&lgd[half], 0, kWaitTimeoutNs, abort_flag);
+          if (!done) latch(err, abort_flag);
+          if (__all_sync(0xffffffffu, done && !*abort_flag)) {
+            ptx::tc_fence_after();
+            uint32_t rz[16];
+            ptx::tmem_ld16(tmem + ((uint32_t)(q * 32) << 16) + LCOL + 16 * half, rz);
+            ptx::tmem_ld_wait();
+            if (gi < M) {
+              float2* zp = reinterpret_cast<float2*>(ep.zpart +
+                                                     ((size_t)(blockIdx.y * HALVES + half) * M + gi) * kLogitClasses);
+#pragma unroll
+              for (int c = 0; c < kLogitClasses; c += 2)
+                zp[c / 2] = make_float2(__uint_as_float(rz[c]), __uint_as_float(rz[c + 1]));
+            }
           }
         }
         if constexpr (LG) {
@@ -734,11 +822,13 @@ __global__ void __launch_bounds__(NTHREADS, 2)
     if (*abort_flag) {
       // MMAs issued before the abort must finish before TMEM is released
       ptx::mbar_wait(tfull, 0, 10000000ull, never_set);
+      if constexpr (LMMA)
+        for (int h = 0; h < 2; ++h) ptx::mbar_wait(&lgd[h], 0, 10000000ull, never_set);
     }
     if constexpr (PAIR)
-      ptx::tmem_dealloc_pair(tmem, C::TMEM_COLS);
+      ptx::tmem_dealloc_pair(tmem, TCOLS);
     else
-      ptx::tmem_dealloc(tmem, C::TMEM_COLS);
+      ptx::tmem_dealloc(tmem, TCOLS);
   }
 }
 
