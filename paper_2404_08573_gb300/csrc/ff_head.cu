@@ -732,6 +732,8 @@ struct ff_head {
   size_t ws2_bytes;
   cudaStream_t side;
   cudaEvent_t ev_start, ev_fwd[2], ev_use[2];
+  // ff_po_train_step: the block's Adam on the side stream (fork, join)
+  cudaEvent_t ev_fork, ev_join;
 };
 
 namespace ff {
@@ -988,6 +990,7 @@ ff_status po_workspace(ff_head* hd, int n, int N, int es, PoWork* w) {
   const size_t oV = off; off += align256((size_t)cdiv(n, kPoRows) * kClasses * N * 4);
   if (off > hd->ws_bytes) {
     FF_TRY(cudaStreamSynchronize(hd->last_stream), "sync before workspace growth");
+    if (hd->side) FF_TRY(cudaStreamSynchronize(hd->side), "sync before workspace growth");
     dev_free(hd->ws);
     hd->ws = nullptr;
     hd->ws_bytes = 0;
@@ -1093,6 +1096,8 @@ ff_status ff_head_destroy(ff_head* hd) {
     cudaStreamSynchronize(hd->side);
     cudaStreamDestroy(hd->side);
     cudaEventDestroy(hd->ev_start);
+    cudaEventDestroy(hd->ev_fork);
+    cudaEventDestroy(hd->ev_join);
     for (int i = 0; i < 2; ++i) {
       cudaEventDestroy(hd->ev_fwd[i]);
       cudaEventDestroy(hd->ev_use[i]);
@@ -1109,6 +1114,16 @@ ff_status ff_head_destroy(ff_head* hd) {
 
 // Rows of stored features ff_head_train_epoch forms per forward pass.
 constexpr int kEpochFeatureRows = 16384;
+
+// The head's side stream and its events (created on first use).
+static ff_status ensure_side(ff_head* hd) {
+  if (hd->side) return FF_OK;
+  FF_TRY(cudaStreamCreateWithFlags(&hd->side, cudaStreamNonBlocking), "head side stream");
+  cudaEvent_t* evs[] = {&hd->ev_start, &hd->ev_fork, &hd->ev_join, &hd->ev_fwd[0], &hd->ev_fwd[1], &hd->ev_use[0],
+                        &hd->ev_use[1]};
+  for (cudaEvent_t* e : evs) FF_TRY(cudaEventCreateWithFlags(e, cudaEventDisableTiming), "head event");
+  return FF_OK;
+}
 
 // The head's part of one train step on n rows of the features in w, starting
 // at row r0 of the stored activities: logits, softmax, loss and dz
@@ -1168,13 +1183,9 @@ ff_status ff_head_train_epoch(ff_head* hd, ff_layer* const* layers, int n_layers
   const int steps_per_chunk = kEpochFeatureRows / B > 0 ? kEpochFeatureRows / B : 1;
   const int R = (int)((long long)steps_per_chunk * B < n ? (long long)steps_per_chunk * B : n);
   const int npass = cdiv(n, R);
-  if (npass > 1 && !hd->side) {
-    FF_TRY(cudaStreamCreateWithFlags(&hd->side, cudaStreamNonBlocking), "head side stream");
-    FF_TRY(cudaEventCreateWithFlags(&hd->ev_start, cudaEventDisableTiming), "head event");
-    for (int i = 0; i < 2; ++i) {
-      FF_TRY(cudaEventCreateWithFlags(&hd->ev_fwd[i], cudaEventDisableTiming), "head event");
-      FF_TRY(cudaEventCreateWithFlags(&hd->ev_use[i], cudaEventDisableTiming), "head event");
-    }
+  if (npass > 1) {
+    s = ensure_side(hd);
+    if (s != FF_OK) return s;
   }
   HeadWork w[2];
   for (int i = 0; i < (npass > 1 ? 2 : 1); ++i) {
@@ -1424,6 +1435,23 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
                  : cudaLaunchKernelEx(&pl.cfg, k_po_grad<float>, pa, static_cast<const float*>(H),
                                       static_cast<float*>(L->dZ))),
             "block gradient into the layer");
+  // The block's Adam needs only what k_po_grad wrote, and nothing later in
+  // this step reads the block's weights: it runs on the head's side stream,
+  // beside the layer's weight gradient and Adam, and `stream` joins it at the
+  // end of the step.
+  s = ensure_side(hd);
+  if (s != FF_OK) return s;
+  FF_TRY(cudaEventRecord(hd->ev_fork, st), "event record");
+  FF_TRY(cudaStreamWaitEvent(hd->side, hd->ev_fork, 0), "stream wait");
+  {
+    const HeadAdamArgs ha =
+        head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, b16 ? kPoRows : kDotRows), n, loss);
+    const int vblocks = cdiv((long long)kClasses * hd->F, 256);
+    PdlLaunch hl(dim3(vblocks + 1), dim3(256), hd->side);
+    FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), hd->side,
+              cudaLaunchKernelEx(&hl.cfg, k_head_adam, ha), "block Adam");
+  }
+  FF_TRY(cudaEventRecord(hd->ev_join, hd->side), "event record");
   if (b16) {
     FF_LAUNCH(K_WGRAD_TC, 2.0 * n * N * K, st,
               tc_gemm_wgrad(static_cast<const bf16*>(L->dZ), L->ldN, static_cast<const bf16*>(X), L->ldK, n, N, K,
@@ -1463,12 +1491,7 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
   aa.discard_dW = !L->cfg.keep_grad && ((uintptr_t)L->dW & 127u) == 0;
   if (!L->cfg.keep_grad) add_dead(aa, L->dZ, (size_t)n * L->ldN * (size_t)es);
   FF_LAUNCH(K_ADAM, (double)N * K * (28.0 + (b16 ? 2.0 : 0.0)), st, launch_adam(aa, st), "layer Adam");
-  const HeadAdamArgs ha =
-      head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, b16 ? kPoRows : kDotRows), n, loss);
-  const int vblocks = cdiv((long long)kClasses * hd->F, 256);
-  PdlLaunch hl(dim3(vblocks + 1), dim3(256), st);
-  FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), st,
-            cudaLaunchKernelEx(&hl.cfg, k_head_adam, ha), "block Adam");
+  FF_TRY(cudaStreamWaitEvent(st, hd->ev_join, 0), "stream wait");
   return FF_OK;
 }
 
