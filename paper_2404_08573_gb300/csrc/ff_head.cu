@@ -1447,9 +1447,10 @@ ff_status ff_po_train_step(ff_layer* L, ff_head* hd, const void* x, int raw_inpu
     const HeadAdamArgs ha =
         head_adam_args(hd, w.dVpart, cdiv(n, kPoRows), w.part, cdiv(n, b16 ? kPoRows : kDotRows), n, loss);
     const int vblocks = cdiv((long long)kClasses * hd->F, 256);
-    PdlLaunch hl(dim3(vblocks + 1), dim3(256), hd->side);
+    // a plain launch: after an event wait, programmatic serialization has
+    // nothing to overlap (griddepcontrol.wait is then a no-op)
     FF_LAUNCH(K_HEAD_ADAM, (double)kClasses * hd->F * (ha.nrb * 4.0 + 28), hd->side,
-              cudaLaunchKernelEx(&hl.cfg, k_head_adam, ha), "block Adam");
+              (k_head_adam<<<vblocks + 1, 256, 0, hd->side>>>(ha), cudaGetLastError()), "block Adam");
   }
   FF_TRY(cudaEventRecord(hd->ev_join, hd->side), "event record");
   if (b16) {
