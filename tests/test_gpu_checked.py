@@ -60,7 +60,34 @@ pff.run(torch.from_numpy(x2).cuda(), torch.from_numpy(np.stack([l2, l2])).cuda()
 torch.cuda.synchronize()
 for l in layers:
     h.update(l.get_state()["W"].tobytes())
-for obj in [l0] + layers + [head, blk]:
+# the local gradient in the forward epilogue (cluster exchange, dZ' store), ragged
+lf = [ff.Layer(784, 264, prec="bf16", init_seed=40), ff.Layer(264, 136, prec="bf16", init_seed=41)]
+for l in lf:
+    l.set_fused_local_grad(True)
+hf, sf = lf[0].new_activation(200), torch.empty(200, device="cuda")
+x2, l2 = pair_inputs(100, seed=42)
+lf[0].train_step(torch.from_numpy(x2).cuda(), labels=torch.from_numpy(l2).cuda(), B=100, h_out=hf, next_scale=sf)
+lf[1].train_step(hf, row_scale=sf, B=100)
+torch.cuda.synchronize()
+for l in lf:
+    h.update(l.get_state()["W"].tobytes())
+# fp32 predict on the tensor cores (three TF32 products)
+l32 = [ff.Layer(784, 200, prec="fp32", init_seed=50), ff.Layer(200, 136, prec="fp32", init_seed=51)]
+G32 = torch.empty(300, 10, device="cuda")
+ff.predict(l32, xs, goodness=G32)
+take(G32)
+# the softmax head's epoch call, and the persistent epoch kernel
+head.train_epoch(layers, xs, ys, 128)
+take(head.predict(layers, xs)[0])
+le = [ff.Layer(784, 256, prec="bf16", init_seed=60), ff.Layer(256, 264, prec="bf16", init_seed=61)]
+ne = ff.Net(le, max_B=128, depth=2)
+parts = [pair_inputs(min(128, 296 - s0), seed=62 + s0) for s0 in range(0, 296, 128)]  # batches of 128, 128, 40 pairs
+xe, le2 = np.concatenate([p[0] for p in parts]), np.concatenate([p[1] for p in parts])
+ne.train_epoch(torch.from_numpy(xe).cuda(), torch.from_numpy(le2).cuda(), 296, 128)
+torch.cuda.synchronize()
+for l in le:
+    h.update(l.get_state()["W"].tobytes())
+for obj in [l0] + layers + lf + l32 + le + [head, blk]:
     obj.check()
 print("digest", h.hexdigest())
 """
