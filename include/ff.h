@@ -301,7 +301,10 @@ FF_API ff_status ff_pff_wait(ff_pff* pff, unsigned int timeout_ms);
  * and one of the block (the block's lr).  h_out / next_scale (or NULL) take
  * the activity and the next layer's row scale from the pre-update weights,
  * as in ff_layer_train_step; loss [1] (device) or NULL.  `block` must have
- * n_features == the layer's out_features, else FF_ERR_INVALID_ARG. */
+ * n_features == the layer's out_features, else FF_ERR_INVALID_ARG.  The
+ * block's Adam step runs on a stream the block owns, beside the layer's
+ * weight gradient and Adam; `stream` waits for it before the call's work
+ * ends there, so everything is ordered before later work on `stream`. */
 FF_API ff_status ff_po_train_step(ff_layer* layer, ff_head* block, const void* x, int raw_input,
                                   const float* row_scale, const int* labels, int n, void* h_out,
                                   float* next_scale, float* loss, void* stream);
