@@ -565,7 +565,7 @@ def run_ours(args):
             "roofline": roof, "kernels": kernels, "e2e": e2e, "gpu_launches": int(launches),
             "clocks": clocks, "final_loss": final_loss,
         }
-        if not args.no_cpu_baseline:
+        if not args.no_cpu_baseline and world == 1:
             out["cpu_baseline"] = cpu_baseline(args.cpu_seconds)
         print(json.dumps(out), flush=True)
     net.close()
