@@ -67,16 +67,19 @@ constexpr int kLgParts = 16;        // goodness partials of a row (128 columns e
 constexpr int kLogitClasses = 10;
 constexpr int kLogitStride = 12;    // floats per column of the staged block weights (three float4)
 
-template <int BN, int NSTAGE, int MT, bool PAIR, int NT = 1, int OPB = 2>
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT = 1, int OPB = 2, int KB = 128>
 struct TcCfg {
   // OPB: bytes per operand element (2: bf16; 4: fp32 through three TF32
-  // products).  A k-block is one 128-byte swizzle row either way: BKE
-  // elements, so tile byte sizes do not depend on the type.
-  static constexpr int BKE = 128 / OPB;
+  // products).  KB: bytes of K per operand row of a stage -- one 128-byte
+  // swizzle row, or (bf16 only) one 64-byte swizzle row, which halves the
+  // stage so that twice as many fit the same ring.  A stage holds BKE = KB /
+  // OPB elements of K, so tile byte sizes do not depend on the type.
+  static constexpr int KBYTES = KB;
+  static constexpr int BKE = KB / OPB;
   static constexpr int TN = NT * BN;                // columns of the tile (NT column subtiles of BN)
-  static constexpr int A_BYTES = MT * BM * 128;     // MT row subtiles of BM rows
+  static constexpr int A_BYTES = MT * BM * KB;      // MT row subtiles of BM rows
   static constexpr int BH = PAIR ? BN / 2 : BN;     // B columns of a column subtile this CTA loads
-  static constexpr int B_BYTES = NT * BH * 128;
+  static constexpr int B_BYTES = NT * BH * KB;
   static constexpr int IN_BYTES = A_BYTES + B_BYTES;  // what TMA brings per stage
   static constexpr int STAGE = (OPB == 4 ? 2 : 1) * IN_BYTES;  // fp32: the lo parts beside
   static constexpr int STAGES = NSTAGE;
@@ -91,6 +94,7 @@ struct TcCfg {
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
   static_assert(OPB == 4 || MT * 4 * 32 * TN * 2 <= STAGES * STAGE, "bf16 epilogue staging must fit in the operand ring");
   static_assert(OPB == 2 || OPB == 4, "bf16 or fp32 operands");
+  static_assert(KB == 128 || (KB == 64 && OPB == 2), "128-byte K rows, or 64-byte ones for bf16");
   static_assert(EPI_WARPS * 8192 <= STAGES * STAGE, "fp32 epilogue staging must fit in the operand ring");
   static_assert(TN % (64 * (EPI_WARPS / 4)) == 0, "each epilogue warp takes whole 64-column groups");
   static_assert(NT == 1 || TN / (EPI_WARPS / 4) == BN, "with column subtiles each epilogue warp reads one accumulator");
@@ -108,18 +112,19 @@ __device__ __forceinline__ void latch(int* err, volatile int* abort_flag) {
 // gradient blocks of the other layers' streams (784-2000x4 epoch -1 %).
 // MODE_FWD_LG: tmD maps dZ' (as tmC maps H) and lg holds the local step's
 // arguments; the grid's column tiles all lie in one cluster (2 x gridDim.y).
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB, int KB>
 __global__ void __launch_bounds__(NTHREADS, 2)
     k_tc_gemm(const __grid_constant__ CUtensorMap tmA, const __grid_constant__ CUtensorMap tmB,
               const __grid_constant__ CUtensorMap tmC, const __grid_constant__ CUtensorMap tmD, int tma_store, int M,
               int N, int K, EpiArgs ep, GradPrepArgs lg, int* err) {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB>;
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB, KB>;
   constexpr bool FWD = MODE != MODE_STORE;
   constexpr bool LOGITS = MODE == MODE_FWD_LOGITS;
   constexpr bool LG = MODE == MODE_FWD_LG;
   constexpr bool TF32 = OPB == 4;
   static_assert(!TF32 || (!A_MN && !B_MN && (MODE == MODE_FWD || MODE == MODE_STORE)),
                 "fp32 operands: K-major forward and store GEMMs");
+  static_assert(KB == 128 || (MODE == MODE_FWD || MODE == MODE_STORE), "64-byte K rows: plain forward and store");
   static_assert(!LG || (PAIR && MT == 1 && NT == 2 && BN == 256 && EPI_WARPS == 8),
                 "the local-gradient epilogue: 128 rows x 512 columns per CTA, a warp per 32 rows x 256 columns");
   // Block logits on the tensor cores (one 128-row subtile per CTA leaves TMEM
@@ -259,17 +264,17 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const int k0 = kb * C::BKE;
         if (!A_MN) {
 #pragma unroll
-          for (int mt = 0; mt < MT; ++mt) load(a + mt * BM * BK * 2, &tmA, s, k0, m0 + BM * mt);
+          for (int mt = 0; mt < MT; ++mt) load(a + mt * BM * C::KBYTES, &tmA, s, k0, m0 + BM * mt);
         } else {
 #pragma unroll
-          for (int j = 0; j < MT * BM / 64; ++j) load(a + j * 64 * BK * 2, &tmA, s, m0 + 64 * j, k0);
+          for (int j = 0; j < MT * BM / 64; ++j) load(a + j * 64 * C::BKE * 2, &tmA, s, m0 + 64 * j, k0);
         }
         if (!B_MN) {
 #pragma unroll
-          for (int nt = 0; nt < NT; ++nt) load(b + nt * C::BH * BK * 2, &tmB, s, k0, nb + nt * BN);
+          for (int nt = 0; nt < NT; ++nt) load(b + nt * C::BH * C::KBYTES, &tmB, s, k0, nb + nt * BN);
         } else {
 #pragma unroll
-          for (int j = 0; j < C::BH / 64; ++j) load(b + j * 64 * BK * 2, &tmB, s, nb + 64 * j, k0);
+          for (int j = 0; j < C::BH / 64; ++j) load(b + j * 64 * C::BKE * 2, &tmB, s, nb + 64 * j, k0);
         }
         issued = kb + 1;
       }
@@ -319,23 +324,26 @@ __global__ void __launch_bounds__(NTHREADS, 2)
         const uint32_t a_base = ptx::smem_u32(sA + s * C::A_BYTES);
         const uint32_t b_base = ptx::smem_u32(sB + s * C::B_BYTES);
 #pragma unroll
-        for (int k = 0; k < BK / 16; ++k) {
+        for (int k = 0; k < C::KBYTES / 32; ++k) {
 #pragma unroll
           for (int nt = 0; nt < NT; ++nt) {
-            // K-major: the 16-element K slice sits 32 bytes further along each
-            // swizzled 128-byte row (SBO = 1024 between 8-row groups).
-            // MN-major: 16 K rows further = 2 x 1024 bytes; LBO = 8192 between
-            // the 64-element MN chunks, SBO = 1024 between 8-row K groups.
-            // Column subtile nt: its own B box, BH rows further.
-            const uint32_t bs = b_base + nt * C::BH * BK * 2;
-            const uint64_t bd = B_MN ? ptx::sdesc_sw128(bs + k * 2048, 64 * BK * 2, 1024)
-                                     : ptx::sdesc_sw128(bs + k * 32, 16, 1024);
+            // K-major: the 32-byte K slice of one MMA sits 32 bytes further
+            // along each swizzled row (SBO = 8 rows: 1024 bytes with 128-byte
+            // rows, 512 with 64-byte ones).  MN-major: 16 K rows further = 2 x
+            // 1024 bytes; LBO = 128 x BKE between the 64-element MN chunks,
+            // SBO = 1024 between 8-row K groups.  Column subtile nt: its own B
+            // box, BH rows further.
+            const uint32_t bs = b_base + nt * C::BH * C::KBYTES;
+            const uint64_t bd = B_MN            ? ptx::sdesc_sw128(bs + k * 2048, 64 * C::BKE * 2, 1024)
+                                : KB == 128     ? ptx::sdesc_sw128(bs + k * 32, 16, 1024)
+                                                : ptx::sdesc_sw64(bs + k * 32, 16, 512);
 #pragma unroll
             for (int mt = 0; mt < MT; ++mt) {
               // row subtile mt: BM rows further in the A stage, its own accumulator
-              const uint32_t as = a_base + mt * BM * BK * 2;
-              const uint64_t ad = A_MN ? ptx::sdesc_sw128(as + k * 2048, 64 * BK * 2, 1024)
-                                       : ptx::sdesc_sw128(as + k * 32, 16, 1024);
+              const uint32_t as = a_base + mt * BM * C::KBYTES;
+              const uint64_t ad = A_MN        ? ptx::sdesc_sw128(as + k * 2048, 64 * C::BKE * 2, 1024)
+                                  : KB == 128 ? ptx::sdesc_sw128(as + k * 32, 16, 1024)
+                                              : ptx::sdesc_sw64(as + k * 32, 16, 512);
               const uint32_t acc = tmem + (uint32_t)((mt * NT + nt) * C::ACC_COLS);
               if constexpr (TF32) {
                 // Ah Bh + Ah Bl + Al Bh (the lo parts LO bytes further on)
@@ -865,10 +873,16 @@ bool encode_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, 
 bool make_map(CUtensorMap* m, const void* ptr, int esize, int cols, int rows, int ld, int box_cols, int box_rows) {
   return encode_map(m, ptr, esize, cols, rows, ld, box_cols, box_rows, CU_TENSOR_MAP_SWIZZLE_128B);
 }
+// A K-major bf16 operand [rows, K] in boxes of box_rows rows and one stage's
+// K row of kb bytes (128: 128-byte swizzle; 64: 64-byte swizzle).
+bool make_kmajor_map(CUtensorMap* m, const bf16* ptr, int K, int rows, int ld, int box_rows, int kb) {
+  return encode_map(m, ptr, 2, K, rows, ld, kb / 2, box_rows,
+                    kb == 128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_64B);
+}
 
-template <int BN, int NSTAGE, int MT, bool PAIR, int NT, int MODE, int OPB>
+template <int BN, int NSTAGE, int MT, bool PAIR, int NT, int MODE, int OPB, int KB>
 constexpr int tc_smem() {
-  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB>;
+  using C = TcCfg<BN, NSTAGE, MT, PAIR, NT, OPB, KB>;
   return C::SMEM + (MODE == MODE_FWD_LOGITS ? BN * kLogitStride * 4 : 0) + (MODE == MODE_FWD_LG ? C::LG_SMEM : 0);
 }
 
@@ -876,9 +890,9 @@ constexpr int tc_smem() {
 // pairs; a padding CTA loads zeros, supplies its half of B and writes
 // nothing), clusters of the pair (LG: of the pair and every column tile),
 // and programmatic stream serialization.
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB = 2>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT, int OPB = 2, int KB = 128>
 struct TcLaunch {
-  static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE, OPB>();
+  static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE, OPB, KB>();
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
   static constexpr int CM = PAIR ? 2 : 1;
   cudaLaunchConfig_t cfg = {};
@@ -898,18 +912,19 @@ struct TcLaunch {
     cfg.attrs = at;
     cfg.numAttrs = 2;
   }
-  static auto kernel() { return k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB>; }
+  static auto kernel() { return k_tc_gemm<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB, KB>; }
   static cudaError_t set_attrs() {
     static cudaError_t e = cudaFuncSetAttribute(kernel(), cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM);
     return e;
   }
 };
 
-template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT = 1, int OPB = 2>
+template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT, int NT = 1, int OPB = 2,
+          int KB = 128>
 cudaError_t launch_tc(const CUtensorMap& ta, const CUtensorMap& tb, const CUtensorMap& tc, int tma_store, int M, int N,
                       int K, const EpiArgs& ep, int* err, cudaStream_t st, const CUtensorMap* td = nullptr,
                       const GradPrepArgs* lg = nullptr) {
-  using Lc = TcLaunch<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB>;
+  using Lc = TcLaunch<BN, A_MN, B_MN, MODE, PAIR, NSTAGE, MT, NT, OPB, KB>;
   const cudaError_t attr = Lc::set_attrs();
   if (attr != cudaSuccess) return attr;
   Lc l(M, N, st);
@@ -931,9 +946,21 @@ constexpr int WGRAD_BN = 256;
 // two layers' GEMMs no longer fit on the GPU side by side (re-measured with
 // dependent launch and the later Adam changes: 9.54 against 8.32 ms); earlier
 // 128 x 256 tiles and 4-CTA multicast clusters measured 9.8 and 11.1 ms.
+// The ring of the two-subtile forward, store and weight-gradient GEMMs holds
+// 144 KB either as 3 stages of 64-deep K steps (128-byte rows) or as 6
+// stages of 32-deep ones (64-byte rows, 24 KB).  The finer ring keeps 120 KB
+// of operand loads in flight instead of 96 KB: an epoch's forward GEMMs, one
+// at a time, 6.61 -> 6.10-6.19 ms; the epoch 8.10 -> 7.95 ms.  Deeper rings of 24 KB
+// stages are faster alone but slower in the epoch, as the 4-stage ring of
+// 48 KB was (7 / 8 stages: 8.00 / 8.57 ms): past ~170 KB a GEMM CTA leaves
+// too little of its SM to the other streams' blocks.  The one-subtile GEMMs
+// below keep 128-byte rows: 8 stages of 16 KB hold fewer bytes in flight than
+// their 6 of 32 KB (layer 1's weight gradient slower, the epoch 7.98 ms).
 constexpr bool USE_PAIR = true;
-constexpr int NSTAGES = 3;       // operand ring depth
+constexpr int NSTAGES = 3;       // operand ring depth with 128-byte K rows (48 KB stages)
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
+constexpr int KB_FULL = 64;      // bytes of K per operand row of a stage, two-subtile GEMMs
+constexpr int NSTAGES_FULL = 6;  // their ring depth
 constexpr int CLUSTER_M = USE_PAIR ? 2 : 1;
 // A GEMM that would get fewer than kSmallGridCtas CTAs with two subtiles per
 // CTA (at most a third of the GPU, e.g. 1216 batch rows of a 2000-wide
@@ -1037,8 +1064,9 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
   Shape sh = shape_of(M, N, FWD_BN);
   if (sh == SHAPE_TINY && !ep.narrow) sh = SHAPE_SMALL;
   const int bn = sh == SHAPE_TINY ? TINY_BN : FWD_BN;
+  const int kb = sh == SHAPE_FULL && !ep.logit_V ? KB_FULL : 128;
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(bn)) ||
+  if (!make_kmajor_map(&ta, A, K, M, lda, BM, kb) || !make_kmajor_map(&tb, B, K, N, ldb, b_box_rows(bn), kb) ||
       !make_map(&tc, ep.out, 2, ep.ldo, M, ep.ldo, 64, 32))
     return cudaErrorInvalidValue;
   if (ep.logit_V) {
@@ -1054,7 +1082,8 @@ cudaError_t tc_gemm_fwd(const bf16* A, int lda, const bf16* B, int ldb, int M, i
     return launch_tc<TINY_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_TINY, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
   if (sh == SHAPE_SMALL)
     return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, 1, M, N, K, ep, err, st);
-  return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, 1, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_FWD, USE_PAIR, NSTAGES_FULL, ROW_SUBTILES, 1, 2, KB_FULL>(ta, tb, tc, 1, M,
+                                                                                                     N, K, ep, err, st);
 }
 
 // fp32 C written through shared memory and TMA when its rows are 16-byte
@@ -1065,32 +1094,40 @@ static bool store_map(CUtensorMap* tc, float* C, int ldc, int rows, int cols) {
 
 cudaError_t tc_gemm_store(const bf16* A, int lda, const bf16* B, int ldb, int M, int N, int K, float* Cm,
                           int ldc, int* err, cudaStream_t st) {
+  const bool full = shape_of(M, N, FWD_BN) == SHAPE_FULL;
+  const int kb = full ? KB_FULL : 128;
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, A, 2, K, M, lda, BK, BM) || !make_map(&tb, B, 2, K, N, ldb, BK, b_box_rows(FWD_BN)))
+  if (!make_kmajor_map(&ta, A, K, M, lda, BM, kb) || !make_kmajor_map(&tb, B, K, N, ldb, b_box_rows(FWD_BN), kb))
     return cudaErrorInvalidValue;
   const int tma = store_map(&tc, Cm, ldc, M, N) ? 1 : 0;
   if (!tma) tc = ta;  // unused
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  if (shape_of(M, N, FWD_BN) != SHAPE_FULL)
+  if (!full)
     return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, M, N, K, ep, err,
                                                                                    st);
-  return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, M, N, K, ep, err, st);
+  return launch_tc<FWD_BN, false, false, MODE_STORE, USE_PAIR, NSTAGES_FULL, ROW_SUBTILES, 1, 2, KB_FULL>(
+      ta, tb, tc, tma, M, N, K, ep, err, st);
 }
 
 cudaError_t tc_gemm_wgrad(const bf16* G, int ldg, const bf16* X, int ldx, int R, int N, int K, float* Cm, int ldc,
                           int* err, cudaStream_t st) {
   // C[N, K] = sum_r G[r, n] X[r, k]: the GEMM's M is N (rows of dW), its N is
   // K (columns of dW), its contraction is R; both operands MN-major.
+  // MN-major boxes: 64 elements (128 bytes, 128-byte swizzle) of M or N by
+  // one stage's K rows
+  const bool full = shape_of(N, K, WGRAD_BN) == SHAPE_FULL;
+  const int bke = (full ? KB_FULL : 128) / 2;
   CUtensorMap ta, tb, tc;
-  if (!make_map(&ta, G, 2, N, R, ldg, 64, BK) || !make_map(&tb, X, 2, K, R, ldx, 64, BK))
+  if (!make_map(&ta, G, 2, N, R, ldg, 64, bke) || !make_map(&tb, X, 2, K, R, ldx, 64, bke))
     return cudaErrorInvalidValue;
   const int tma = store_map(&tc, Cm, ldc, N, K) ? 1 : 0;
   if (!tma) tc = ta;
   EpiArgs ep{nullptr, nullptr, Cm, ldc, nullptr};
-  if (shape_of(N, K, WGRAD_BN) != SHAPE_FULL)
+  if (!full)
     return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES_SMALL, 1>(ta, tb, tc, tma, N, K, R, ep, err,
                                                                                    st);
-  return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES, ROW_SUBTILES>(ta, tb, tc, tma, N, K, R, ep, err, st);
+  return launch_tc<WGRAD_BN, true, true, MODE_STORE, USE_PAIR, NSTAGES_FULL, ROW_SUBTILES, 1, 2, KB_FULL>(
+      ta, tb, tc, tma, N, K, R, ep, err, st);
 }
 
 // ------------------------------------------------ fp32 operands (3 x TF32)
