@@ -894,6 +894,11 @@ template <int BN, bool A_MN, bool B_MN, int MODE, bool PAIR, int NSTAGE, int MT,
 struct TcLaunch {
   static constexpr int SMEM = tc_smem<BN, NSTAGE, MT, PAIR, NT, MODE, OPB, KB>();
   static_assert(SMEM <= 227 * 1024, "shared memory per CTA");
+  // More than half of an SM's 228 KB (with the 1 KB each CTA reserves): no
+  // two GEMM CTAs, of this or any other instance, share an SM, so no TMEM
+  // allocation waits for another CTA's (a pair waiting on a pair could
+  // otherwise deadlock).
+  static_assert(SMEM > 113 * 1024, "a GEMM CTA must hold more than half of its SM's shared memory");
   static constexpr int CM = PAIR ? 2 : 1;
   cudaLaunchConfig_t cfg = {};
   cudaLaunchAttribute at[2];
@@ -953,9 +958,7 @@ constexpr int WGRAD_BN = 256;
 // at a time, 6.61 -> 6.10-6.19 ms; the epoch 8.10 -> 7.95 ms.  Deeper rings of 24 KB
 // stages are faster alone but slower in the epoch, as the 4-stage ring of
 // 48 KB was (7 / 8 stages: 8.00 / 8.57 ms): past ~170 KB a GEMM CTA leaves
-// too little of its SM to the other streams' blocks.  The one-subtile GEMMs
-// below keep 128-byte rows: 8 stages of 16 KB hold fewer bytes in flight than
-// their 6 of 32 KB (layer 1's weight gradient slower, the epoch 7.98 ms).
+// too little of its SM to the other streams' blocks.
 constexpr bool USE_PAIR = true;
 constexpr int NSTAGES = 3;       // operand ring depth with 128-byte K rows (48 KB stages)
 constexpr int ROW_SUBTILES = 2;  // 128-row subtiles per CTA (each with its own TMEM accumulator)
@@ -965,11 +968,17 @@ constexpr int CLUSTER_M = USE_PAIR ? 2 : 1;
 // A GEMM that would get fewer than kSmallGridCtas CTAs with two subtiles per
 // CTA (at most a third of the GPU, e.g. 1216 batch rows of a 2000-wide
 // layer) runs with one subtile per CTA instead: twice the CTAs, each with a
-// 6-stage ring of 32 KB stages.  One whose one-subtile grid still fills at
-// most half the SMs (1024 rows of a 2000-wide layer: 64 CTAs) also halves
-// the tile width to 128 columns (128 CTAs, 8-stage ring of 24 KB stages).
+// 4-stage ring of 32 KB stages (128-byte rows).  One whose one-subtile grid
+// still fills at most half the SMs (1024 rows of a 2000-wide layer: 64 CTAs)
+// also halves the tile width to 128 columns (128 CTAs, 8-stage ring of 24 KB
+// stages).  The one-subtile ring, on the epoch (layer 1's weight gradient):
+// 6 / 5 / 4 stages of 32 KB 7.90 / 7.89 / 7.81 ms -- the smaller footprint
+// again leaves more of the SM to the other streams; 8 stages of 16 KB
+// (64-byte rows, 128 KB) 7.98 ms.  Every ring keeps a CTA above half an
+// SM's shared memory, so two GEMM CTAs, whose TMEM allocations could then
+// wait on each other, never share an SM.
 constexpr int kSmallGridCtas = 64;
-constexpr int NSTAGES_SMALL = 6;
+constexpr int NSTAGES_SMALL = 4;
 constexpr int TINY_BN = 128;
 constexpr int kTinyGridCtas = 152 / 2;
 constexpr int NSTAGES_TINY = 8;
