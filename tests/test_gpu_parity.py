@@ -132,6 +132,9 @@ STEP_CASES = [
     ("fp32", 64, 784, 500, True), ("bf16", 64, 784, 500, True), ("bf16", 3, 11, 5, True), ("fp32", 1, 11, 5, True),
     ("bf16", 1024, 784, 2000, True), ("bf16", 1024, 2000, 2000, False), ("fp32", 150, 2000, 300, False),
     ("bf16", 608, 2000, 2000, False),
+    # two-subtile GEMMs with ragged row tiles and a partial last 32-deep K step of the
+    # weight gradient (2000 batch rows)
+    ("bf16", 1000, 2000, 2000, False),
     # the Adam update's element-wise form (N*K not a multiple of 8, or a padded bf16 copy of W)
     ("fp32", 33, 20, 7, False), ("bf16", 40, 20, 6, False),
 ]
