@@ -389,6 +389,45 @@ def test_net_on_streams_is_bitwise_sequential(env):
             assert np.array_equal(sa[k], sb[k]), k
 
 
+def test_net_on_streams_is_bitwise_sequential_full_width(env):
+    """The same at the width the epoch runs: 784-2000-2000-2000, batches of
+    1000 and 1024 pairs, so the layers' two-subtile GEMMs (ragged row tiles,
+    a partial last K step of the weight gradient) run concurrently on the
+    layer streams; every layer's loss and state bitwise equal to the layers
+    stepped one after another."""
+    torch, ff = env
+    dims, Bs = (784, 2000, 2000, 2000), (1000, 1024, 1000)
+    L = len(dims) - 1
+    mk = lambda: [ff.Layer(dims[i], dims[i + 1], prec="bf16", init_seed=140 + i) for i in range(L)]
+    par, seq = mk(), mk()
+    net = ff.Net(par, max_B=max(Bs), depth=2)
+    hs = [seq[k].new_activation(2 * max(Bs)) for k in range(L - 1)]
+    ss = [torch.empty(2 * max(Bs), device="cuda") for _ in range(L - 1)]
+    lp = torch.empty(len(Bs), L, device="cuda")
+    ls = torch.empty(len(Bs), L, device="cuda")
+    xs = []
+    for t, B in enumerate(Bs):
+        x2, l2 = pair_inputs(B, seed=300 + t)
+        xs.append((torch.from_numpy(x2).cuda(), torch.from_numpy(l2).cuda()))
+    for t, B in enumerate(Bs):
+        net.train_step(xs[t][0], xs[t][1], B=B, loss=lp[t])
+    net.sync()
+    for t, B in enumerate(Bs):
+        M = 2 * B
+        seq[0].train_step(xs[t][0], labels=xs[t][1], B=B, h_out=hs[0][:M], next_scale=ss[0][:M], loss=ls[t, 0:1])
+        for k in range(1, L):
+            last = k == L - 1
+            seq[k].train_step(hs[k - 1][:M], row_scale=ss[k - 1][:M], B=B,
+                              h_out=None if last else hs[k][:M], next_scale=None if last else ss[k][:M],
+                              loss=ls[t, k:k + 1])
+    torch.cuda.synchronize()
+    assert torch.equal(lp, ls)
+    for a, b in zip(par, seq):
+        sa, sb = a.get_state(), b.get_state()
+        for k in ("W", "b", "mW", "vW"):
+            assert np.array_equal(sa[k], sb[k]), k
+
+
 def test_repeat_runs_are_bitwise_equal(env):
     torch, ff = env
     B = 256
