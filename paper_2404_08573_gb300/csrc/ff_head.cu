@@ -517,7 +517,21 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   const int lane = threadIdx.x, tid = threadIdx.y * 32 + threadIdx.x;
   const int c0 = blockIdx.x * 256;
   const int cg = c0 + lane * 8;
+  const bool cols_ok = cg < a.ld;
   ptx::griddep_wait();  // launched with programmatic stream serialization
+  // this thread's activity (rows y, y+8, y+16, y+24; 8 columns), loaded first
+  // so that its latency overlaps the logits and softmax below
+  float hv[4][8];
+#pragma unroll
+  for (int k = 0; k < 4; ++k) {
+    const int i = r0 + threadIdx.y + 8 * k;
+    if (cols_ok && i < a.n) {
+      Vec8<T>::load(H + (size_t)i * a.ld + cg, hv[k]);
+    } else {
+#pragma unroll
+      for (int e = 0; e < 8; ++e) hv[k][e] = 0.f;
+    }
+  }
   for (int idx = tid; idx < kClasses * 256; idx += 256) {
     const int c = idx / 256, j = idx % 256;
     Vsh[c][j % 8][j / 8] = (c0 + j < a.N) ? __ldg(a.V + (size_t)c * a.N + c0 + j) : 0.f;
@@ -587,7 +601,6 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
     a.ds->bc2 = (float)(1.0 - a.ds->pow2);
   }
   __syncthreads();
-  const bool cols_ok = cg < a.ld;
   float db[8];
 #pragma unroll
   for (int e = 0; e < 8; ++e) db[e] = 0.f;
@@ -595,13 +608,8 @@ __global__ void __launch_bounds__(256) k_po_grad(PoGradArgs a, const T* __restri
   for (int k = 0; k < 4; ++k) {
     const int li = threadIdx.y + 8 * k;
     const int i = r0 + li;
-    float h[8], z[8];
-    if (cols_ok && i < a.n) {
-      Vec8<T>::load(H + (size_t)i * a.ld + cg, h);
-    } else {
-#pragma unroll
-      for (int e = 0; e < 8; ++e) h[e] = 0.f;
-    }
+    const float(&h)[8] = hv[k];
+    float z[8];
     Vec8<T>::store(&Hs[li][lane * 8], h);
     if (!cols_ok || i >= a.n) continue;
     const float si = __ldg(a.s + i);
