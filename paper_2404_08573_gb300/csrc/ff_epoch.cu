@@ -331,17 +331,6 @@ __device__ void signal_done(const EpochP& P, uint2 t) {
 }
 
 
-__device__ __forceinline__ void load_h8(const bf16* p, float (&v)[8]) {
-  const uint4 u = ldcg16(p);
-  const __nv_bfloat162* h = reinterpret_cast<const __nv_bfloat162*>(&u);
-#pragma unroll
-  for (int e = 0; e < 4; ++e) {
-    const float2 f = __bfloat1622float2(h[e]);
-    v[2 * e] = f.x;
-    v[2 * e + 1] = f.y;
-  }
-}
-
 // ------------------------------------------------------------- stream tasks
 // s: streamer thread 0..NSTR-1 (s >> 5 its warp, lane its lane).
 
